@@ -1,0 +1,445 @@
+#!/usr/bin/env python
+"""Benchmark of the region-sparse DiT denoising step on GB300.
+
+Workload: PixArt-alpha-shaped DiT at 1024 px (64 x 64 = 4096 image tokens,
+28 blocks, hidden 1152, 16 heads of 72, MLP 4608, 120 text tokens, 20
+timesteps), batch 1, bf16 weights and a bf16 per-(layer, timestep) K/V/hidden
+cache of 15.85 GB resident in HBM.  The dirty region of each sweep point is a
+union of 1-3 seeded ellipses covering 5 / 10 / 20 / 40 % of the tokens,
+presented to the localisation kernel as a cross-attention score map.
+
+One step = localisation mask (rc_localize_mask) + one region-sparse
+denoising step (rc_step, mode SPARSE) at timestep t = step mod 20; the
+headline value is steps/s at 20 % dirty.  The library's own dense path
+(rc_step_dense) and every sweep point are reported beside it.
+
+Usage: python bench.py [--gpus N --steps K --warmup W] [--impl reference]
+For N > 1 launch with torch.distributed.run: every rank runs an independent
+replica (its own session and cache); value = all ranks' steps / max time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2608_29809_gb300 import synth  # noqa: E402
+
+METRIC = "region-reuse DiT steps/s @4096 tok vs dirty %; % of BF16 tensor peak"
+UNIT = "steps/s"
+SEED = 1234 + 300
+FRACS = (0.05, 0.10, 0.20, 0.40)
+HEADLINE = 0.20
+WORKLOAD = "pixart-alpha-1024px: 4096 tokens, 28 blocks, 20 timesteps, batch 1"
+L2_NOTE = ("inputs larger than L2: each step streams 1.04 GB of weights and a different "
+           "28 x 28.3 MB cache slice per timestep")
+
+
+def linear_flops_per_token_block(d: synth.Dims) -> float:
+    """2 x (3h^2 + h^2 + h^2 + h^2 + hF + Fh) multiply-adds per dirty token and block."""
+    h, F = d.hidden, d.mlp
+    return 2.0 * (6 * h * h + 2 * h * F)
+
+
+def attn_flops_per_token_block(d: synth.Dims) -> float:
+    """Self-attention (4 N h) plus cross-attention (4 M h) per dirty token and block."""
+    return 4.0 * d.tokens * d.hidden + 4.0 * d.text_len * d.hidden
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            j = json.load(f)
+        return {"hbm_gbs": j["hbm_gbs"], "bf16_tflops": j["bf16_tflops"],
+                "bf16_tflops_sustained": j.get("bf16_tflops_sustained", j["bf16_tflops"]),
+                "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "source": "fallback"}
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi samples (200 ms) of SM clock and throttle reasons."""
+
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-i", str(self.index)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in out.strip().splitlines():
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx.append(float(f[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[4:8]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------ distributed
+def dist_setup(n_gpus: int):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world != n_gpus:
+        raise SystemExit(f"--gpus {n_gpus} but WORLD_SIZE={world}; launch N>1 with torchrun")
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------ our arm
+class Workload:
+    def __init__(self, R, d: synth.Dims, seed: int, dev: str):
+        self.R, self.d, self.dev = R, d, dev
+        w = synth.make_weights(d, seed, device=dev)
+        self.model = R.Model(d, w, sessions=1, device=dev)
+        ctx, cache = self.model.ctx, self.model.cache
+        for t in range(d.timesteps):
+            for l in range(d.layers):
+                H, K, V = synth.make_cache_slice(d, seed, 0, l, t, device=dev)
+                R.rc_cache_fill(cache, 0, l, t, H, K, V)
+        torch.cuda.synchronize()
+        self.text = synth.make_text(d, seed, dev)
+        R.rc_set_text(ctx, cache, 0, self.text)
+        tv, ab = synth.ddim_tables(d.timesteps)
+        R.rc_set_schedule(ctx, tv, ab)
+        self.latent0 = synth.make_latent(d, seed, dev)
+        self.latent = self.latent0.clone()
+        N = d.tokens
+        self.mask = torch.zeros(N, dtype=torch.uint8, device=dev)
+        self.idx = torch.zeros(N, dtype=torch.int32, device=dev)
+        self.cnt = torch.zeros(1, dtype=torch.int32, device=dev)
+        self.ws = torch.empty(R.rc_localize_workspace_size(N, 8), dtype=torch.uint8, device=dev)
+        self.sparse = np.full(d.timesteps, R.RC_MODE_SPARSE, np.uint8)
+        self.scores = {}
+        for f in FRACS:
+            blobs = synth.ellipse_blobs(d, seed, f)
+            A, ids = synth.indicator_scores(d, blobs, seed)
+            self.scores[f] = (torch.from_numpy(A).to(dev), ids, A)
+
+    def localize(self, f, A=None):
+        d = self.d
+        A_dev, ids, _ = self.scores[f]
+        self.R.rc_localize_mask(A_dev if A is None else A, 1, d.tokens, d.text_len, d.grid_h,
+                                d.grid_w, ids, 0.5, 0, self.mask, self.idx, self.cnt, self.ws)
+
+    def step(self, i, f):
+        t = i % self.d.timesteps
+        if t == 0:
+            self.latent.copy_(self.latent0)
+        self.localize(f)
+        self.R.rc_step(self.model.ctx, self.model.cache, 0, self.latent, t, self.sparse, self.idx,
+                       -1, self.cnt)
+
+    def step_dense(self, i):
+        t = i % self.d.timesteps
+        if t == 0:
+            self.latent.copy_(self.latent0)
+        self.R.rc_step_dense(self.model.ctx, self.model.cache, 0, self.latent, t)
+
+
+def timed(fn, K, W, world):
+    for i in range(W):
+        fn(i)
+    torch.cuda.synchronize()
+    barrier(world)
+    torch.cuda.synchronize()
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record()
+    for i in range(K):
+        fn(W + i)
+    e.record()
+    torch.cuda.synchronize()
+    barrier(world)
+    return s.elapsed_time(e)  # ms
+
+
+def run_ours(args, world, rank, local):
+    from paper_2608_29809_gb300 import regioncache as R
+    torch.cuda.set_device(local)
+    dev = f"cuda:{local}"
+    d = synth.PIXART_1024
+    K, W = args.steps, args.warmup
+    wl = Workload(R, d, SEED + rank, dev)
+    peaks = load_peaks()
+
+    # headline: 20 % dirty, with the GEMM probe and the clock sampler running
+    R.rc_probe_enable(wl.model.ctx, R.RC_PROBE_GEMM, K * d.layers * 6)
+    for i in range(W):
+        wl.step(i, HEADLINE)
+    torch.cuda.synchronize()
+    R.rc_probe_read(wl.model.ctx)  # drop warm-up launches
+    clocks = ClockSampler(local)
+    clocks.start()
+    n0 = R.rc_launch_count()
+    ms = timed(lambda i: wl.step(i, HEADLINE), K, 0, world)
+    launches = R.rc_launch_count() - n0
+    clk = clocks.stop()
+    gemm_ms, gemm_n = R.rc_probe_read(wl.model.ctx)
+    R.rc_probe_enable(wl.model.ctx, R.RC_PROBE_OFF, 0)
+    R.rc_sync(wl.model.ctx)
+    D = int(wl.cnt.item())
+    ms_max = max_over_ranks(ms, world)
+    value = K * world / (ms_max / 1e3)
+
+    # attention probe (separate pass over the same workload)
+    R.rc_probe_enable(wl.model.ctx, R.RC_PROBE_ATTENTION, K * d.layers * 2)
+    timed(lambda i: wl.step(i, HEADLINE), K, 0, 1)
+    att_ms, att_n = R.rc_probe_read(wl.model.ctx)
+    R.rc_probe_enable(wl.model.ctx, R.RC_PROBE_OFF, 0)
+
+    # sweep and dense baseline
+    sweep, dirty = {}, {}
+    for f in FRACS:
+        m = timed(lambda i, f=f: wl.step(i, f), K, W, world)
+        sweep[f"{f:.2f}"] = round(K * world / (max_over_ranks(m, world) / 1e3), 3)
+        dirty[f"{f:.2f}"] = int(wl.cnt.item())
+    m = timed(wl.step_dense, max(2, K // 2), min(W, 3), world)
+    dense = max(2, K // 2) * world / (max_over_ranks(m, world) / 1e3)
+    R.rc_sync(wl.model.ctx)
+
+    # end to end through the C ABI with host buffers: per step the score map
+    # and the latent go host -> device, the updated latent comes back
+    A_host = torch.from_numpy(wl.scores[HEADLINE][2]).pin_memory()
+    lat_host = wl.latent0.cpu().pin_memory()
+    A_dev = torch.empty_like(A_host, device=dev)
+
+    def e2e_step(i):
+        t = i % d.timesteps
+        if t == 0:
+            lat_host.copy_(wl.latent0.cpu())
+        A_dev.copy_(A_host, non_blocking=True)
+        wl.latent.copy_(lat_host, non_blocking=True)
+        wl.localize(HEADLINE, A_dev)
+        R.rc_step(wl.model.ctx, wl.model.cache, 0, wl.latent, t, wl.sparse, wl.idx, -1, wl.cnt)
+        lat_host.copy_(wl.latent, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+
+    for i in range(W):
+        e2e_step(i)
+    barrier(world)
+    t0 = time.perf_counter()
+    for i in range(K):
+        e2e_step(i)
+    e2e_s = max_over_ranks(time.perf_counter() - t0, world)
+    barrier(world)
+    e2e = {"value": round(K * world / e2e_s, 3), "unit": UNIT,
+           "h2d_bytes_per_step": int(A_host.numel() * 4 + lat_host.numel() * 4),
+           "d2h_bytes_per_step": int(lat_host.numel() * 4)}
+
+    lin_flops_launch = linear_flops_per_token_block(d) * D * d.layers / (6 * d.layers)
+    gemm_avg_ms = gemm_ms / max(gemm_n, 1)
+    gemm_tflops = linear_flops_per_token_block(d) * D * d.layers * K / (gemm_ms / 1e3) / 1e12
+    peak = peaks["bf16_tflops_sustained"]
+    att_tflops = (attn_flops_per_token_block(d) * D * d.layers * K) / (att_ms / 1e3) / 1e12
+    roofline = {"bound": "tensor", "achieved": round(gemm_tflops, 2), "peak": peak,
+                "unit": "TFLOP/s", "frac": round(gemm_tflops / peak, 4), "traffic": None,
+                "kernel": "gemm (QKV, out, cross-q, cross-out, fc1, fc2 of every block)",
+                "launches": gemm_n, "avg_launch_ms": round(gemm_avg_ms, 5),
+                "flops_per_launch": lin_flops_launch,
+                "peak_source": f"{peaks['source']} bf16_tflops_sustained"}
+    roof_att = {"bound": "tensor", "achieved": round(att_tflops, 2), "peak": peak,
+                "unit": "TFLOP/s", "frac": round(att_tflops / peak, 4), "launches": att_n,
+                "avg_launch_ms": round(att_ms / max(att_n, 1), 5)}
+    out = {
+        "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
+        "steps": K, "warmup": W, "ms_per_step": round(ms_max / K, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic: seeded random-init PixArt-alpha-shaped weights, cache, text, "
+                "latent and ellipse-blob score maps",
+        "config": {"workload": WORKLOAD, "tokens": d.tokens, "dirty_frac": HEADLINE,
+                   "dirty_tokens": D, "layers": d.layers, "timesteps": d.timesteps,
+                   "sessions_per_gpu": 1, "parallelism": "replicas" if world > 1 else "single",
+                   "l2": L2_NOTE, "step": "rc_localize_mask + rc_step(SPARSE)"},
+        "sweep_steps_per_s": sweep, "sweep_dirty_tokens": dirty,
+        "dense_steps_per_s": round(dense, 3),
+        "speedup_vs_dense": {k: round(v / dense, 3) for k, v in sweep.items()},
+        "roofline": roofline, "roofline_attention": roof_att,
+        "e2e": e2e, "gpu_launches": int(launches), "clocks": clk,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(d, SEED, HEADLINE, layers_sample=args.cpu_layers)
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    wl.model.close()
+
+
+# ------------------------------------------------------------- oracle arm
+def oracle_sample(d: synth.Dims, seed: int, f: float, layers_sample: int):
+    """Oracle inputs for the first `layers_sample` blocks of the workload."""
+    import oracle as O
+    from dataclasses import replace
+    ds = replace(d, layers=layers_sample)
+    w = synth.make_weights(ds, seed)
+    layers = [{k: O.to64(v) for k, v in L.items()} for L in w.layers]
+    G = {k: O.to64(v) for k, v in w.glob.items()}
+    pos = O.to64(w.pos)
+    ctx = O.to64(synth.make_text(d, seed))
+    tkv = [O.text_kv(ctx, L) for L in layers]
+    cache = [dict(zip("HKV", (O.to64(a) for a in synth.make_cache_slice(d, seed, 0, l, 0))))
+             for l in range(layers_sample)]
+    blobs = synth.ellipse_blobs(d, seed, f)
+    A, ids = synth.indicator_scores(d, blobs, seed)
+    lat = O.to64(synth.make_latent(d, seed))
+    return O, ds, layers, G, pos, tkv, cache, A, ids, lat
+
+
+def cpu_baseline(d, seed, f, layers_sample=2):
+    """The oracle, as it stands, on the host cores: localisation, `layers_sample`
+    region blocks and the final layer of one step of the headline workload,
+    scaled to a full 28-block step."""
+    O, ds, layers, G, pos, tkv, cache, A, ids, lat = oracle_sample(d, seed, f, layers_sample)
+    t0 = time.perf_counter()
+    _, idx = O.localize_mask(A, ids, d.grid_h, d.grid_w, 0.5, 0)
+    t_loc = time.perf_counter() - t0
+    temb = O.t_embed(999.0, G)
+    tb = O.t_block(temb, G)
+    x = O.patch_embed(lat, idx, G, pos, d.patch)
+    t0 = time.perf_counter()
+    for l in range(layers_sample):
+        _, x = O.region_block(x, idx, cache[l], layers[l], layers[l]["table"] + tb, tkv[l],
+                              d.heads)
+    t_blk = (time.perf_counter() - t0) / layers_sample
+    t0 = time.perf_counter()
+    eps = O.final_layer(cache[-1]["H"], temb, G, d.grid_h, d.grid_w, d.patch, d.in_ch)
+    O.ddim_update(lat, eps, 0.5, 0.6)
+    t_fin = time.perf_counter() - t0
+    step_s = t_loc + d.layers * t_blk + t_fin
+    return {"value": round(1.0 / step_s, 6), "unit": UNIT, "cores": os.cpu_count(),
+            "kind": "oracle",
+            "sample": f"one step of the headline workload ({int(f * 100)} % dirty, D={len(idx)}) "
+                      f"timed as localisation + {layers_sample} of {d.layers} region blocks "
+                      f"(scaled x{d.layers}/{layers_sample}) + final layer; float64 numpy",
+            "seconds_per_step": round(step_s, 3)}
+
+
+def run_reference(args, world, rank):
+    if rank != 0:
+        return
+    d = synth.PIXART_1024
+    layers_sample = 2
+    O, ds, layers, G, pos, tkv, cache, A, ids, lat = oracle_sample(d, SEED, HEADLINE,
+                                                                   layers_sample)
+    t0 = time.perf_counter()
+    _, idx = O.localize_mask(A, ids, d.grid_h, d.grid_w, 0.5, 0)
+    temb = O.t_embed(999.0, G)
+    tb = O.t_block(temb, G)
+    x = O.patch_embed(lat, idx, G, pos, d.patch)
+    eps = O.final_layer(cache[-1]["H"], temb, G, d.grid_h, d.grid_w, d.patch, d.in_ch)
+    O.ddim_update(lat, eps, 0.5, 0.6)
+    t_fixed = time.perf_counter() - t0
+
+    def one(i):
+        l = i % layers_sample
+        s = time.perf_counter()
+        O.region_block(x, idx, cache[l], layers[l], layers[l]["table"] + tb, tkv[l], d.heads)
+        return time.perf_counter() - s
+
+    for i in range(args.warmup):
+        one(i)
+    ts = [one(i) for i in range(args.steps)]
+    step_s = t_fixed + d.layers * (sum(ts) / len(ts))
+    v = 1.0 / step_s
+    sample = (f"each timed step is one of {layers_sample} oracle region blocks of the headline "
+              f"workload ({int(HEADLINE * 100)} % dirty, D={len(idx)}); steps/s = 1 / "
+              f"({d.layers} x mean block time + localisation + final layer)")
+    out = {"metric": METRIC, "value": round(v, 6), "unit": UNIT, "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_s * 1e3, 3),
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+           "data": "synthetic", "impl": "reference",
+           "config": {"workload": WORKLOAD, "tokens": d.tokens, "dirty_frac": HEADLINE,
+                      "dirty_tokens": int(len(idx)), "layers": d.layers,
+                      "timesteps": d.timesteps},
+           "cpu_baseline": {"value": round(v, 6), "unit": UNIT, "cores": os.cpu_count(),
+                            "kind": "oracle", "sample": sample},
+           "e2e": {"value": round(v, 6), "unit": UNIT, "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-layers", type=int, default=2)
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        raise SystemExit("--warmup must be >= 3")
+    world, rank, local = dist_setup(args.gpus)
+    try:
+        if args.impl == "reference":
+            run_reference(args, world, rank)
+        else:
+            run_ours(args, world, rank, local)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

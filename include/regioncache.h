@@ -1,0 +1,263 @@
+/*
+ * regioncache.h -- C ABI of the GB300 (sm_103a) region-sparse DiT step.
+ *
+ * The library implements the hot path of RegionCache (semantic-aware region
+ * reuse for multi-turn image editing): a cross-attention localisation pass
+ * turns the prompt-delta text tokens into a token-level dirty mask
+ * (Section 3.2, R_edit); only dirty image tokens are recomputed through each
+ * PixArt-alpha-shaped block, their queries attending over every token's
+ * keys/values, where clean tokens' K/V and hidden states come from a
+ * per-(layer, timestep) cache (Section 3.3, Region-Level Sparse Attention);
+ * fresh K/V rows are written straight to their cache rows by the projection
+ * GEMM (Section 3.4, Kernel Fusing); a step follows a per-step reuse
+ * schedule given as input (Section 3.3, Eq. 2).
+ *
+ * Conventions for every entry point:
+ *   - Return value: rc_status; RC_OK (0) on success.  No C++ exception ever
+ *     crosses this boundary.  rc_last_error() gives a thread-local message
+ *     for the last failing call on the calling thread.
+ *   - Host arguments are validated before anything is launched; a failing
+ *     validation launches nothing and changes no memory.
+ *   - Pointers named *_host are host memory.  Every other tensor pointer is a
+ *     device pointer owned by the caller, who keeps it alive and unmodified
+ *     until the work queued on `stream` has finished.  Weights are borrowed
+ *     for the lifetime of the rc_ctx.
+ *   - Work is queued asynchronously on `stream` (a cudaStream_t; 0 is the
+ *     legacy default stream).  Device-side argument errors (an index out of
+ *     range, a count above its bound) are recorded in a library-owned error
+ *     word and reported by rc_sync().
+ *   - Dtypes: "bf16" = bfloat16 (2 bytes), "f32" = IEEE float.  Matrices are
+ *     row-major.  Linear weights are [out][in]: y = x W^T + b.
+ */
+#ifndef REGIONCACHE_H
+#define REGIONCACHE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int rc_status;
+#define RC_OK 0
+#define RC_ERR_INVALID_ARG 1   /* null pointer, value out of range           */
+#define RC_ERR_SHAPE 2         /* sizes inconsistent with the rc_dims         */
+#define RC_ERR_OOM 3           /* device allocation failed                    */
+#define RC_ERR_CUDA 4          /* a CUDA runtime call failed                  */
+#define RC_ERR_TIMEOUT 5       /* a bounded device wait gave up               */
+#define RC_ERR_DEVICE_ASSERT 6 /* a kernel found a bad index / count          */
+#define RC_ERR_STATE 7         /* call order violated (e.g. no weights set)   */
+
+/* Per-step modes of a reuse schedule (Section 3.3, Eq. 2). */
+#define RC_MODE_DENSE 0  /* every token recomputed; cache rows overwritten    */
+#define RC_MODE_SPARSE 1 /* only the dirty tokens recomputed                  */
+#define RC_MODE_REUSE 2  /* no block runs; the last hidden state is cached    */
+
+typedef void* rc_stream; /* cudaStream_t */
+
+/* Model and problem sizes.  PixArt-alpha: hidden 1152, heads 16 (head_dim
+ * 72), mlp 4608, layers 28, patch 2, in_ch 4, out_ch 8, text_len 120,
+ * freq_dim 256.  N = grid_h * grid_w image tokens. */
+typedef struct rc_dims {
+  int hidden, heads, mlp, layers;
+  int grid_h, grid_w, patch, in_ch, out_ch;
+  int text_len, timesteps, freq_dim;
+} rc_dims;
+
+/* One block's weights (device pointers, borrowed).  W_* bf16 [out][in];
+ * b_* f32 [out]; table f32 [6][hidden] = the adaLN-single scale-shift table
+ * whose rows are (shift_msa, scale_msa, gate_msa, shift_mlp, scale_mlp,
+ * gate_mlp).  W_qkv's outputs are q | k | v; W_xkv's are k | v. */
+typedef struct rc_layer_weights {
+  const void* W_qkv; const float* b_qkv;  /* [3h][h], [3h] */
+  const void* W_o;   const float* b_o;    /* [h][h],  [h]  */
+  const void* W_xq;  const float* b_xq;   /* [h][h],  [h]  */
+  const void* W_xkv; const float* b_xkv;  /* [2h][h], [2h] */
+  const void* W_xo;  const float* b_xo;   /* [h][h],  [h]  */
+  const void* W_1;   const float* b_1;    /* [F][h],  [F]  */
+  const void* W_2;   const float* b_2;    /* [h][F],  [h]  */
+  const float* table;                     /* [6][h]        */
+} rc_layer_weights;
+
+/* Model-level weights (device pointers, borrowed).  W_e: patch embedding as a
+ * linear map of the patch vector ordered (channel, py, px), bf16
+ * [h][in_ch*p*p]; pos f32 [N][h] fixed positional table; timestep MLP
+ * W_t1 [h][freq_dim], W_t2 [h][h]; adaLN-single W_tb [6h][h]; final layer
+ * table_f f32 [2][h] (shift, scale), W_f bf16 [p*p*out_ch][h] with outputs
+ * ordered (py, px, channel). */
+typedef struct rc_global_weights {
+  const void* W_e;  const float* b_e;  const float* pos;
+  const void* W_t1; const float* b_t1;
+  const void* W_t2; const float* b_t2;
+  const void* W_tb; const float* b_tb;
+  const float* table_f;
+  const void* W_f;  const float* b_f;
+} rc_global_weights;
+
+typedef struct rc_ctx rc_ctx;     /* model + device scratch, one per stream user */
+typedef struct rc_cache rc_cache; /* library-owned per-(session, t, layer) cache */
+
+/* ---------------------------------------------------------------- context */
+
+/* Creates a context on the current CUDA device and allocates its scratch
+ * (sized for N tokens).  Errors: RC_ERR_INVALID_ARG (null, a dimension <= 0),
+ * RC_ERR_SHAPE (hidden % heads != 0, head_dim not 72 or 64, hidden not a
+ * multiple of 128 or above 1536, mlp not a multiple of 128, N > 16384,
+ * in_ch * patch^2 > 16, out_ch < in_ch), RC_ERR_OOM.  Validation happens
+ * before any CUDA call. */
+rc_status rc_create(const rc_dims* dims, rc_ctx** out);
+void rc_destroy(rc_ctx* ctx);
+
+/* Registers (borrows) the weights of block `layer` / of the model. */
+rc_status rc_set_layer_weights(rc_ctx* ctx, int layer, const rc_layer_weights* w);
+rc_status rc_set_global_weights(rc_ctx* ctx, const rc_global_weights* w);
+
+/* Sampling schedule, copied: timestep values t_values_host[timesteps] fed to
+ * the timestep embedding, and cumulative alphas alpha_bar_host[timesteps+1]
+ * (entry timesteps is the value after the last step, normally 1) for the
+ * DDIM (eta = 0) update after step t: alpha_bar[t] -> alpha_bar[t+1]. */
+rc_status rc_set_schedule(rc_ctx* ctx, const float* t_values_host, const float* alpha_bar_host);
+
+/* ------------------------------------------------------------------ cache */
+
+/* Cache pool of Section 3.2 (Hidden-State-Oriented Caching): for every
+ * session s, timestep t and layer l, the block output H^{l+1}, keys K^l and
+ * values V^l of all N tokens, bf16 [N][hidden] each, plus the per-session
+ * text keys/values of every layer.  Library-owned device memory:
+ * sessions * timesteps * layers * 3 * N * hidden * 2 bytes (15.85 GB for one
+ * PixArt-alpha session at 4096 tokens and 20 steps). */
+rc_status rc_cache_create(rc_ctx* ctx, int sessions, rc_cache** out);
+void rc_cache_destroy(rc_cache* cache);
+
+/* Copies caller bf16 [N][hidden] device buffers into / out of the (session,
+ * layer, t) slot.  Any of H, K, V may be null to skip it. */
+rc_status rc_cache_fill(rc_cache* cache, int session, int layer, int t,
+                        const void* H, const void* K, const void* V, rc_stream stream);
+rc_status rc_cache_read(rc_cache* cache, int session, int layer, int t,
+                        void* H, void* K, void* V, rc_stream stream);
+
+/* Text conditioning of one session for an editing turn: ctx_bf16 is the
+ * text context, bf16 [text_len][hidden].  Computes every layer's
+ * cross-attention keys/values (ctx W_xkv^T + b_xkv) into the session's
+ * cache.  Must precede rc_step / rc_block_forward_region for the session. */
+rc_status rc_set_text(rc_ctx* ctx, rc_cache* cache, int session, const void* ctx_bf16,
+                      rc_stream stream);
+
+/* ----------------------------------------------------------- localisation */
+
+/* Bytes of device workspace rc_localize_mask needs for N tokens and
+ * n_delta delta tokens. */
+size_t rc_localize_workspace_size(int N, int n_delta);
+
+/* Edit region R_edit of Section 3.2 as a dirty mask and a compact list.
+ *   xattn        f32 [S][N][M] cross-attention scores (S slices, e.g. heads
+ *                x layers, averaged: summed in ascending s, divided by S).
+ *   delta_ids_host  int32 [n_delta], the new/modified text tokens, each in
+ *                [0, M); 1 <= n_delta <= 64.
+ *   threshold    per delta token j the scores are min-max normalised over the
+ *                N tokens and token i is in j's region iff the normalised
+ *                value is >= threshold; a constant column gives no token.
+ *   dilation     the union over j is dilated by a (2r+1)^2 square on the
+ *                grid_h x grid_w token grid (r = dilation, 0..8), neighbours
+ *                outside the grid ignored.
+ *   mask         out, u8 [N] 0/1.
+ *   dirty_idx    out, int32 [N] capacity; the first D entries are the dirty
+ *                tokens in ascending order.
+ *   dirty_count  out, int32 [1] device: D.
+ *   workspace    device scratch of rc_localize_workspace_size() bytes.
+ * The comparison is taken in f32 with round-to-nearest subtraction and
+ * division, so the result is bit-identical to a float32 evaluation of the
+ * same definition.  Errors: RC_ERR_INVALID_ARG, RC_ERR_SHAPE
+ * (N != grid_h * grid_w, N > 16384, M < 1). */
+rc_status rc_localize_mask(const float* xattn, int S, int N, int M, int grid_h, int grid_w,
+                           const int32_t* delta_ids_host, int n_delta, float threshold,
+                           int dilation, uint8_t* mask, int32_t* dirty_idx,
+                           int32_t* dirty_count, void* workspace, size_t workspace_bytes,
+                           rc_stream stream);
+
+/* ------------------------------------------------------------ block / step */
+
+/* Region-level sparse forward of block `layer` at timestep slot `t` of
+ * `session` (Section 3.3, Region-Level Sparse Attention; Section 3.4, Kernel
+ * Fusing).
+ *   hidden       f32 [N][hidden], in/out: rows dirty_idx[r] are the dirty
+ *                tokens' block inputs and are overwritten with their block
+ *                outputs; other rows are neither read nor written.
+ *   dirty_idx    int32 device, distinct token indices in [0, N) (any order).
+ *   D            number of dirty tokens, 0..N; with dirty_count non-null it
+ *                is only an upper bound (-1 = N) and *dirty_count is used.
+ *   mod6         f32 [6][hidden] device: this block's adaLN-single vector
+ *                (table + timestep projection).
+ * Effect on the cache slot (session, layer, t): K and V rows of the dirty
+ * tokens are replaced by their fresh projections before the attention (the
+ * dirty queries attend over all N keys: cached for clean tokens, fresh for
+ * dirty ones); H rows of the dirty tokens are replaced by their block
+ * outputs (bf16), so H holds the merged H^{l+1}.  Clean rows are untouched.
+ * D = 0 is legal and changes nothing.  Errors: RC_ERR_INVALID_ARG,
+ * RC_ERR_STATE (weights or text not set). */
+rc_status rc_block_forward_region(rc_ctx* ctx, rc_cache* cache, int session, int layer, int t,
+                                  float* hidden, const int32_t* dirty_idx, int D,
+                                  const int32_t* dirty_count, const float* mod6,
+                                  rc_stream stream);
+
+/* One denoising step t of `session` following the reuse schedule
+ * schedule_host[timesteps] (modes RC_MODE_*; Section 3.3, Eq. 2):
+ *   DENSE   every token is embedded and pushed through all blocks; every
+ *           cache row of (session, *, t) is overwritten.
+ *   SPARSE  only the dirty tokens (dirty_idx / D / dirty_count as in
+ *           rc_block_forward_region) are embedded and recomputed through all
+ *           blocks; clean rows come from the cache.
+ *   REUSE   no block runs; the final layer reads the cached H of the last
+ *           block.
+ * Then the final layer (LayerNorm, modulation by the timestep embedding,
+ * linear to p*p*out_ch) gives eps (the first in_ch output channels) for all
+ * tokens and the latent is updated in place by DDIM (eta = 0).
+ *   latent  f32 [in_ch][grid_h*patch][grid_w*patch], in/out.
+ * Errors: RC_ERR_INVALID_ARG, RC_ERR_STATE (weights, schedule or text not
+ * set). */
+rc_status rc_step(rc_ctx* ctx, rc_cache* cache, int session, float* latent, int t,
+                  const uint8_t* schedule_host, const int32_t* dirty_idx, int D,
+                  const int32_t* dirty_count, rc_stream stream);
+
+/* Full-recompute baseline: rc_step with mode DENSE. */
+rc_status rc_step_dense(rc_ctx* ctx, rc_cache* cache, int session, float* latent, int t,
+                        rc_stream stream);
+
+/* ------------------------------------------------------------- auxiliary */
+
+/* The tensor-core GEMM of the block on its own: y = x W^T + b.
+ *   x bf16 [rows][k], W bf16 [n][k], b f32 [n] (may be null), y f32 [rows][n].
+ *   k % 64 == 0, n % 64 == 0, rows >= 0.
+ * Provided so the GEMM can be checked and timed in isolation. */
+rc_status rc_linear(rc_ctx* ctx, const void* x, const void* W, const float* b, float* y,
+                    int rows, int n, int k, rc_stream stream);
+
+/* Waits for `stream`, then reports (and clears) the context's device error
+ * word: RC_ERR_DEVICE_ASSERT if a kernel met a bad index or count,
+ * RC_ERR_TIMEOUT if a bounded wait gave up, RC_ERR_CUDA on a CUDA error. */
+rc_status rc_sync(rc_ctx* ctx, rc_stream stream);
+
+/* Timing probe.  rc_probe_enable(ctx, which, capacity) makes the context
+ * record a pair of CUDA events on the launching stream around each of the
+ * next `capacity` launches of kernel class `which` (RC_PROBE_GEMM: every
+ * tensor-core GEMM of a block; RC_PROBE_ATTENTION: every attention launch);
+ * which = RC_PROBE_OFF disables it.  rc_probe_read waits for the recorded
+ * events and returns the summed device time (ms) and the number of launches
+ * recorded, then rearms the ring.  Errors: RC_ERR_INVALID_ARG, RC_ERR_CUDA. */
+#define RC_PROBE_OFF 0
+#define RC_PROBE_GEMM 1
+#define RC_PROBE_ATTENTION 2
+rc_status rc_probe_enable(rc_ctx* ctx, int which, int capacity);
+rc_status rc_probe_read(rc_ctx* ctx, double* total_ms, int* launches);
+
+/* Number of kernels this library has launched in the calling process. */
+uint64_t rc_launch_count(void);
+
+const char* rc_status_string(rc_status s);
+const char* rc_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* REGIONCACHE_H */

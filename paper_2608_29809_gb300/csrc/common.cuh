@@ -1,0 +1,56 @@
+// Shared device helpers of the region-sparse DiT library (sm_103a).
+#pragma once
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace rc {
+
+// Device error-word bits (reported by rc_sync).
+enum : unsigned {
+  DEVERR_INDEX = 1u,    // a dirty index outside [0, N)
+  DEVERR_COUNT = 2u,    // a device dirty count outside [0, bound]
+  DEVERR_TIMEOUT = 4u,  // a bounded wait gave up
+};
+
+__device__ __forceinline__ float bf2f(__nv_bfloat16 v) { return __bfloat162float(v); }
+__device__ __forceinline__ __nv_bfloat16 f2bf(float v) { return __float2bfloat16_rn(v); }
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ __forceinline__ float2 unpack_bf16x2(uint32_t u) {
+  __nv_bfloat162 v = *reinterpret_cast<__nv_bfloat162*>(&u);
+  return __bfloat1622float2(v);
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ float gelu_tanh(float z) {
+  const float k0 = 0.7978845608028654f;  // sqrt(2/pi)
+  float inner = k0 * (z + 0.044715f * z * z * z);
+  return 0.5f * z * (1.0f + tanhf(inner));
+}
+
+__device__ __forceinline__ float silu(float z) { return z / (1.0f + expf(-z)); }
+
+// Resolves the live dirty count: the device count when given (checked against
+// the bound; a bad value raises DEVERR_COUNT and is treated as 0), else the
+// host count.
+__device__ __forceinline__ int live_count(const int* dcount, int bound, unsigned* err) {
+  if (dcount == nullptr) return bound;
+  int d = *dcount;
+  if (d < 0 || d > bound) {
+    if (err) atomicOr(err, DEVERR_COUNT);
+    return 0;
+  }
+  return d;
+}
+
+}  // namespace rc

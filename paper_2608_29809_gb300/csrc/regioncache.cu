@@ -1,0 +1,677 @@
+// C ABI of the region-sparse DiT step (see include/regioncache.h): context and
+// cache management, host-side validation, and the launch sequence of a block
+// and a denoising step.  Every compute step runs in this library's kernels.
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <atomic>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "../../include/regioncache.h"
+#include "common.cuh"
+#include "kernels.h"
+
+using rc::bf16;
+
+namespace {
+
+thread_local std::string g_last_error;
+std::atomic<uint64_t> g_launches{0};
+
+rc_status fail(rc_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return s;
+}
+
+rc_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(e == cudaErrorMemoryAllocation ? RC_ERR_OOM : RC_ERR_CUDA, "%s: %s", what,
+              cudaGetErrorString(e));
+}
+
+#define RC_CUDA(call, what)                        \
+  do {                                             \
+    cudaError_t e_ = (call);                       \
+    if (e_ != cudaSuccess) return cuda_fail(e_, what); \
+  } while (0)
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+namespace rc {
+void count_launches(int n) { g_launches.fetch_add(uint64_t(n), std::memory_order_relaxed); }
+}  // namespace rc
+
+struct rc_ctx {
+  rc_dims dims;
+  int N, d, F, dh, L, T, M;
+  int device;
+  std::vector<rc_layer_weights> lw;
+  std::vector<char> lw_set;
+  rc_global_weights gw;
+  bool gw_set = false;
+  std::vector<float> t_values, alpha_bar;
+  bool sched_set = false;
+  // device scratch
+  float* xf = nullptr;   // [N][d] residual rows of the dirty tokens (compact)
+  bf16* xb = nullptr;    // [N][d] GEMM input: modulated rows / residual copy
+  bf16* ob = nullptr;    // [N][d] attention output
+  bf16* q = nullptr;     // [N][d] queries (self, then cross)
+  bf16* u = nullptr;     // [N][F] MLP hidden
+  float* fbuf = nullptr; // [freq_dim]
+  float* h1 = nullptr;   // [d]
+  float* temb = nullptr; // [d]
+  float* tb = nullptr;   // [6d]
+  int* iota = nullptr;   // [N] identity row map (dense path)
+  unsigned* err = nullptr;
+  // timing probe
+  int probe_which = RC_PROBE_OFF;
+  int probe_n = 0;
+  std::vector<cudaEvent_t> probe_ev;  // 2 * capacity
+};
+
+struct rc_cache {
+  rc_ctx* ctx;
+  int sessions;
+  bf16* base = nullptr;  // [sessions][T][L][3 (H,K,V)][N][d]
+  bf16* text = nullptr;  // [sessions][L][M][2d]
+  std::vector<char> text_set;
+
+  size_t slot_elems() const { return size_t(ctx->N) * ctx->d; }
+  bf16* slot(int s, int l, int t, int which) const {
+    size_t i = ((size_t(s) * ctx->T + t) * ctx->L + l) * 3 + which;
+    return base + i * slot_elems();
+  }
+  bf16* text_kv(int s, int l) const {
+    return text + (size_t(s) * ctx->L + l) * size_t(ctx->M) * 2 * ctx->d;
+  }
+};
+
+namespace {
+
+__global__ void iota_kernel(int* p, int n) {
+  int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) p[i] = i;
+}
+
+template <class T>
+rc_status dalloc(T** p, size_t count, const char* what) {
+  void* v = nullptr;
+  cudaError_t e = cudaMalloc(&v, count * sizeof(T));
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return fail(RC_ERR_OOM, "cudaMalloc(%s, %zu bytes): %s", what, count * sizeof(T),
+                cudaGetErrorString(e));
+  }
+  *p = static_cast<T*>(v);
+  return RC_OK;
+}
+
+void probe_free(rc_ctx* c) {
+  for (cudaEvent_t e : c->probe_ev) cudaEventDestroy(e);
+  c->probe_ev.clear();
+  c->probe_n = 0;
+  c->probe_which = RC_PROBE_OFF;
+}
+
+// Brackets one launch of kernel class `which` with probe events.
+struct Probe {
+  rc_ctx* c;
+  cudaStream_t st;
+  bool on;
+  Probe(rc_ctx* c_, int which, cudaStream_t st_)
+      : c(c_), st(st_),
+        on(c_->probe_which == which && 2 * (c_->probe_n + 1) <= int(c_->probe_ev.size())) {
+    if (on) cudaEventRecord(c->probe_ev[2 * c->probe_n], st);
+  }
+  ~Probe() {
+    if (on) {
+      cudaEventRecord(c->probe_ev[2 * c->probe_n + 1], st);
+      ++c->probe_n;
+    }
+  }
+};
+
+void free_ctx(rc_ctx* c) {
+  if (!c) return;
+  probe_free(c);
+  void* ps[] = {c->xf, c->xb, c->ob, c->q, c->u, c->fbuf, c->h1, c->temb, c->tb, c->iota, c->err};
+  for (void* p : ps)
+    if (p) cudaFree(p);
+  delete c;
+}
+
+rc_status check_session(const rc_cache* cache, int session) {
+  if (session < 0 || session >= cache->sessions)
+    return fail(RC_ERR_INVALID_ARG, "session %d outside [0, %d)", session, cache->sessions);
+  return RC_OK;
+}
+
+rc_status check_ready(const rc_ctx* c, const rc_cache* cache, int session, bool need_sched) {
+  for (int l = 0; l < c->L; ++l)
+    if (!c->lw_set[l]) return fail(RC_ERR_STATE, "weights of layer %d not set", l);
+  if (!c->gw_set) return fail(RC_ERR_STATE, "global weights not set");
+  if (need_sched && !c->sched_set) return fail(RC_ERR_STATE, "schedule not set");
+  if (!cache->text_set[session])
+    return fail(RC_ERR_STATE, "text of session %d not set (rc_set_text)", session);
+  return RC_OK;
+}
+
+// Row map of a call: the dirty rows (idx, D bound, optional device count).
+struct Rows {
+  const int* idx;
+  int bound;
+  const int* dcount;
+};
+
+// One region-sparse block on the compact residual rows c->xf (Section 3.3,
+// Region-Level Sparse Attention; Section 3.4, Kernel Fusing).  tab / tbv give
+// the modulation vector as tab (+ tbv), each [6][d] (tbv may be null).
+rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows& rw,
+                    const float* tab, const float* tbv, cudaStream_t st) {
+  const int d = c->d, F = c->F, N = c->N;
+  const rc_layer_weights& w = c->lw[l];
+  auto mv = [&](const float* base, int k) { return base ? base + size_t(k) * d : nullptr; };
+  bf16* Kc = cache->slot(s, l, t, 1);
+  bf16* Vc = cache->slot(s, l, t, 2);
+  bf16* Hc = cache->slot(s, l, t, 0);
+  const bf16* tk = cache->text_kv(s, l);
+  const bf16* tv = tk + d;
+
+  // x_hat = LN(x)(1 + scale_msa) + shift_msa
+  RC_CUDA(rc::launch_ln_mod(c->xf, d, mv(tab, 0), mv(tbv, 0), mv(tab, 1), mv(tbv, 1), c->xb, d,
+                            rw.bound, rw.dcount, d, c->err, st), "ln_mod(msa)");
+  // [q | k | v] = x_hat W_qkv^T + b; k, v rows go straight to cache rows idx[r]
+  rc::GemmEpi e{};
+  e.mode = rc::EPI_QKV;
+  e.bias = w.b_qkv;
+  e.out_bf = c->q;
+  e.ld_out = d;
+  e.kc = Kc;
+  e.vc = Vc;
+  e.ld_kv = d;
+  e.dsplit = d;
+  e.idx = rw.idx;
+  e.n_tokens = N;
+  e.err = c->err;
+  {
+    Probe pr(c, RC_PROBE_GEMM, st);
+    RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_qkv), rw.bound, rw.dcount, 3 * d,
+                            d, e, st), "gemm(qkv)");
+  }
+  // dirty queries over all N keys / values of (l, t)
+  {
+    Probe pr(c, RC_PROBE_ATTENTION, st);
+    RC_CUDA(rc::launch_attention(c->q, d, Kc, Vc, d, N, c->ob, d, c->dims.heads, c->dh, rw.bound,
+                                 rw.dcount, c->err, st), "attention(self)");
+  }
+  // x += gate_msa (o W_o^T + b_o); bf16 copy of x for the cross-attention query
+  e = rc::GemmEpi{};
+  e.mode = rc::EPI_GATE_RES;
+  e.bias = w.b_o;
+  e.xf = c->xf;
+  e.ld_xf = d;
+  e.gate_tab = mv(tab, 2);
+  e.gate_tb = mv(tbv, 2);
+  e.copy_bf = c->xb;
+  e.ld_copy = d;
+  e.err = c->err;
+  {
+    Probe pr(c, RC_PROBE_GEMM, st);
+    RC_CUDA(rc::launch_gemm(c->ob, d, static_cast<const bf16*>(w.W_o), rw.bound, rw.dcount, d, d, e,
+                            st), "gemm(out)");
+  }
+  // q' = x W_xq^T + b
+  e = rc::GemmEpi{};
+  e.mode = rc::EPI_BIAS_BF16;
+  e.bias = w.b_xq;
+  e.out_bf = c->q;
+  e.ld_out = d;
+  e.err = c->err;
+  {
+    Probe pr(c, RC_PROBE_GEMM, st);
+    RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_xq), rw.bound, rw.dcount, d, d,
+                            e, st), "gemm(xq)");
+  }
+  {
+    Probe pr(c, RC_PROBE_ATTENTION, st);
+    RC_CUDA(rc::launch_attention(c->q, d, tk, tv, 2 * d, c->M, c->ob, d, c->dims.heads, c->dh,
+                                 rw.bound, rw.dcount, c->err, st), "attention(cross)");
+  }
+  // x += o' W_xo^T + b
+  e = rc::GemmEpi{};
+  e.mode = rc::EPI_GATE_RES;
+  e.bias = w.b_xo;
+  e.xf = c->xf;
+  e.ld_xf = d;
+  e.err = c->err;
+  {
+    Probe pr(c, RC_PROBE_GEMM, st);
+    RC_CUDA(rc::launch_gemm(c->ob, d, static_cast<const bf16*>(w.W_xo), rw.bound, rw.dcount, d, d,
+                            e, st), "gemm(xo)");
+  }
+  // MLP
+  RC_CUDA(rc::launch_ln_mod(c->xf, d, mv(tab, 3), mv(tbv, 3), mv(tab, 4), mv(tbv, 4), c->xb, d,
+                            rw.bound, rw.dcount, d, c->err, st), "ln_mod(mlp)");
+  e = rc::GemmEpi{};
+  e.mode = rc::EPI_GELU_BF16;
+  e.bias = w.b_1;
+  e.out_bf = c->u;
+  e.ld_out = F;
+  e.err = c->err;
+  {
+    Probe pr(c, RC_PROBE_GEMM, st);
+    RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_1), rw.bound, rw.dcount, F, d, e,
+                            st), "gemm(fc1)");
+  }
+  // x += gate_mlp (u W_2^T + b_2); merged H^{l+1}: row idx[r] of the cache
+  e = rc::GemmEpi{};
+  e.mode = rc::EPI_GATE_RES;
+  e.bias = w.b_2;
+  e.xf = c->xf;
+  e.ld_xf = d;
+  e.gate_tab = mv(tab, 5);
+  e.gate_tb = mv(tbv, 5);
+  e.scat = Hc;
+  e.ld_kv = d;
+  e.idx = rw.idx;
+  e.n_tokens = N;
+  e.err = c->err;
+  {
+    Probe pr(c, RC_PROBE_GEMM, st);
+    RC_CUDA(rc::launch_gemm(c->u, F, static_cast<const bf16*>(w.W_2), rw.bound, rw.dcount, d, F, e,
+                            st), "gemm(fc2)");
+  }
+  return RC_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* rc_status_string(rc_status s) {
+  switch (s) {
+    case RC_OK: return "ok";
+    case RC_ERR_INVALID_ARG: return "invalid argument";
+    case RC_ERR_SHAPE: return "shape mismatch";
+    case RC_ERR_OOM: return "out of device memory";
+    case RC_ERR_CUDA: return "CUDA error";
+    case RC_ERR_TIMEOUT: return "device wait timed out";
+    case RC_ERR_DEVICE_ASSERT: return "device-side index/count check failed";
+    case RC_ERR_STATE: return "call order violated";
+    default: return "unknown status";
+  }
+}
+
+const char* rc_last_error(void) { return g_last_error.c_str(); }
+
+uint64_t rc_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+rc_status rc_create(const rc_dims* dims, rc_ctx** out) {
+  if (!dims || !out) return fail(RC_ERR_INVALID_ARG, "rc_create: null argument");
+  *out = nullptr;
+  const rc_dims& D = *dims;
+  if (D.hidden <= 0 || D.heads <= 0 || D.mlp <= 0 || D.layers <= 0 || D.grid_h <= 0 ||
+      D.grid_w <= 0 || D.patch <= 0 || D.in_ch <= 0 || D.out_ch <= 0 || D.text_len <= 0 ||
+      D.timesteps <= 0 || D.freq_dim <= 0)
+    return fail(RC_ERR_INVALID_ARG, "rc_create: every dimension must be positive");
+  if (D.hidden % D.heads) return fail(RC_ERR_SHAPE, "hidden %% heads != 0");
+  const int dh = D.hidden / D.heads;
+  if (dh != 72 && dh != 64) return fail(RC_ERR_SHAPE, "head_dim %d not in {64, 72}", dh);
+  if (D.hidden % 128 || D.hidden > 1536)
+    return fail(RC_ERR_SHAPE, "hidden %d must be a multiple of 128 and <= 1536", D.hidden);
+  if (D.mlp % 128) return fail(RC_ERR_SHAPE, "mlp %d must be a multiple of 128", D.mlp);
+  if (D.freq_dim % 8 || D.freq_dim > 4096) return fail(RC_ERR_SHAPE, "freq_dim %d", D.freq_dim);
+  const long long N = 1LL * D.grid_h * D.grid_w;
+  if (N > 16384) return fail(RC_ERR_SHAPE, "N = %lld tokens > 16384", N);
+  if (D.in_ch * D.patch * D.patch > 16 || D.out_ch < D.in_ch)
+    return fail(RC_ERR_SHAPE, "in_ch * patch^2 must be <= 16 and out_ch >= in_ch");
+
+  rc_ctx* c = new (std::nothrow) rc_ctx();
+  if (!c) return fail(RC_ERR_OOM, "host allocation");
+  c->dims = D;
+  c->N = int(N);
+  c->d = D.hidden;
+  c->F = D.mlp;
+  c->dh = dh;
+  c->L = D.layers;
+  c->T = D.timesteps;
+  c->M = D.text_len;
+  cudaGetDevice(&c->device);
+  c->lw.resize(c->L);
+  c->lw_set.assign(c->L, 0);
+  rc_status s = RC_OK;
+  const size_t Nd = size_t(N) * D.hidden;
+  if ((s = dalloc(&c->xf, Nd, "xf")) || (s = dalloc(&c->xb, Nd, "xb")) ||
+      (s = dalloc(&c->ob, Nd, "ob")) || (s = dalloc(&c->q, Nd, "q")) ||
+      (s = dalloc(&c->u, size_t(N) * D.mlp, "u")) || (s = dalloc(&c->fbuf, D.freq_dim, "f")) ||
+      (s = dalloc(&c->h1, D.hidden, "h1")) || (s = dalloc(&c->temb, D.hidden, "temb")) ||
+      (s = dalloc(&c->tb, 6 * size_t(D.hidden), "tb")) || (s = dalloc(&c->iota, N, "iota")) ||
+      (s = dalloc(&c->err, 1, "err"))) {
+    free_ctx(c);
+    return s;
+  }
+  iota_kernel<<<int((N + 255) / 256), 256>>>(c->iota, int(N));
+  rc::count_launches(1);
+  cudaError_t e = cudaMemset(c->err, 0, sizeof(unsigned));
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) {
+    free_ctx(c);
+    return cuda_fail(e, "rc_create");
+  }
+  *out = c;
+  return RC_OK;
+}
+
+void rc_destroy(rc_ctx* ctx) { free_ctx(ctx); }
+
+rc_status rc_set_layer_weights(rc_ctx* c, int layer, const rc_layer_weights* w) {
+  if (!c || !w) return fail(RC_ERR_INVALID_ARG, "rc_set_layer_weights: null argument");
+  if (layer < 0 || layer >= c->L)
+    return fail(RC_ERR_INVALID_ARG, "layer %d outside [0, %d)", layer, c->L);
+  const void* ps[] = {w->W_qkv, w->b_qkv, w->W_o, w->b_o, w->W_xq, w->b_xq, w->W_xkv, w->b_xkv,
+                      w->W_xo,  w->b_xo,  w->W_1, w->b_1, w->W_2,  w->b_2,  w->table};
+  for (const void* p : ps)
+    if (!p || !aligned16(p))
+      return fail(RC_ERR_INVALID_ARG, "layer %d: null or unaligned (16 B) weight", layer);
+  c->lw[layer] = *w;
+  c->lw_set[layer] = 1;
+  return RC_OK;
+}
+
+rc_status rc_set_global_weights(rc_ctx* c, const rc_global_weights* w) {
+  if (!c || !w) return fail(RC_ERR_INVALID_ARG, "rc_set_global_weights: null argument");
+  const void* ps[] = {w->W_e, w->b_e,  w->pos,     w->W_t1, w->b_t1, w->W_t2,
+                      w->b_t2, w->W_tb, w->b_tb, w->table_f, w->W_f, w->b_f};
+  for (const void* p : ps)
+    if (!p || !aligned16(p))
+      return fail(RC_ERR_INVALID_ARG, "global weights: null or unaligned (16 B) pointer");
+  c->gw = *w;
+  c->gw_set = true;
+  return RC_OK;
+}
+
+rc_status rc_set_schedule(rc_ctx* c, const float* tv, const float* ab) {
+  if (!c || !tv || !ab) return fail(RC_ERR_INVALID_ARG, "rc_set_schedule: null argument");
+  for (int i = 0; i <= c->T; ++i)
+    if (!(ab[i] > 0.f && ab[i] <= 1.f))
+      return fail(RC_ERR_INVALID_ARG, "alpha_bar[%d] = %g outside (0, 1]", i, double(ab[i]));
+  c->t_values.assign(tv, tv + c->T);
+  c->alpha_bar.assign(ab, ab + c->T + 1);
+  c->sched_set = true;
+  return RC_OK;
+}
+
+rc_status rc_cache_create(rc_ctx* c, int sessions, rc_cache** out) {
+  if (!c || !out) return fail(RC_ERR_INVALID_ARG, "rc_cache_create: null argument");
+  *out = nullptr;
+  if (sessions <= 0) return fail(RC_ERR_INVALID_ARG, "sessions = %d", sessions);
+  rc_cache* k = new (std::nothrow) rc_cache();
+  if (!k) return fail(RC_ERR_OOM, "host allocation");
+  k->ctx = c;
+  k->sessions = sessions;
+  k->text_set.assign(sessions, 0);
+  const size_t n = size_t(sessions) * c->T * c->L * 3 * k->slot_elems();
+  rc_status s = dalloc(&k->base, n, "cache");
+  if (s == RC_OK) s = dalloc(&k->text, size_t(sessions) * c->L * c->M * 2 * c->d, "text kv");
+  if (s != RC_OK) {
+    if (k->base) cudaFree(k->base);
+    delete k;
+    return s;
+  }
+  *out = k;
+  return RC_OK;
+}
+
+void rc_cache_destroy(rc_cache* k) {
+  if (!k) return;
+  if (k->base) cudaFree(k->base);
+  if (k->text) cudaFree(k->text);
+  delete k;
+}
+
+static rc_status cache_copy(rc_cache* k, int s, int l, int t, void* H, void* K, void* V,
+                            bool fill, cudaStream_t st) {
+  if (!k) return fail(RC_ERR_INVALID_ARG, "null cache");
+  rc_status r = check_session(k, s);
+  if (r) return r;
+  if (l < 0 || l >= k->ctx->L || t < 0 || t >= k->ctx->T)
+    return fail(RC_ERR_INVALID_ARG, "layer %d / t %d out of range", l, t);
+  void* ps[3] = {H, K, V};
+  const size_t bytes = k->slot_elems() * sizeof(bf16);
+  for (int w = 0; w < 3; ++w) {
+    if (!ps[w]) continue;
+    bf16* slot = k->slot(s, l, t, w);
+    RC_CUDA(cudaMemcpyAsync(fill ? static_cast<void*>(slot) : ps[w],
+                            fill ? static_cast<const void*>(ps[w]) : slot, bytes,
+                            cudaMemcpyDeviceToDevice, st),
+            "cache copy");
+  }
+  return RC_OK;
+}
+
+rc_status rc_cache_fill(rc_cache* k, int s, int l, int t, const void* H, const void* K,
+                        const void* V, rc_stream st) {
+  return cache_copy(k, s, l, t, const_cast<void*>(H), const_cast<void*>(K), const_cast<void*>(V),
+                    true, static_cast<cudaStream_t>(st));
+}
+
+rc_status rc_cache_read(rc_cache* k, int s, int l, int t, void* H, void* K, void* V,
+                        rc_stream st) {
+  return cache_copy(k, s, l, t, H, K, V, false, static_cast<cudaStream_t>(st));
+}
+
+rc_status rc_set_text(rc_ctx* c, rc_cache* k, int s, const void* ctx_bf16, rc_stream stream) {
+  if (!c || !k || !ctx_bf16) return fail(RC_ERR_INVALID_ARG, "rc_set_text: null argument");
+  if (k->ctx != c) return fail(RC_ERR_INVALID_ARG, "cache belongs to another context");
+  rc_status r = check_session(k, s);
+  if (r) return r;
+  if (!aligned16(ctx_bf16)) return fail(RC_ERR_INVALID_ARG, "text context not 16-B aligned");
+  for (int l = 0; l < c->L; ++l)
+    if (!c->lw_set[l]) return fail(RC_ERR_STATE, "weights of layer %d not set", l);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  for (int l = 0; l < c->L; ++l) {
+    rc::GemmEpi e{};
+    e.mode = rc::EPI_BIAS_BF16;
+    e.bias = c->lw[l].b_xkv;
+    e.out_bf = k->text_kv(s, l);
+    e.ld_out = 2 * c->d;
+    e.err = c->err;
+    RC_CUDA(rc::launch_gemm(static_cast<const bf16*>(ctx_bf16), c->d,
+                            static_cast<const bf16*>(c->lw[l].W_xkv), c->M, nullptr, 2 * c->d,
+                            c->d, e, st), "gemm(text kv)");
+  }
+  k->text_set[s] = 1;
+  return RC_OK;
+}
+
+size_t rc_localize_workspace_size(int N, int n_delta) {
+  if (N <= 0 || n_delta <= 0) return 0;
+  return rc::localize_workspace_bytes(N, n_delta);
+}
+
+rc_status rc_localize_mask(const float* xattn, int S, int N, int M, int grid_h, int grid_w,
+                           const int32_t* delta_ids_host, int n_delta, float threshold,
+                           int dilation, uint8_t* mask, int32_t* dirty_idx, int32_t* dirty_count,
+                           void* workspace, size_t workspace_bytes, rc_stream stream) {
+  if (!xattn || !delta_ids_host || !mask || !dirty_idx || !dirty_count || !workspace)
+    return fail(RC_ERR_INVALID_ARG, "rc_localize_mask: null pointer");
+  if (S < 1 || M < 1 || N < 1 || grid_h < 1 || grid_w < 1)
+    return fail(RC_ERR_SHAPE, "rc_localize_mask: S, M, N and the grid must be positive");
+  if (1LL * grid_h * grid_w != N) return fail(RC_ERR_SHAPE, "N != grid_h * grid_w");
+  if (N > 16384) return fail(RC_ERR_SHAPE, "N = %d > 16384", N);
+  if (n_delta < 1 || n_delta > 64) return fail(RC_ERR_INVALID_ARG, "n_delta %d not in 1..64", n_delta);
+  if (dilation < 0 || dilation > 8) return fail(RC_ERR_INVALID_ARG, "dilation %d not in 0..8", dilation);
+  if (!(threshold == threshold) || threshold > 3.4e38f || threshold < -3.4e38f)
+    return fail(RC_ERR_INVALID_ARG, "threshold is not finite");
+  if (workspace_bytes < rc::localize_workspace_bytes(N, n_delta))
+    return fail(RC_ERR_INVALID_ARG, "workspace of %zu bytes < %zu", workspace_bytes,
+                rc::localize_workspace_bytes(N, n_delta));
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
+    return fail(RC_ERR_INVALID_ARG, "workspace not 256-B aligned");
+  rc::DeltaIds ids{};
+  ids.n = n_delta;
+  for (int j = 0; j < n_delta; ++j) {
+    if (delta_ids_host[j] < 0 || delta_ids_host[j] >= M)
+      return fail(RC_ERR_INVALID_ARG, "delta id %d outside [0, %d)", delta_ids_host[j], M);
+    ids.id[j] = delta_ids_host[j];
+  }
+  RC_CUDA(rc::launch_localize(xattn, S, N, M, grid_h, grid_w, ids, threshold, dilation, mask,
+                              dirty_idx, dirty_count, workspace, static_cast<cudaStream_t>(stream)),
+          "localize");
+  return RC_OK;
+}
+
+static rc_status rows_of(const rc_ctx* c, const int32_t* idx, int D, const int32_t* dcount,
+                         Rows* rw) {
+  if (D < -1 || D > c->N) return fail(RC_ERR_INVALID_ARG, "D = %d outside [-1, %d]", D, c->N);
+  if (D == -1 && !dcount) return fail(RC_ERR_INVALID_ARG, "D = -1 needs a device dirty_count");
+  const int bound = D < 0 ? c->N : D;
+  if (bound > 0 && !idx) return fail(RC_ERR_INVALID_ARG, "dirty_idx is null");
+  rw->idx = idx;
+  rw->bound = bound;
+  rw->dcount = dcount;
+  return RC_OK;
+}
+
+rc_status rc_block_forward_region(rc_ctx* c, rc_cache* k, int s, int l, int t, float* hidden,
+                                  const int32_t* dirty_idx, int D, const int32_t* dirty_count,
+                                  const float* mod6, rc_stream stream) {
+  if (!c || !k || !hidden || !mod6)
+    return fail(RC_ERR_INVALID_ARG, "rc_block_forward_region: null argument");
+  if (k->ctx != c) return fail(RC_ERR_INVALID_ARG, "cache belongs to another context");
+  rc_status r = check_session(k, s);
+  if (r) return r;
+  if (l < 0 || l >= c->L || t < 0 || t >= c->T)
+    return fail(RC_ERR_INVALID_ARG, "layer %d / t %d out of range", l, t);
+  if (!aligned16(hidden) || !aligned16(mod6))
+    return fail(RC_ERR_INVALID_ARG, "hidden / mod6 not 16-B aligned");
+  if ((r = check_ready(c, k, s, false))) return r;
+  Rows rw;
+  if ((r = rows_of(c, dirty_idx, D, dirty_count, &rw))) return r;
+  if (rw.bound == 0) return RC_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  RC_CUDA(rc::launch_rows_f32(hidden, c->xf, rw.idx, rw.bound, rw.dcount, c->d, c->N, false,
+                              c->err, st), "gather");
+  if ((r = run_block(c, k, s, l, t, rw, mod6, nullptr, st))) return r;
+  RC_CUDA(rc::launch_rows_f32(c->xf, hidden, rw.idx, rw.bound, rw.dcount, c->d, c->N, true,
+                              c->err, st), "scatter");
+  return RC_OK;
+}
+
+rc_status rc_step(rc_ctx* c, rc_cache* k, int s, float* latent, int t,
+                  const uint8_t* schedule_host, const int32_t* dirty_idx, int D,
+                  const int32_t* dirty_count, rc_stream stream) {
+  if (!c || !k || !latent || !schedule_host)
+    return fail(RC_ERR_INVALID_ARG, "rc_step: null argument");
+  if (k->ctx != c) return fail(RC_ERR_INVALID_ARG, "cache belongs to another context");
+  rc_status r = check_session(k, s);
+  if (r) return r;
+  if (t < 0 || t >= c->T) return fail(RC_ERR_INVALID_ARG, "t %d outside [0, %d)", t, c->T);
+  if (!aligned16(latent)) return fail(RC_ERR_INVALID_ARG, "latent not 16-B aligned");
+  const int mode = schedule_host[t];
+  if (mode != RC_MODE_DENSE && mode != RC_MODE_SPARSE && mode != RC_MODE_REUSE)
+    return fail(RC_ERR_INVALID_ARG, "schedule[%d] = %d is not a mode", t, mode);
+  if ((r = check_ready(c, k, s, true))) return r;
+  Rows rw{c->iota, c->N, nullptr};
+  if (mode == RC_MODE_SPARSE && (r = rows_of(c, dirty_idx, D, dirty_count, &rw))) return r;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const rc_global_weights& g = c->gw;
+  const int d = c->d;
+  RC_CUDA(rc::launch_t_embed(c->t_values[t], c->dims.freq_dim, d,
+                             static_cast<const bf16*>(g.W_t1), g.b_t1,
+                             static_cast<const bf16*>(g.W_t2), g.b_t2,
+                             static_cast<const bf16*>(g.W_tb), g.b_tb, c->fbuf, c->h1, c->temb,
+                             c->tb, st), "t_embed");
+  if (mode != RC_MODE_REUSE && rw.bound > 0) {
+    RC_CUDA(rc::launch_patch_embed(latent, c->dims.grid_h, c->dims.grid_w, c->dims.patch,
+                                   c->dims.in_ch, static_cast<const bf16*>(g.W_e), g.b_e, g.pos,
+                                   rw.idx, rw.bound, rw.dcount, c->xf, d, c->err, st),
+            "patch_embed");
+    for (int l = 0; l < c->L; ++l)
+      if ((r = run_block(c, k, s, l, t, rw, c->lw[l].table, c->tb, st))) return r;
+  }
+  RC_CUDA(rc::launch_final_ddim(k->slot(s, c->L - 1, t, 0), c->temb, g.table_f,
+                                static_cast<const bf16*>(g.W_f), g.b_f, latent, c->dims.grid_h,
+                                c->dims.grid_w, c->dims.patch, c->dims.in_ch, c->dims.out_ch, d,
+                                c->alpha_bar[t], c->alpha_bar[t + 1], st), "final_ddim");
+  return RC_OK;
+}
+
+rc_status rc_step_dense(rc_ctx* c, rc_cache* k, int s, float* latent, int t, rc_stream stream) {
+  if (!c) return fail(RC_ERR_INVALID_ARG, "rc_step_dense: null context");
+  std::vector<uint8_t> sched(size_t(c->T), uint8_t(RC_MODE_DENSE));
+  return rc_step(c, k, s, latent, t, sched.data(), nullptr, 0, nullptr, stream);
+}
+
+rc_status rc_linear(rc_ctx* c, const void* x, const void* W, const float* b, float* y, int rows,
+                    int n, int kdim, rc_stream stream) {
+  if (!c || !x || !W || !y) return fail(RC_ERR_INVALID_ARG, "rc_linear: null argument");
+  if (rows < 0 || n <= 0 || kdim <= 0 || n % 128 || kdim % 64)
+    return fail(RC_ERR_SHAPE, "rc_linear: rows %d n %d k %d (n %% 128, k %% 64 must be 0)", rows,
+                n, kdim);
+  if (!aligned16(x) || !aligned16(W) || !aligned16(y) || (b && !aligned16(b)))
+    return fail(RC_ERR_INVALID_ARG, "rc_linear: pointers must be 16-B aligned");
+  rc::GemmEpi e{};
+  e.mode = rc::EPI_F32;
+  e.bias = b;
+  e.out_f = y;
+  e.ld_out = n;
+  e.err = c->err;
+  RC_CUDA(rc::launch_gemm(static_cast<const bf16*>(x), kdim, static_cast<const bf16*>(W), rows,
+                          nullptr, n, kdim, e, static_cast<cudaStream_t>(stream)), "gemm(linear)");
+  return RC_OK;
+}
+
+rc_status rc_probe_enable(rc_ctx* c, int which, int capacity) {
+  if (!c) return fail(RC_ERR_INVALID_ARG, "rc_probe_enable: null context");
+  if (which < RC_PROBE_OFF || which > RC_PROBE_ATTENTION || capacity < 0 || capacity > 1 << 20)
+    return fail(RC_ERR_INVALID_ARG, "rc_probe_enable: which %d capacity %d", which, capacity);
+  probe_free(c);
+  if (which == RC_PROBE_OFF) return RC_OK;
+  c->probe_ev.resize(size_t(2) * capacity);
+  for (auto& e : c->probe_ev) RC_CUDA(cudaEventCreate(&e), "cudaEventCreate");
+  c->probe_which = which;
+  return RC_OK;
+}
+
+rc_status rc_probe_read(rc_ctx* c, double* total_ms, int* launches) {
+  if (!c || !total_ms || !launches) return fail(RC_ERR_INVALID_ARG, "rc_probe_read: null");
+  double tot = 0.0;
+  for (int i = 0; i < c->probe_n; ++i) {
+    RC_CUDA(cudaEventSynchronize(c->probe_ev[2 * i + 1]), "cudaEventSynchronize");
+    float ms = 0.f;
+    RC_CUDA(cudaEventElapsedTime(&ms, c->probe_ev[2 * i], c->probe_ev[2 * i + 1]),
+            "cudaEventElapsedTime");
+    tot += ms;
+  }
+  *total_ms = tot;
+  *launches = c->probe_n;
+  c->probe_n = 0;
+  return RC_OK;
+}
+
+rc_status rc_sync(rc_ctx* c, rc_stream stream) {
+  if (!c) return fail(RC_ERR_INVALID_ARG, "rc_sync: null context");
+  RC_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)), "stream sync");
+  unsigned w = 0;
+  RC_CUDA(cudaMemcpy(&w, c->err, sizeof(w), cudaMemcpyDeviceToHost), "read error word");
+  if (w) {
+    RC_CUDA(cudaMemset(c->err, 0, sizeof(unsigned)), "clear error word");
+    if (w & rc::DEVERR_TIMEOUT) return fail(RC_ERR_TIMEOUT, "a bounded device wait gave up");
+    return fail(RC_ERR_DEVICE_ASSERT, "device check failed (bits 0x%x: %s%s)", w,
+                (w & rc::DEVERR_INDEX) ? "index out of range " : "",
+                (w & rc::DEVERR_COUNT) ? "count out of range" : "");
+  }
+  return RC_OK;
+}
+
+}  // extern "C"

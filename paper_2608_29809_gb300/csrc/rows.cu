@@ -1,0 +1,518 @@
+// Row-wise and reduction kernels of the region-sparse DiT step: the
+// localisation mask (Section 3.2, R_edit), adaLN modulation, patch embedding,
+// timestep embedding, final layer + DDIM update, row gather/scatter.
+// All of them are HBM- or latency-bound; rows are read with 128-bit loads.
+#include <float.h>
+#include <math.h>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace rc {
+
+static inline int cdiv(int a, int b) { return (a + b - 1) / b; }
+
+// ============================================================ localisation
+// Workspace: abar f32 [n_delta][N] | part f32x2 [nblk][n_delta] | union u8 [N]
+// | cnt int [nblk].  One thread per token, MASK_ROWS tokens per CTA.
+constexpr int MASK_ROWS = 256;
+
+static size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+size_t localize_workspace_bytes(int N, int n_delta) {
+  int nblk = cdiv(N, MASK_ROWS);
+  return align256(sizeof(float) * size_t(n_delta) * N) +
+         align256(sizeof(float2) * size_t(nblk) * n_delta) + align256(size_t(N)) +
+         align256(sizeof(int) * size_t(nblk));
+}
+
+struct MaskWs {
+  float* abar;
+  float2* part;
+  uint8_t* uni;
+  int* cnt;
+};
+
+static MaskWs carve(void* ws, int N, int n_delta) {
+  int nblk = cdiv(N, MASK_ROWS);
+  char* p = static_cast<char*>(ws);
+  MaskWs w;
+  w.abar = reinterpret_cast<float*>(p);
+  p += align256(sizeof(float) * size_t(n_delta) * N);
+  w.part = reinterpret_cast<float2*>(p);
+  p += align256(sizeof(float2) * size_t(nblk) * n_delta);
+  w.uni = reinterpret_cast<uint8_t*>(p);
+  p += align256(size_t(N));
+  w.cnt = reinterpret_cast<int*>(p);
+  return w;
+}
+
+// Pass 1: a_j(i) = (sum_s A[s][i][j]) / S for each delta token j (summed in
+// ascending s, f32 round-to-nearest), and per-CTA min / max of each column.
+__global__ void __launch_bounds__(MASK_ROWS)
+mask_colstats_kernel(const float* __restrict__ A, int S, int N, int M, DeltaIds ids,
+                     float* __restrict__ abar, float2* __restrict__ part) {
+  __shared__ float smin[MASK_ROWS / 32], smax[MASK_ROWS / 32];
+  const int i = blockIdx.x * MASK_ROWS + threadIdx.x;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const size_t plane = size_t(N) * M;
+  for (int j = 0; j < ids.n; ++j) {
+    const int col = ids.id[j];
+    float lo = FLT_MAX, hi = -FLT_MAX;
+    if (i < N) {
+      float a = __ldg(A + size_t(i) * M + col);
+      for (int s = 1; s < S; ++s) a = __fadd_rn(a, __ldg(A + s * plane + size_t(i) * M + col));
+      a = __fdiv_rn(a, float(S));
+      abar[size_t(j) * N + i] = a;
+      lo = hi = a;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+      hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+    }
+    if (lane == 0) { smin[warp] = lo; smax[warp] = hi; }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      for (int w = 1; w < MASK_ROWS / 32; ++w) { lo = fminf(lo, smin[w]); hi = fmaxf(hi, smax[w]); }
+      part[size_t(blockIdx.x) * ids.n + j] = make_float2(lo, hi);
+    }
+    __syncthreads();
+  }
+}
+
+// Pass 2: column min / max over all CTAs (exact, order-free), then the
+// thresholded union over the delta tokens: ((a - mn) / (mx - mn)) >= tau.
+__global__ void __launch_bounds__(MASK_ROWS)
+mask_threshold_kernel(const float* __restrict__ abar, const float2* __restrict__ part, int nblk,
+                      int N, DeltaIds ids, float tau, uint8_t* __restrict__ uni) {
+  __shared__ float s_mn[64], s_rng[64];
+  __shared__ int s_ok[64];
+  if (threadIdx.x < ids.n) {
+    const int j = threadIdx.x;
+    float lo = FLT_MAX, hi = -FLT_MAX;
+    for (int b = 0; b < nblk; ++b) {
+      float2 v = part[size_t(b) * ids.n + j];
+      lo = fminf(lo, v.x);
+      hi = fmaxf(hi, v.y);
+    }
+    float rng = __fsub_rn(hi, lo);
+    s_mn[j] = lo;
+    s_rng[j] = rng;
+    s_ok[j] = rng > 0.0f;
+  }
+  __syncthreads();
+  const int i = blockIdx.x * MASK_ROWS + threadIdx.x;
+  if (i >= N) return;
+  uint8_t u = 0;
+  for (int j = 0; j < ids.n; ++j) {
+    if (!s_ok[j]) continue;
+    float nv = __fdiv_rn(__fsub_rn(abar[size_t(j) * N + i], s_mn[j]), s_rng[j]);
+    u |= (nv >= tau) ? 1 : 0;
+  }
+  uni[i] = u;
+}
+
+// Pass 3: (2r+1)^2 dilation on the grid, and the per-CTA dirty count.
+__global__ void __launch_bounds__(MASK_ROWS)
+mask_dilate_kernel(const uint8_t* __restrict__ uni, int gh, int gw, int r,
+                   uint8_t* __restrict__ mask, int* __restrict__ cnt) {
+  const int N = gh * gw;
+  const int i = blockIdx.x * MASK_ROWS + threadIdx.x;
+  int m = 0;
+  if (i < N) {
+    const int y = i / gw, x = i - (i / gw) * gw;
+    const int y0 = max(0, y - r), y1 = min(gh - 1, y + r);
+    const int x0 = max(0, x - r), x1 = min(gw - 1, x + r);
+    for (int yy = y0; yy <= y1 && !m; ++yy)
+      for (int xx = x0; xx <= x1; ++xx)
+        if (uni[yy * gw + xx]) { m = 1; break; }
+    mask[i] = uint8_t(m);
+  }
+  int c = __syncthreads_count(m);
+  if (threadIdx.x == 0) cnt[blockIdx.x] = c;
+}
+
+// Pass 4: compaction.  Each CTA sums the counts of the CTAs before it, then a
+// warp ballot + prefix over warps gives each dirty token its slot; the
+// indices come out in ascending token order.
+__global__ void __launch_bounds__(MASK_ROWS)
+mask_compact_kernel(const uint8_t* __restrict__ mask, const int* __restrict__ cnt, int N,
+                    int32_t* __restrict__ idx, int32_t* __restrict__ count) {
+  __shared__ int s_warp[MASK_ROWS / 32];
+  __shared__ int s_base;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (threadIdx.x < 32) {
+    int acc = 0;
+    for (int b = lane; b < int(blockIdx.x); b += 32) acc += cnt[b];
+    acc = __reduce_add_sync(0xffffffffu, acc);
+    if (lane == 0) s_base = acc;
+  }
+  const int i = blockIdx.x * MASK_ROWS + threadIdx.x;
+  const int m = (i < N) ? mask[i] : 0;
+  const unsigned bal = __ballot_sync(0xffffffffu, m);
+  if (lane == 0) s_warp[warp] = __popc(bal);
+  __syncthreads();
+  int before = s_base;
+  for (int w = 0; w < warp; ++w) before += s_warp[w];
+  if (m) idx[before + __popc(bal & ((1u << lane) - 1u))] = i;
+  if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0) {
+    int total = s_base;
+    for (int w = 0; w < MASK_ROWS / 32; ++w) total += s_warp[w];
+    *count = total;
+  }
+}
+
+cudaError_t launch_localize(const float* A, int S, int N, int M, int gh, int gw,
+                            const DeltaIds& ids, float tau, int dilation, uint8_t* mask,
+                            int32_t* idx, int32_t* count, void* ws, cudaStream_t st) {
+  const int nblk = cdiv(N, MASK_ROWS);
+  MaskWs w = carve(ws, N, ids.n);
+  mask_colstats_kernel<<<nblk, MASK_ROWS, 0, st>>>(A, S, N, M, ids, w.abar, w.part);
+  mask_threshold_kernel<<<nblk, MASK_ROWS, 0, st>>>(w.abar, w.part, nblk, N, ids, tau, w.uni);
+  mask_dilate_kernel<<<nblk, MASK_ROWS, 0, st>>>(w.uni, gh, gw, dilation, mask, w.cnt);
+  mask_compact_kernel<<<nblk, MASK_ROWS, 0, st>>>(mask, w.cnt, N, idx, count);
+  count_launches(4);
+  return cudaGetLastError();
+}
+
+// ================================================================= LN + mod
+// One warp per row; the row stays in registers (hidden <= 1536, % 128 == 0).
+constexpr int LN_WARPS = 8;
+constexpr int LN_MAXV = 12;  // float4 per lane
+
+__global__ void __launch_bounds__(LN_WARPS * 32)
+ln_mod_kernel(const float* __restrict__ x, int ldx, const float* __restrict__ tab_sh,
+              const float* __restrict__ tb_sh, const float* __restrict__ tab_sc,
+              const float* __restrict__ tb_sc, bf16* __restrict__ out, int ldo, int Dbound,
+              const int* __restrict__ dcount, int d, unsigned* err) {
+  const int D = live_count(dcount, Dbound, err);
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * LN_WARPS + (threadIdx.x >> 5);
+  if (r >= D) return;
+  const int nv = d / 128;
+  const float4* xr = reinterpret_cast<const float4*>(x + size_t(r) * ldx);
+  float4 v[LN_MAXV];
+  float s = 0.f;
+#pragma unroll
+  for (int k = 0; k < LN_MAXV; ++k)
+    if (k < nv) {
+      v[k] = xr[lane + 32 * k];
+      s += (v[k].x + v[k].y) + (v[k].z + v[k].w);
+    }
+  const float mean = warp_sum(s) / float(d);
+  float q = 0.f;
+#pragma unroll
+  for (int k = 0; k < LN_MAXV; ++k)
+    if (k < nv) {
+      float a = v[k].x - mean, b = v[k].y - mean, c = v[k].z - mean, e = v[k].w - mean;
+      q += (a * a + b * b) + (c * c + e * e);
+    }
+  const float rstd = 1.0f / sqrtf(warp_sum(q) / float(d) + 1e-6f);
+  uint2* orow = reinterpret_cast<uint2*>(out + size_t(r) * ldo);
+#pragma unroll
+  for (int k = 0; k < LN_MAXV; ++k)
+    if (k < nv) {
+      const int c = 4 * (lane + 32 * k);
+      float4 sh = *reinterpret_cast<const float4*>(tab_sh + c);
+      float4 sc = *reinterpret_cast<const float4*>(tab_sc + c);
+      if (tb_sh) {
+        float4 a = *reinterpret_cast<const float4*>(tb_sh + c);
+        sh.x += a.x; sh.y += a.y; sh.z += a.z; sh.w += a.w;
+      }
+      if (tb_sc) {
+        float4 a = *reinterpret_cast<const float4*>(tb_sc + c);
+        sc.x += a.x; sc.y += a.y; sc.z += a.z; sc.w += a.w;
+      }
+      float y0 = (v[k].x - mean) * rstd * (1.f + sc.x) + sh.x;
+      float y1 = (v[k].y - mean) * rstd * (1.f + sc.y) + sh.y;
+      float y2 = (v[k].z - mean) * rstd * (1.f + sc.z) + sh.z;
+      float y3 = (v[k].w - mean) * rstd * (1.f + sc.w) + sh.w;
+      orow[lane + 32 * k] = make_uint2(pack_bf16x2(y0, y1), pack_bf16x2(y2, y3));
+    }
+}
+
+cudaError_t launch_ln_mod(const float* x, int ldx, const float* tab_sh, const float* tb_sh,
+                          const float* tab_sc, const float* tb_sc, bf16* out, int ldo,
+                          int Dbound, const int* dcount, int d, unsigned* err, cudaStream_t st) {
+  if (Dbound <= 0) return cudaSuccess;
+  ln_mod_kernel<<<cdiv(Dbound, LN_WARPS), LN_WARPS * 32, 0, st>>>(
+      x, ldx, tab_sh, tb_sh, tab_sc, tb_sc, out, ldo, Dbound, dcount, d, err);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+// ============================================================ patch embed
+// One CTA per dirty token: gathers its p x p x C latent patch (ordered
+// channel, py, px) and applies the linear patch embedding + bias + position.
+__global__ void __launch_bounds__(256)
+patch_embed_kernel(const float* __restrict__ latent, int gh, int gw, int p, int C,
+                   const bf16* __restrict__ We, const float* __restrict__ be,
+                   const float* __restrict__ pos, const int* __restrict__ idx, int Dbound,
+                   const int* __restrict__ dcount, float* __restrict__ xf, int d, unsigned* err) {
+  __shared__ float patch[64];
+  const int D = live_count(dcount, Dbound, err);
+  const int r = blockIdx.x;
+  if (r >= D) return;
+  const int N = gh * gw;
+  int i = idx ? idx[r] : r;
+  if (i < 0 || i >= N) {
+    if (threadIdx.x == 0) atomicOr(err, DEVERR_INDEX);
+    return;
+  }
+  const int P = C * p * p;
+  const int gy = i / gw, gx = i - gy * gw;
+  const int W = gw * p, H = gh * p;
+  if (threadIdx.x < P) {
+    const int c = threadIdx.x / (p * p), rem = threadIdx.x - c * p * p;
+    const int py = rem / p, px = rem - py * p;
+    patch[threadIdx.x] = latent[(size_t(c) * H + gy * p + py) * W + gx * p + px];
+  }
+  __syncthreads();
+  for (int o = threadIdx.x; o < d; o += blockDim.x) {
+    float acc = 0.f;
+    const bf16* w = We + size_t(o) * P;
+    for (int k = 0; k < P; ++k) acc = fmaf(bf2f(w[k]), patch[k], acc);
+    xf[size_t(r) * d + o] = acc + be[o] + pos[size_t(i) * d + o];
+  }
+}
+
+cudaError_t launch_patch_embed(const float* latent, int gh, int gw, int p, int C,
+                               const bf16* We, const float* be, const float* pos,
+                               const int* idx, int Dbound, const int* dcount, float* xf, int d,
+                               unsigned* err, cudaStream_t st) {
+  if (Dbound <= 0) return cudaSuccess;
+  patch_embed_kernel<<<Dbound, 256, 0, st>>>(latent, gh, gw, p, C, We, be, pos, idx, Dbound,
+                                             dcount, xf, d, err);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+// ======================================================== timestep embed
+// f[k] = cos(t w_k), f[half + k] = sin(t w_k), w_k = 10000^(-k/half); double
+// precision for the argument so large timesteps keep their phase.
+__global__ void sinusoid_kernel(float t, int dim, float* f) {
+  const int half = dim / 2;
+  for (int k = threadIdx.x; k < half; k += blockDim.x) {
+    double w = exp(-log(10000.0) * double(k) / double(half));
+    double a = double(t) * w;
+    f[k] = float(cos(a));
+    f[half + k] = float(sin(a));
+  }
+}
+
+// out[o] = sum_k W[o][k] act(in[k]) + b[o], act = SiLU when silu_in.  One warp
+// per output; 16-byte weight loads.
+__global__ void __launch_bounds__(256)
+matvec_kernel(const bf16* __restrict__ W, const float* __restrict__ b,
+              const float* __restrict__ in, float* __restrict__ out, int in_dim, int out_dim,
+              int silu_in) {
+  extern __shared__ float s_in[];
+  for (int k = threadIdx.x; k < in_dim; k += blockDim.x) {
+    float v = in[k];
+    s_in[k] = silu_in ? silu(v) : v;
+  }
+  __syncthreads();
+  const int lane = threadIdx.x & 31;
+  const int o = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (o >= out_dim) return;
+  const bf16* w = W + size_t(o) * in_dim;
+  float acc = 0.f;
+  for (int k = lane * 8; k < in_dim; k += 256) {
+    uint4 u = *reinterpret_cast<const uint4*>(w + k);
+    float2 a0 = unpack_bf16x2(u.x), a1 = unpack_bf16x2(u.y);
+    float2 a2 = unpack_bf16x2(u.z), a3 = unpack_bf16x2(u.w);
+    acc = fmaf(a0.x, s_in[k + 0], acc);
+    acc = fmaf(a0.y, s_in[k + 1], acc);
+    acc = fmaf(a1.x, s_in[k + 2], acc);
+    acc = fmaf(a1.y, s_in[k + 3], acc);
+    acc = fmaf(a2.x, s_in[k + 4], acc);
+    acc = fmaf(a2.y, s_in[k + 5], acc);
+    acc = fmaf(a3.x, s_in[k + 6], acc);
+    acc = fmaf(a3.y, s_in[k + 7], acc);
+  }
+  acc = warp_sum(acc);
+  if (lane == 0) out[o] = acc + b[o];
+}
+
+cudaError_t launch_t_embed(float t_value, int freq_dim, int d, const bf16* Wt1, const float* bt1,
+                           const bf16* Wt2, const float* bt2, const bf16* Wtb, const float* btb,
+                           float* fbuf, float* h1, float* temb, float* tb, cudaStream_t st) {
+  sinusoid_kernel<<<1, 128, 0, st>>>(t_value, freq_dim, fbuf);
+  matvec_kernel<<<cdiv(d, 8), 256, freq_dim * sizeof(float), st>>>(Wt1, bt1, fbuf, h1, freq_dim,
+                                                                    d, 0);
+  matvec_kernel<<<cdiv(d, 8), 256, d * sizeof(float), st>>>(Wt2, bt2, h1, temb, d, d, 1);
+  matvec_kernel<<<cdiv(6 * d, 8), 256, d * sizeof(float), st>>>(Wtb, btb, temb, tb, d, 6 * d, 1);
+  count_launches(4);
+  return cudaGetLastError();
+}
+
+// ===================================================== final layer + DDIM
+// One warp per token.  The eps outputs (py, px, c < c_in) of the final linear
+// are computed for all tokens from the last block's hidden state; each updates
+// one latent element: x0 = (x - sqrt(1-ab_t) eps) / sqrt(ab_t),
+// x' = sqrt(ab_next) x0 + sqrt(1-ab_next) eps.
+constexpr int FIN_WARPS = 8;
+constexpr int FIN_MAXV = 12;  // 4-element groups per lane (hidden <= 1536)
+constexpr int FIN_MAXO = 16;  // eps outputs per token (p*p*c_in)
+
+__global__ void __launch_bounds__(FIN_WARPS * 32)
+final_ddim_kernel(const bf16* __restrict__ H, const float* __restrict__ temb,
+                  const float* __restrict__ table_f, const bf16* __restrict__ Wf,
+                  const float* __restrict__ bfin, float* __restrict__ latent, int gh, int gw,
+                  int p, int c_in, int c_out, int d, float ab_t, float ab_next) {
+  extern __shared__ uint8_t smem_raw[];
+  float* s_shift = reinterpret_cast<float*>(smem_raw);
+  float* s_scale = s_shift + d;
+  bf16* s_w = reinterpret_cast<bf16*>(s_scale + d);  // [n_eps][d]
+  const int n_eps = p * p * c_in;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    s_shift[c] = table_f[c] + temb[c];
+    s_scale[c] = table_f[d + c] + temb[c];
+  }
+  for (int e = 0; e < n_eps; ++e) {
+    const int sub = e / c_in, ch = e - sub * c_in;
+    const bf16* src = Wf + size_t(sub * c_out + ch) * d;
+    for (int c = threadIdx.x; c < d; c += blockDim.x) s_w[size_t(e) * d + c] = src[c];
+  }
+  __syncthreads();
+  const int N = gh * gw;
+  const int lane = threadIdx.x & 31;
+  const int nv = d / 128;
+  const float sa = sqrtf(ab_t), sn = sqrtf(1.f - ab_t);
+  const float ta = sqrtf(ab_next), tn = sqrtf(1.f - ab_next);
+  const int W = gw * p, Hh = gh * p;
+  for (int i = blockIdx.x * FIN_WARPS + (threadIdx.x >> 5); i < N; i += gridDim.x * FIN_WARPS) {
+    const uint2* hr = reinterpret_cast<const uint2*>(H + size_t(i) * d);
+    float y[FIN_MAXV][4];
+    float s = 0.f;
+#pragma unroll
+    for (int k = 0; k < FIN_MAXV; ++k)
+      if (k < nv) {
+        uint2 u = hr[lane + 32 * k];
+        float2 a = unpack_bf16x2(u.x), b = unpack_bf16x2(u.y);
+        y[k][0] = a.x; y[k][1] = a.y; y[k][2] = b.x; y[k][3] = b.y;
+        s += (a.x + a.y) + (b.x + b.y);
+      }
+    const float mean = warp_sum(s) / float(d);
+    float q = 0.f;
+#pragma unroll
+    for (int k = 0; k < FIN_MAXV; ++k)
+      if (k < nv)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) { float a = y[k][j] - mean; q += a * a; }
+    const float rstd = 1.0f / sqrtf(warp_sum(q) / float(d) + 1e-6f);
+#pragma unroll
+    for (int k = 0; k < FIN_MAXV; ++k)
+      if (k < nv)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int c = 4 * (lane + 32 * k) + j;
+          y[k][j] = (y[k][j] - mean) * rstd * (1.f + s_scale[c]) + s_shift[c];
+        }
+    const int gy = i / gw, gx = i - gy * gw;
+    for (int e = 0; e < n_eps; ++e) {
+      const bf16* w = s_w + size_t(e) * d;
+      float acc = 0.f;
+#pragma unroll
+      for (int k = 0; k < FIN_MAXV; ++k)
+        if (k < nv) {
+          const int c = 4 * (lane + 32 * k);
+          uint2 u = *reinterpret_cast<const uint2*>(w + c);
+          float2 a = unpack_bf16x2(u.x), b = unpack_bf16x2(u.y);
+          acc = fmaf(y[k][0], a.x, acc);
+          acc = fmaf(y[k][1], a.y, acc);
+          acc = fmaf(y[k][2], b.x, acc);
+          acc = fmaf(y[k][3], b.y, acc);
+        }
+      acc = warp_sum(acc);
+      if (lane == (e & 31)) {
+        const int sub = e / c_in, ch = e - sub * c_in;
+        const int py = sub / p, px = sub - py * p;
+        const float eps = acc + bfin[sub * c_out + ch];
+        float* xp = latent + (size_t(ch) * Hh + gy * p + py) * W + gx * p + px;
+        const float x0 = (*xp - sn * eps) / sa;
+        *xp = ta * x0 + tn * eps;
+      }
+    }
+  }
+}
+
+cudaError_t launch_final_ddim(const bf16* H, const float* temb, const float* table_f,
+                              const bf16* Wf, const float* bf, float* latent, int gh, int gw,
+                              int p, int c_in, int c_out, int d, float ab_t, float ab_next,
+                              cudaStream_t st) {
+  const int n_eps = p * p * c_in;
+  const size_t smem = size_t(2) * d * sizeof(float) + size_t(n_eps) * d * sizeof(bf16);
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaFuncSetAttribute(final_ddim_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         64 * 1024);
+    attr_set = true;
+  }
+  const int N = gh * gw;
+  int grid = cdiv(N, FIN_WARPS * 4);
+  if (grid > 1024) grid = 1024;
+  final_ddim_kernel<<<grid, FIN_WARPS * 32, smem, st>>>(H, temb, table_f, Wf, bf, latent, gh, gw,
+                                                        p, c_in, c_out, d, ab_t, ab_next);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+// ======================================================= gather / scatter
+__global__ void __launch_bounds__(256)
+rows_f32_kernel(const float* __restrict__ src, float* __restrict__ dst,
+                const int* __restrict__ idx, int Dbound, const int* __restrict__ dcount, int d,
+                int N, int scatter, unsigned* err) {
+  const int D = live_count(dcount, Dbound, err);
+  const int r = blockIdx.x;
+  if (r >= D) return;
+  const int i = idx[r];
+  if (i < 0 || i >= N) {
+    if (threadIdx.x == 0) atomicOr(err, DEVERR_INDEX);
+    return;
+  }
+  const float4* s = reinterpret_cast<const float4*>(src + size_t(scatter ? r : i) * d);
+  float4* t = reinterpret_cast<float4*>(dst + size_t(scatter ? i : r) * d);
+  for (int c = threadIdx.x; c < d / 4; c += blockDim.x) t[c] = s[c];
+}
+
+__global__ void __launch_bounds__(256)
+scatter_bf16_kernel(const float* __restrict__ src, bf16* __restrict__ dst,
+                    const int* __restrict__ idx, int Dbound, const int* __restrict__ dcount,
+                    int d, int N, unsigned* err) {
+  const int D = live_count(dcount, Dbound, err);
+  const int r = blockIdx.x;
+  if (r >= D) return;
+  const int i = idx ? idx[r] : r;
+  if (i < 0 || i >= N) {
+    if (threadIdx.x == 0) atomicOr(err, DEVERR_INDEX);
+    return;
+  }
+  const float4* s = reinterpret_cast<const float4*>(src + size_t(r) * d);
+  uint2* t = reinterpret_cast<uint2*>(dst + size_t(i) * d);
+  for (int c = threadIdx.x; c < d / 4; c += blockDim.x) {
+    float4 v = s[c];
+    t[c] = make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
+  }
+}
+
+cudaError_t launch_rows_f32(const float* src, float* dst, const int* idx, int Dbound,
+                            const int* dcount, int d, int N, bool scatter, unsigned* err,
+                            cudaStream_t st) {
+  if (Dbound <= 0) return cudaSuccess;
+  rows_f32_kernel<<<Dbound, 256, 0, st>>>(src, dst, idx, Dbound, dcount, d, N, scatter ? 1 : 0,
+                                          err);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_scatter_bf16(const float* src, bf16* dst, const int* idx, int Dbound,
+                                const int* dcount, int d, int N, unsigned* err, cudaStream_t st) {
+  if (Dbound <= 0) return cudaSuccess;
+  scatter_bf16_kernel<<<Dbound, 256, 0, st>>>(src, dst, idx, Dbound, dcount, d, N, err);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+}  // namespace rc
