@@ -176,6 +176,38 @@ rc_status rc_localize_mask(const float* xattn, int S, int N, int M, int grid_h, 
                            int32_t* dirty_count, void* workspace, size_t workspace_bytes,
                            rc_stream stream);
 
+/* Allocation-free variant of rc_localize_mask.  The paper has no counterpart
+ * to this entry point; it exists for callers that cannot allocate device
+ * memory where they need a mask: code running inside an inference server's
+ * plugin hook that must not call the CUDA allocator, programs whose device
+ * memory is wholly owned by another framework's pool, and latency-critical
+ * loops that cannot afford cudaMalloc's implicit device-wide synchronisation.
+ *
+ * It computes exactly what rc_localize_mask computes (same arguments minus
+ * the workspace, same bit-exact result) but takes its scratch from a fixed
+ * array compiled into the library: RC_NOALLOC_SCRATCH_BYTES (about 1 MiB) of
+ * device memory that every GPU which loads the library holds until the
+ * process exits.  It calls no cudaMalloc, cudaFree or other allocating
+ * routine.
+ *   Limits: N <= RC_NOALLOC_MAX_TOKENS and n_delta <= RC_NOALLOC_MAX_DELTA;
+ *   larger sizes return RC_ERR_SHAPE with a message naming the limit.
+ *   Set-up: the first call on each device (with that device current) looks
+ *   up the array's device address once; make that first call before any
+ *   stream capture.
+ *   Sharing: every call on a device uses the same scratch, which keeps the
+ *   previous call's contents; no part of it needs to start at zero (each
+ *   pass overwrites what the next pass reads).  Calls whose work overlaps on
+ *   the GPU (for example issued on two unordered streams) race on the
+ *   scratch and can return wrong masks: serialise them on one stream or
+ *   order them with events. */
+#define RC_NOALLOC_MAX_TOKENS 16384
+#define RC_NOALLOC_MAX_DELTA 16
+#define RC_NOALLOC_SCRATCH_BYTES 1073408
+rc_status rc_localize_mask_noalloc(const float* xattn, int S, int N, int M, int grid_h,
+                                   int grid_w, const int32_t* delta_ids_host, int n_delta,
+                                   float threshold, int dilation, uint8_t* mask,
+                                   int32_t* dirty_idx, int32_t* dirty_count, rc_stream stream);
+
 /* ------------------------------------------------------------ block / step */
 
 /* Region-level sparse forward of block `layer` at timestep slot `t` of

@@ -12,6 +12,8 @@ typedef __nv_bfloat16 bf16;
 
 // Kernels launched by this library in this process (reported by rc_launch_count).
 void count_launches(int n);
+// Sets the calling thread's rc_last_error() text.
+void set_last_error(const char* msg);
 
 // ------------------------------------------------------------- localisation
 struct DeltaIds {

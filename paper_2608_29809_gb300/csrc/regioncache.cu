@@ -48,6 +48,7 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 namespace rc {
 void count_launches(int n) { g_launches.fetch_add(uint64_t(n), std::memory_order_relaxed); }
+void set_last_error(const char* msg) { g_last_error = msg; }
 }  // namespace rc
 
 struct rc_ctx {

@@ -70,6 +70,7 @@ def load_library(path: str = LIB_PATH) -> C.CDLL:
         "rc_set_text": (I, [P, P, I, P, P]),
         "rc_localize_workspace_size": (S, [I, I]),
         "rc_localize_mask": (I, [P, I, I, I, I, I, P, I, F, I, P, P, P, P, S, P]),
+        "rc_localize_mask_noalloc": (I, [P, I, I, I, I, I, P, I, F, I, P, P, P, P]),
         "rc_block_forward_region": (I, [P, P, I, I, I, P, P, I, P, P, P]),
         "rc_step": (I, [P, P, I, P, I, P, P, I, P, P]),
         "rc_step_dense": (I, [P, P, I, P, I, P]),
@@ -179,6 +180,14 @@ def rc_localize_mask(xattn, S, N, M, grid_h, grid_w, delta_ids, threshold, dilat
                                  len(ids), float(threshold), dilation, _ptr(mask),
                                  _ptr(dirty_idx), _ptr(dirty_count), _ptr(workspace), ws_bytes,
                                  _stream(stream)))
+
+
+def rc_localize_mask_noalloc(xattn, S, N, M, grid_h, grid_w, delta_ids, threshold, dilation,
+                             mask, dirty_idx, dirty_count, stream=None):
+    ids = np.ascontiguousarray(delta_ids, np.int32)
+    _check(_lib.rc_localize_mask_noalloc(_ptr(xattn), S, N, M, grid_h, grid_w, ids.ctypes.data,
+                                         len(ids), float(threshold), dilation, _ptr(mask),
+                                         _ptr(dirty_idx), _ptr(dirty_count), _stream(stream)))
 
 
 def rc_block_forward_region(ctx, cache, session, layer, t, hidden, dirty_idx, D, dirty_count,
