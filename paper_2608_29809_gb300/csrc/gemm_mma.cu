@@ -218,8 +218,8 @@ gemm_mma_kernel(const bf16* __restrict__ A, int lda, const bf16* __restrict__ W,
 
 }  // namespace
 
-cudaError_t launch_gemm(const bf16* A, int lda, const bf16* W, int Mbound, const int* dcount,
-                        int n, int k, const GemmEpi& ep, cudaStream_t st) {
+cudaError_t launch_gemm_mma(const bf16* A, int lda, const bf16* W, int Mbound, const int* dcount,
+                            int n, int k, const GemmEpi& ep, cudaStream_t st) {
   if (Mbound <= 0) return cudaSuccess;
   static int attr_dev = -1;
   int dev = 0;

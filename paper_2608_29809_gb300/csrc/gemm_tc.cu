@@ -1,0 +1,555 @@
+// Tensor-core GEMM of the region-sparse block on sm_103a: tcgen05.mma with
+// TMEM accumulators, operands staged by TMA (128-byte swizzle), persistent
+// warp-specialised CTAs, and the block's epilogues fused (bias, tanh-GELU,
+// gated residual, QKV with K/V rows written straight into the cache rows of
+// the dirty tokens -- Section 3.4, Kernel Fusing -- and the merged hidden
+// state written into the cache's H rows).
+//
+// C[M][n] = A[M][k] W[n][k]^T, A and W K-major bf16, f32 accumulation.
+// M (the dirty-token count) may live on the device: every CTA reads it, derives
+// the tile list and, when the tiles cannot fill the grid, a split of K.  A
+// split-K tile's partial sums go to a workspace; the last split to finish
+// (an atomic ticket, no waiting) adds them in split order and runs the
+// epilogue, so the result is deterministic.
+//
+// CTA = 6 warps: warp 0 issues TMA loads, warp 1 owns TMEM and issues the
+// MMAs (one thread), warps 2..5 drain the accumulator (one TMEM lane = one
+// output row per thread).  Two TMEM accumulators of 128 columns let the
+// epilogue of one tile overlap the main loop of the next.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <stdlib.h>
+
+#include <mutex>
+#include <unordered_map>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace rc {
+
+namespace {
+
+constexpr int BM = 128, BN = 128, BK = 64, STAGES = 6;
+constexpr int THREADS = 192;
+constexpr int STAGE_A = BM * BK * 2;   // bytes
+constexpr int STAGE_B = BN * BK * 2;
+constexpr int TMEM_COLS = 2 * BN;      // two accumulators
+constexpr int MAX_SPLIT = 4;
+constexpr int MIN_KB_PER_SPLIT = 4;
+constexpr size_t SMEM_BYTES = size_t(STAGES) * (STAGE_A + STAGE_B) + 1024 + 256;
+constexpr unsigned long long WAIT_NS = 2000000000ull;  // bounded waits: 2 s
+
+// ---------------------------------------------------------------- PTX glue
+__device__ __forceinline__ uint32_t saddr(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ unsigned long long globaltimer() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Waits for the phase of parity `parity`; gives up (returns false) when the
+// CTA's abort flag is raised or after WAIT_NS.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const unsigned long long t0 = globaltimer();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (globaltimer() - t0 > WAIT_NS) return false;
+  }
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
+                                            int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y)
+      : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                          uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+      : "memory");
+}
+// 32 consecutive f32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+        "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+        "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Shared-memory matrix descriptor of a K-major bf16 tile written by TMA with
+// the 128-byte swizzle: rows of 128 B, 8-row groups 1024 B apart (stride byte
+// offset), descriptor version 1, layout SWIZZLE_128B.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t addr) {
+  uint64_t d = 0;
+  d |= uint64_t((addr & 0x3FFFFu) >> 4);
+  d |= uint64_t(16 >> 4) << 16;
+  d |= uint64_t(1024 >> 4) << 32;
+  d |= uint64_t(1) << 46;
+  d |= uint64_t(2) << 61;
+  return d;
+}
+
+// Instruction descriptor, kind::f16: D f32, A and B bf16, both K-major.
+constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(BN >> 3) << 17) |
+                           (uint32_t(BM >> 4) << 24);
+
+// ---------------------------------------------------------------- epilogue
+__device__ __forceinline__ void load32(const float* p, float* v) {
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    float4 a = __ldg(reinterpret_cast<const float4*>(p) + i);
+    v[4 * i] = a.x; v[4 * i + 1] = a.y; v[4 * i + 2] = a.z; v[4 * i + 3] = a.w;
+  }
+}
+__device__ __forceinline__ void store32_bf16(bf16* p, const float* v) {
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    uint4 u;
+    u.x = pack_bf16x2(v[8 * i + 0], v[8 * i + 1]);
+    u.y = pack_bf16x2(v[8 * i + 2], v[8 * i + 3]);
+    u.z = pack_bf16x2(v[8 * i + 4], v[8 * i + 5]);
+    u.w = pack_bf16x2(v[8 * i + 6], v[8 * i + 7]);
+    reinterpret_cast<uint4*>(p)[i] = u;
+  }
+}
+
+// Applies the epilogue to columns c0 .. c0+31 of output row r (r < M).
+__device__ __forceinline__ void epilogue32(const GemmEpi& ep, int r, int c0, float* v) {
+  if (ep.bias) {
+    float b[32];
+    load32(ep.bias + c0, b);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] += b[i];
+  }
+  switch (ep.mode) {
+    case EPI_F32: {
+      float4* o = reinterpret_cast<float4*>(ep.out_f + size_t(r) * ep.ld_out + c0);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+      break;
+    }
+    case EPI_BIAS_BF16:
+      store32_bf16(ep.out_bf + size_t(r) * ep.ld_out + c0, v);
+      break;
+    case EPI_GELU_BF16:
+#pragma unroll
+      for (int i = 0; i < 32; ++i) v[i] = gelu_tanh(v[i]);
+      store32_bf16(ep.out_bf + size_t(r) * ep.ld_out + c0, v);
+      break;
+    case EPI_GATE_RES: {
+      if (ep.gate_tab) {
+        float g[32];
+        load32(ep.gate_tab + c0, g);
+        if (ep.gate_tb) {
+          float g2[32];
+          load32(ep.gate_tb + c0, g2);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) g[i] += g2[i];
+        }
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] *= g[i];
+      }
+      float4* xp = reinterpret_cast<float4*>(ep.xf + size_t(r) * ep.ld_xf + c0);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        float4 x = xp[i];
+        x.x += v[4 * i]; x.y += v[4 * i + 1]; x.z += v[4 * i + 2]; x.w += v[4 * i + 3];
+        xp[i] = x;
+        v[4 * i] = x.x; v[4 * i + 1] = x.y; v[4 * i + 2] = x.z; v[4 * i + 3] = x.w;
+      }
+      if (ep.copy_bf) store32_bf16(ep.copy_bf + size_t(r) * ep.ld_copy + c0, v);
+      if (ep.scat) {
+        const int tok = ep.idx ? ep.idx[r] : r;
+        if (tok >= 0 && tok < ep.n_tokens)
+          store32_bf16(ep.scat + size_t(tok) * ep.ld_kv + c0, v);
+        else
+          atomicOr(ep.err, DEVERR_INDEX);
+      }
+      break;
+    }
+    case EPI_QKV: {
+      const int part = c0 / ep.dsplit;
+      const int cc = c0 - part * ep.dsplit;
+      if (part == 0) {
+        store32_bf16(ep.out_bf + size_t(r) * ep.ld_out + cc, v);
+      } else {
+        const int tok = ep.idx ? ep.idx[r] : r;
+        if (tok >= 0 && tok < ep.n_tokens)
+          store32_bf16((part == 1 ? ep.kc : ep.vc) + size_t(tok) * ep.ld_kv + cc, v);
+        else
+          atomicOr(ep.err, DEVERR_INDEX);
+      }
+      break;
+    }
+  }
+}
+
+struct Sched {
+  int mt, nt, tiles, split, kb_total, units;
+  __device__ void init(int M, int n, int k, int grid) {
+    mt = (M + BM - 1) / BM;
+    nt = n / BN;
+    tiles = mt * nt;
+    kb_total = k / BK;
+    split = 1;
+    if (tiles > 0 && tiles < grid) {
+      split = grid / tiles;
+      if (split > MAX_SPLIT) split = MAX_SPLIT;
+      int cap = kb_total / MIN_KB_PER_SPLIT;
+      if (split > cap) split = cap < 1 ? 1 : cap;
+    }
+    units = tiles * split;
+  }
+  // unit -> (m, n, s); m varies fastest so concurrent CTAs share W tiles in L2
+  __device__ void decode(int u, int& m, int& nn, int& s, int& kb0, int& kb1) const {
+    m = u % mt;
+    int rest = u / mt;
+    s = rest % split;
+    nn = rest / split;
+    kb0 = (kb_total * s) / split;
+    kb1 = (kb_total * (s + 1)) / split;
+  }
+};
+
+__global__ void __launch_bounds__(THREADS, 1)
+gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+               int Mbound, const int* __restrict__ dcount, int n, int k, GemmEpi ep,
+               float* __restrict__ ws, int* __restrict__ tickets, int ws_units) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  // 1024-aligned operand stages, then barriers
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + STAGES * STAGE_A;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sB + STAGES * STAGE_B);
+  // bars: full[STAGES], empty[STAGES], tfull[2], tempty[2]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 4);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  int* last_flag = reinterpret_cast<int*>(tmem_slot + 2);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t full0 = saddr(bars), empty0 = saddr(bars + STAGES);
+  const uint32_t tfull0 = saddr(bars + 2 * STAGES), tempty0 = saddr(bars + 2 * STAGES + 2);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tfull0 + 8 * a, 1);
+      mbar_init(tempty0 + 8 * a, 128);
+    }
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     saddr(tmem_slot)),
+                 "r"(TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  if (warp == 0 && lane == 0) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int M = live_count(dcount, Mbound, ep.err);
+  Sched sc;
+  sc.init(M, n, k, min(int(gridDim.x), ws_units));
+
+  if (warp == 0) {
+    // ------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int u = blockIdx.x; u < sc.units; u += gridDim.x) {
+        int m, nn, s, kb0, kb1;
+        sc.decode(u, m, nn, s, kb0, kb1);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(empty0 + 8 * stage, phase ^ 1, abort_flag)) goto timeout;
+          mbar_expect_tx(full0 + 8 * stage, STAGE_A + STAGE_B);
+          tma_load_2d(saddr(sA + stage * STAGE_A), &tmA, full0 + 8 * stage, kb * BK, m * BM);
+          tma_load_2d(saddr(sB + stage * STAGE_B), &tmB, full0 + 8 * stage, kb * BK, nn * BN);
+          if (++stage == STAGES) { stage = 0; phase ^= 1; }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      for (int u = blockIdx.x; u < sc.units; u += gridDim.x) {
+        int m, nn, s, kb0, kb1;
+        sc.decode(u, m, nn, s, kb0, kb1);
+        if (!mbar_wait(tempty0 + 8 * acc, acc_phase ^ 1, abort_flag)) goto timeout;
+        tc_fence_after();
+        const uint32_t dtm = tmem_base + uint32_t(acc * BN);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(full0 + 8 * stage, phase, abort_flag)) goto timeout;
+          tc_fence_after();
+          const uint32_t a0 = saddr(sA + stage * STAGE_A), b0 = saddr(sB + stage * STAGE_B);
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk)
+            umma_bf16(dtm, sw128_desc(a0 + 32 * kk), sw128_desc(b0 + 32 * kk), IDESC,
+                      (kb > kb0 || kk > 0) ? 1u : 0u);
+          umma_commit(empty0 + 8 * stage);
+          if (++stage == STAGES) { stage = 0; phase ^= 1; }
+        }
+        umma_commit(tfull0 + 8 * acc);
+        if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+      }
+    }
+  } else {
+    // ------------------------------------------------------- epilogue (warps 2..5)
+    const int sp = warp & 3;  // TMEM lane sub-partition this warp may access
+    const int et = threadIdx.x - 64;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int u = blockIdx.x; u < sc.units; u += gridDim.x) {
+      int m, nn, s, kb0, kb1;
+      sc.decode(u, m, nn, s, kb0, kb1);
+      if (!mbar_wait(tfull0 + 8 * acc, acc_phase, abort_flag)) goto timeout;
+      __syncwarp();
+      tc_fence_after();
+      const int row = sp * 32 + lane;
+      const int r = m * BM + row;
+      const uint32_t tbase = tmem_base + uint32_t(acc * BN) + (uint32_t(sp * 32) << 16);
+      const int tile = nn * sc.mt + m;
+      float* part = ws + (size_t(tile) * sc.split + s) * (BM * BN) + size_t(row) * BN;
+#pragma unroll 1
+      for (int ch = 0; ch < BN / 32; ++ch) {
+        float v[32];
+        tmem_ld32(tbase + uint32_t(ch * 32), v);
+        if (sc.split == 1) {
+          if (r < M) epilogue32(ep, r, nn * BN + ch * 32, v);
+        } else {
+          float4* p4 = reinterpret_cast<float4*>(part + ch * 32);
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            __stcg(p4 + i, make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]));
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(tempty0 + 8 * acc);
+      if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+      if (sc.split > 1) {
+        __threadfence();
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+        if (et == 0) {
+          const int prev = atomicAdd(tickets + tile, 1);
+          const int last = (prev == sc.split - 1);
+          if (last) tickets[tile] = 0;  // re-armed for the next launch
+          *last_flag = last;
+        }
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+        if (*last_flag) {
+          __threadfence();
+          const float* base = ws + size_t(tile) * sc.split * (BM * BN) + size_t(row) * BN;
+#pragma unroll 1
+          for (int ch = 0; ch < BN / 32; ++ch) {
+            float v[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = 0.f;
+            for (int q = 0; q < sc.split; ++q) {
+              const float4* p4 = reinterpret_cast<const float4*>(base + size_t(q) * (BM * BN) + ch * 32);
+#pragma unroll
+              for (int i = 0; i < 8; ++i) {
+                float4 a = __ldcg(p4 + i);
+                v[4 * i] += a.x; v[4 * i + 1] += a.y; v[4 * i + 2] += a.z; v[4 * i + 3] += a.w;
+              }
+            }
+            if (r < M) epilogue32(ep, r, nn * BN + ch * 32, v);
+          }
+        }
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+      }
+    }
+  }
+  goto done;
+timeout:
+  *abort_flag = 1;
+  atomicOr(ep.err, DEVERR_TIMEOUT);
+done:
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                 "r"(TMEM_COLS)
+                 : "memory");
+  }
+}
+
+// ------------------------------------------------------------------- host
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+struct MapKey {
+  const void* p;
+  uint64_t rows, cols, ld;
+  int box_rows;
+  bool operator==(const MapKey& o) const {
+    return p == o.p && rows == o.rows && cols == o.cols && ld == o.ld && box_rows == o.box_rows;
+  }
+};
+struct MapKeyHash {
+  size_t operator()(const MapKey& k) const {
+    return std::hash<const void*>()(k.p) ^ (k.rows * 1000003ull) ^ (k.cols * 7919ull) ^
+           (k.ld * 131ull) ^ size_t(k.box_rows);
+  }
+};
+
+// 2-D bf16 row-major [rows][cols] (row stride ld elements), box BK x box_rows,
+// 128-byte swizzle; out-of-range rows read as zero.
+cudaError_t tensor_map(const bf16* p, int rows, int cols, int ld, int box_rows, CUtensorMap* out) {
+  static std::mutex mu;
+  static std::unordered_map<MapKey, CUtensorMap, MapKeyHash> cache;
+  MapKey key{p, uint64_t(rows), uint64_t(cols), uint64_t(ld), box_rows};
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    auto it = cache.find(key);
+    if (it != cache.end()) {
+      *out = it->second;
+      return cudaSuccess;
+    }
+  }
+  auto fn = encode_fn();
+  if (!fn) return cudaErrorNotSupported;
+  cuuint64_t dims[2] = {cuuint64_t(cols), cuuint64_t(rows)};
+  cuuint64_t strides[1] = {cuuint64_t(ld) * sizeof(bf16)};
+  cuuint32_t box[2] = {cuuint32_t(BK), cuuint32_t(box_rows)};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<bf16*>(p), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+  std::lock_guard<std::mutex> lock(mu);
+  if (cache.size() > 4096) cache.clear();
+  cache.emplace(key, *out);
+  return cudaSuccess;
+}
+
+int device_sms() {
+  static int sms[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  if (!sms[dev]) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    if (cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             int(SMEM_BYTES)) != cudaSuccess)
+      return 0;
+    sms[dev] = v;
+  }
+  return sms[dev];
+}
+
+constexpr int MAX_TILES = 4096;
+
+}  // namespace
+
+cudaError_t gemm_scratch_shape(int* units, int* max_tiles) {
+  const int sms = device_sms();
+  if (!sms) return cudaErrorInvalidDevice;
+  *units = sms;
+  *max_tiles = MAX_TILES;
+  return cudaSuccess;
+}
+
+cudaError_t launch_gemm(const bf16* A, int lda, const bf16* W, int Mbound, const int* dcount,
+                        int n, int k, const GemmEpi& ep, const GemmScratch& gs, cudaStream_t st) {
+  if (Mbound <= 0) return cudaSuccess;
+  static const bool use_mma = [] {
+    const char* v = getenv("RC_GEMM_IMPL");
+    return v && v[0] == 'm';
+  }();
+  if (use_mma) return launch_gemm_mma(A, lda, W, Mbound, dcount, n, k, ep, st);
+  if (n % BN || k % BK) return cudaErrorInvalidValue;
+  if (((Mbound + BM - 1) / BM) * (n / BN) > gs.max_tiles) return cudaErrorInvalidValue;
+  const int sms = device_sms();
+  if (!sms) return cudaErrorInvalidDevice;
+  cudaError_t e;
+  CUtensorMap ta, tb;
+  if ((e = tensor_map(A, Mbound, k, lda, BM, &ta)) != cudaSuccess) return e;
+  if ((e = tensor_map(W, n, k, k, BN, &tb)) != cudaSuccess) return e;
+  gemm_tc_kernel<<<sms, THREADS, SMEM_BYTES, st>>>(ta, tb, Mbound, dcount, n, k, ep, gs.ws,
+                                                   gs.tickets, gs.units);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+}  // namespace rc

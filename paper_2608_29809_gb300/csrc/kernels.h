@@ -83,10 +83,24 @@ struct GemmEpi {
   unsigned* err;
 };
 
+// Split-K scratch of one context: `units` partial 128x128 f32 tiles and
+// per-tile tickets (zero between launches).
+struct GemmScratch {
+  float* ws;
+  int* tickets;
+  int units;
+  int max_tiles;
+};
+// Partial tiles / tickets a context should allocate on the current device.
+cudaError_t gemm_scratch_shape(int* units, int* max_tiles);
+
 // C[M][n] = A[M][k] W[n][k]^T, epilogue `ep`.  M = *dcount if non-null (bounded
-// by Mbound) else Mbound.  n % 128 == 0, k % 64 == 0.
+// by Mbound) else Mbound.  n % 128 == 0, k % 64 == 0.  Launches on one
+// GemmScratch must be stream-ordered.
 cudaError_t launch_gemm(const bf16* A, int lda, const bf16* W, int Mbound, const int* dcount,
-                        int n, int k, const GemmEpi& ep, cudaStream_t st);
+                        int n, int k, const GemmEpi& ep, const GemmScratch& gs, cudaStream_t st);
+cudaError_t launch_gemm_mma(const bf16* A, int lda, const bf16* W, int Mbound, const int* dcount,
+                            int n, int k, const GemmEpi& ep, cudaStream_t st);
 
 // ----------------------------------------------------------------- attention
 // O[r][h*dh..] = softmax(Q_r K^T / sqrt(dh)) V per head, over Nk keys.

@@ -73,6 +73,7 @@ struct rc_ctx {
   float* tb = nullptr;   // [6d]
   int* iota = nullptr;   // [N] identity row map (dense path)
   unsigned* err = nullptr;
+  rc::GemmScratch gs{};  // split-K partial tiles + tickets
   // timing probe
   int probe_which = RC_PROBE_OFF;
   int probe_n = 0;
@@ -144,7 +145,9 @@ struct Probe {
 void free_ctx(rc_ctx* c) {
   if (!c) return;
   probe_free(c);
-  void* ps[] = {c->xf, c->xb, c->ob, c->q, c->u, c->fbuf, c->h1, c->temb, c->tb, c->iota, c->err};
+  void* ps[] = {c->xf,   c->xb,  c->ob,   c->q,        c->u,         c->fbuf,
+                c->h1,   c->temb, c->tb,  c->iota,     c->err,       c->gs.ws,
+                c->gs.tickets};
   for (void* p : ps)
     if (p) cudaFree(p);
   delete c;
@@ -206,7 +209,7 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
   {
     Probe pr(c, RC_PROBE_GEMM, st);
     RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_qkv), rw.bound, rw.dcount, 3 * d,
-                            d, e, st), "gemm(qkv)");
+                            d, e, c->gs, st), "gemm(qkv)");
   }
   // dirty queries over all N keys / values of (l, t)
   {
@@ -228,7 +231,7 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
   {
     Probe pr(c, RC_PROBE_GEMM, st);
     RC_CUDA(rc::launch_gemm(c->ob, d, static_cast<const bf16*>(w.W_o), rw.bound, rw.dcount, d, d, e,
-                            st), "gemm(out)");
+                            c->gs, st), "gemm(out)");
   }
   // q' = x W_xq^T + b
   e = rc::GemmEpi{};
@@ -240,7 +243,7 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
   {
     Probe pr(c, RC_PROBE_GEMM, st);
     RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_xq), rw.bound, rw.dcount, d, d,
-                            e, st), "gemm(xq)");
+                            e, c->gs, st), "gemm(xq)");
   }
   {
     Probe pr(c, RC_PROBE_ATTENTION, st);
@@ -257,7 +260,7 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
   {
     Probe pr(c, RC_PROBE_GEMM, st);
     RC_CUDA(rc::launch_gemm(c->ob, d, static_cast<const bf16*>(w.W_xo), rw.bound, rw.dcount, d, d,
-                            e, st), "gemm(xo)");
+                            e, c->gs, st), "gemm(xo)");
   }
   // MLP
   RC_CUDA(rc::launch_ln_mod(c->xf, d, mv(tab, 3), mv(tbv, 3), mv(tab, 4), mv(tbv, 4), c->xb, d,
@@ -271,7 +274,7 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
   {
     Probe pr(c, RC_PROBE_GEMM, st);
     RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_1), rw.bound, rw.dcount, F, d, e,
-                            st), "gemm(fc1)");
+                            c->gs, st), "gemm(fc1)");
   }
   // x += gate_mlp (u W_2^T + b_2); merged H^{l+1}: row idx[r] of the cache
   e = rc::GemmEpi{};
@@ -289,7 +292,7 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
   {
     Probe pr(c, RC_PROBE_GEMM, st);
     RC_CUDA(rc::launch_gemm(c->u, F, static_cast<const bf16*>(w.W_2), rw.bound, rw.dcount, d, F, e,
-                            st), "gemm(fc2)");
+                            c->gs, st), "gemm(fc2)");
   }
   return RC_OK;
 }
@@ -359,6 +362,22 @@ rc_status rc_create(const rc_dims* dims, rc_ctx** out) {
       (s = dalloc(&c->err, 1, "err"))) {
     free_ctx(c);
     return s;
+  }
+  {
+    int units = 0, max_tiles = 0;
+    cudaError_t e0 = rc::gemm_scratch_shape(&units, &max_tiles);
+    if (e0 != cudaSuccess) {
+      free_ctx(c);
+      return cuda_fail(e0, "rc_create: device query");
+    }
+    c->gs.units = units;
+    c->gs.max_tiles = max_tiles;
+    if ((s = dalloc(&c->gs.ws, size_t(units) * 128 * 128, "gemm split-K partials")) ||
+        (s = dalloc(&c->gs.tickets, size_t(max_tiles), "gemm tickets"))) {
+      free_ctx(c);
+      return s;
+    }
+    cudaMemset(c->gs.tickets, 0, sizeof(int) * size_t(max_tiles));
   }
   iota_kernel<<<int((N + 255) / 256), 256>>>(c->iota, int(N));
   rc::count_launches(1);
@@ -488,7 +507,7 @@ rc_status rc_set_text(rc_ctx* c, rc_cache* k, int s, const void* ctx_bf16, rc_st
     e.err = c->err;
     RC_CUDA(rc::launch_gemm(static_cast<const bf16*>(ctx_bf16), c->d,
                             static_cast<const bf16*>(c->lw[l].W_xkv), c->M, nullptr, 2 * c->d,
-                            c->d, e, st), "gemm(text kv)");
+                            c->d, e, c->gs, st), "gemm(text kv)");
   }
   k->text_set[s] = 1;
   return RC_OK;
@@ -628,7 +647,8 @@ rc_status rc_linear(rc_ctx* c, const void* x, const void* W, const float* b, flo
   e.ld_out = n;
   e.err = c->err;
   RC_CUDA(rc::launch_gemm(static_cast<const bf16*>(x), kdim, static_cast<const bf16*>(W), rows,
-                          nullptr, n, kdim, e, static_cast<cudaStream_t>(stream)), "gemm(linear)");
+                          nullptr, n, kdim, e, c->gs, static_cast<cudaStream_t>(stream)),
+          "gemm(linear)");
   return RC_OK;
 }
 
