@@ -219,7 +219,8 @@ def run_ours(args, world, rank, local):
     from paper_2608_29809_gb300 import regioncache as R
     torch.cuda.set_device(local)
     dev = f"cuda:{local}"
-    d = synth.PIXART_1024
+    from dataclasses import replace
+    d = replace(synth.PIXART_1024, timesteps=args.resident_steps)
     K, W = args.steps, args.warmup
     wl = Workload(R, d, SEED + rank, dev)
     peaks = load_peaks()
@@ -242,6 +243,14 @@ def run_ours(args, world, rank, local):
     D = int(wl.cnt.item())
     ms_max = max_over_ranks(ms, world)
     value = K * world / (ms_max / 1e3)
+    if args.quick:
+        if rank == 0:
+            print(json.dumps({"metric": METRIC, "value": round(value, 3), "unit": UNIT,
+                              "quick": True, "ms_per_step": round(ms_max / K, 4),
+                              "dirty_tokens": D, "gemm_ms": gemm_ms, "gemm_launches": gemm_n,
+                              "gpu_launches": int(launches)}), flush=True)
+        wl.model.close()
+        return
 
     # attention probe (separate pass over the same workload)
     R.rc_probe_enable(wl.model.ctx, R.RC_PROBE_ATTENTION, K * d.layers * 2)
@@ -426,6 +435,10 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-layers", type=int, default=2)
+    ap.add_argument("--quick", action="store_true",
+                    help="headline only: no attention probe, sweep, dense, e2e or cpu baseline")
+    ap.add_argument("--resident-steps", type=int, default=20,
+                    help="timesteps held in the cache (1 keeps a profiling run to ~2 GB)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         raise SystemExit("--warmup must be >= 3")
