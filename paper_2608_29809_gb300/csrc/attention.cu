@@ -4,10 +4,13 @@
 // whose dirty rows the QKV GEMM has just refreshed; in the text cross-
 // attention they are the 120 per-layer text keys / values.
 //
-// One CTA = 64 queries of one head (4 warps x 16 rows); K/V tiles of 64 keys
-// are double-buffered in shared memory with cp.async; S = Q K^T and O += P V
-// run on mma.sync (m16n8k16, plus m16n8k8 for the 8-wide tail of head_dim
-// 72); the softmax is online, in registers, in base 2.
+// One CTA = 64 queries of one head (4 warps x 16 rows) over one split of the
+// keys; K/V tiles of 64 keys are double-buffered in shared memory with
+// cp.async; S = Q K^T and O += P V run on mma.sync (m16n8k16, plus m16n8k8 for
+// the 8-wide tail of head_dim 72); the softmax is online, in registers, in
+// base 2.  With several key splits, each split stores its unnormalised output
+// and row max / sum; the last split of a (query tile, head) to finish (an
+// atomic ticket, no waiting) merges them in split order.
 #include <math.h>
 
 #include "common.cuh"
@@ -85,15 +88,18 @@ template <int DH>
 __global__ void __launch_bounds__(THREADS)
 attn_kernel(const bf16* __restrict__ Q, int ldq, const bf16* __restrict__ Kp,
             const bf16* __restrict__ Vp, int ldkv, int Nk, bf16* __restrict__ O, int ldo,
-            int Dbound, const int* __restrict__ dcount, float scale_log2, unsigned* err) {
+            int Dbound, const int* __restrict__ dcount, float scale_log2, unsigned* err,
+            float* __restrict__ part, int* __restrict__ tickets) {
   using C = Cfg<DH>;
   __shared__ __align__(128) bf16 sQ[BQ * C::SROW];
   __shared__ __align__(128) bf16 sK[2][BKV * C::SROW];
   __shared__ __align__(128) bf16 sV[2][BKV * C::SROW];
+  __shared__ int s_last;
 
   const int D = live_count(dcount, Dbound, err);
   const int q0 = blockIdx.x * BQ;
   const int h = blockIdx.y;
+  const int nsplit = gridDim.z, split = blockIdx.z;
   if (q0 >= D) return;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int hoff = h * DH;
@@ -115,8 +121,12 @@ attn_kernel(const bf16* __restrict__ Q, int ldq, const bf16* __restrict__ Kp,
       cp_async16(smem_u32(sV[buf] + row * C::SROW + ch * 8), Vp + off, ok ? 16 : 0);
     }
   };
-  const int nkb = (Nk + BKV - 1) / BKV;
-  load_kv(0, 0);
+  const int nkb_all = (Nk + BKV - 1) / BKV;
+  const int per = (nkb_all + nsplit - 1) / nsplit;
+  const int kb_begin = split * per;
+  const int kb_end = min(nkb_all, kb_begin + per);
+  const int nkb = kb_end > kb_begin ? kb_end - kb_begin : 0;
+  if (nkb > 0) load_kv(0, kb_begin);
   cp_async_commit();
 
   uint32_t qa[C::KS16][4];
@@ -129,7 +139,7 @@ attn_kernel(const bf16* __restrict__ Q, int ldq, const bf16* __restrict__ Kp,
 
   for (int kb = 0; kb < nkb; ++kb) {
     const int buf = kb & 1;
-    if (kb + 1 < nkb) load_kv(buf ^ 1, kb + 1);
+    if (kb + 1 < nkb) load_kv(buf ^ 1, kb_begin + kb + 1);
     cp_async_commit();
     cp_async_wait<1>();
     __syncthreads();
@@ -180,7 +190,7 @@ attn_kernel(const bf16* __restrict__ Q, int ldq, const bf16* __restrict__ Kp,
 
     // ---- mask the ragged key tail, online softmax (base 2)
     const int g = lane >> 2, t4 = lane & 3;
-    const int kbase_idx = kb * BKV;
+    const int kbase_idx = (kb_begin + kb) * BKV;
     float mx[2] = {mrow[0], mrow[1]};
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt) {
@@ -255,8 +265,66 @@ attn_kernel(const bf16* __restrict__ Q, int ldq, const bf16* __restrict__ Kp,
     __syncthreads();  // buffer `buf` is refilled by the next iteration's prefetch
   }
 
-  // ---- normalise and store
+  cp_async_wait<0>();
   const int g = lane >> 2, t4 = lane & 3;
+  if (nsplit > 1) {
+    // ---- partial result of this split, then the merge by the last split
+    constexpr int SLOT = BQ * (DH + 2);
+    const int tile = blockIdx.x * gridDim.y + h;
+    float* mine = part + (size_t(tile) * nsplit + split) * SLOT;
+    const int rr = warp * 16 + g;
+#pragma unroll
+    for (int nt = 0; nt < C::NT; ++nt) {
+      const int c = nt * 8 + 2 * t4;
+      __stcg(reinterpret_cast<float2*>(mine + rr * DH + c), make_float2(o[nt][0], o[nt][1]));
+      __stcg(reinterpret_cast<float2*>(mine + (rr + 8) * DH + c), make_float2(o[nt][2], o[nt][3]));
+    }
+    if (t4 == 0) {
+      __stcg(mine + BQ * DH + rr, mrow[0]);
+      __stcg(mine + BQ * DH + rr + 8, mrow[1]);
+      __stcg(mine + BQ * DH + BQ + rr, lrow[0]);
+      __stcg(mine + BQ * DH + BQ + rr + 8, lrow[1]);
+    }
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) {
+      const int prev = atomicAdd(tickets + tile, 1);
+      s_last = (prev == nsplit - 1);
+      if (s_last) tickets[tile] = 0;  // re-armed for the next launch
+    }
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    const float* base = part + size_t(tile) * nsplit * SLOT;
+    const int r = tid >> 1, c0 = (tid & 1) * (DH / 2);
+    if (q0 + r >= D) return;
+    float M = -INFINITY;
+    for (int q = 0; q < nsplit; ++q) M = fmaxf(M, __ldcg(base + q * SLOT + BQ * DH + r));
+    const float Msub = (M == -INFINITY) ? 0.f : M;
+    float L = 0.f;
+    float acc[DH / 2];
+#pragma unroll
+    for (int c = 0; c < DH / 2; ++c) acc[c] = 0.f;
+    for (int q = 0; q < nsplit; ++q) {
+      const float* sl = base + q * SLOT;
+      const float w = exp2f(__ldcg(sl + BQ * DH + r) - Msub);
+      L += w * __ldcg(sl + BQ * DH + BQ + r);
+#pragma unroll
+      for (int c = 0; c < DH / 2; c += 2) {
+        const float2 v = __ldcg(reinterpret_cast<const float2*>(sl + r * DH + c0 + c));
+        acc[c] += w * v.x;
+        acc[c + 1] += w * v.y;
+      }
+    }
+    const float inv = L > 0.f ? 1.f / L : 0.f;
+    bf16* orow = O + size_t(q0 + r) * ldo + hoff + c0;
+#pragma unroll
+    for (int c = 0; c < DH / 2; c += 2)
+      *reinterpret_cast<uint32_t*>(orow + c) = pack_bf16x2(acc[c] * inv, acc[c + 1] * inv);
+    return;
+  }
+
+  // ---- normalise and store
   const float inv0 = lrow[0] > 0.f ? 1.f / lrow[0] : 0.f;
   const float inv1 = lrow[1] > 0.f ? 1.f / lrow[1] : 0.f;
   const int r0 = q0 + warp * 16 + g;
@@ -274,18 +342,29 @@ attn_kernel(const bf16* __restrict__ Q, int ldq, const bf16* __restrict__ Kp,
 
 }  // namespace
 
+size_t attention_split_floats(int Nmax, int heads, int dh) {
+  return size_t((Nmax + BQ - 1) / BQ) * heads * ATTN_MAX_SPLIT * BQ * (dh + 2);
+}
+
+int attention_tickets(int Nmax, int heads) { return ((Nmax + BQ - 1) / BQ) * heads; }
+
 cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* V, int ldkv,
                              int Nk, bf16* O, int ldo, int heads, int dh, int Dbound,
-                             const int* dcount, unsigned* err, cudaStream_t st) {
+                             const int* dcount, unsigned* err, const AttnScratch& as,
+                             cudaStream_t st) {
   if (Dbound <= 0) return cudaSuccess;
   const float scale_log2 = float(1.4426950408889634 / sqrt(double(dh)));
-  dim3 grid((Dbound + BQ - 1) / BQ, heads);
+  // keys per split >= 1024: 4 splits at 4096 keys, none for the 120 text keys
+  int nsplit = Nk / 1024;
+  if (nsplit > ATTN_MAX_SPLIT) nsplit = ATTN_MAX_SPLIT;
+  if (nsplit < 1 || !as.part || (Dbound + BQ - 1) / BQ > as.max_qtiles) nsplit = 1;
+  dim3 grid((Dbound + BQ - 1) / BQ, heads, nsplit);
   if (dh == 72) {
     attn_kernel<72><<<grid, THREADS, 0, st>>>(Q, ldq, K, V, ldkv, Nk, O, ldo, Dbound, dcount,
-                                               scale_log2, err);
+                                               scale_log2, err, as.part, as.tickets);
   } else if (dh == 64) {
     attn_kernel<64><<<grid, THREADS, 0, st>>>(Q, ldq, K, V, ldkv, Nk, O, ldo, Dbound, dcount,
-                                               scale_log2, err);
+                                               scale_log2, err, as.part, as.tickets);
   } else {
     return cudaErrorInvalidValue;
   }

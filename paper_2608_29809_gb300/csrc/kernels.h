@@ -103,10 +103,22 @@ cudaError_t launch_gemm_mma(const bf16* A, int lda, const bf16* W, int Mbound, c
                             int n, int k, const GemmEpi& ep, cudaStream_t st);
 
 // ----------------------------------------------------------------- attention
+constexpr int ATTN_MAX_SPLIT = 4;
+// Key-split scratch of one context: partial outputs and per-(query tile,
+// head) tickets (zero between launches).
+struct AttnScratch {
+  float* part;
+  int* tickets;
+  int max_qtiles;
+};
+size_t attention_split_floats(int Nmax, int heads, int dh);
+int attention_tickets(int Nmax, int heads);
+
 // O[r][h*dh..] = softmax(Q_r K^T / sqrt(dh)) V per head, over Nk keys.
 // Q/O compact rows (r < D), K/V rows 0..Nk-1 with row stride ldkv.
 cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* V, int ldkv,
                              int Nk, bf16* O, int ldo, int heads, int dh, int Dbound,
-                             const int* dcount, unsigned* err, cudaStream_t st);
+                             const int* dcount, unsigned* err, const AttnScratch& as,
+                             cudaStream_t st);
 
 }  // namespace rc

@@ -74,6 +74,7 @@ struct rc_ctx {
   int* iota = nullptr;   // [N] identity row map (dense path)
   unsigned* err = nullptr;
   rc::GemmScratch gs{};  // split-K partial tiles + tickets
+  rc::AttnScratch as{};  // key-split partial outputs + tickets
   // timing probe
   int probe_which = RC_PROBE_OFF;
   int probe_n = 0;
@@ -147,7 +148,7 @@ void free_ctx(rc_ctx* c) {
   probe_free(c);
   void* ps[] = {c->xf,   c->xb,  c->ob,   c->q,        c->u,         c->fbuf,
                 c->h1,   c->temb, c->tb,  c->iota,     c->err,       c->gs.ws,
-                c->gs.tickets};
+                c->gs.tickets, c->as.part, c->as.tickets};
   for (void* p : ps)
     if (p) cudaFree(p);
   delete c;
@@ -215,7 +216,7 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
   {
     Probe pr(c, RC_PROBE_ATTENTION, st);
     RC_CUDA(rc::launch_attention(c->q, d, Kc, Vc, d, N, c->ob, d, c->dims.heads, c->dh, rw.bound,
-                                 rw.dcount, c->err, st), "attention(self)");
+                                 rw.dcount, c->err, c->as, st), "attention(self)");
   }
   // x += gate_msa (o W_o^T + b_o); bf16 copy of x for the cross-attention query
   e = rc::GemmEpi{};
@@ -248,7 +249,7 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
   {
     Probe pr(c, RC_PROBE_ATTENTION, st);
     RC_CUDA(rc::launch_attention(c->q, d, tk, tv, 2 * d, c->M, c->ob, d, c->dims.heads, c->dh,
-                                 rw.bound, rw.dcount, c->err, st), "attention(cross)");
+                                 rw.bound, rw.dcount, c->err, c->as, st), "attention(cross)");
   }
   // x += o' W_xo^T + b
   e = rc::GemmEpi{};
@@ -378,6 +379,14 @@ rc_status rc_create(const rc_dims* dims, rc_ctx** out) {
       return s;
     }
     cudaMemset(c->gs.tickets, 0, sizeof(int) * size_t(max_tiles));
+    const int nt = rc::attention_tickets(int(N), D.heads);
+    if ((s = dalloc(&c->as.part, rc::attention_split_floats(int(N), D.heads, dh), "attn part")) ||
+        (s = dalloc(&c->as.tickets, size_t(nt), "attn tickets"))) {
+      free_ctx(c);
+      return s;
+    }
+    cudaMemset(c->as.tickets, 0, sizeof(int) * size_t(nt));
+    c->as.max_qtiles = int((N + 63) / 64);
   }
   iota_kernel<<<int((N + 255) / 256), 256>>>(c->iota, int(N));
   rc::count_launches(1);

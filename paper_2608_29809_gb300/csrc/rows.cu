@@ -411,29 +411,42 @@ final_ddim_kernel(const bf16* __restrict__ H, const float* __restrict__ temb,
           y[k][j] = (y[k][j] - mean) * rstd * (1.f + s_scale[c]) + s_shift[c];
         }
     const int gy = i / gw, gx = i - gy * gw;
-    for (int e = 0; e < n_eps; ++e) {
-      const bf16* w = s_w + size_t(e) * d;
-      float acc = 0.f;
+    // all eps dot products first (independent reductions), then one batched
+    // latent update: lane e < n_eps owns output e
+    float acc[FIN_MAXO];
 #pragma unroll
-      for (int k = 0; k < FIN_MAXV; ++k)
-        if (k < nv) {
-          const int c = 4 * (lane + 32 * k);
-          uint2 u = *reinterpret_cast<const uint2*>(w + c);
-          float2 a = unpack_bf16x2(u.x), b = unpack_bf16x2(u.y);
-          acc = fmaf(y[k][0], a.x, acc);
-          acc = fmaf(y[k][1], a.y, acc);
-          acc = fmaf(y[k][2], b.x, acc);
-          acc = fmaf(y[k][3], b.y, acc);
-        }
-      acc = warp_sum(acc);
-      if (lane == (e & 31)) {
-        const int sub = e / c_in, ch = e - sub * c_in;
-        const int py = sub / p, px = sub - py * p;
-        const float eps = acc + bfin[sub * c_out + ch];
-        float* xp = latent + (size_t(ch) * Hh + gy * p + py) * W + gx * p + px;
-        const float x0 = (*xp - sn * eps) / sa;
-        *xp = ta * x0 + tn * eps;
+    for (int e = 0; e < FIN_MAXO; ++e) {
+      acc[e] = 0.f;
+      if (e < n_eps) {
+        const bf16* w = s_w + size_t(e) * d;
+#pragma unroll
+        for (int k = 0; k < FIN_MAXV; ++k)
+          if (k < nv) {
+            const int c = 4 * (lane + 32 * k);
+            uint2 u = *reinterpret_cast<const uint2*>(w + c);
+            float2 a = unpack_bf16x2(u.x), b = unpack_bf16x2(u.y);
+            acc[e] = fmaf(y[k][0], a.x, acc[e]);
+            acc[e] = fmaf(y[k][1], a.y, acc[e]);
+            acc[e] = fmaf(y[k][2], b.x, acc[e]);
+            acc[e] = fmaf(y[k][3], b.y, acc[e]);
+          }
       }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+      for (int e = 0; e < FIN_MAXO; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], o);
+    float mine = 0.f;
+#pragma unroll
+    for (int e = 0; e < FIN_MAXO; ++e)
+      if (lane == e) mine = acc[e];
+    if (lane < n_eps) {
+      const int sub = lane / c_in, ch = lane - (lane / c_in) * c_in;
+      const int py = sub / p, px = sub - py * p;
+      const float eps = mine + bfin[sub * c_out + ch];
+      float* xp = latent + (size_t(ch) * Hh + gy * p + py) * W + gx * p + px;
+      const float x0 = (*xp - sn * eps) / sa;
+      *xp = ta * x0 + tn * eps;
     }
   }
 }
