@@ -14,8 +14,9 @@
 //
 // CTA = 6 warps: warp 0 issues TMA loads, warp 1 owns TMEM and issues the
 // MMAs (one thread), warps 2..5 drain the accumulator (one TMEM lane = one
-// output row per thread).  Two TMEM accumulators of 128 columns let the
-// epilogue of one tile overlap the main loop of the next.
+// output row per thread).  Two TMEM accumulators (tiles of 128 x 192, or
+// 128 x 128 when 192 does not divide n) let the epilogue of one tile overlap
+// the main loop of the next.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -31,15 +32,27 @@ namespace rc {
 
 namespace {
 
-constexpr int BM = 128, BN = 128, BK = 64, STAGES = 6;
+constexpr int BM = 128, BK = 64;
 constexpr int THREADS = 192;
 constexpr int STAGE_A = BM * BK * 2;   // bytes
-constexpr int STAGE_B = BN * BK * 2;
-constexpr int TMEM_COLS = 2 * BN;      // two accumulators
 constexpr int MAX_SPLIT = 4;
 constexpr int MIN_KB_PER_SPLIT = 4;
-constexpr size_t SMEM_BYTES = size_t(STAGES) * (STAGE_A + STAGE_B) + 1024 + 256;
+constexpr int MAX_BN = 192;
 constexpr unsigned long long WAIT_NS = 2000000000ull;  // bounded waits: 2 s
+
+// Tile width BN (output features per tile): 192 when it divides n (every
+// PixArt-alpha width: 1152, 2304, 3456, 4608), else 128.
+template <int BN>
+struct TileCfg {
+  static constexpr int STAGE_B = BN * BK * 2;
+  static constexpr int STAGES = (200 * 1024) / (STAGE_A + STAGE_B);  // 6 for 128, 5 for 192
+  static constexpr int TMEM_COLS = (2 * BN <= 256) ? 256 : 512;     // two accumulators
+  static constexpr size_t SMEM_BYTES = size_t(STAGES) * (STAGE_A + STAGE_B) + 1024 + 256;
+  // Instruction descriptor, kind::f16: D f32, A and B bf16, both K-major,
+  // N >> 3 at bit 17, M >> 4 at bit 24.
+  static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
+                                    (uint32_t(BN >> 3) << 17) | (uint32_t(BM >> 4) << 24);
+};
 
 // ---------------------------------------------------------------- PTX glue
 __device__ __forceinline__ uint32_t saddr(const void* p) {
@@ -142,9 +155,6 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t addr) {
   return d;
 }
 
-// Instruction descriptor, kind::f16: D f32, A and B bf16, both K-major.
-constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(BN >> 3) << 17) |
-                           (uint32_t(BM >> 4) << 24);
 
 // ---------------------------------------------------------------- epilogue
 __device__ __forceinline__ void load32(const float* p, float* v) {
@@ -237,6 +247,7 @@ __device__ __forceinline__ void epilogue32(const GemmEpi& ep, int r, int c0, flo
   }
 }
 
+template <int BN>
 struct Sched {
   int mt, nt, tiles, split, kb_total, units;
   __device__ void init(int M, int n, int k, int grid) {
@@ -264,10 +275,13 @@ struct Sched {
   }
 };
 
+template <int BN>
 __global__ void __launch_bounds__(THREADS, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                int Mbound, const int* __restrict__ dcount, int n, int k, GemmEpi ep,
                float* __restrict__ ws, int* __restrict__ tickets, int ws_units) {
+  using TC = TileCfg<BN>;
+  constexpr int STAGES = TC::STAGES, STAGE_B = TC::STAGE_B, TMEM_COLS = TC::TMEM_COLS;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 1024-aligned operand stages, then barriers
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -313,7 +327,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   const uint32_t tmem_base = *tmem_slot;
 
   const int M = live_count(dcount, Mbound, ep.err);
-  Sched sc;
+  Sched<BN> sc;
   sc.init(M, n, k, min(int(gridDim.x), ws_units));
 
   if (warp == 0) {
@@ -345,14 +359,14 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         sc.decode(u, m, nn, s, kb0, kb1);
         if (!mbar_wait(tempty0 + 8 * acc, acc_phase ^ 1, abort_flag)) goto timeout;
         tc_fence_after();
-        const uint32_t dtm = tmem_base + uint32_t(acc * BN);
+        const uint32_t dtm = tmem_base + uint32_t(acc * (TMEM_COLS / 2));
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(full0 + 8 * stage, phase, abort_flag)) goto timeout;
           tc_fence_after();
           const uint32_t a0 = saddr(sA + stage * STAGE_A), b0 = saddr(sB + stage * STAGE_B);
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk)
-            umma_bf16(dtm, sw128_desc(a0 + 32 * kk), sw128_desc(b0 + 32 * kk), IDESC,
+            umma_bf16(dtm, sw128_desc(a0 + 32 * kk), sw128_desc(b0 + 32 * kk), TC::IDESC,
                       (kb > kb0 || kk > 0) ? 1u : 0u);
           umma_commit(empty0 + 8 * stage);
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
@@ -375,7 +389,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       tc_fence_after();
       const int row = sp * 32 + lane;
       const int r = m * BM + row;
-      const uint32_t tbase = tmem_base + uint32_t(acc * BN) + (uint32_t(sp * 32) << 16);
+      const uint32_t tbase = tmem_base + uint32_t(acc * (TMEM_COLS / 2)) + (uint32_t(sp * 32) << 16);
       const int tile = nn * sc.mt + m;
       float* part = ws + (size_t(tile) * sc.split + s) * (BM * BN) + size_t(row) * BN;
 #pragma unroll 1
@@ -510,8 +524,10 @@ int device_sms() {
   if (!sms[dev]) {
     int v = 0;
     if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-    if (cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             int(SMEM_BYTES)) != cudaSuccess)
+    if (cudaFuncSetAttribute(gemm_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             int(TileCfg<128>::SMEM_BYTES)) != cudaSuccess ||
+        cudaFuncSetAttribute(gemm_tc_kernel<192>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             int(TileCfg<192>::SMEM_BYTES)) != cudaSuccess)
       return 0;
     sms[dev] = v;
   }
@@ -522,11 +538,12 @@ constexpr int MAX_TILES = 4096;
 
 }  // namespace
 
-cudaError_t gemm_scratch_shape(int* units, int* max_tiles) {
+cudaError_t gemm_scratch_shape(int* units, int* max_tiles, size_t* ws_floats) {
   const int sms = device_sms();
   if (!sms) return cudaErrorInvalidDevice;
   *units = sms;
   *max_tiles = MAX_TILES;
+  *ws_floats = size_t(sms) * BM * MAX_BN;
   return cudaSuccess;
 }
 
@@ -538,16 +555,22 @@ cudaError_t launch_gemm(const bf16* A, int lda, const bf16* W, int Mbound, const
     return v && v[0] == 'm';
   }();
   if (use_mma) return launch_gemm_mma(A, lda, W, Mbound, dcount, n, k, ep, st);
-  if (n % BN || k % BK) return cudaErrorInvalidValue;
-  if (((Mbound + BM - 1) / BM) * (n / BN) > gs.max_tiles) return cudaErrorInvalidValue;
+  if (n % 128 || k % BK) return cudaErrorInvalidValue;
   const int sms = device_sms();
   if (!sms) return cudaErrorInvalidDevice;
+  const int BN = (n % 192 == 0) ? 192 : 128;
   cudaError_t e;
   CUtensorMap ta, tb;
   if ((e = tensor_map(A, Mbound, k, lda, BM, &ta)) != cudaSuccess) return e;
   if ((e = tensor_map(W, n, k, k, BN, &tb)) != cudaSuccess) return e;
-  gemm_tc_kernel<<<sms, THREADS, SMEM_BYTES, st>>>(ta, tb, Mbound, dcount, n, k, ep, gs.ws,
-                                                   gs.tickets, gs.units);
+  // split-K only runs when the tiles do not fill the grid; its tickets cover them
+  const int units = min(gs.units, gs.max_tiles);
+  if (BN == 192)
+    gemm_tc_kernel<192><<<sms, THREADS, TileCfg<192>::SMEM_BYTES, st>>>(
+        ta, tb, Mbound, dcount, n, k, ep, gs.ws, gs.tickets, units);
+  else
+    gemm_tc_kernel<128><<<sms, THREADS, TileCfg<128>::SMEM_BYTES, st>>>(
+        ta, tb, Mbound, dcount, n, k, ep, gs.ws, gs.tickets, units);
   count_launches(1);
   return cudaGetLastError();
 }

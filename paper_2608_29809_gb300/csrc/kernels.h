@@ -91,8 +91,9 @@ struct GemmScratch {
   int units;
   int max_tiles;
 };
-// Partial tiles / tickets a context should allocate on the current device.
-cudaError_t gemm_scratch_shape(int* units, int* max_tiles);
+// Partial tiles / tickets / workspace floats a context should allocate on the
+// current device.
+cudaError_t gemm_scratch_shape(int* units, int* max_tiles, size_t* ws_floats);
 
 // C[M][n] = A[M][k] W[n][k]^T, epilogue `ep`.  M = *dcount if non-null (bounded
 // by Mbound) else Mbound.  n % 128 == 0, k % 64 == 0.  Launches on one

@@ -366,14 +366,15 @@ rc_status rc_create(const rc_dims* dims, rc_ctx** out) {
   }
   {
     int units = 0, max_tiles = 0;
-    cudaError_t e0 = rc::gemm_scratch_shape(&units, &max_tiles);
+    size_t ws_floats = 0;
+    cudaError_t e0 = rc::gemm_scratch_shape(&units, &max_tiles, &ws_floats);
     if (e0 != cudaSuccess) {
       free_ctx(c);
       return cuda_fail(e0, "rc_create: device query");
     }
     c->gs.units = units;
     c->gs.max_tiles = max_tiles;
-    if ((s = dalloc(&c->gs.ws, size_t(units) * 128 * 128, "gemm split-K partials")) ||
+    if ((s = dalloc(&c->gs.ws, ws_floats, "gemm split-K partials")) ||
         (s = dalloc(&c->gs.tickets, size_t(max_tiles), "gemm tickets"))) {
       free_ctx(c);
       return s;
