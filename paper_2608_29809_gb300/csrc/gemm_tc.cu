@@ -7,10 +7,11 @@
 //
 // C[M][n] = A[M][k] W[n][k]^T, A and W K-major bf16, f32 accumulation.
 // M (the dirty-token count) may live on the device: every CTA reads it, derives
-// the tile list and, when the tiles cannot fill the grid, a split of K.  A
-// split-K tile's partial sums go to a workspace; the last split to finish
-// (an atomic ticket, no waiting) adds them in split order and runs the
-// epilogue, so the result is deterministic.
+// the tile list and, when the tiles cannot fill the grid, a split of K.  The
+// gated residual (x += gate (C + b)) is written as vector reductions into x,
+// so the splits of K simply add up; for the other epilogues the splits reduce
+// into a zeroed f32 tile and the last split to arrive (an atomic ticket, no
+// waiting) reads it once, zeroes it and applies the epilogue.
 //
 // CTA = 6 warps: warp 0 issues TMA loads, warp 1 owns TMEM and issues the
 // MMAs (one thread), warps 2..5 drain the accumulator (one TMEM lane = one
@@ -19,8 +20,6 @@
 // the main loop of the next.
 #include <cuda.h>
 #include <cudaTypedefs.h>
-
-#include <stdlib.h>
 
 #include <mutex>
 #include <unordered_map>
@@ -176,9 +175,18 @@ __device__ __forceinline__ void store32_bf16(bf16* p, const float* v) {
   }
 }
 
-// Applies the epilogue to columns c0 .. c0+31 of output row r (r < M).
-__device__ __forceinline__ void epilogue32(const GemmEpi& ep, int r, int c0, float* v) {
-  if (ep.bias) {
+__device__ __forceinline__ void red_add_v4(float* p, float a, float b, float c, float d) {
+  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(p), "f"(a), "f"(b), "f"(c),
+               "f"(d)
+               : "memory");
+}
+
+// Applies the epilogue to columns c0 .. c0+31 of output row r (r < M).  The
+// bias is added when with_bias (the gated residual adds it from split 0 only:
+// its update is a sum over splits).
+__device__ __forceinline__ void epilogue32(const GemmEpi& ep, int r, int c0, float* v,
+                                           bool with_bias) {
+  if (ep.bias && with_bias) {
     float b[32];
     load32(ep.bias + c0, b);
 #pragma unroll
@@ -200,6 +208,8 @@ __device__ __forceinline__ void epilogue32(const GemmEpi& ep, int r, int c0, flo
       store32_bf16(ep.out_bf + size_t(r) * ep.ld_out + c0, v);
       break;
     case EPI_GATE_RES: {
+      // x += gate (acc + b), as vector reductions: no read of x, and the
+      // partial sums of a split K add up in place
       if (ep.gate_tab) {
         float g[32];
         load32(ep.gate_tab + c0, g);
@@ -212,22 +222,9 @@ __device__ __forceinline__ void epilogue32(const GemmEpi& ep, int r, int c0, flo
 #pragma unroll
         for (int i = 0; i < 32; ++i) v[i] *= g[i];
       }
-      float4* xp = reinterpret_cast<float4*>(ep.xf + size_t(r) * ep.ld_xf + c0);
+      float* xp = ep.xf + size_t(r) * ep.ld_xf + c0;
 #pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        float4 x = xp[i];
-        x.x += v[4 * i]; x.y += v[4 * i + 1]; x.z += v[4 * i + 2]; x.w += v[4 * i + 3];
-        xp[i] = x;
-        v[4 * i] = x.x; v[4 * i + 1] = x.y; v[4 * i + 2] = x.z; v[4 * i + 3] = x.w;
-      }
-      if (ep.copy_bf) store32_bf16(ep.copy_bf + size_t(r) * ep.ld_copy + c0, v);
-      if (ep.scat) {
-        const int tok = ep.idx ? ep.idx[r] : r;
-        if (tok >= 0 && tok < ep.n_tokens)
-          store32_bf16(ep.scat + size_t(tok) * ep.ld_kv + c0, v);
-        else
-          atomicOr(ep.err, DEVERR_INDEX);
-      }
+      for (int i = 0; i < 8; ++i) red_add_v4(xp + 4 * i, v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
       break;
     }
     case EPI_QKV: {
@@ -391,24 +388,26 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       const int r = m * BM + row;
       const uint32_t tbase = tmem_base + uint32_t(acc * (TMEM_COLS / 2)) + (uint32_t(sp * 32) << 16);
       const int tile = nn * sc.mt + m;
-      float* part = ws + (size_t(tile) * sc.split + s) * (BM * BN) + size_t(row) * BN;
+      const bool additive = ep.mode == EPI_GATE_RES;
+      // split K, non-additive epilogue: partial sums reduce into a zeroed
+      // f32 tile; the last split reads it once, zeroes it and runs the epilogue
+      float* acc_row = ws + size_t(tile) * (BM * BN) + size_t(row) * BN;
 #pragma unroll 1
       for (int ch = 0; ch < BN / 32; ++ch) {
         float v[32];
         tmem_ld32(tbase + uint32_t(ch * 32), v);
-        if (sc.split == 1) {
-          if (r < M) epilogue32(ep, r, nn * BN + ch * 32, v);
+        if (sc.split == 1 || additive) {
+          if (r < M) epilogue32(ep, r, nn * BN + ch * 32, v, s == 0);
         } else {
-          float4* p4 = reinterpret_cast<float4*>(part + ch * 32);
 #pragma unroll
           for (int i = 0; i < 8; ++i)
-            __stcg(p4 + i, make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]));
+            red_add_v4(acc_row + ch * 32 + 4 * i, v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
         }
       }
       tc_fence_before();
       mbar_arrive(tempty0 + 8 * acc);
       if (++acc == 2) { acc = 0; acc_phase ^= 1; }
-      if (sc.split > 1) {
+      if (sc.split > 1 && !additive) {
         __threadfence();
         asm volatile("bar.sync 1, 128;" ::: "memory");
         if (et == 0) {
@@ -420,21 +419,21 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         asm volatile("bar.sync 1, 128;" ::: "memory");
         if (*last_flag) {
           __threadfence();
-          const float* base = ws + size_t(tile) * sc.split * (BM * BN) + size_t(row) * BN;
 #pragma unroll 1
-          for (int ch = 0; ch < BN / 32; ++ch) {
-            float v[32];
+          for (int ch = 0; ch < BN / 32; ch += 2) {
+            float v[64];
+            float4* p4 = reinterpret_cast<float4*>(acc_row + ch * 32);
 #pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = 0.f;
-            for (int q = 0; q < sc.split; ++q) {
-              const float4* p4 = reinterpret_cast<const float4*>(base + size_t(q) * (BM * BN) + ch * 32);
-#pragma unroll
-              for (int i = 0; i < 8; ++i) {
-                float4 a = __ldcg(p4 + i);
-                v[4 * i] += a.x; v[4 * i + 1] += a.y; v[4 * i + 2] += a.z; v[4 * i + 3] += a.w;
-              }
+            for (int i = 0; i < 16; ++i) {
+              const float4 a = __ldcg(p4 + i);
+              v[4 * i] = a.x; v[4 * i + 1] = a.y; v[4 * i + 2] = a.z; v[4 * i + 3] = a.w;
             }
-            if (r < M) epilogue32(ep, r, nn * BN + ch * 32, v);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) __stcg(p4 + i, make_float4(0.f, 0.f, 0.f, 0.f));
+            if (r < M) {
+              epilogue32(ep, r, nn * BN + ch * 32, v, true);
+              epilogue32(ep, r, nn * BN + ch * 32 + 32, v + 32, true);
+            }
           }
         }
         asm volatile("bar.sync 1, 128;" ::: "memory");
@@ -550,11 +549,6 @@ cudaError_t gemm_scratch_shape(int* units, int* max_tiles, size_t* ws_floats) {
 cudaError_t launch_gemm(const bf16* A, int lda, const bf16* W, int Mbound, const int* dcount,
                         int n, int k, const GemmEpi& ep, const GemmScratch& gs, cudaStream_t st) {
   if (Mbound <= 0) return cudaSuccess;
-  static const bool use_mma = [] {
-    const char* v = getenv("RC_GEMM_IMPL");
-    return v && v[0] == 'm';
-  }();
-  if (use_mma) return launch_gemm_mma(A, lda, W, Mbound, dcount, n, k, ep, st);
   if (n % 128 || k % BK) return cudaErrorInvalidValue;
   const int sms = device_sms();
   if (!sms) return cudaErrorInvalidDevice;

@@ -27,10 +27,16 @@ cudaError_t launch_localize(const float* A, int S, int N, int M, int gh, int gw,
 
 // --------------------------------------------------------------- row kernels
 // out[r] = bf16(LN(x[r]) * (1 + scale) + shift) for r < D; scale = tab_sc (+ tb_sc),
-// shift = tab_sh (+ tb_sh) (the tb_* terms may be null).
+// shift = tab_sh (+ tb_sh) (the tb_* terms may be null).  With hprev non-null
+// the row itself is also stored as bf16 to hprev[idx[r]] (the previous
+// block's merged hidden state, Section 3.3).
 cudaError_t launch_ln_mod(const float* x, int ldx, const float* tab_sh, const float* tb_sh,
                           const float* tab_sc, const float* tb_sc, bf16* out, int ldo,
-                          int Dbound, const int* dcount, int d, unsigned* err, cudaStream_t st);
+                          int Dbound, const int* dcount, int d, bf16* hprev, const int* idx,
+                          int n_tokens, unsigned* err, cudaStream_t st);
+// out[r] = bf16(x[r]) for r < D.
+cudaError_t launch_cast_rows(const float* x, int ldx, bf16* out, int ldo, int Dbound,
+                             const int* dcount, int d, unsigned* err, cudaStream_t st);
 
 // xf[r] = W_e patch(idx[r]) + b_e + pos[idx[r]]  (idx null: identity)
 cudaError_t launch_patch_embed(const float* latent, int gh, int gw, int p, int C,
@@ -71,9 +77,6 @@ struct GemmEpi {
   int ld_xf;
   const float* gate_tab;   // gate = gate_tab[c] (+ gate_tb[c]); null tab = no gate
   const float* gate_tb;
-  bf16* copy_bf;           // GATE_RES: optional bf16 copy of the new residual row r
-  int ld_copy;
-  bf16* scat;              // GATE_RES: optional bf16 copy to row idx[r] (cache H)
   bf16* kc;                // QKV: K rows idx[r] (cache)
   bf16* vc;                // QKV: V rows idx[r] (cache)
   int ld_kv;
@@ -83,8 +86,8 @@ struct GemmEpi {
   unsigned* err;
 };
 
-// Split-K scratch of one context: `units` partial 128x128 f32 tiles and
-// per-tile tickets (zero between launches).
+// Split-K scratch of one context: `units` f32 accumulator tiles (zero
+// between launches) and per-tile tickets (zero between launches).
 struct GemmScratch {
   float* ws;
   int* tickets;
@@ -100,8 +103,7 @@ cudaError_t gemm_scratch_shape(int* units, int* max_tiles, size_t* ws_floats);
 // GemmScratch must be stream-ordered.
 cudaError_t launch_gemm(const bf16* A, int lda, const bf16* W, int Mbound, const int* dcount,
                         int n, int k, const GemmEpi& ep, const GemmScratch& gs, cudaStream_t st);
-cudaError_t launch_gemm_mma(const bf16* A, int lda, const bf16* W, int Mbound, const int* dcount,
-                            int n, int k, const GemmEpi& ep, cudaStream_t st);
+
 
 // ----------------------------------------------------------------- attention
 constexpr int ATTN_MAX_SPLIT = 4;

@@ -181,19 +181,20 @@ struct Rows {
 // Region-Level Sparse Attention; Section 3.4, Kernel Fusing).  tab / tbv give
 // the modulation vector as tab (+ tbv), each [6][d] (tbv may be null).
 rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows& rw,
-                    const float* tab, const float* tbv, cudaStream_t st) {
+                    const float* tab, const float* tbv, bf16* hprev, cudaStream_t st) {
   const int d = c->d, F = c->F, N = c->N;
   const rc_layer_weights& w = c->lw[l];
   auto mv = [&](const float* base, int k) { return base ? base + size_t(k) * d : nullptr; };
   bf16* Kc = cache->slot(s, l, t, 1);
   bf16* Vc = cache->slot(s, l, t, 2);
-  bf16* Hc = cache->slot(s, l, t, 0);
   const bf16* tk = cache->text_kv(s, l);
   const bf16* tv = tk + d;
 
-  // x_hat = LN(x)(1 + scale_msa) + shift_msa
+  // x_hat = LN(x)(1 + scale_msa) + shift_msa; x itself is the previous
+  // block's output H^l of the dirty rows, written to their cache rows here
   RC_CUDA(rc::launch_ln_mod(c->xf, d, mv(tab, 0), mv(tbv, 0), mv(tab, 1), mv(tbv, 1), c->xb, d,
-                            rw.bound, rw.dcount, d, c->err, st), "ln_mod(msa)");
+                            rw.bound, rw.dcount, d, hprev, rw.idx, N, c->err, st),
+          "ln_mod(msa)");
   // [q | k | v] = x_hat W_qkv^T + b; k, v rows go straight to cache rows idx[r]
   rc::GemmEpi e{};
   e.mode = rc::EPI_QKV;
@@ -218,7 +219,7 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
     RC_CUDA(rc::launch_attention(c->q, d, Kc, Vc, d, N, c->ob, d, c->dims.heads, c->dh, rw.bound,
                                  rw.dcount, c->err, c->as, st), "attention(self)");
   }
-  // x += gate_msa (o W_o^T + b_o); bf16 copy of x for the cross-attention query
+  // x += gate_msa (o W_o^T + b_o)
   e = rc::GemmEpi{};
   e.mode = rc::EPI_GATE_RES;
   e.bias = w.b_o;
@@ -226,15 +227,14 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
   e.ld_xf = d;
   e.gate_tab = mv(tab, 2);
   e.gate_tb = mv(tbv, 2);
-  e.copy_bf = c->xb;
-  e.ld_copy = d;
   e.err = c->err;
   {
     Probe pr(c, RC_PROBE_GEMM, st);
     RC_CUDA(rc::launch_gemm(c->ob, d, static_cast<const bf16*>(w.W_o), rw.bound, rw.dcount, d, d, e,
                             c->gs, st), "gemm(out)");
   }
-  // q' = x W_xq^T + b
+  // q' = x W_xq^T + b (on a bf16 copy of x)
+  RC_CUDA(rc::launch_cast_rows(c->xf, d, c->xb, d, rw.bound, rw.dcount, d, c->err, st), "cast");
   e = rc::GemmEpi{};
   e.mode = rc::EPI_BIAS_BF16;
   e.bias = w.b_xq;
@@ -265,7 +265,8 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
   }
   // MLP
   RC_CUDA(rc::launch_ln_mod(c->xf, d, mv(tab, 3), mv(tbv, 3), mv(tab, 4), mv(tbv, 4), c->xb, d,
-                            rw.bound, rw.dcount, d, c->err, st), "ln_mod(mlp)");
+                            rw.bound, rw.dcount, d, nullptr, nullptr, N, c->err, st),
+          "ln_mod(mlp)");
   e = rc::GemmEpi{};
   e.mode = rc::EPI_GELU_BF16;
   e.bias = w.b_1;
@@ -277,7 +278,7 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
     RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_1), rw.bound, rw.dcount, F, d, e,
                             c->gs, st), "gemm(fc1)");
   }
-  // x += gate_mlp (u W_2^T + b_2); merged H^{l+1}: row idx[r] of the cache
+  // x += gate_mlp (u W_2^T + b_2); the caller stores x as the merged H^{l+1}
   e = rc::GemmEpi{};
   e.mode = rc::EPI_GATE_RES;
   e.bias = w.b_2;
@@ -285,10 +286,6 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
   e.ld_xf = d;
   e.gate_tab = mv(tab, 5);
   e.gate_tb = mv(tbv, 5);
-  e.scat = Hc;
-  e.ld_kv = d;
-  e.idx = rw.idx;
-  e.n_tokens = N;
   e.err = c->err;
   {
     Probe pr(c, RC_PROBE_GEMM, st);
@@ -380,6 +377,7 @@ rc_status rc_create(const rc_dims* dims, rc_ctx** out) {
       return s;
     }
     cudaMemset(c->gs.tickets, 0, sizeof(int) * size_t(max_tiles));
+    cudaMemset(c->gs.ws, 0, sizeof(float) * ws_floats);  // split-K accumulators start at zero
     const int nt = rc::attention_tickets(int(N), D.heads);
     if ((s = dalloc(&c->as.part, rc::attention_split_floats(int(N), D.heads, dh), "attn part")) ||
         (s = dalloc(&c->as.tickets, size_t(nt), "attn tickets"))) {
@@ -591,7 +589,9 @@ rc_status rc_block_forward_region(rc_ctx* c, rc_cache* k, int s, int l, int t, f
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   RC_CUDA(rc::launch_rows_f32(hidden, c->xf, rw.idx, rw.bound, rw.dcount, c->d, c->N, false,
                               c->err, st), "gather");
-  if ((r = run_block(c, k, s, l, t, rw, mod6, nullptr, st))) return r;
+  if ((r = run_block(c, k, s, l, t, rw, mod6, nullptr, nullptr, st))) return r;
+  RC_CUDA(rc::launch_scatter_bf16(c->xf, k->slot(s, l, t, 0), rw.idx, rw.bound, rw.dcount, c->d,
+                                  c->N, c->err, st), "H scatter");
   RC_CUDA(rc::launch_rows_f32(c->xf, hidden, rw.idx, rw.bound, rw.dcount, c->d, c->N, true,
                               c->err, st), "scatter");
   return RC_OK;
@@ -627,7 +627,11 @@ rc_status rc_step(rc_ctx* c, rc_cache* k, int s, float* latent, int t,
                                    rw.idx, rw.bound, rw.dcount, c->xf, d, c->err, st),
             "patch_embed");
     for (int l = 0; l < c->L; ++l)
-      if ((r = run_block(c, k, s, l, t, rw, c->lw[l].table, c->tb, st))) return r;
+      if ((r = run_block(c, k, s, l, t, rw, c->lw[l].table, c->tb,
+                         l > 0 ? k->slot(s, l - 1, t, 0) : nullptr, st)))
+        return r;
+    RC_CUDA(rc::launch_scatter_bf16(c->xf, k->slot(s, c->L - 1, t, 0), rw.idx, rw.bound,
+                                    rw.dcount, d, c->N, c->err, st), "H scatter");
   }
   RC_CUDA(rc::launch_final_ddim(k->slot(s, c->L - 1, t, 0), c->temb, g.table_f,
                                 static_cast<const bf16*>(g.W_f), g.b_f, latent, c->dims.grid_h,

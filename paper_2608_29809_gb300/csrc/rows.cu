@@ -185,7 +185,8 @@ __global__ void __launch_bounds__(LN_WARPS * 32)
 ln_mod_kernel(const float* __restrict__ x, int ldx, const float* __restrict__ tab_sh,
               const float* __restrict__ tb_sh, const float* __restrict__ tab_sc,
               const float* __restrict__ tb_sc, bf16* __restrict__ out, int ldo, int Dbound,
-              const int* __restrict__ dcount, int d, unsigned* err) {
+              const int* __restrict__ dcount, int d, bf16* __restrict__ hprev,
+              const int* __restrict__ idx, int n_tokens, unsigned* err) {
   const int D = live_count(dcount, Dbound, err);
   const int lane = threadIdx.x & 31;
   const int r = blockIdx.x * LN_WARPS + (threadIdx.x >> 5);
@@ -200,6 +201,18 @@ ln_mod_kernel(const float* __restrict__ x, int ldx, const float* __restrict__ ta
       v[k] = xr[lane + 32 * k];
       s += (v[k].x + v[k].y) + (v[k].z + v[k].w);
     }
+  if (hprev) {
+    const int tok = idx ? idx[r] : r;
+    if (tok >= 0 && tok < n_tokens) {
+      uint2* hrow = reinterpret_cast<uint2*>(hprev + size_t(tok) * d);
+#pragma unroll
+      for (int k = 0; k < LN_MAXV; ++k)
+        if (k < nv)
+          hrow[lane + 32 * k] = make_uint2(pack_bf16x2(v[k].x, v[k].y), pack_bf16x2(v[k].z, v[k].w));
+    } else if (lane == 0) {
+      atomicOr(err, DEVERR_INDEX);
+    }
+  }
   const float mean = warp_sum(s) / float(d);
   float q = 0.f;
 #pragma unroll
@@ -234,10 +247,36 @@ ln_mod_kernel(const float* __restrict__ x, int ldx, const float* __restrict__ ta
 
 cudaError_t launch_ln_mod(const float* x, int ldx, const float* tab_sh, const float* tb_sh,
                           const float* tab_sc, const float* tb_sc, bf16* out, int ldo,
-                          int Dbound, const int* dcount, int d, unsigned* err, cudaStream_t st) {
+                          int Dbound, const int* dcount, int d, bf16* hprev, const int* idx,
+                          int n_tokens, unsigned* err, cudaStream_t st) {
   if (Dbound <= 0) return cudaSuccess;
   ln_mod_kernel<<<cdiv(Dbound, LN_WARPS), LN_WARPS * 32, 0, st>>>(
-      x, ldx, tab_sh, tb_sh, tab_sc, tb_sc, out, ldo, Dbound, dcount, d, err);
+      x, ldx, tab_sh, tb_sh, tab_sc, tb_sc, out, ldo, Dbound, dcount, d, hprev, idx, n_tokens,
+      err);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+// out[r] = bf16(x[r]); one warp per row, 16-byte loads.
+__global__ void __launch_bounds__(LN_WARPS * 32)
+cast_rows_kernel(const float* __restrict__ x, int ldx, bf16* __restrict__ out, int ldo,
+                 int Dbound, const int* __restrict__ dcount, int d, unsigned* err) {
+  const int D = live_count(dcount, Dbound, err);
+  const int r = blockIdx.x * LN_WARPS + (threadIdx.x >> 5);
+  if (r >= D) return;
+  const float4* xr = reinterpret_cast<const float4*>(x + size_t(r) * ldx);
+  uint2* orow = reinterpret_cast<uint2*>(out + size_t(r) * ldo);
+  for (int c = threadIdx.x & 31; c < d / 4; c += 32) {
+    const float4 v = xr[c];
+    orow[c] = make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
+  }
+}
+
+cudaError_t launch_cast_rows(const float* x, int ldx, bf16* out, int ldo, int Dbound,
+                             const int* dcount, int d, unsigned* err, cudaStream_t st) {
+  if (Dbound <= 0) return cudaSuccess;
+  cast_rows_kernel<<<cdiv(Dbound, LN_WARPS), LN_WARPS * 32, 0, st>>>(x, ldx, out, ldo, Dbound,
+                                                                     dcount, d, err);
   count_launches(1);
   return cudaGetLastError();
 }
