@@ -96,6 +96,8 @@ attn_kernel(const bf16* __restrict__ Q, int ldq, const bf16* __restrict__ Kp,
   __shared__ __align__(128) bf16 sV[2][BKV * C::SROW];
   __shared__ int s_last;
 
+  pdl_wait();
+  pdl_trigger();
   const int D = live_count(dcount, Dbound, err);
   const int q0 = blockIdx.x * BQ;
   const int h = blockIdx.y;
@@ -360,16 +362,16 @@ cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* 
   if (nsplit < 1 || !as.part || (Dbound + BQ - 1) / BQ > as.max_qtiles) nsplit = 1;
   dim3 grid((Dbound + BQ - 1) / BQ, heads, nsplit);
   if (dh == 72) {
-    attn_kernel<72><<<grid, THREADS, 0, st>>>(Q, ldq, K, V, ldkv, Nk, O, ldo, Dbound, dcount,
-                                               scale_log2, err, as.part, as.tickets);
+    RC_TRY(launch_k(attn_kernel<72>, grid, dim3(THREADS), 0, st, Q, ldq, K, V, ldkv, Nk, O, ldo,
+                    Dbound, dcount, scale_log2, err, as.part, as.tickets));
   } else if (dh == 64) {
-    attn_kernel<64><<<grid, THREADS, 0, st>>>(Q, ldq, K, V, ldkv, Nk, O, ldo, Dbound, dcount,
-                                               scale_log2, err, as.part, as.tickets);
+    RC_TRY(launch_k(attn_kernel<64>, grid, dim3(THREADS), 0, st, Q, ldq, K, V, ldkv, Nk, O, ldo,
+                    Dbound, dcount, scale_log2, err, as.part, as.tickets));
   } else {
     return cudaErrorInvalidValue;
   }
   count_launches(1);
-  return cudaGetLastError();
+  return cudaSuccess;
 }
 
 }  // namespace rc

@@ -323,6 +323,10 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
+  // everything above is private set-up; inputs written by earlier kernels
+  // are read only after the predecessor has completed
+  pdl_wait();
+  pdl_trigger();
   const int M = live_count(dcount, Mbound, ep.err);
   Sched<BN> sc;
   sc.init(M, n, k, min(int(gridDim.x), ws_units));
@@ -560,13 +564,13 @@ cudaError_t launch_gemm(const bf16* A, int lda, const bf16* W, int Mbound, const
   // split-K only runs when the tiles do not fill the grid; its tickets cover them
   const int units = min(gs.units, gs.max_tiles);
   if (BN == 192)
-    gemm_tc_kernel<192><<<sms, THREADS, TileCfg<192>::SMEM_BYTES, st>>>(
-        ta, tb, Mbound, dcount, n, k, ep, gs.ws, gs.tickets, units);
+    RC_TRY(launch_k(gemm_tc_kernel<192>, dim3(sms), dim3(THREADS), TileCfg<192>::SMEM_BYTES, st, ta,
+                    tb, Mbound, dcount, n, k, ep, gs.ws, gs.tickets, units));
   else
-    gemm_tc_kernel<128><<<sms, THREADS, TileCfg<128>::SMEM_BYTES, st>>>(
-        ta, tb, Mbound, dcount, n, k, ep, gs.ws, gs.tickets, units);
+    RC_TRY(launch_k(gemm_tc_kernel<128>, dim3(sms), dim3(THREADS), TileCfg<128>::SMEM_BYTES, st, ta,
+                    tb, Mbound, dcount, n, k, ep, gs.ws, gs.tickets, units));
   count_launches(1);
-  return cudaGetLastError();
+  return cudaSuccess;
 }
 
 }  // namespace rc

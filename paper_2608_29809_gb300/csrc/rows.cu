@@ -52,6 +52,8 @@ static MaskWs carve(void* ws, int N, int n_delta) {
 __global__ void __launch_bounds__(MASK_ROWS)
 mask_colstats_kernel(const float* __restrict__ A, int S, int N, int M, DeltaIds ids,
                      float* __restrict__ abar, float2* __restrict__ part) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float smin[MASK_ROWS / 32], smax[MASK_ROWS / 32];
   const int i = blockIdx.x * MASK_ROWS + threadIdx.x;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -86,6 +88,8 @@ mask_colstats_kernel(const float* __restrict__ A, int S, int N, int M, DeltaIds 
 __global__ void __launch_bounds__(MASK_ROWS)
 mask_threshold_kernel(const float* __restrict__ abar, const float2* __restrict__ part, int nblk,
                       int N, DeltaIds ids, float tau, uint8_t* __restrict__ uni) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float s_mn[64], s_rng[64];
   __shared__ int s_ok[64];
   if (threadIdx.x < ids.n) {
@@ -117,6 +121,8 @@ mask_threshold_kernel(const float* __restrict__ abar, const float2* __restrict__
 __global__ void __launch_bounds__(MASK_ROWS)
 mask_dilate_kernel(const uint8_t* __restrict__ uni, int gh, int gw, int r,
                    uint8_t* __restrict__ mask, int* __restrict__ cnt) {
+  pdl_wait();
+  pdl_trigger();
   const int N = gh * gw;
   const int i = blockIdx.x * MASK_ROWS + threadIdx.x;
   int m = 0;
@@ -139,6 +145,8 @@ mask_dilate_kernel(const uint8_t* __restrict__ uni, int gh, int gw, int r,
 __global__ void __launch_bounds__(MASK_ROWS)
 mask_compact_kernel(const uint8_t* __restrict__ mask, const int* __restrict__ cnt, int N,
                     int32_t* __restrict__ idx, int32_t* __restrict__ count) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ int s_warp[MASK_ROWS / 32];
   __shared__ int s_base;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -168,12 +176,16 @@ cudaError_t launch_localize(const float* A, int S, int N, int M, int gh, int gw,
                             int32_t* idx, int32_t* count, void* ws, cudaStream_t st) {
   const int nblk = cdiv(N, MASK_ROWS);
   MaskWs w = carve(ws, N, ids.n);
-  mask_colstats_kernel<<<nblk, MASK_ROWS, 0, st>>>(A, S, N, M, ids, w.abar, w.part);
-  mask_threshold_kernel<<<nblk, MASK_ROWS, 0, st>>>(w.abar, w.part, nblk, N, ids, tau, w.uni);
-  mask_dilate_kernel<<<nblk, MASK_ROWS, 0, st>>>(w.uni, gh, gw, dilation, mask, w.cnt);
-  mask_compact_kernel<<<nblk, MASK_ROWS, 0, st>>>(mask, w.cnt, N, idx, count);
+  RC_TRY(launch_k(mask_colstats_kernel, dim3(nblk), dim3(MASK_ROWS), 0, st, A, S, N, M, ids,
+                  w.abar, w.part));
+  RC_TRY(launch_k(mask_threshold_kernel, dim3(nblk), dim3(MASK_ROWS), 0, st, w.abar, w.part, nblk,
+                  N, ids, tau, w.uni));
+  RC_TRY(launch_k(mask_dilate_kernel, dim3(nblk), dim3(MASK_ROWS), 0, st, w.uni, gh, gw, dilation,
+                  mask, w.cnt));
+  RC_TRY(launch_k(mask_compact_kernel, dim3(nblk), dim3(MASK_ROWS), 0, st, mask, w.cnt, N, idx,
+                  count));
   count_launches(4);
-  return cudaGetLastError();
+  return cudaSuccess;
 }
 
 // ================================================================= LN + mod
@@ -187,6 +199,8 @@ ln_mod_kernel(const float* __restrict__ x, int ldx, const float* __restrict__ ta
               const float* __restrict__ tb_sc, bf16* __restrict__ out, int ldo, int Dbound,
               const int* __restrict__ dcount, int d, bf16* __restrict__ hprev,
               const int* __restrict__ idx, int n_tokens, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   const int D = live_count(dcount, Dbound, err);
   const int lane = threadIdx.x & 31;
   const int r = blockIdx.x * LN_WARPS + (threadIdx.x >> 5);
@@ -250,17 +264,19 @@ cudaError_t launch_ln_mod(const float* x, int ldx, const float* tab_sh, const fl
                           int Dbound, const int* dcount, int d, bf16* hprev, const int* idx,
                           int n_tokens, unsigned* err, cudaStream_t st) {
   if (Dbound <= 0) return cudaSuccess;
-  ln_mod_kernel<<<cdiv(Dbound, LN_WARPS), LN_WARPS * 32, 0, st>>>(
-      x, ldx, tab_sh, tb_sh, tab_sc, tb_sc, out, ldo, Dbound, dcount, d, hprev, idx, n_tokens,
-      err);
+  RC_TRY(launch_k(ln_mod_kernel, dim3(cdiv(Dbound, LN_WARPS)), dim3(LN_WARPS * 32), 0, st, x, ldx,
+                  tab_sh, tb_sh, tab_sc, tb_sc, out, ldo, Dbound, dcount, d, hprev, idx, n_tokens,
+                  err));
   count_launches(1);
-  return cudaGetLastError();
+  return cudaSuccess;
 }
 
 // out[r] = bf16(x[r]); one warp per row, 16-byte loads.
 __global__ void __launch_bounds__(LN_WARPS * 32)
 cast_rows_kernel(const float* __restrict__ x, int ldx, bf16* __restrict__ out, int ldo,
                  int Dbound, const int* __restrict__ dcount, int d, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   const int D = live_count(dcount, Dbound, err);
   const int r = blockIdx.x * LN_WARPS + (threadIdx.x >> 5);
   if (r >= D) return;
@@ -275,10 +291,10 @@ cast_rows_kernel(const float* __restrict__ x, int ldx, bf16* __restrict__ out, i
 cudaError_t launch_cast_rows(const float* x, int ldx, bf16* out, int ldo, int Dbound,
                              const int* dcount, int d, unsigned* err, cudaStream_t st) {
   if (Dbound <= 0) return cudaSuccess;
-  cast_rows_kernel<<<cdiv(Dbound, LN_WARPS), LN_WARPS * 32, 0, st>>>(x, ldx, out, ldo, Dbound,
-                                                                     dcount, d, err);
+  RC_TRY(launch_k(cast_rows_kernel, dim3(cdiv(Dbound, LN_WARPS)), dim3(LN_WARPS * 32), 0, st, x,
+                  ldx, out, ldo, Dbound, dcount, d, err));
   count_launches(1);
-  return cudaGetLastError();
+  return cudaSuccess;
 }
 
 // ============================================================ patch embed
@@ -289,6 +305,8 @@ patch_embed_kernel(const float* __restrict__ latent, int gh, int gw, int p, int 
                    const bf16* __restrict__ We, const float* __restrict__ be,
                    const float* __restrict__ pos, const int* __restrict__ idx, int Dbound,
                    const int* __restrict__ dcount, float* __restrict__ xf, int d, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ float patch[64];
   const int D = live_count(dcount, Dbound, err);
   const int r = blockIdx.x;
@@ -321,16 +339,18 @@ cudaError_t launch_patch_embed(const float* latent, int gh, int gw, int p, int C
                                const int* idx, int Dbound, const int* dcount, float* xf, int d,
                                unsigned* err, cudaStream_t st) {
   if (Dbound <= 0) return cudaSuccess;
-  patch_embed_kernel<<<Dbound, 256, 0, st>>>(latent, gh, gw, p, C, We, be, pos, idx, Dbound,
-                                             dcount, xf, d, err);
+  RC_TRY(launch_k(patch_embed_kernel, dim3(Dbound), dim3(256), 0, st, latent, gh, gw, p, C, We, be,
+                  pos, idx, Dbound, dcount, xf, d, err));
   count_launches(1);
-  return cudaGetLastError();
+  return cudaSuccess;
 }
 
 // ======================================================== timestep embed
 // f[k] = cos(t w_k), f[half + k] = sin(t w_k), w_k = 10000^(-k/half); double
 // precision for the argument so large timesteps keep their phase.
 __global__ void sinusoid_kernel(float t, int dim, float* f) {
+  pdl_wait();
+  pdl_trigger();
   const int half = dim / 2;
   for (int k = threadIdx.x; k < half; k += blockDim.x) {
     double w = exp(-log(10000.0) * double(k) / double(half));
@@ -346,6 +366,8 @@ __global__ void __launch_bounds__(256)
 matvec_kernel(const bf16* __restrict__ W, const float* __restrict__ b,
               const float* __restrict__ in, float* __restrict__ out, int in_dim, int out_dim,
               int silu_in) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ float s_in[];
   for (int k = threadIdx.x; k < in_dim; k += blockDim.x) {
     float v = in[k];
@@ -377,13 +399,15 @@ matvec_kernel(const bf16* __restrict__ W, const float* __restrict__ b,
 cudaError_t launch_t_embed(float t_value, int freq_dim, int d, const bf16* Wt1, const float* bt1,
                            const bf16* Wt2, const float* bt2, const bf16* Wtb, const float* btb,
                            float* fbuf, float* h1, float* temb, float* tb, cudaStream_t st) {
-  sinusoid_kernel<<<1, 128, 0, st>>>(t_value, freq_dim, fbuf);
-  matvec_kernel<<<cdiv(d, 8), 256, freq_dim * sizeof(float), st>>>(Wt1, bt1, fbuf, h1, freq_dim,
-                                                                    d, 0);
-  matvec_kernel<<<cdiv(d, 8), 256, d * sizeof(float), st>>>(Wt2, bt2, h1, temb, d, d, 1);
-  matvec_kernel<<<cdiv(6 * d, 8), 256, d * sizeof(float), st>>>(Wtb, btb, temb, tb, d, 6 * d, 1);
+  RC_TRY(launch_k(sinusoid_kernel, dim3(1), dim3(128), 0, st, t_value, freq_dim, fbuf));
+  RC_TRY(launch_k(matvec_kernel, dim3(cdiv(d, 8)), dim3(256), freq_dim * sizeof(float), st, Wt1,
+                  bt1, fbuf, h1, freq_dim, d, 0));
+  RC_TRY(launch_k(matvec_kernel, dim3(cdiv(d, 8)), dim3(256), d * sizeof(float), st, Wt2, bt2, h1,
+                  temb, d, d, 1));
+  RC_TRY(launch_k(matvec_kernel, dim3(cdiv(6 * d, 8)), dim3(256), d * sizeof(float), st, Wtb, btb,
+                  temb, tb, d, 6 * d, 1));
   count_launches(4);
-  return cudaGetLastError();
+  return cudaSuccess;
 }
 
 // ===================================================== final layer + DDIM
@@ -400,6 +424,8 @@ final_ddim_kernel(const bf16* __restrict__ H, const float* __restrict__ temb,
                   const float* __restrict__ table_f, const bf16* __restrict__ Wf,
                   const float* __restrict__ bfin, float* __restrict__ latent, int gh, int gw,
                   int p, int c_in, int c_out, int d, float ab_t, float ab_next) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ uint8_t smem_raw[];
   float* s_shift = reinterpret_cast<float*>(smem_raw);
   float* s_scale = s_shift + d;
@@ -505,10 +531,10 @@ cudaError_t launch_final_ddim(const bf16* H, const float* temb, const float* tab
   const int N = gh * gw;
   int grid = cdiv(N, FIN_WARPS * 4);
   if (grid > 1024) grid = 1024;
-  final_ddim_kernel<<<grid, FIN_WARPS * 32, smem, st>>>(H, temb, table_f, Wf, bf, latent, gh, gw,
-                                                        p, c_in, c_out, d, ab_t, ab_next);
+  RC_TRY(launch_k(final_ddim_kernel, dim3(grid), dim3(FIN_WARPS * 32), smem, st, H, temb, table_f,
+                  Wf, bf, latent, gh, gw, p, c_in, c_out, d, ab_t, ab_next));
   count_launches(1);
-  return cudaGetLastError();
+  return cudaSuccess;
 }
 
 // ======================================================= gather / scatter
@@ -516,6 +542,8 @@ __global__ void __launch_bounds__(256)
 rows_f32_kernel(const float* __restrict__ src, float* __restrict__ dst,
                 const int* __restrict__ idx, int Dbound, const int* __restrict__ dcount, int d,
                 int N, int scatter, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   const int D = live_count(dcount, Dbound, err);
   const int r = blockIdx.x;
   if (r >= D) return;
@@ -533,6 +561,8 @@ __global__ void __launch_bounds__(256)
 scatter_bf16_kernel(const float* __restrict__ src, bf16* __restrict__ dst,
                     const int* __restrict__ idx, int Dbound, const int* __restrict__ dcount,
                     int d, int N, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
   const int D = live_count(dcount, Dbound, err);
   const int r = blockIdx.x;
   if (r >= D) return;
@@ -553,18 +583,19 @@ cudaError_t launch_rows_f32(const float* src, float* dst, const int* idx, int Db
                             const int* dcount, int d, int N, bool scatter, unsigned* err,
                             cudaStream_t st) {
   if (Dbound <= 0) return cudaSuccess;
-  rows_f32_kernel<<<Dbound, 256, 0, st>>>(src, dst, idx, Dbound, dcount, d, N, scatter ? 1 : 0,
-                                          err);
+  RC_TRY(launch_k(rows_f32_kernel, dim3(Dbound), dim3(256), 0, st, src, dst, idx, Dbound, dcount,
+                  d, N, scatter ? 1 : 0, err));
   count_launches(1);
-  return cudaGetLastError();
+  return cudaSuccess;
 }
 
 cudaError_t launch_scatter_bf16(const float* src, bf16* dst, const int* idx, int Dbound,
                                 const int* dcount, int d, int N, unsigned* err, cudaStream_t st) {
   if (Dbound <= 0) return cudaSuccess;
-  scatter_bf16_kernel<<<Dbound, 256, 0, st>>>(src, dst, idx, Dbound, dcount, d, N, err);
+  RC_TRY(launch_k(scatter_bf16_kernel, dim3(Dbound), dim3(256), 0, st, src, dst, idx, Dbound,
+                  dcount, d, N, err));
   count_launches(1);
-  return cudaGetLastError();
+  return cudaSuccess;
 }
 
 }  // namespace rc
