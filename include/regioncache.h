@@ -265,6 +265,16 @@ rc_status rc_step_dense(rc_ctx* ctx, rc_cache* cache, int session, float* latent
 rc_status rc_linear(rc_ctx* ctx, const void* x, const void* W, const float* b, float* y,
                     int rows, int n, int k, rc_stream stream);
 
+/* The dirty-query attention of the block on its own (Section 3.3,
+ * Region-Level Sparse Attention): for each of the context's heads h,
+ * O[r][h*dh..] = softmax(Q_r,h K_h^T / sqrt(dh)) V_h over the Nk keys.
+ *   Q bf16 [Nq][ldq], K and V bf16 [Nk][ldkv] (head h in columns h*dh ..
+ *   h*dh+dh-1), O bf16 [Nq][ldo].  ldq, ldkv, ldo multiples of 8, >= heads*dh;
+ *   pointers 16-byte aligned; Nq, Nk >= 0.
+ * Provided so the attention kernel can be checked and timed in isolation. */
+rc_status rc_attention(rc_ctx* ctx, const void* Q, int ldq, const void* K, const void* V,
+                       int ldkv, int Nq, int Nk, void* O, int ldo, rc_stream stream);
+
 /* Waits for `stream`, then reports (and clears) the context's device error
  * word: RC_ERR_DEVICE_ASSERT if a kernel met a bad index or count,
  * RC_ERR_TIMEOUT if a bounded wait gave up, RC_ERR_CUDA on a CUDA error. */

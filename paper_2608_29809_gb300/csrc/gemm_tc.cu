@@ -10,8 +10,9 @@
 // the tile list and, when the tiles cannot fill the grid, a split of K.  The
 // gated residual (x += gate (C + b)) is written as vector reductions into x,
 // so the splits of K simply add up; for the other epilogues the splits reduce
-// into a zeroed f32 tile and the last split to arrive (an atomic ticket, no
-// waiting) reads it once, zeroes it and applies the epilogue.
+// into a zeroed f32 tile and, row by row, the last split to arrive (an atomic
+// ticket per row, no waiting) reads the row once, zeroes it and applies the
+// epilogue.
 //
 // CTA = 6 warps: warp 0 issues TMA loads, warp 1 owns TMEM and issues the
 // MMAs (one thread), warps 2..5 drain the accumulator (one TMEM lane = one
@@ -26,10 +27,13 @@
 
 #include "common.cuh"
 #include "kernels.h"
+#include "tc_common.cuh"
 
 namespace rc {
 
 namespace {
+
+using namespace rc::tc;
 
 constexpr int BM = 128, BK = 64;
 constexpr int THREADS = 192;
@@ -37,7 +41,6 @@ constexpr int STAGE_A = BM * BK * 2;   // bytes
 constexpr int MAX_SPLIT = 4;
 constexpr int MIN_KB_PER_SPLIT = 4;
 constexpr int MAX_BN = 192;
-constexpr unsigned long long WAIT_NS = 2000000000ull;  // bounded waits: 2 s
 
 // Tile width BN (output features per tile): 192 when it divides n (every
 // PixArt-alpha width: 1152, 2304, 3456, 4608), else 128.
@@ -52,108 +55,6 @@ struct TileCfg {
   static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
                                     (uint32_t(BN >> 3) << 17) | (uint32_t(BM >> 4) << 24);
 };
-
-// ---------------------------------------------------------------- PTX glue
-__device__ __forceinline__ uint32_t saddr(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-__device__ __forceinline__ unsigned long long globaltimer() {
-  unsigned long long t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-// Waits for the phase of parity `parity`; gives up (returns false) when the
-// CTA's abort flag is raised or after WAIT_NS.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const unsigned long long t0 = globaltimer();
-  while (true) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if (*abort_flag) return false;
-    if (globaltimer() - t0 > WAIT_NS) return false;
-  }
-}
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
-                                            int x, int y) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y)
-      : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() {
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
-                                          uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-__device__ __forceinline__ void umma_commit(uint32_t bar) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
-      : "memory");
-}
-// 32 consecutive f32 columns of this thread's TMEM lane.
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
-  uint32_t r[32];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
-        "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
-        "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
-        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
-        "=r"(r[31])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-}
-
-// Shared-memory matrix descriptor of a K-major bf16 tile written by TMA with
-// the 128-byte swizzle: rows of 128 B, 8-row groups 1024 B apart (stride byte
-// offset), descriptor version 1, layout SWIZZLE_128B.
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t addr) {
-  uint64_t d = 0;
-  d |= uint64_t((addr & 0x3FFFFu) >> 4);
-  d |= uint64_t(16 >> 4) << 16;
-  d |= uint64_t(1024 >> 4) << 32;
-  d |= uint64_t(1) << 46;
-  d |= uint64_t(2) << 61;
-  return d;
-}
-
 
 // ---------------------------------------------------------------- epilogue
 __device__ __forceinline__ void load32(const float* p, float* v) {
@@ -289,7 +190,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   // bars: full[STAGES], empty[STAGES], tfull[2], tempty[2]
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 4);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  int* last_flag = reinterpret_cast<int*>(tmem_slot + 2);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t full0 = saddr(bars), empty0 = saddr(bars + STAGES);
@@ -379,14 +279,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   } else {
     // ------------------------------------------------------- epilogue (warps 2..5)
     const int sp = warp & 3;  // TMEM lane sub-partition this warp may access
-    const int et = threadIdx.x - 64;
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int u = blockIdx.x; u < sc.units; u += gridDim.x) {
       int m, nn, s, kb0, kb1;
       sc.decode(u, m, nn, s, kb0, kb1);
-      if (!mbar_wait(tfull0 + 8 * acc, acc_phase, abort_flag)) goto timeout;
-      __syncwarp();
+      if (!mbar_wait_warp(tfull0 + 8 * acc, acc_phase, abort_flag)) goto timeout;
       tc_fence_after();
       const int row = sp * 32 + lane;
       const int r = m * BM + row;
@@ -412,16 +310,13 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       mbar_arrive(tempty0 + 8 * acc);
       if (++acc == 2) { acc = 0; acc_phase ^= 1; }
       if (sc.split > 1 && !additive) {
+        // per-row ticket: the last split to finish a row reduces it (no
+        // cross-warp barrier, no waiting)
         __threadfence();
-        asm volatile("bar.sync 1, 128;" ::: "memory");
-        if (et == 0) {
-          const int prev = atomicAdd(tickets + tile, 1);
-          const int last = (prev == sc.split - 1);
-          if (last) tickets[tile] = 0;  // re-armed for the next launch
-          *last_flag = last;
-        }
-        asm volatile("bar.sync 1, 128;" ::: "memory");
-        if (*last_flag) {
+        int* tk = tickets + size_t(tile) * BM + row;
+        const bool last = atomicAdd(tk, 1) == sc.split - 1;
+        if (last) {
+          *tk = 0;  // re-armed for the next launch
           __threadfence();
 #pragma unroll 1
           for (int ch = 0; ch < BN / 32; ch += 2) {
@@ -440,7 +335,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             }
           }
         }
-        asm volatile("bar.sync 1, 128;" ::: "memory");
       }
     }
   }
@@ -537,7 +431,7 @@ int device_sms() {
   return sms[dev];
 }
 
-constexpr int MAX_TILES = 4096;
+constexpr int MAX_TILES = 4096;  // tickets: MAX_TILES x BM rows
 
 }  // namespace
 
@@ -545,7 +439,7 @@ cudaError_t gemm_scratch_shape(int* units, int* max_tiles, size_t* ws_floats) {
   const int sms = device_sms();
   if (!sms) return cudaErrorInvalidDevice;
   *units = sms;
-  *max_tiles = MAX_TILES;
+  *max_tiles = MAX_TILES;  // the context allocates MAX_TILES * 128 row tickets
   *ws_floats = size_t(sms) * BM * MAX_BN;
   return cudaSuccess;
 }

@@ -106,13 +106,12 @@ cudaError_t launch_gemm(const bf16* A, int lda, const bf16* W, int Mbound, const
 
 
 // ----------------------------------------------------------------- attention
-constexpr int ATTN_MAX_SPLIT = 4;
 // Key-split scratch of one context: partial outputs and per-(query tile,
 // head) tickets (zero between launches).
 struct AttnScratch {
   float* part;
+  size_t part_floats;
   int* tickets;
-  int max_qtiles;
 };
 size_t attention_split_floats(int Nmax, int heads, int dh);
 int attention_tickets(int Nmax, int heads);

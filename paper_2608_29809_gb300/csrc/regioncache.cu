@@ -372,20 +372,20 @@ rc_status rc_create(const rc_dims* dims, rc_ctx** out) {
     c->gs.units = units;
     c->gs.max_tiles = max_tiles;
     if ((s = dalloc(&c->gs.ws, ws_floats, "gemm split-K partials")) ||
-        (s = dalloc(&c->gs.tickets, size_t(max_tiles), "gemm tickets"))) {
+        (s = dalloc(&c->gs.tickets, size_t(max_tiles) * 128, "gemm tickets"))) {
       free_ctx(c);
       return s;
     }
-    cudaMemset(c->gs.tickets, 0, sizeof(int) * size_t(max_tiles));
+    cudaMemset(c->gs.tickets, 0, sizeof(int) * size_t(max_tiles) * 128);
     cudaMemset(c->gs.ws, 0, sizeof(float) * ws_floats);  // split-K accumulators start at zero
     const int nt = rc::attention_tickets(int(N), D.heads);
-    if ((s = dalloc(&c->as.part, rc::attention_split_floats(int(N), D.heads, dh), "attn part")) ||
-        (s = dalloc(&c->as.tickets, size_t(nt), "attn tickets"))) {
+    c->as.part_floats = rc::attention_split_floats(int(N), D.heads, dh);
+    if ((s = dalloc(&c->as.part, c->as.part_floats, "attn part")) ||
+        (s = dalloc(&c->as.tickets, size_t(nt) * 128, "attn tickets"))) {
       free_ctx(c);
       return s;
     }
-    cudaMemset(c->as.tickets, 0, sizeof(int) * size_t(nt));
-    c->as.max_qtiles = int((N + 63) / 64);
+    cudaMemset(c->as.tickets, 0, sizeof(int) * size_t(nt) * 128);
   }
   iota_kernel<<<int((N + 255) / 256), 256>>>(c->iota, int(N));
   rc::count_launches(1);
@@ -663,6 +663,27 @@ rc_status rc_linear(rc_ctx* c, const void* x, const void* W, const float* b, flo
   RC_CUDA(rc::launch_gemm(static_cast<const bf16*>(x), kdim, static_cast<const bf16*>(W), rows,
                           nullptr, n, kdim, e, c->gs, static_cast<cudaStream_t>(stream)),
           "gemm(linear)");
+  return RC_OK;
+}
+
+rc_status rc_attention(rc_ctx* c, const void* Q, int ldq, const void* K, const void* V, int ldkv,
+                       int Nq, int Nk, void* O, int ldo, rc_stream stream) {
+  if (!c || !Q || !K || !V || !O) return fail(RC_ERR_INVALID_ARG, "rc_attention: null argument");
+  const int hd = c->dims.heads * c->dh;
+  if (Nq < 0 || Nk < 0 || ldq < hd || ldkv < hd || ldo < hd || ldq % 8 || ldkv % 8 || ldo % 8)
+    return fail(RC_ERR_SHAPE, "rc_attention: Nq %d Nk %d ldq %d ldkv %d ldo %d", Nq, Nk, ldq,
+                ldkv, ldo);
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O))
+    return fail(RC_ERR_INVALID_ARG, "rc_attention: pointers must be 16-B aligned");
+  if (Nq == 0) return RC_OK;
+  if (Nk == 0) return fail(RC_ERR_SHAPE, "rc_attention: Nk = 0 with queries");
+  if ((Nq + 127) / 128 > (c->N + 127) / 128)
+    return fail(RC_ERR_SHAPE, "rc_attention: Nq %d above the context's %d tokens", Nq, c->N);
+  RC_CUDA(rc::launch_attention(static_cast<const bf16*>(Q), ldq, static_cast<const bf16*>(K),
+                               static_cast<const bf16*>(V), ldkv, Nk, static_cast<bf16*>(O), ldo,
+                               c->dims.heads, c->dh, Nq, nullptr, c->err, c->as,
+                               static_cast<cudaStream_t>(stream)),
+          "attention");
   return RC_OK;
 }
 

@@ -75,6 +75,7 @@ def load_library(path: str = LIB_PATH) -> C.CDLL:
         "rc_step": (I, [P, P, I, P, I, P, P, I, P, P]),
         "rc_step_dense": (I, [P, P, I, P, I, P]),
         "rc_linear": (I, [P, P, P, P, P, I, I, I, P]),
+        "rc_attention": (I, [P, P, I, P, P, I, I, I, P, I, P]),
         "rc_sync": (I, [P, P]),
         "rc_probe_enable": (I, [P, I, I]),
         "rc_probe_read": (I, [P, C.POINTER(C.c_double), C.POINTER(I)]),
@@ -209,6 +210,11 @@ def rc_step_dense(ctx, cache, session, latent, t, stream=None):
 
 def rc_linear(ctx, x, W, b, y, rows, n, k, stream=None):
     _check(_lib.rc_linear(ctx, _ptr(x), _ptr(W), _ptr(b), _ptr(y), rows, n, k, _stream(stream)))
+
+
+def rc_attention(ctx, Q, ldq, K, V, ldkv, Nq, Nk, O, ldo, stream=None):
+    _check(_lib.rc_attention(ctx, _ptr(Q), ldq, _ptr(K), _ptr(V), ldkv, Nq, Nk, _ptr(O), ldo,
+                             _stream(stream)))
 
 
 def rc_sync(ctx, stream=None):

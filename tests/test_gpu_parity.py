@@ -110,6 +110,29 @@ def test_linear_matches_fp64(R, rows, n, k):
     assert np.max(np.abs(got - ref)) <= 1e-4 * (1 + np.max(np.abs(ref)))
 
 
+# --------------------------------------------------------------- attention
+@pytest.mark.parametrize("Nq,Nk,ld_kv", [(1, 120, 2304), (37, 256, 1152), (200, 1024, 1152),
+                                         (831, 4096, 1152), (128, 120, 2304), (300, 4096, 1152)])
+def test_attention_matches_fp64(R, Nq, Nk, ld_kv):
+    d = synth.PIXART_1024
+    g = torch.Generator().manual_seed(Nq * 31 + Nk)
+    h = d.hidden
+    Q = torch.randn(Nq, h, generator=g).to(torch.bfloat16)
+    KV = (torch.randn(Nk, ld_kv, generator=g) * 1.5).to(torch.bfloat16)
+    Vsrc = torch.randn(Nk, ld_kv, generator=g).to(torch.bfloat16)
+    ctx = R.rc_create(R.dims_struct(d))
+    try:
+        out = torch.full((Nq, h), float("nan"), dtype=torch.bfloat16, device="cuda")
+        Kd, Vd = KV.cuda(), Vsrc.cuda()
+        R.rc_attention(ctx, Q.cuda(), h, Kd, Vd, ld_kv, Nq, Nk, out, h)
+        R.rc_sync(ctx)
+    finally:
+        R.rc_destroy(ctx)
+    got = out.cpu().double().numpy()
+    want = O.multihead_attention(O.to64(Q), O.to64(KV[:, :h]), O.to64(Vsrc[:, :h]), d.heads)
+    block_close(got, want, f"attention Nq={Nq} Nk={Nk}")
+
+
 # ------------------------------------------------------------- one block
 @pytest.fixture(scope="module")
 def block_problem(R):
