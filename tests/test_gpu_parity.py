@@ -130,7 +130,16 @@ def test_attention_matches_fp64(R, Nq, Nk, ld_kv):
         R.rc_destroy(ctx)
     got = out.cpu().double().numpy()
     want = O.multihead_attention(O.to64(Q), O.to64(KV[:, :h]), O.to64(Vsrc[:, :h]), d.heads)
-    block_close(got, want, f"attention Nq={Nq} Nk={Nk}")
+    # Raw attention outputs, not block outputs: P and O are bf16, so each
+    # element carries ~2^-9 of its own size in rounding while the output RMS
+    # shrinks like 1/sqrt(effective keys).  Bound: relative L2 <= 1e-2,
+    # max |err| <= 8e-2 x RMS, cosine >= 0.9999.
+    err = got - want
+    rms = np.sqrt(np.mean(want ** 2))
+    assert np.linalg.norm(err) <= 1e-2 * np.linalg.norm(want), f"Nq={Nq} Nk={Nk} rel L2"
+    assert np.max(np.abs(err)) <= 8e-2 * rms, f"Nq={Nq} Nk={Nk}: {np.max(np.abs(err)):.2e}"
+    cos = float((got * want).sum() / (np.linalg.norm(got) * np.linalg.norm(want)))
+    assert cos >= 0.9999, cos
 
 
 # ------------------------------------------------------------- one block
