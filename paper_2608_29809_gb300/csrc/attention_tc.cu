@@ -6,19 +6,22 @@
 //
 // One work unit = 128 queries of one head over one split of the keys.  CTAs
 // are persistent (one per SM) and warp-specialised:
-//   warp 0     TMA: Q once per unit, then K/V blocks of 128 keys (3 stages).
-//              Every operand is loaded as 16-wide head-dim blocks through a
-//              3-D tensor map (head_dim, head, row) whose head_dim extent is
-//              the true 72: the pad to 80 reads as zero, so the padded
-//              columns add nothing to Q K^T.
-//   warp 1     TMEM owner and MMA issuer: S = Q K^T (M=128, N=128, 5 K-steps
-//              of 16) into one of two TMEM S buffers, one block ahead of
-//              O += P V (M=128, N=80, K=128; V is an MN-major operand).
+//   warp 0     TMA: Q once per unit, then K/V blocks of 64 keys (3 stages).
+//              Every operand comes through 3-D tensor maps (head_dim, head,
+//              row) as a 64-wide 128B-swizzled tile plus a 16-wide 32B-
+//              swizzled tail; the head_dim extent is the true 72, so the pad
+//              to 80 reads as zero and adds nothing to Q K^T.
+//   warp 1     TMEM owner and MMA issuer: S = Q K^T (M=128, N=64, 5 K-steps
+//              of 16) into one of two TMEM S buffers, ahead of O += P V
+//              (M=128, N=64 + 16, K=64; V is an MN-major operand) whenever
+//              the next block's K/V have landed.
 //   warps 2-5  softmax, one thread per query row: reads its S row from TMEM,
 //              online softmax in base 2 with lazy rescaling (O in TMEM is
 //              rescaled only when the running max grows by more than 2^8),
 //              writes its P row (bf16) to a 128-byte-swizzled shared buffer,
 //              and at the end normalises O and stores it.
+// Two CTAs share an SM (256 TMEM columns and ~94 KB of shared memory each), so
+// the softmax of one overlaps the MMAs and exponentials of the other.
 // Key splits of the same (query tile, head) leave their unnormalised O and
 // row max / sum in a workspace; for each row, the last split to finish (an
 // atomic ticket per row, no waiting) merges them in split order.
@@ -39,26 +42,41 @@ namespace {
 
 using namespace rc::tc;
 
-constexpr int BQ = 128, BKV = 128, THREADS = 192;
+constexpr int BQ = 128, BKV = 64, THREADS = 192;
 constexpr int KV_STAGES = 3;
-constexpr int BLK = BQ * 32;       // one [128 rows][16 bf16] block, 32-byte swizzled
-constexpr int P_BYTES = BQ * BKV * 2;
+constexpr int P_BYTES = BQ * BKV * 2;  // [128][64] bf16, 128-byte swizzle (one buffer)
+constexpr int TMEM_COLS = 256;     // S0 | S1 (64 columns each) | O (<= 128)
+constexpr int CTAS_PER_SM = 2;
 constexpr int PART_STRIDE = 76;    // floats per row of a split's partial result
 constexpr float LAZY_RESCALE = 8.f;
 
+// 2^x on the special-function unit (flushes subnormal results to zero; the
+// argument is at most 8 here).
+__device__ __forceinline__ float ex2_ftz(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 template <int DH>
 struct ACfg {
-  static constexpr int NB = (DH + 15) / 16;  // head-dim blocks (5 for 72)
-  static constexpr int DHP = NB * 16;        // padded head dim (80)
-  static constexpr int Q_BYTES = NB * BLK;
-  static constexpr int KV_BYTES = 2 * NB * BLK;
-  static constexpr size_t SMEM = size_t(Q_BYTES) + KV_STAGES * KV_BYTES + 2 * P_BYTES + 1024 + 256;
+  static_assert(DH == 64 || DH == 72, "head_dim 64 or 72");
+  static constexpr bool TAIL = DH > 64;          // head dims 64..79 (72..79 read as zero)
+  static constexpr int DHP = TAIL ? 80 : 64;     // padded head dim of the PV accumulator
+  // shared-memory operand tiles: a 64-wide 128B-swizzled part, a 16-wide
+  // 32B-swizzled tail
+  static constexpr int Q128 = BQ * 128, Q32 = TAIL ? BQ * 32 : 0;
+  static constexpr int K128 = BKV * 128, K32 = TAIL ? BKV * 32 : 0;
+  static constexpr int Q_BYTES = Q128 + Q32;
+  static constexpr int KV_BYTES = 2 * (K128 + K32);  // K then V
+  static constexpr size_t SMEM = size_t(Q_BYTES) + KV_STAGES * KV_BYTES + P_BYTES + 1024 + 256;
   // kind::f16, D f32, A/B bf16; S: both K-major; PV: B (V) MN-major (bit 16)
   static constexpr uint32_t IDESC_S = (1u << 4) | (1u << 7) | (1u << 10) |
                                       (uint32_t(BKV >> 3) << 17) | (uint32_t(BQ >> 4) << 24);
-  static constexpr uint32_t IDESC_PV = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) |
-                                       (uint32_t(DHP >> 3) << 17) | (uint32_t(BQ >> 4) << 24);
-  static_assert(DHP <= 128 && DH + 2 <= PART_STRIDE, "head dim too large");
+  static constexpr uint32_t IDESC_PV64 = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) |
+                                         (uint32_t(64 >> 3) << 17) | (uint32_t(BQ >> 4) << 24);
+  static constexpr uint32_t IDESC_PV16 = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) |
+                                         (uint32_t(16 >> 3) << 17) | (uint32_t(BQ >> 4) << 24);
 };
 
 // Work list of one launch, identical in every thread.
@@ -69,7 +87,7 @@ struct AttnSched {
     pairs = qtiles * heads;
     nkb = (Nk + BKV - 1) / BKV;
     split = 1;
-    while (split < 8 && pairs * split < 2 * grid && split * 2 <= nkb &&
+    while (split < 16 && pairs * split < 2 * grid && split * 4 <= nkb &&
            pairs * split * 2 <= ws_units)
       split *= 2;
     per = (nkb + split - 1) / split;
@@ -89,29 +107,30 @@ struct AttnSched {
 };
 
 template <int DH>
-__global__ void __launch_bounds__(THREADS, 1)
-attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-               const __grid_constant__ CUtensorMap tmV, int Nk, bf16* __restrict__ O, int ldo,
-               int heads, int Dbound, const int* __restrict__ dcount, float scale_log2,
-               unsigned* err, float* __restrict__ part, int* __restrict__ tickets, int ws_units) {
+__global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
+attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmQt,
+               const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmKt,
+               const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmVt,
+               int Nk, bf16* __restrict__ O, int ldo, int heads, int Dbound,
+               const int* __restrict__ dcount, float scale_log2, unsigned* err,
+               float* __restrict__ part, int* __restrict__ tickets, int ws_units) {
   using C = ACfg<DH>;
-  constexpr int NB = C::NB;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   uint8_t* sQ = smem;
   uint8_t* sKV = sQ + C::Q_BYTES;
   uint8_t* sP = sKV + KV_STAGES * C::KV_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + 2 * P_BYTES);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 18);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + P_BYTES);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 16);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   // barrier addresses
   const uint32_t b0 = saddr(bars);
   const uint32_t q_full = b0, q_empty = b0 + 8;
   const uint32_t kv_full = b0 + 16, kv_empty = kv_full + 8 * KV_STAGES;
   const uint32_t s_full = kv_empty + 8 * KV_STAGES, s_free = s_full + 16;
-  const uint32_t p_ready = s_free + 16, p_free = p_ready + 16;
-  const uint32_t o_full = p_free + 16, o_free = o_full + 8;
+  const uint32_t p_ready = s_free + 16, p_free = p_ready + 8;
+  const uint32_t o_full = p_free + 8, o_free = o_full + 8;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -124,25 +143,30 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     for (int b = 0; b < 2; ++b) {
       mbar_init(s_full + 8 * b, 1);
       mbar_init(s_free + 8 * b, 128);
-      mbar_init(p_ready + 8 * b, 128);
-      mbar_init(p_free + 8 * b, 1);
     }
+    mbar_init(p_ready, 128);
+    mbar_init(p_free, 1);
     mbar_init(o_full, 1);
     mbar_init(o_free, 128);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 1) tmem_alloc(saddr(tmem_slot), 512);
+  if (warp == 1) tmem_alloc(saddr(tmem_slot), TMEM_COLS);
   if (warp == 0 && lane == 0) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmQ)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+    if (C::TAIL) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmQt)) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmKt)) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmVt)) : "memory");
+    }
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const uint32_t tS0 = tmem_base, tO = tmem_base + 256;
+  const uint32_t tS0 = tmem_base, tO = tmem_base + 2 * BKV;
 
   pdl_wait();
   pdl_trigger();
@@ -159,18 +183,18 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         sc.decode(u, qt, h, sp, kb0, kb1);
         if (!mbar_wait(q_empty, (uc + 1) & 1, abort_flag)) goto timeout;
         mbar_expect_tx(q_full, C::Q_BYTES);
-        for (int jj = 0; jj < NB; ++jj)
-          tma_load_3d(saddr(sQ + jj * BLK), &tmQ, q_full, jj * 16, h, qt * BQ);
+        tma_load_3d(saddr(sQ), &tmQ, q_full, 0, h, qt * BQ);
+        if (C::TAIL) tma_load_3d(saddr(sQ + C::Q128), &tmQt, q_full, 64, h, qt * BQ);
         for (int kb = kb0; kb < kb1; ++kb, ++g) {
           const int st = g % KV_STAGES;
           if (!mbar_wait(kv_empty + 8 * st, ((g / KV_STAGES) & 1) ^ 1, abort_flag)) goto timeout;
           mbar_expect_tx(kv_full + 8 * st, C::KV_BYTES);
           uint8_t* base = sKV + st * C::KV_BYTES;
-          for (int jj = 0; jj < NB; ++jj)
-            tma_load_3d(saddr(base + jj * BLK), &tmK, kv_full + 8 * st, jj * 16, h, kb * BKV);
-          for (int jj = 0; jj < NB; ++jj)
-            tma_load_3d(saddr(base + (NB + jj) * BLK), &tmV, kv_full + 8 * st, jj * 16, h,
-                        kb * BKV);
+          const uint32_t fb = kv_full + 8 * st;
+          tma_load_3d(saddr(base), &tmK, fb, 0, h, kb * BKV);
+          if (C::TAIL) tma_load_3d(saddr(base + C::K128), &tmKt, fb, 64, h, kb * BKV);
+          tma_load_3d(saddr(base + C::K128 + C::K32), &tmV, fb, 0, h, kb * BKV);
+          if (C::TAIL) tma_load_3d(saddr(base + 2 * C::K128 + C::K32), &tmVt, fb, 64, h, kb * BKV);
         }
       }
     }
@@ -185,38 +209,60 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         const int n = kb1 - kb0;
         if (!mbar_wait(q_full, uc & 1, abort_flag)) goto timeout;
         tc_fence_after();
-        for (int j = -1; j < n; ++j) {
-          // S for block j + 1, one block ahead of P V for block j
-          if (j + 1 < n) {
-            const int gg = g + j + 1;
-            const int st = gg % KV_STAGES;
-            if (!mbar_wait(kv_full + 8 * st, (gg / KV_STAGES) & 1, abort_flag)) goto timeout;
-            if (!mbar_wait(s_free + 8 * (gg & 1), ((gg >> 1) + 1) & 1, abort_flag)) goto timeout;
-            tc_fence_after();
-            const uint32_t kbase = saddr(sKV + st * C::KV_BYTES);
-            for (int jj = 0; jj < NB; ++jj)
-              umma_bf16(tS0 + 128u * uint32_t(gg & 1), sw32_kmajor_desc(qb + jj * BLK),
-                        sw32_kmajor_desc(kbase + jj * BLK), C::IDESC_S, jj > 0 ? 1u : 0u);
-            umma_commit(s_full + 8 * (gg & 1));
-            if (j + 2 == n) umma_commit(q_empty);  // last S of the unit issued
+        int s_issued = 0;
+        // S = Q K^T for block s_issued of the unit.  Non-blocking form: only
+        // if its K/V have landed and its S buffer is free.  Returns false on
+        // timeout.
+        auto issue_S = [&](bool block, bool& done) -> bool {
+          const int gg = g + s_issued;
+          const int st = gg % KV_STAGES;
+          const uint32_t kvp = (gg / KV_STAGES) & 1, sfp = ((gg >> 1) + 1) & 1;
+          if (block) {
+            if (!mbar_wait(kv_full + 8 * st, kvp, abort_flag)) return false;
+            if (!mbar_wait(s_free + 8 * (gg & 1), sfp, abort_flag)) return false;
+          } else if (!mbar_test(kv_full + 8 * st, kvp) || !mbar_test(s_free + 8 * (gg & 1), sfp)) {
+            done = false;
+            return true;
           }
-          if (j < 0) continue;
+          tc_fence_after();
+          const uint32_t kb = saddr(sKV + st * C::KV_BYTES);
+          const uint32_t sd = tS0 + uint32_t(BKV) * uint32_t(gg & 1);
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            umma_bf16(sd, sw128_desc(qb + 32 * kk), sw128_desc(kb + 32 * kk), C::IDESC_S,
+                      kk > 0 ? 1u : 0u);
+          if (C::TAIL)
+            umma_bf16(sd, sw32_kmajor_desc(qb + C::Q128), sw32_kmajor_desc(kb + C::K128),
+                      C::IDESC_S, 1u);
+          umma_commit(s_full + 8 * (gg & 1));
+          if (++s_issued == n) umma_commit(q_empty);  // last S of the unit issued
+          done = true;
+          return true;
+        };
+        bool done = false;
+        if (!issue_S(true, done)) goto timeout;
+        for (int j = 0; j < n; ++j) {
           const int gj = g + j;
-          if (j == 0) {
-            if (!mbar_wait(o_free, (uc + 1) & 1, abort_flag)) goto timeout;
-          }
-          if (!mbar_wait(p_ready + 8 * (gj & 1), (gj >> 1) & 1, abort_flag)) goto timeout;
+          // S of the next block early if its data is already here
+          if (s_issued == j + 1 && j + 1 < n && !issue_S(false, done)) goto timeout;
+          if (j == 0 && !mbar_wait(o_free, (uc + 1) & 1, abort_flag)) goto timeout;
+          if (!mbar_wait(p_ready, gj & 1, abort_flag)) goto timeout;
           tc_fence_after();
           const int st = gj % KV_STAGES;
-          const uint32_t vb = saddr(sKV + st * C::KV_BYTES + NB * BLK);
-          const uint32_t pb = saddr(sP + (gj & 1) * P_BYTES);
+          const uint32_t vb = saddr(sKV + st * C::KV_BYTES + C::K128 + C::K32);
+          const uint32_t pb = saddr(sP);
 #pragma unroll
-          for (int kk = 0; kk < BKV / 16; ++kk)
-            umma_bf16(tO, sw128_desc(pb + (kk >> 2) * (BQ * 128) + (kk & 3) * 32),
-                      sw32_mnmajor_desc(vb + kk * 16 * 32, BLK), C::IDESC_PV,
-                      (j > 0 || kk > 0) ? 1u : 0u);
-          umma_commit(p_free + 8 * (gj & 1));
+          for (int kk = 0; kk < BKV / 16; ++kk) {
+            const uint32_t acc = (j > 0 || kk > 0) ? 1u : 0u;
+            umma_bf16(tO, sw128_desc(pb + 32 * kk), sw128_mnmajor_desc(vb + kk * 16 * 128),
+                      C::IDESC_PV64, acc);
+            if (C::TAIL)
+              umma_bf16(tO + 64, sw128_desc(pb + 32 * kk),
+                        sw32_mnmajor_desc(vb + C::K128 + kk * 16 * 32, 16), C::IDESC_PV16, acc);
+          }
+          umma_commit(p_free);
           umma_commit(kv_empty + 8 * st);
+          if (s_issued == j + 1 && j + 1 < n && !issue_S(true, done)) goto timeout;
         }
         g += n;
         umma_commit(o_full);
@@ -239,30 +285,37 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         uint32_t r[BKV];
 #pragma unroll
         for (int i = 0; i < BKV / 16; ++i)
-          tmem_ld16_nowait(tS0 + 128u * uint32_t(g & 1) + lane_off + 16u * i, r + 16 * i);
+          tmem_ld16_nowait(tS0 + uint32_t(BKV) * uint32_t(g & 1) + lane_off + 16u * i, r + 16 * i);
         tmem_wait_ld();
         tc_fence_before();
         mbar_arrive(s_free + 8 * (g & 1));
+        // raw scores: the running max m is kept in scaled base-2 units; the
+        // scale (log2 e / sqrt(dh) > 0) commutes with the max, and
+        // p = 2^(s * scale - m) is one FFMA + ex2 per element
         const int valid = Nk - (kb0 + j) * BKV;
-        float mx = -INFINITY;
+        float mx8[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) mx8[q] = -INFINITY;
 #pragma unroll
         for (int c = 0; c < BKV; ++c) {
-          const float v = c < valid ? __uint_as_float(r[c]) * scale_log2 : -INFINITY;
+          const float v = c < valid ? __uint_as_float(r[c]) : -INFINITY;
           r[c] = __float_as_uint(v);
-          mx = fmaxf(mx, v);
+          mx8[c & 7] = fmaxf(mx8[c & 7], v);
         }
+        float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                         fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]))) * scale_log2;
+        // the single P buffer is free once P V of the previous block is done
+        // (that is also when O may be rescaled)
+        if (!mbar_wait_warp(p_free, (g + 1) & 1, abort_flag)) goto timeout;
         if (j == 0) {
           m = mx;
         } else if (__any_sync(0xffffffffu, mx > m + LAZY_RESCALE)) {
           // (warp-uniform branch: the TMEM accesses below are warp-wide)
           mx = fmaxf(mx, m);
-          // O holds P V of blocks < j: wait for the last of them, then rescale
-          if (!mbar_wait_warp(p_free + 8 * ((g - 1) & 1), ((g - 1) >> 1) & 1, abort_flag))
-            goto timeout;
           tc_fence_after();
-          const float alpha = exp2f(m - mx);
+          const float alpha = ex2_ftz(m - mx);
 #pragma unroll
-          for (int i = 0; i < NB; ++i) {
+          for (int i = 0; i < C::DHP / 16; ++i) {
             uint32_t o16[16];
             tmem_ld16_nowait(tO + lane_off + 16u * i, o16);
             tmem_wait_ld();
@@ -274,37 +327,38 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
           l *= alpha;
           m = mx;
         }
-        float sum = 0.f;
+        const float negm = -m;
+        float sum8[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) sum8[q] = 0.f;
 #pragma unroll
         for (int c = 0; c < BKV; ++c) {
-          const float p = exp2f(__uint_as_float(r[c]) - m);
+          const float p = ex2_ftz(fmaf(__uint_as_float(r[c]), scale_log2, negm));
           r[c] = __float_as_uint(p);
-          sum += p;
+          sum8[c & 7] += p;
         }
-        l += sum;
-        // P buffer (g & 1) is free once P V of block g - 2 is done
-        if (!mbar_wait_warp(p_free + 8 * (g & 1), ((g >> 1) + 1) & 1, abort_flag)) goto timeout;
-        uint8_t* prow = sP + (g & 1) * P_BYTES + row * 128;
+        l += ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) + ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
+        // P row: 64 keys = one 128-byte row of the 128B-swizzled A tile
+        uint8_t* prow = sP + row * 128;
 #pragma unroll
-        for (int c16 = 0; c16 < BKV / 8; ++c16) {
+        for (int ch = 0; ch < BKV / 8; ++ch) {
           uint4 w;
-          w.x = pack_bf16x2(__uint_as_float(r[8 * c16 + 0]), __uint_as_float(r[8 * c16 + 1]));
-          w.y = pack_bf16x2(__uint_as_float(r[8 * c16 + 2]), __uint_as_float(r[8 * c16 + 3]));
-          w.z = pack_bf16x2(__uint_as_float(r[8 * c16 + 4]), __uint_as_float(r[8 * c16 + 5]));
-          w.w = pack_bf16x2(__uint_as_float(r[8 * c16 + 6]), __uint_as_float(r[8 * c16 + 7]));
-          const int atom = c16 >> 3, ch = c16 & 7;
-          *reinterpret_cast<uint4*>(prow + atom * (BQ * 128) + ((ch ^ (row & 7)) << 4)) = w;
+          w.x = pack_bf16x2(__uint_as_float(r[8 * ch + 0]), __uint_as_float(r[8 * ch + 1]));
+          w.y = pack_bf16x2(__uint_as_float(r[8 * ch + 2]), __uint_as_float(r[8 * ch + 3]));
+          w.z = pack_bf16x2(__uint_as_float(r[8 * ch + 4]), __uint_as_float(r[8 * ch + 5]));
+          w.w = pack_bf16x2(__uint_as_float(r[8 * ch + 6]), __uint_as_float(r[8 * ch + 7]));
+          *reinterpret_cast<uint4*>(prow + ((ch ^ (row & 7)) << 4)) = w;
         }
         fence_proxy_async_smem();
         tc_fence_before();
-        mbar_arrive(p_ready + 8 * (g & 1));
+        mbar_arrive(p_ready);
       }
       // ---- unit epilogue
       if (!mbar_wait_warp(o_full, uc & 1, abort_flag)) goto timeout;
       tc_fence_after();
       uint32_t o[C::DHP];
 #pragma unroll
-      for (int i = 0; i < NB; ++i) tmem_ld16_nowait(tO + lane_off + 16u * i, o + 16 * i);
+      for (int i = 0; i < C::DHP / 16; ++i) tmem_ld16_nowait(tO + lane_off + 16u * i, o + 16 * i);
       tmem_wait_ld();
       tc_fence_before();
       mbar_arrive(o_free);
@@ -391,7 +445,7 @@ done:
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tmem_base, 512);
+    tmem_dealloc(tmem_base, TMEM_COLS);
   }
 }
 
@@ -425,12 +479,14 @@ struct HeadMapHash {
 };
 
 // (head_dim, head, row) view of a row-major [rows][ld] bf16 matrix whose row
-// holds `heads` blocks of dh; boxes of 16 x 1 x 128, 32-byte swizzle; reads
-// outside the view (head_dim >= dh, row >= rows) return zero.
-cudaError_t head_map(const bf16* p, int rows, int ld, int heads, int dh, CUtensorMap* out) {
+// holds `heads` blocks of dh; boxes of box_w x 1 x box_rows (box_w 64 with the
+// 128-byte swizzle, 16 with the 32-byte swizzle); reads outside the view
+// (head_dim >= dh, row >= rows) return zero.
+cudaError_t head_map(const bf16* p, int rows, int ld, int heads, int dh, int box_w, int box_rows,
+                     CUtensorMap* out) {
   static std::mutex mu;
   static std::unordered_map<HeadMapKey, CUtensorMap, HeadMapHash> cache;
-  HeadMapKey key{p, rows, ld, heads, dh};
+  HeadMapKey key{p, rows, ld, heads, (dh * 1024 + box_rows) * 256 + box_w};
   {
     std::lock_guard<std::mutex> lock(mu);
     auto it = cache.find(key);
@@ -443,10 +499,11 @@ cudaError_t head_map(const bf16* p, int rows, int ld, int heads, int dh, CUtenso
   if (!fn) return cudaErrorNotSupported;
   cuuint64_t dims[3] = {cuuint64_t(dh), cuuint64_t(heads), cuuint64_t(rows)};
   cuuint64_t strides[2] = {cuuint64_t(dh) * sizeof(bf16), cuuint64_t(ld) * sizeof(bf16)};
-  cuuint32_t box[3] = {16, 1, cuuint32_t(BQ)};
+  cuuint32_t box[3] = {cuuint32_t(box_w), 1, cuuint32_t(box_rows)};
   cuuint32_t estr[3] = {1, 1, 1};
   CUresult r = fn(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<bf16*>(p), dims, strides,
-                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_32B,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  box_w == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_32B,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
   std::lock_guard<std::mutex> lock(mu);
@@ -479,7 +536,7 @@ size_t attention_split_floats(int Nmax, int heads, int dh) {
   (void)heads;
   (void)dh;
   const int sms = device_sms_attn();
-  return size_t(4) * (sms > 0 ? sms : 160) * BQ * PART_STRIDE;
+  return size_t(8) * (sms > 0 ? sms : 160) * BQ * PART_STRIDE;
 }
 
 // (query tile, head) pairs; the context allocates 128 row tickets per pair
@@ -493,20 +550,24 @@ cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* 
   if (dh != 72 && dh != 64) return cudaErrorInvalidValue;
   const int sms = device_sms_attn();
   if (!sms) return cudaErrorInvalidDevice;
-  CUtensorMap tq, tk, tv;
-  RC_TRY(head_map(Q, Dbound, ldq, heads, dh, &tq));
-  RC_TRY(head_map(K, Nk, ldkv, heads, dh, &tk));
-  RC_TRY(head_map(V, Nk, ldkv, heads, dh, &tv));
+  // a 64-wide 128B-swizzled map and a 16-wide 32B-swizzled tail map per operand
+  CUtensorMap tq, tqt, tk, tkt, tv, tvt;
+  RC_TRY(head_map(Q, Dbound, ldq, heads, dh, 64, BQ, &tq));
+  RC_TRY(head_map(K, Nk, ldkv, heads, dh, 64, BKV, &tk));
+  RC_TRY(head_map(V, Nk, ldkv, heads, dh, 64, BKV, &tv));
+  RC_TRY(head_map(Q, Dbound, ldq, heads, dh, 16, BQ, &tqt));
+  RC_TRY(head_map(K, Nk, ldkv, heads, dh, 16, BKV, &tkt));
+  RC_TRY(head_map(V, Nk, ldkv, heads, dh, 16, BKV, &tvt));
   const float scale_log2 = float(1.4426950408889634 / sqrt(double(dh)));
   const int ws_units = int(as.part_floats / (size_t(BQ) * PART_STRIDE));
   if (dh == 72)
-    RC_TRY(launch_k(attn_tc_kernel<72>, dim3(sms), dim3(THREADS), ACfg<72>::SMEM, st, tq, tk, tv,
-                    Nk, O, ldo, heads, Dbound, dcount, scale_log2, err, as.part, as.tickets,
-                    ws_units));
+    RC_TRY(launch_k(attn_tc_kernel<72>, dim3(CTAS_PER_SM * sms), dim3(THREADS), ACfg<72>::SMEM,
+                    st, tq, tqt, tk, tkt, tv, tvt, Nk, O, ldo, heads, Dbound, dcount, scale_log2,
+                    err, as.part, as.tickets, ws_units));
   else
-    RC_TRY(launch_k(attn_tc_kernel<64>, dim3(sms), dim3(THREADS), ACfg<64>::SMEM, st, tq, tk, tv,
-                    Nk, O, ldo, heads, Dbound, dcount, scale_log2, err, as.part, as.tickets,
-                    ws_units));
+    RC_TRY(launch_k(attn_tc_kernel<64>, dim3(CTAS_PER_SM * sms), dim3(THREADS), ACfg<64>::SMEM,
+                    st, tq, tqt, tk, tkt, tv, tvt, Nk, O, ldo, heads, Dbound, dcount, scale_log2,
+                    err, as.part, as.tickets, ws_units));
   count_launches(1);
   return cudaSuccess;
 }

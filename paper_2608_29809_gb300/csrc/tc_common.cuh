@@ -153,6 +153,32 @@ __device__ __forceinline__ uint64_t sw32_mnmajor_desc(uint32_t addr, uint32_t lb
   return d;
 }
 
+// MN-major bf16 operand with the 128-byte swizzle: 64 MN-contiguous elements
+// per 128-byte row, consecutive K rows 128 B apart, 8-row K groups 1024 B
+// apart (a single 64-wide MN group: the leading offset is unused).
+__device__ __forceinline__ uint64_t sw128_mnmajor_desc(uint32_t addr) {
+  uint64_t d = 0;
+  d |= uint64_t((addr & 0x3FFFFu) >> 4);
+  d |= uint64_t(16 >> 4) << 16;
+  d |= uint64_t(1024 >> 4) << 32;
+  d |= uint64_t(1) << 46;
+  d |= uint64_t(2) << 61;
+  return d;
+}
+
+// Non-blocking check that the phase of parity `parity` has completed.
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
 // 16 consecutive f32 columns of this thread's TMEM lane (no wait).
 __device__ __forceinline__ void tmem_ld16_nowait(uint32_t taddr, uint32_t* r) {
   asm volatile(
