@@ -23,8 +23,8 @@
 // Two CTAs share an SM (256 TMEM columns and ~94 KB of shared memory each), so
 // the softmax of one overlaps the MMAs and exponentials of the other.
 // Key splits of the same (query tile, head) leave their unnormalised O and
-// row max / sum in a workspace; for each row, the last split to finish (an
-// atomic ticket per row, no waiting) merges them in split order.
+// row max / sum in a workspace; a small combine kernel, launched right after,
+// merges them (one warp per row, coalesced).
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <math.h>
@@ -49,6 +49,7 @@ constexpr int TMEM_COLS = 256;     // S0 | S1 (64 columns each) | O (<= 128)
 constexpr int CTAS_PER_SM = 2;
 constexpr int PART_STRIDE = 76;    // floats per row of a split's partial result
 constexpr float LAZY_RESCALE = 8.f;
+constexpr int MAX_SPLIT = 16;
 
 // 2^x on the special-function unit (flushes subnormal results to zero; the
 // argument is at most 8 here).
@@ -87,7 +88,7 @@ struct AttnSched {
     pairs = qtiles * heads;
     nkb = (Nk + BKV - 1) / BKV;
     split = 1;
-    while (split < 16 && pairs * split < 2 * grid && split * 4 <= nkb &&
+    while (split < MAX_SPLIT && pairs * split < 2 * grid && split * 4 <= nkb &&
            pairs * split * 2 <= ws_units)
       split *= 2;
     per = (nkb + split - 1) / split;
@@ -113,7 +114,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmVt,
                int Nk, bf16* __restrict__ O, int ldo, int heads, int Dbound,
                const int* __restrict__ dcount, float scale_log2, unsigned* err,
-               float* __restrict__ part, int* __restrict__ tickets, int ws_units) {
+               float* __restrict__ part, int ws_units) {
   using C = ACfg<DH>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -378,6 +379,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
           }
         }
       } else {
+        // split of the keys: unnormalised O with its row max and sum; the
+        // combine kernel merges the splits
         const int pair = u / sc.split;
         float* mine = part + (size_t(pair) * sc.split + sp) * (BQ * PART_STRIDE) +
                       size_t(row) * PART_STRIDE;
@@ -387,51 +390,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                  make_float4(__uint_as_float(o[4 * c4]), __uint_as_float(o[4 * c4 + 1]),
                              __uint_as_float(o[4 * c4 + 2]), __uint_as_float(o[4 * c4 + 3])));
         __stcg(reinterpret_cast<float2*>(mine + DH), make_float2(m, l));
-        // per-row ticket: the last split to finish this row merges it (no
-        // cross-warp barrier, no waiting)
-        __threadfence();
-        int* tk = tickets + size_t(pair) * BQ + row;
-        const bool last = atomicAdd(tk, 1) == sc.split - 1;
-        if (last) {
-          *tk = 0;  // re-armed for the next launch
-          if (qrow < D) {
-            __threadfence();
-            const float* base = part + size_t(pair) * sc.split * (BQ * PART_STRIDE) +
-                                size_t(row) * PART_STRIDE;
-            float M = -INFINITY;
-            for (int q = 0; q < sc.split; ++q)
-              M = fmaxf(M, __ldcg(base + size_t(q) * (BQ * PART_STRIDE) + DH));
-            float L = 0.f;
-            float acc[DH];
-#pragma unroll
-            for (int c = 0; c < DH; ++c) acc[c] = 0.f;
-            for (int q = 0; q < sc.split; ++q) {
-              const float* sl = base + size_t(q) * (BQ * PART_STRIDE);
-              const float2 ml = __ldcg(reinterpret_cast<const float2*>(sl + DH));
-              const float w = exp2f(ml.x - M);
-              L += w * ml.y;
-#pragma unroll
-              for (int c4 = 0; c4 < DH / 4; ++c4) {
-                const float4 v = __ldcg(reinterpret_cast<const float4*>(sl) + c4);
-                acc[4 * c4] += w * v.x;
-                acc[4 * c4 + 1] += w * v.y;
-                acc[4 * c4 + 2] += w * v.z;
-                acc[4 * c4 + 3] += w * v.w;
-              }
-            }
-            const float inv = L > 0.f ? 1.f / L : 0.f;
-            uint4* dst = reinterpret_cast<uint4*>(O + size_t(qrow) * ldo + h * DH);
-#pragma unroll
-            for (int c8 = 0; c8 < DH / 8; ++c8) {
-              uint4 w;
-              w.x = pack_bf16x2(acc[8 * c8 + 0] * inv, acc[8 * c8 + 1] * inv);
-              w.y = pack_bf16x2(acc[8 * c8 + 2] * inv, acc[8 * c8 + 3] * inv);
-              w.z = pack_bf16x2(acc[8 * c8 + 4] * inv, acc[8 * c8 + 5] * inv);
-              w.w = pack_bf16x2(acc[8 * c8 + 6] * inv, acc[8 * c8 + 7] * inv);
-              dst[c8] = w;
-            }
-          }
-        }
       }
     }
   }
@@ -447,6 +405,53 @@ done:
     tc_fence_after();
     tmem_dealloc(tmem_base, TMEM_COLS);
   }
+}
+
+// Merge of the key splits: one warp per query row; lane q < split reads that
+// split's row max / sum, the warp reduces the max, then every lane
+// accumulates its 4 head-dim columns over the splits.
+template <int DH>
+__global__ void __launch_bounds__(256)
+attn_combine_kernel(const float* __restrict__ part, bf16* __restrict__ O, int ldo, int heads,
+                    int Dbound, const int* __restrict__ dcount, int Nk, int attn_grid,
+                    int ws_units, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
+  const int D = live_count(dcount, Dbound, err);
+  AttnSched sc;
+  sc.init(D, heads, Nk, attn_grid, ws_units);
+  if (sc.split == 1) return;
+  const int lane = threadIdx.x & 31;
+  const int gw = blockIdx.x * 8 + (threadIdx.x >> 5);  // (pair, row)
+  if (gw >= sc.pairs * BQ) return;
+  const int pair = gw / BQ, row = gw - pair * BQ;
+  const int qt = pair % sc.qtiles, h = pair / sc.qtiles;
+  const int qrow = qt * BQ + row;
+  if (qrow >= D) return;
+  const float* base = part + size_t(pair) * sc.split * (BQ * PART_STRIDE) + size_t(row) * PART_STRIDE;
+  float2 ml = make_float2(-INFINITY, 0.f);
+  if (lane < sc.split) ml = __ldcg(reinterpret_cast<const float2*>(base + size_t(lane) * (BQ * PART_STRIDE) + DH));
+  float M = ml.x;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  const float w = lane < sc.split ? ex2_ftz(ml.x - M) : 0.f;
+  float L = w * ml.y;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+  if (lane >= DH / 4) return;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+  for (int q = 0; q < sc.split; ++q) {
+    const float wq = __shfl_sync((1u << (DH / 4)) - 1u, w, q);
+    const float4 v = __ldcg(reinterpret_cast<const float4*>(base + size_t(q) * (BQ * PART_STRIDE)) + lane);
+    acc.x += wq * v.x;
+    acc.y += wq * v.y;
+    acc.z += wq * v.z;
+    acc.w += wq * v.w;
+  }
+  const float inv = L > 0.f ? 1.f / L : 0.f;
+  *reinterpret_cast<uint2*>(O + size_t(qrow) * ldo + h * DH + 4 * lane) =
+      make_uint2(pack_bf16x2(acc.x * inv, acc.y * inv), pack_bf16x2(acc.z * inv, acc.w * inv));
 }
 
 // ------------------------------------------------------------------- host
@@ -560,15 +565,27 @@ cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* 
   RC_TRY(head_map(V, Nk, ldkv, heads, dh, 16, BKV, &tvt));
   const float scale_log2 = float(1.4426950408889634 / sqrt(double(dh)));
   const int ws_units = int(as.part_floats / (size_t(BQ) * PART_STRIDE));
+  const int grid = CTAS_PER_SM * sms;
   if (dh == 72)
-    RC_TRY(launch_k(attn_tc_kernel<72>, dim3(CTAS_PER_SM * sms), dim3(THREADS), ACfg<72>::SMEM,
-                    st, tq, tqt, tk, tkt, tv, tvt, Nk, O, ldo, heads, Dbound, dcount, scale_log2,
-                    err, as.part, as.tickets, ws_units));
+    RC_TRY(launch_k(attn_tc_kernel<72>, dim3(grid), dim3(THREADS), ACfg<72>::SMEM, st, tq, tqt,
+                    tk, tkt, tv, tvt, Nk, O, ldo, heads, Dbound, dcount, scale_log2, err, as.part,
+                    ws_units));
   else
-    RC_TRY(launch_k(attn_tc_kernel<64>, dim3(CTAS_PER_SM * sms), dim3(THREADS), ACfg<64>::SMEM,
-                    st, tq, tqt, tk, tkt, tv, tvt, Nk, O, ldo, heads, Dbound, dcount, scale_log2,
-                    err, as.part, as.tickets, ws_units));
+    RC_TRY(launch_k(attn_tc_kernel<64>, dim3(grid), dim3(THREADS), ACfg<64>::SMEM, st, tq, tqt,
+                    tk, tkt, tv, tvt, Nk, O, ldo, heads, Dbound, dcount, scale_log2, err, as.part,
+                    ws_units));
   count_launches(1);
+  // key splits happen only with at least 4 key blocks per split
+  if ((Nk + BKV - 1) / BKV >= 8) {
+    const int warps = ((Dbound + BQ - 1) / BQ) * heads * BQ;
+    if (dh == 72)
+      RC_TRY(launch_k(attn_combine_kernel<72>, dim3((warps + 7) / 8), dim3(256), 0, st, as.part, O,
+                      ldo, heads, Dbound, dcount, Nk, grid, ws_units, err));
+    else
+      RC_TRY(launch_k(attn_combine_kernel<64>, dim3((warps + 7) / 8), dim3(256), 0, st, as.part, O,
+                      ldo, heads, Dbound, dcount, Nk, grid, ws_units, err));
+    count_launches(1);
+  }
   return cudaSuccess;
 }
 

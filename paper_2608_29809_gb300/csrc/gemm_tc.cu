@@ -311,13 +311,11 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       if (++acc == 2) { acc = 0; acc_phase ^= 1; }
       if (sc.split > 1 && !additive) {
         // per-row ticket: the last split to finish a row reduces it (no
-        // cross-warp barrier, no waiting)
-        __threadfence();
+        // cross-warp barrier, no waiting); acq_rel orders the reductions
         int* tk = tickets + size_t(tile) * BM + row;
-        const bool last = atomicAdd(tk, 1) == sc.split - 1;
+        const bool last = ticket_add(tk, 1) == sc.split - 1;
         if (last) {
           *tk = 0;  // re-armed for the next launch
-          __threadfence();
 #pragma unroll 1
           for (int ch = 0; ch < BN / 32; ch += 2) {
             float v[64];

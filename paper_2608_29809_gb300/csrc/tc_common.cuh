@@ -38,17 +38,34 @@ __device__ __forceinline__ unsigned long long globaltimer() {
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
   return t;
 }
-// Waits for the phase of parity `parity`; gives up (returns false) when the
-// CTA's abort flag is raised or after WAIT_NS.
+// Non-blocking check that the phase of parity `parity` has completed.
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Waits for the phase of parity `parity` by polling (test_wait: the thread is
+// never parked, so it resumes as soon as the phase completes); gives up
+// (returns false) when the CTA's abort flag is raised or after WAIT_NS.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
-  if (mbar_try_wait(bar, parity)) return true;
+  if (mbar_test(bar, parity)) return true;
   const unsigned long long t0 = globaltimer();
-  while (true) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if (*abort_flag) return false;
-    if (globaltimer() - t0 > WAIT_NS) return false;
+  for (unsigned n = 1;; ++n) {
+    if (mbar_test(bar, parity)) return true;
+    if ((n & 63) == 0) {
+      if (*abort_flag) return false;
+      if (globaltimer() - t0 > WAIT_NS) return false;
+    }
   }
 }
+
 // mbar_wait taken by every lane of a warp; the outcome is made warp-uniform
 // so that a timeout never leaves part of a warp at a warp-wide instruction.
 __device__ __forceinline__ bool mbar_wait_warp(uint32_t bar, uint32_t parity,
@@ -164,19 +181,6 @@ __device__ __forceinline__ uint64_t sw128_mnmajor_desc(uint32_t addr) {
   d |= uint64_t(1) << 46;
   d |= uint64_t(2) << 61;
   return d;
-}
-
-// Non-blocking check that the phase of parity `parity` has completed.
-__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0;
 }
 
 // 16 consecutive f32 columns of this thread's TMEM lane (no wait).
