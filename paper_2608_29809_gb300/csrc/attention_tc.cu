@@ -50,6 +50,7 @@ constexpr int CTAS_PER_SM = 2;
 constexpr int PART_STRIDE = 76;    // floats per row of a split's partial result
 constexpr float LAZY_RESCALE = 8.f;
 constexpr int MAX_SPLIT = 16;
+constexpr int MIN_KB_PER_SPLIT = 4;  // key blocks per split, at least
 
 // 2^x on the special-function unit (flushes subnormal results to zero; the
 // argument is at most 8 here).
@@ -88,7 +89,7 @@ struct AttnSched {
     pairs = qtiles * heads;
     nkb = (Nk + BKV - 1) / BKV;
     split = 1;
-    while (split < MAX_SPLIT && pairs * split < 2 * grid && split * 4 <= nkb &&
+    while (split < MAX_SPLIT && pairs * split < 2 * grid && split * 2 * MIN_KB_PER_SPLIT <= nkb &&
            pairs * split * 2 <= ws_units)
       split *= 2;
     per = (nkb + split - 1) / split;
@@ -575,8 +576,8 @@ cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* 
                     tk, tkt, tv, tvt, Nk, O, ldo, heads, Dbound, dcount, scale_log2, err, as.part,
                     ws_units));
   count_launches(1);
-  // key splits happen only with at least 4 key blocks per split
-  if ((Nk + BKV - 1) / BKV >= 8) {
+  // key splits happen only with at least MIN_KB_PER_SPLIT key blocks per split
+  if ((Nk + BKV - 1) / BKV >= 2 * MIN_KB_PER_SPLIT) {
     const int warps = ((Dbound + BQ - 1) / BQ) * heads * BQ;
     if (dh == 72)
       RC_TRY(launch_k(attn_combine_kernel<72>, dim3((warps + 7) / 8), dim3(256), 0, st, as.part, O,
