@@ -423,12 +423,11 @@ attn_combine_kernel(const float* __restrict__ part, bf16* __restrict__ O, int ld
   sc.init(D, heads, Nk, attn_grid, ws_units);
   if (sc.split == 1) return;
   const int lane = threadIdx.x & 31;
-  const int gw = blockIdx.x * 8 + (threadIdx.x >> 5);  // (pair, row)
-  if (gw >= sc.pairs * BQ) return;
+  for (int gw = blockIdx.x * 8 + (threadIdx.x >> 5); gw < sc.pairs * BQ; gw += gridDim.x * 8) {
   const int pair = gw / BQ, row = gw - pair * BQ;
   const int qt = pair % sc.qtiles, h = pair / sc.qtiles;
   const int qrow = qt * BQ + row;
-  if (qrow >= D) return;
+  if (qrow >= D) continue;
   const float* base = part + size_t(pair) * sc.split * (BQ * PART_STRIDE) + size_t(row) * PART_STRIDE;
   float2 ml = make_float2(-INFINITY, 0.f);
   if (lane < sc.split) ml = __ldcg(reinterpret_cast<const float2*>(base + size_t(lane) * (BQ * PART_STRIDE) + DH));
@@ -439,7 +438,7 @@ attn_combine_kernel(const float* __restrict__ part, bf16* __restrict__ O, int ld
   float L = w * ml.y;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-  if (lane >= DH / 4) return;
+  if (lane < DH / 4) {
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll 4
   for (int q = 0; q < sc.split; ++q) {
@@ -453,6 +452,8 @@ attn_combine_kernel(const float* __restrict__ part, bf16* __restrict__ O, int ld
   const float inv = L > 0.f ? 1.f / L : 0.f;
   *reinterpret_cast<uint2*>(O + size_t(qrow) * ldo + h * DH + 4 * lane) =
       make_uint2(pack_bf16x2(acc.x * inv, acc.y * inv), pack_bf16x2(acc.z * inv, acc.w * inv));
+  }
+  }
 }
 
 // ------------------------------------------------------------------- host
@@ -545,8 +546,6 @@ size_t attention_split_floats(int Nmax, int heads, int dh) {
   return size_t(8) * (sms > 0 ? sms : 160) * BQ * PART_STRIDE;
 }
 
-// (query tile, head) pairs; the context allocates 128 row tickets per pair
-int attention_tickets(int Nmax, int heads) { return ((Nmax + BQ - 1) / BQ) * heads; }
 
 cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* V, int ldkv,
                              int Nk, bf16* O, int ldo, int heads, int dh, int Dbound,
@@ -579,11 +578,12 @@ cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* 
   // key splits happen only with at least MIN_KB_PER_SPLIT key blocks per split
   if ((Nk + BKV - 1) / BKV >= 2 * MIN_KB_PER_SPLIT) {
     const int warps = ((Dbound + BQ - 1) / BQ) * heads * BQ;
+    const int cgrid = min((warps + 7) / 8, 4 * sms);
     if (dh == 72)
-      RC_TRY(launch_k(attn_combine_kernel<72>, dim3((warps + 7) / 8), dim3(256), 0, st, as.part, O,
+      RC_TRY(launch_k(attn_combine_kernel<72>, dim3(cgrid), dim3(256), 0, st, as.part, O,
                       ldo, heads, Dbound, dcount, Nk, grid, ws_units, err));
     else
-      RC_TRY(launch_k(attn_combine_kernel<64>, dim3((warps + 7) / 8), dim3(256), 0, st, as.part, O,
+      RC_TRY(launch_k(attn_combine_kernel<64>, dim3(cgrid), dim3(256), 0, st, as.part, O,
                       ldo, heads, Dbound, dcount, Nk, grid, ws_units, err));
     count_launches(1);
   }

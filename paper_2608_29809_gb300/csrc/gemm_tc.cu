@@ -6,13 +6,13 @@
 // state written into the cache's H rows).
 //
 // C[M][n] = A[M][k] W[n][k]^T, A and W K-major bf16, f32 accumulation.
-// M (the dirty-token count) may live on the device: every CTA reads it, derives
-// the tile list and, when the tiles cannot fill the grid, a split of K.  The
-// gated residual (x += gate (C + b)) is written as vector reductions into x,
-// so the splits of K simply add up; for the other epilogues the splits reduce
-// into a zeroed f32 tile and, row by row, the last split to arrive (an atomic
-// ticket per row, no waiting) reads the row once, zeroes it and applies the
-// epilogue.
+// M (the dirty-token count) may live on the device: every CTA reads it and
+// derives a stream-K schedule (equal shares of all tiles' k-blocks, so small
+// and ragged tile counts still fill the GPU).  The gated residual
+// (x += gate (C + b)) is written as vector reductions into x, so pieces of a
+// tile simply add up; for the other epilogues the pieces of a split tile
+// reduce into a zeroed f32 workspace tile and a small finish kernel, launched
+// right after, applies the epilogue and zeroes the tile again.
 //
 // CTA = 6 warps: warp 0 issues TMA loads, warp 1 owns TMEM and issues the
 // MMAs (one thread), warps 2..5 drain the accumulator (one TMEM lane = one
@@ -38,8 +38,7 @@ using namespace rc::tc;
 constexpr int BM = 128, BK = 64;
 constexpr int THREADS = 192;
 constexpr int STAGE_A = BM * BK * 2;   // bytes
-constexpr int MAX_SPLIT = 4;
-constexpr int MIN_KB_PER_SPLIT = 4;
+constexpr int MIN_KB_PER_CTA = 4;
 constexpr int MAX_BN = 192;
 
 // Tile width BN (output features per tile): 192 when it divides n (every
@@ -145,31 +144,33 @@ __device__ __forceinline__ void epilogue32(const GemmEpi& ep, int r, int c0, flo
   }
 }
 
+// Stream-K schedule: the tiles' k-blocks are laid end to end (tile t =
+// nn * mt + m, m fastest so neighbouring CTAs share weight tiles in L2) and
+// CTA c takes the contiguous range [bound(c), bound(c+1)); a tile cut by a
+// range boundary is "split".  At least MIN_KB_PER_CTA k-blocks per CTA.
 template <int BN>
 struct Sched {
-  int mt, nt, tiles, split, kb_total, units;
+  int mt, nt, tiles, kbt, G;
+  long long work;
   __device__ void init(int M, int n, int k, int grid) {
     mt = (M + BM - 1) / BM;
     nt = n / BN;
     tiles = mt * nt;
-    kb_total = k / BK;
-    split = 1;
-    if (tiles > 0 && tiles < grid) {
-      split = grid / tiles;
-      if (split > MAX_SPLIT) split = MAX_SPLIT;
-      int cap = kb_total / MIN_KB_PER_SPLIT;
-      if (split > cap) split = cap < 1 ? 1 : cap;
-    }
-    units = tiles * split;
+    kbt = k / BK;
+    work = (long long)tiles * kbt;
+    long long g = work / MIN_KB_PER_CTA;
+    if (g < 1) g = 1;
+    G = int(g < grid ? g : grid);
   }
-  // unit -> (m, n, s); m varies fastest so concurrent CTAs share W tiles in L2
-  __device__ void decode(int u, int& m, int& nn, int& s, int& kb0, int& kb1) const {
-    m = u % mt;
-    int rest = u / mt;
-    s = rest % split;
-    nn = rest / split;
-    kb0 = (kb_total * s) / split;
-    kb1 = (kb_total * (s + 1)) / split;
+  __device__ long long bound(int c) const { return work * c / G; }
+  // Workspace slot of tile t when a CTA range starts strictly inside it (the
+  // first such CTA index, 1..G-1), else -1.
+  __device__ int split_slot(int t) const {
+    const long long lo = (long long)t * kbt, hi = lo + kbt;
+    long long c = ((lo + 1) * G + work - 1) / work;
+    while (c > 1 && bound(int(c - 1)) > lo) --c;
+    while (c < G && bound(int(c)) <= lo) ++c;
+    return (c < G && bound(int(c)) < hi) ? int(c) : -1;
   }
 };
 
@@ -177,7 +178,7 @@ template <int BN>
 __global__ void __launch_bounds__(THREADS, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                int Mbound, const int* __restrict__ dcount, int n, int k, GemmEpi ep,
-               float* __restrict__ ws, int* __restrict__ tickets, int ws_units) {
+               float* __restrict__ ws, int ws_units) {
   using TC = TileCfg<BN>;
   constexpr int STAGES = TC::STAGES, STAGE_B = TC::STAGE_B, TMEM_COLS = TC::TMEM_COLS;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -230,15 +231,20 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   const int M = live_count(dcount, Mbound, ep.err);
   Sched<BN> sc;
   sc.init(M, n, k, min(int(gridDim.x), ws_units));
+  const long long seg_beg = blockIdx.x < sc.G ? sc.bound(blockIdx.x) : 0;
+  const long long seg_end = blockIdx.x < sc.G ? sc.bound(blockIdx.x + 1) : 0;
 
   if (warp == 0) {
     // ------------------------------------------------------- TMA producer
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
-      for (int u = blockIdx.x; u < sc.units; u += gridDim.x) {
-        int m, nn, s, kb0, kb1;
-        sc.decode(u, m, nn, s, kb0, kb1);
+      for (long long cur = seg_beg; cur < seg_end;) {
+        const int t = int(cur / sc.kbt);
+        const int kb0 = int(cur - (long long)t * sc.kbt);
+        const int kb1 = int(min((long long)sc.kbt, kb0 + (seg_end - cur)));
+        cur += kb1 - kb0;
+        const int m = t % sc.mt, nn = t / sc.mt;
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(empty0 + 8 * stage, phase ^ 1, abort_flag)) goto timeout;
           mbar_expect_tx(full0 + 8 * stage, STAGE_A + STAGE_B);
@@ -255,9 +261,11 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       uint32_t phase = 0;
       int acc = 0;
       uint32_t acc_phase = 0;
-      for (int u = blockIdx.x; u < sc.units; u += gridDim.x) {
-        int m, nn, s, kb0, kb1;
-        sc.decode(u, m, nn, s, kb0, kb1);
+      for (long long cur = seg_beg; cur < seg_end;) {
+        const int t = int(cur / sc.kbt);
+        const int kb0 = int(cur - (long long)t * sc.kbt);
+        const int kb1 = int(min((long long)sc.kbt, kb0 + (seg_end - cur)));
+        cur += kb1 - kb0;
         if (!mbar_wait(tempty0 + 8 * acc, acc_phase ^ 1, abort_flag)) goto timeout;
         tc_fence_after();
         const uint32_t dtm = tmem_base + uint32_t(acc * (TMEM_COLS / 2));
@@ -281,25 +289,28 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     const int sp = warp & 3;  // TMEM lane sub-partition this warp may access
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int u = blockIdx.x; u < sc.units; u += gridDim.x) {
-      int m, nn, s, kb0, kb1;
-      sc.decode(u, m, nn, s, kb0, kb1);
+    for (long long cur = seg_beg; cur < seg_end;) {
+      const int t = int(cur / sc.kbt);
+      const int kb0 = int(cur - (long long)t * sc.kbt);
+      const int kb1 = int(min((long long)sc.kbt, kb0 + (seg_end - cur)));
+      cur += kb1 - kb0;
+      const int m = t % sc.mt, nn = t / sc.mt;
       if (!mbar_wait_warp(tfull0 + 8 * acc, acc_phase, abort_flag)) goto timeout;
       tc_fence_after();
       const int row = sp * 32 + lane;
       const int r = m * BM + row;
       const uint32_t tbase = tmem_base + uint32_t(acc * (TMEM_COLS / 2)) + (uint32_t(sp * 32) << 16);
-      const int tile = nn * sc.mt + m;
-      const bool additive = ep.mode == EPI_GATE_RES;
-      // split K, non-additive epilogue: partial sums reduce into a zeroed
-      // f32 tile; the last split reads it once, zeroes it and runs the epilogue
-      float* acc_row = ws + size_t(tile) * (BM * BN) + size_t(row) * BN;
+      // a whole tile, or any piece of a gated residual (its update is a sum),
+      // goes straight to the epilogue; a piece of another epilogue reduces
+      // into the tile's workspace slot and the finish kernel completes it
+      const bool direct = (kb0 == 0 && kb1 == sc.kbt) || ep.mode == EPI_GATE_RES;
+      float* acc_row = direct ? nullptr : ws + size_t(sc.split_slot(t)) * (BM * BN) + size_t(row) * BN;
 #pragma unroll 1
       for (int ch = 0; ch < BN / 32; ++ch) {
         float v[32];
         tmem_ld32(tbase + uint32_t(ch * 32), v);
-        if (sc.split == 1 || additive) {
-          if (r < M) epilogue32(ep, r, nn * BN + ch * 32, v, s == 0);
+        if (direct) {
+          if (r < M) epilogue32(ep, r, nn * BN + ch * 32, v, kb0 == 0);
         } else {
 #pragma unroll
           for (int i = 0; i < 8; ++i)
@@ -309,31 +320,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       tc_fence_before();
       mbar_arrive(tempty0 + 8 * acc);
       if (++acc == 2) { acc = 0; acc_phase ^= 1; }
-      if (sc.split > 1 && !additive) {
-        // per-row ticket: the last split to finish a row reduces it (no
-        // cross-warp barrier, no waiting); acq_rel orders the reductions
-        int* tk = tickets + size_t(tile) * BM + row;
-        const bool last = ticket_add(tk, 1) == sc.split - 1;
-        if (last) {
-          *tk = 0;  // re-armed for the next launch
-#pragma unroll 1
-          for (int ch = 0; ch < BN / 32; ch += 2) {
-            float v[64];
-            float4* p4 = reinterpret_cast<float4*>(acc_row + ch * 32);
-#pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              const float4 a = __ldcg(p4 + i);
-              v[4 * i] = a.x; v[4 * i + 1] = a.y; v[4 * i + 2] = a.z; v[4 * i + 3] = a.w;
-            }
-#pragma unroll
-            for (int i = 0; i < 16; ++i) __stcg(p4 + i, make_float4(0.f, 0.f, 0.f, 0.f));
-            if (r < M) {
-              epilogue32(ep, r, nn * BN + ch * 32, v, true);
-              epilogue32(ep, r, nn * BN + ch * 32 + 32, v + 32, true);
-            }
-          }
-        }
-      }
     }
   }
   goto done;
@@ -349,6 +335,41 @@ done:
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
                  "r"(TMEM_COLS)
                  : "memory");
+  }
+}
+
+// Completes the split tiles of a non-additive epilogue: reads the reduced
+// f32 tile from its workspace slot, zeroes it, applies the epilogue.  One
+// thread per (slot, row, 32-column chunk), grid-stride.
+template <int BN>
+__global__ void __launch_bounds__(256)
+gemm_finish_kernel(float* __restrict__ ws, int Mbound, const int* __restrict__ dcount, int n,
+                   int k, int grid, GemmEpi ep) {
+  pdl_wait();
+  pdl_trigger();
+  const int M = live_count(dcount, Mbound, ep.err);
+  Sched<BN> sc;
+  sc.init(M, n, k, grid);
+  constexpr int CH = BN / 32;
+  // split tiles = tiles whose first inner CTA boundary is c (c = 1 .. G-1)
+  const int items = (sc.G - 1) * BM * CH;
+  for (int it = blockIdx.x * 256 + threadIdx.x; it < items; it += gridDim.x * 256) {
+    const int c = 1 + it / (BM * CH);
+    const int rem = it - (c - 1) * (BM * CH);
+    const int row = rem / CH, ch = rem - (rem / CH) * CH;
+    const int t = int(sc.bound(c) / sc.kbt);
+    if (sc.split_slot(t) != c) continue;
+    float4* p4 = reinterpret_cast<float4*>(ws + size_t(c) * (BM * BN) + size_t(row) * BN + ch * 32);
+    float v[32];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float4 a = __ldcg(p4 + i);
+      v[4 * i] = a.x; v[4 * i + 1] = a.y; v[4 * i + 2] = a.z; v[4 * i + 3] = a.w;
+      __stcg(p4 + i, make_float4(0.f, 0.f, 0.f, 0.f));
+    }
+    const int m = t % sc.mt, nn = t / sc.mt;
+    const int r = m * BM + row;
+    if (r < M) epilogue32(ep, r, nn * BN + ch * 32, v, true);
   }
 }
 
@@ -429,15 +450,12 @@ int device_sms() {
   return sms[dev];
 }
 
-constexpr int MAX_TILES = 4096;  // tickets: MAX_TILES x BM rows
-
 }  // namespace
 
-cudaError_t gemm_scratch_shape(int* units, int* max_tiles, size_t* ws_floats) {
+cudaError_t gemm_scratch_shape(int* units, size_t* ws_floats) {
   const int sms = device_sms();
   if (!sms) return cudaErrorInvalidDevice;
   *units = sms;
-  *max_tiles = MAX_TILES;  // the context allocates MAX_TILES * 128 row tickets
   *ws_floats = size_t(sms) * BM * MAX_BN;
   return cudaSuccess;
 }
@@ -453,15 +471,24 @@ cudaError_t launch_gemm(const bf16* A, int lda, const bf16* W, int Mbound, const
   CUtensorMap ta, tb;
   if ((e = tensor_map(A, Mbound, k, lda, BM, &ta)) != cudaSuccess) return e;
   if ((e = tensor_map(W, n, k, k, BN, &tb)) != cudaSuccess) return e;
-  // split-K only runs when the tiles do not fill the grid; its tickets cover them
-  const int units = min(gs.units, gs.max_tiles);
+  // one workspace slot per CTA range boundary
+  const int grid = min(sms, gs.units);
   if (BN == 192)
-    RC_TRY(launch_k(gemm_tc_kernel<192>, dim3(sms), dim3(THREADS), TileCfg<192>::SMEM_BYTES, st, ta,
-                    tb, Mbound, dcount, n, k, ep, gs.ws, gs.tickets, units));
+    RC_TRY(launch_k(gemm_tc_kernel<192>, dim3(grid), dim3(THREADS), TileCfg<192>::SMEM_BYTES, st,
+                    ta, tb, Mbound, dcount, n, k, ep, gs.ws, grid));
   else
-    RC_TRY(launch_k(gemm_tc_kernel<128>, dim3(sms), dim3(THREADS), TileCfg<128>::SMEM_BYTES, st, ta,
-                    tb, Mbound, dcount, n, k, ep, gs.ws, gs.tickets, units));
+    RC_TRY(launch_k(gemm_tc_kernel<128>, dim3(grid), dim3(THREADS), TileCfg<128>::SMEM_BYTES, st,
+                    ta, tb, Mbound, dcount, n, k, ep, gs.ws, grid));
   count_launches(1);
+  if (ep.mode != EPI_GATE_RES) {
+    if (BN == 192)
+      RC_TRY(launch_k(gemm_finish_kernel<192>, dim3(2 * sms), dim3(256), 0, st, gs.ws, Mbound,
+                      dcount, n, k, grid, ep));
+    else
+      RC_TRY(launch_k(gemm_finish_kernel<128>, dim3(2 * sms), dim3(256), 0, st, gs.ws, Mbound,
+                      dcount, n, k, grid, ep));
+    count_launches(1);
+  }
   return cudaSuccess;
 }
 

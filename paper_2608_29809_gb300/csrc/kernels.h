@@ -86,17 +86,14 @@ struct GemmEpi {
   unsigned* err;
 };
 
-// Split-K scratch of one context: `units` f32 accumulator tiles (zero
-// between launches) and per-tile tickets (zero between launches).
+// Stream-K scratch of one context: `units` f32 accumulator tiles (zero
+// between launches), one per CTA range boundary.
 struct GemmScratch {
   float* ws;
-  int* tickets;
   int units;
-  int max_tiles;
 };
-// Partial tiles / tickets / workspace floats a context should allocate on the
-// current device.
-cudaError_t gemm_scratch_shape(int* units, int* max_tiles, size_t* ws_floats);
+// Workspace tiles and floats a context should allocate on the current device.
+cudaError_t gemm_scratch_shape(int* units, size_t* ws_floats);
 
 // C[M][n] = A[M][k] W[n][k]^T, epilogue `ep`.  M = *dcount if non-null (bounded
 // by Mbound) else Mbound.  n % 128 == 0, k % 64 == 0.  Launches on one
@@ -106,15 +103,12 @@ cudaError_t launch_gemm(const bf16* A, int lda, const bf16* W, int Mbound, const
 
 
 // ----------------------------------------------------------------- attention
-// Key-split scratch of one context: partial outputs and per-(query tile,
-// head) tickets (zero between launches).
+// Key-split scratch of one context: partial outputs of the key splits.
 struct AttnScratch {
   float* part;
   size_t part_floats;
-  int* tickets;
 };
 size_t attention_split_floats(int Nmax, int heads, int dh);
-int attention_tickets(int Nmax, int heads);
 
 // O[r][h*dh..] = softmax(Q_r K^T / sqrt(dh)) V per head, over Nk keys.
 // Q/O compact rows (r < D), K/V rows 0..Nk-1 with row stride ldkv.

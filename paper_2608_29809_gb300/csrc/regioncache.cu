@@ -73,8 +73,8 @@ struct rc_ctx {
   float* tb = nullptr;   // [6d]
   int* iota = nullptr;   // [N] identity row map (dense path)
   unsigned* err = nullptr;
-  rc::GemmScratch gs{};  // split-K partial tiles + tickets
-  rc::AttnScratch as{};  // key-split partial outputs + tickets
+  rc::GemmScratch gs{};  // stream-K workspace tiles
+  rc::AttnScratch as{};  // key-split partial outputs
   // timing probe
   int probe_which = RC_PROBE_OFF;
   int probe_n = 0;
@@ -148,7 +148,7 @@ void free_ctx(rc_ctx* c) {
   probe_free(c);
   void* ps[] = {c->xf,   c->xb,  c->ob,   c->q,        c->u,         c->fbuf,
                 c->h1,   c->temb, c->tb,  c->iota,     c->err,       c->gs.ws,
-                c->gs.tickets, c->as.part, c->as.tickets};
+                c->as.part};
   for (void* p : ps)
     if (p) cudaFree(p);
   delete c;
@@ -362,30 +362,21 @@ rc_status rc_create(const rc_dims* dims, rc_ctx** out) {
     return s;
   }
   {
-    int units = 0, max_tiles = 0;
+    int units = 0;
     size_t ws_floats = 0;
-    cudaError_t e0 = rc::gemm_scratch_shape(&units, &max_tiles, &ws_floats);
+    cudaError_t e0 = rc::gemm_scratch_shape(&units, &ws_floats);
     if (e0 != cudaSuccess) {
       free_ctx(c);
       return cuda_fail(e0, "rc_create: device query");
     }
     c->gs.units = units;
-    c->gs.max_tiles = max_tiles;
-    if ((s = dalloc(&c->gs.ws, ws_floats, "gemm split-K partials")) ||
-        (s = dalloc(&c->gs.tickets, size_t(max_tiles) * 128, "gemm tickets"))) {
-      free_ctx(c);
-      return s;
-    }
-    cudaMemset(c->gs.tickets, 0, sizeof(int) * size_t(max_tiles) * 128);
-    cudaMemset(c->gs.ws, 0, sizeof(float) * ws_floats);  // split-K accumulators start at zero
-    const int nt = rc::attention_tickets(int(N), D.heads);
     c->as.part_floats = rc::attention_split_floats(int(N), D.heads, dh);
-    if ((s = dalloc(&c->as.part, c->as.part_floats, "attn part")) ||
-        (s = dalloc(&c->as.tickets, size_t(nt) * 128, "attn tickets"))) {
+    if ((s = dalloc(&c->gs.ws, ws_floats, "gemm workspace")) ||
+        (s = dalloc(&c->as.part, c->as.part_floats, "attn part"))) {
       free_ctx(c);
       return s;
     }
-    cudaMemset(c->as.tickets, 0, sizeof(int) * size_t(nt) * 128);
+    cudaMemset(c->gs.ws, 0, sizeof(float) * ws_floats);  // workspace tiles start at zero
   }
   iota_kernel<<<int((N + 255) / 256), 256>>>(c->iota, int(N));
   rc::count_launches(1);

@@ -12,6 +12,28 @@ namespace rc {
 
 static inline int cdiv(int a, int b) { return (a + b - 1) / b; }
 
+int device_sm_count() {
+  static int sms[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 128;
+  if (!sms[dev]) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v <= 0)
+      v = 128;
+    sms[dev] = v;
+  }
+  return sms[dev];
+}
+
+// Grid of a row kernel: enough CTAs for the row bound, at most `per_sm` per
+// SM; the kernels loop over rows, so a device-side row count below the bound
+// costs no empty CTAs.
+static inline int row_grid(int rows_bound, int rows_per_cta, int per_sm) {
+  const int want = cdiv(rows_bound, rows_per_cta);
+  const int cap = per_sm * device_sm_count();
+  return want < cap ? want : cap;
+}
+
 // ============================================================ localisation
 // Workspace: abar f32 [n_delta][N] | part f32x2 [nblk][n_delta] | union u8 [N]
 // | cnt int [nblk].  One thread per token, MASK_ROWS tokens per CTA.
@@ -203,9 +225,8 @@ ln_mod_kernel(const float* __restrict__ x, int ldx, const float* __restrict__ ta
   pdl_trigger();
   const int D = live_count(dcount, Dbound, err);
   const int lane = threadIdx.x & 31;
-  const int r = blockIdx.x * LN_WARPS + (threadIdx.x >> 5);
-  if (r >= D) return;
   const int nv = d / 128;
+  for (int r = blockIdx.x * LN_WARPS + (threadIdx.x >> 5); r < D; r += gridDim.x * LN_WARPS) {
   const float4* xr = reinterpret_cast<const float4*>(x + size_t(r) * ldx);
   float4 v[LN_MAXV];
   float s = 0.f;
@@ -257,6 +278,7 @@ ln_mod_kernel(const float* __restrict__ x, int ldx, const float* __restrict__ ta
       float y3 = (v[k].w - mean) * rstd * (1.f + sc.w) + sh.w;
       orow[lane + 32 * k] = make_uint2(pack_bf16x2(y0, y1), pack_bf16x2(y2, y3));
     }
+  }
 }
 
 cudaError_t launch_ln_mod(const float* x, int ldx, const float* tab_sh, const float* tb_sh,
@@ -264,7 +286,7 @@ cudaError_t launch_ln_mod(const float* x, int ldx, const float* tab_sh, const fl
                           int Dbound, const int* dcount, int d, bf16* hprev, const int* idx,
                           int n_tokens, unsigned* err, cudaStream_t st) {
   if (Dbound <= 0) return cudaSuccess;
-  RC_TRY(launch_k(ln_mod_kernel, dim3(cdiv(Dbound, LN_WARPS)), dim3(LN_WARPS * 32), 0, st, x, ldx,
+  RC_TRY(launch_k(ln_mod_kernel, dim3(row_grid(Dbound, LN_WARPS, 4)), dim3(LN_WARPS * 32), 0, st, x, ldx,
                   tab_sh, tb_sh, tab_sc, tb_sc, out, ldo, Dbound, dcount, d, hprev, idx, n_tokens,
                   err));
   count_launches(1);
@@ -278,59 +300,85 @@ cast_rows_kernel(const float* __restrict__ x, int ldx, bf16* __restrict__ out, i
   pdl_wait();
   pdl_trigger();
   const int D = live_count(dcount, Dbound, err);
-  const int r = blockIdx.x * LN_WARPS + (threadIdx.x >> 5);
-  if (r >= D) return;
-  const float4* xr = reinterpret_cast<const float4*>(x + size_t(r) * ldx);
-  uint2* orow = reinterpret_cast<uint2*>(out + size_t(r) * ldo);
-  for (int c = threadIdx.x & 31; c < d / 4; c += 32) {
-    const float4 v = xr[c];
-    orow[c] = make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
+  for (int r = blockIdx.x * LN_WARPS + (threadIdx.x >> 5); r < D; r += gridDim.x * LN_WARPS) {
+    const float4* xr = reinterpret_cast<const float4*>(x + size_t(r) * ldx);
+    uint2* orow = reinterpret_cast<uint2*>(out + size_t(r) * ldo);
+    for (int c = threadIdx.x & 31; c < d / 4; c += 32) {
+      const float4 v = xr[c];
+      orow[c] = make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
+    }
   }
 }
 
 cudaError_t launch_cast_rows(const float* x, int ldx, bf16* out, int ldo, int Dbound,
                              const int* dcount, int d, unsigned* err, cudaStream_t st) {
   if (Dbound <= 0) return cudaSuccess;
-  RC_TRY(launch_k(cast_rows_kernel, dim3(cdiv(Dbound, LN_WARPS)), dim3(LN_WARPS * 32), 0, st, x,
+  RC_TRY(launch_k(cast_rows_kernel, dim3(row_grid(Dbound, LN_WARPS, 4)), dim3(LN_WARPS * 32), 0, st, x,
                   ldx, out, ldo, Dbound, dcount, d, err));
   count_launches(1);
   return cudaSuccess;
 }
 
 // ============================================================ patch embed
-// One CTA per dirty token: gathers its p x p x C latent patch (ordered
-// channel, py, px) and applies the linear patch embedding + bias + position.
-__global__ void __launch_bounds__(256)
+// x_r = W_e patch(idx[r]) + b_e + pos[idx[r]], the patch vector ordered
+// (channel, py, px).  W_e (<= 16 inputs per output) sits in shared memory;
+// one warp per dirty token, grid-stride over the tokens.
+constexpr int PE_WARPS = 8;
+constexpr int PE_MAXD = 1536;
+
+__global__ void __launch_bounds__(PE_WARPS * 32)
 patch_embed_kernel(const float* __restrict__ latent, int gh, int gw, int p, int C,
                    const bf16* __restrict__ We, const float* __restrict__ be,
                    const float* __restrict__ pos, const int* __restrict__ idx, int Dbound,
                    const int* __restrict__ dcount, float* __restrict__ xf, int d, unsigned* err) {
   pdl_wait();
   pdl_trigger();
-  __shared__ float patch[64];
-  const int D = live_count(dcount, Dbound, err);
-  const int r = blockIdx.x;
-  if (r >= D) return;
-  const int N = gh * gw;
-  int i = idx ? idx[r] : r;
-  if (i < 0 || i >= N) {
-    if (threadIdx.x == 0) atomicOr(err, DEVERR_INDEX);
-    return;
-  }
-  const int P = C * p * p;
-  const int gy = i / gw, gx = i - gy * gw;
-  const int W = gw * p, H = gh * p;
-  if (threadIdx.x < P) {
-    const int c = threadIdx.x / (p * p), rem = threadIdx.x - c * p * p;
-    const int py = rem / p, px = rem - py * p;
-    patch[threadIdx.x] = latent[(size_t(c) * H + gy * p + py) * W + gx * p + px];
+  extern __shared__ __align__(16) uint8_t pe_smem[];
+  bf16* s_w = reinterpret_cast<bf16*>(pe_smem);  // [d][16], zero beyond P
+  const int P = C * p * p;                         // <= 16
+  for (int e = threadIdx.x; e < d * 16; e += blockDim.x) {
+    const int o = e >> 4, k = e & 15;
+    s_w[e] = k < P ? We[size_t(o) * P + k] : f2bf(0.f);
   }
   __syncthreads();
-  for (int o = threadIdx.x; o < d; o += blockDim.x) {
-    float acc = 0.f;
-    const bf16* w = We + size_t(o) * P;
-    for (int k = 0; k < P; ++k) acc = fmaf(bf2f(w[k]), patch[k], acc);
-    xf[size_t(r) * d + o] = acc + be[o] + pos[size_t(i) * d + o];
+  const int D = live_count(dcount, Dbound, err);
+  const int lane = threadIdx.x & 31;
+  const int N = gh * gw, W = gw * p, H = gh * p;
+  for (int r = blockIdx.x * PE_WARPS + (threadIdx.x >> 5); r < D; r += gridDim.x * PE_WARPS) {
+    const int i = idx ? idx[r] : r;
+    if (i < 0 || i >= N) {
+      if (lane == 0) atomicOr(err, DEVERR_INDEX);
+      continue;
+    }
+    const int gy = i / gw, gx = i - gy * gw;
+    float pv = 0.f;
+    if (lane < P) {
+      const int c = lane / (p * p), rem = lane - c * p * p;
+      const int py = rem / p, px = rem - py * p;
+      pv = latent[(size_t(c) * H + gy * p + py) * W + gx * p + px];
+    }
+    float patch[16];
+#pragma unroll
+    for (int k = 0; k < 16; ++k) patch[k] = __shfl_sync(0xffffffffu, pv, k);
+    for (int o = lane; o < d; o += 32) {
+      const uint4* w4 = reinterpret_cast<const uint4*>(s_w + o * 16);
+      float acc = 0.f;
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        const uint4 w = w4[q];
+        const float2 a = unpack_bf16x2(w.x), b = unpack_bf16x2(w.y);
+        const float2 c2 = unpack_bf16x2(w.z), e2 = unpack_bf16x2(w.w);
+        acc = fmaf(a.x, patch[8 * q], acc);
+        acc = fmaf(a.y, patch[8 * q + 1], acc);
+        acc = fmaf(b.x, patch[8 * q + 2], acc);
+        acc = fmaf(b.y, patch[8 * q + 3], acc);
+        acc = fmaf(c2.x, patch[8 * q + 4], acc);
+        acc = fmaf(c2.y, patch[8 * q + 5], acc);
+        acc = fmaf(e2.x, patch[8 * q + 6], acc);
+        acc = fmaf(e2.y, patch[8 * q + 7], acc);
+      }
+      xf[size_t(r) * d + o] = acc + be[o] + pos[size_t(i) * d + o];
+    }
   }
 }
 
@@ -339,8 +387,10 @@ cudaError_t launch_patch_embed(const float* latent, int gh, int gw, int p, int C
                                const int* idx, int Dbound, const int* dcount, float* xf, int d,
                                unsigned* err, cudaStream_t st) {
   if (Dbound <= 0) return cudaSuccess;
-  RC_TRY(launch_k(patch_embed_kernel, dim3(Dbound), dim3(256), 0, st, latent, gh, gw, p, C, We, be,
-                  pos, idx, Dbound, dcount, xf, d, err));
+  if (d > PE_MAXD || C * p * p > 16) return cudaErrorInvalidValue;
+  RC_TRY(launch_k(patch_embed_kernel, dim3(row_grid(Dbound, PE_WARPS, 1)), dim3(PE_WARPS * 32),
+                  size_t(d) * 16 * sizeof(bf16), st, latent, gh, gw, p, C, We, be, pos, idx, Dbound,
+                  dcount, xf, d, err));
   count_launches(1);
   return cudaSuccess;
 }
@@ -538,44 +588,49 @@ cudaError_t launch_final_ddim(const bf16* H, const float* temb, const float* tab
 }
 
 // ======================================================= gather / scatter
-__global__ void __launch_bounds__(256)
+// One warp per row, grid-stride over the rows.
+constexpr int RW_WARPS = 8;
+
+__global__ void __launch_bounds__(RW_WARPS * 32)
 rows_f32_kernel(const float* __restrict__ src, float* __restrict__ dst,
                 const int* __restrict__ idx, int Dbound, const int* __restrict__ dcount, int d,
                 int N, int scatter, unsigned* err) {
   pdl_wait();
   pdl_trigger();
   const int D = live_count(dcount, Dbound, err);
-  const int r = blockIdx.x;
-  if (r >= D) return;
-  const int i = idx[r];
-  if (i < 0 || i >= N) {
-    if (threadIdx.x == 0) atomicOr(err, DEVERR_INDEX);
-    return;
+  const int lane = threadIdx.x & 31;
+  for (int r = blockIdx.x * RW_WARPS + (threadIdx.x >> 5); r < D; r += gridDim.x * RW_WARPS) {
+    const int i = idx[r];
+    if (i < 0 || i >= N) {
+      if (lane == 0) atomicOr(err, DEVERR_INDEX);
+      continue;
+    }
+    const float4* s4 = reinterpret_cast<const float4*>(src + size_t(scatter ? r : i) * d);
+    float4* t4 = reinterpret_cast<float4*>(dst + size_t(scatter ? i : r) * d);
+    for (int c = lane; c < d / 4; c += 32) t4[c] = s4[c];
   }
-  const float4* s = reinterpret_cast<const float4*>(src + size_t(scatter ? r : i) * d);
-  float4* t = reinterpret_cast<float4*>(dst + size_t(scatter ? i : r) * d);
-  for (int c = threadIdx.x; c < d / 4; c += blockDim.x) t[c] = s[c];
 }
 
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(RW_WARPS * 32)
 scatter_bf16_kernel(const float* __restrict__ src, bf16* __restrict__ dst,
                     const int* __restrict__ idx, int Dbound, const int* __restrict__ dcount,
                     int d, int N, unsigned* err) {
   pdl_wait();
   pdl_trigger();
   const int D = live_count(dcount, Dbound, err);
-  const int r = blockIdx.x;
-  if (r >= D) return;
-  const int i = idx ? idx[r] : r;
-  if (i < 0 || i >= N) {
-    if (threadIdx.x == 0) atomicOr(err, DEVERR_INDEX);
-    return;
-  }
-  const float4* s = reinterpret_cast<const float4*>(src + size_t(r) * d);
-  uint2* t = reinterpret_cast<uint2*>(dst + size_t(i) * d);
-  for (int c = threadIdx.x; c < d / 4; c += blockDim.x) {
-    float4 v = s[c];
-    t[c] = make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
+  const int lane = threadIdx.x & 31;
+  for (int r = blockIdx.x * RW_WARPS + (threadIdx.x >> 5); r < D; r += gridDim.x * RW_WARPS) {
+    const int i = idx ? idx[r] : r;
+    if (i < 0 || i >= N) {
+      if (lane == 0) atomicOr(err, DEVERR_INDEX);
+      continue;
+    }
+    const float4* s4 = reinterpret_cast<const float4*>(src + size_t(r) * d);
+    uint2* t2 = reinterpret_cast<uint2*>(dst + size_t(i) * d);
+    for (int c = lane; c < d / 4; c += 32) {
+      const float4 v = s4[c];
+      t2[c] = make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
+    }
   }
 }
 
@@ -583,8 +638,8 @@ cudaError_t launch_rows_f32(const float* src, float* dst, const int* idx, int Db
                             const int* dcount, int d, int N, bool scatter, unsigned* err,
                             cudaStream_t st) {
   if (Dbound <= 0) return cudaSuccess;
-  RC_TRY(launch_k(rows_f32_kernel, dim3(Dbound), dim3(256), 0, st, src, dst, idx, Dbound, dcount,
-                  d, N, scatter ? 1 : 0, err));
+  RC_TRY(launch_k(rows_f32_kernel, dim3(row_grid(Dbound, RW_WARPS, 4)), dim3(RW_WARPS * 32), 0, st,
+                  src, dst, idx, Dbound, dcount, d, N, scatter ? 1 : 0, err));
   count_launches(1);
   return cudaSuccess;
 }
@@ -592,8 +647,8 @@ cudaError_t launch_rows_f32(const float* src, float* dst, const int* idx, int Db
 cudaError_t launch_scatter_bf16(const float* src, bf16* dst, const int* idx, int Dbound,
                                 const int* dcount, int d, int N, unsigned* err, cudaStream_t st) {
   if (Dbound <= 0) return cudaSuccess;
-  RC_TRY(launch_k(scatter_bf16_kernel, dim3(Dbound), dim3(256), 0, st, src, dst, idx, Dbound,
-                  dcount, d, N, err));
+  RC_TRY(launch_k(scatter_bf16_kernel, dim3(row_grid(Dbound, RW_WARPS, 4)), dim3(RW_WARPS * 32), 0,
+                  st, src, dst, idx, Dbound, dcount, d, N, err));
   count_launches(1);
   return cudaSuccess;
 }
