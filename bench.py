@@ -252,14 +252,15 @@ def run_ours(args, world, rank, local):
     # launching stream; they serialise the launches they bracket, so these
     # passes are kept out of the headline)
     def probe(which, per_step):
-        R.rc_probe_enable(wl.model.ctx, which, K * d.layers * per_step)
+        cap = K * d.layers * per_step
+        R.rc_probe_enable(wl.model.ctx, which, cap)
         timed(lambda i: wl.step(i, HEADLINE), K, 0, 1)
-        out = R.rc_probe_read(wl.model.ctx)
+        each = R.rc_probe_read_each(wl.model.ctx, cap)
         R.rc_probe_enable(wl.model.ctx, R.RC_PROBE_OFF, 0)
-        return out
+        return sum(each), len(each), each
 
-    gemm_ms, gemm_n = probe(R.RC_PROBE_GEMM, 6)
-    att_ms, att_n = probe(R.RC_PROBE_ATTENTION, 2)
+    gemm_ms, gemm_n, gemm_each = probe(R.RC_PROBE_GEMM, 6)
+    att_ms, att_n, att_each = probe(R.RC_PROBE_ATTENTION, 2)
 
     # sweep and dense baseline
     sweep, dirty = {}, {}
@@ -315,6 +316,25 @@ def run_ours(args, world, rank, local):
     roof_att = {"bound": "tensor", "achieved": round(att_tflops, 2), "peak": peak,
                 "unit": "TFLOP/s", "frac": round(att_tflops / peak, 4), "launches": att_n,
                 "avg_launch_ms": round(att_ms / max(att_n, 1), 5)}
+    # per-launch breakdown: launches come in block order (GEMMs: QKV, out,
+    # cross-q, cross-out, fc1, fc2; attention: self, cross)
+    h, F = d.hidden, d.mlp
+    gemm_shapes = [("qkv", 3 * h, h), ("out", h, h), ("cross_q", h, h), ("cross_out", h, h),
+                   ("fc1", F, h), ("fc2", h, F)]
+    per_gemm = {}
+    for j, (name, n_, k_) in enumerate(gemm_shapes):
+        ts = gemm_each[j::6]
+        us = 1e3 * sum(ts) / max(len(ts), 1)
+        per_gemm[name] = {"shape": [D, n_, k_], "avg_us": round(us, 2),
+                          "tflops": round(2.0 * D * n_ * k_ / (us * 1e-6) / 1e12, 1)}
+    per_attn = {}
+    for j, (name, nk) in enumerate([("self", d.tokens), ("cross", d.text_len)]):
+        ts = att_each[j::2]
+        us = 1e3 * sum(ts) / max(len(ts), 1)
+        per_attn[name] = {"queries": D, "keys": nk, "avg_us": round(us, 2),
+                          "tflops": round(4.0 * D * nk * h / (us * 1e-6) / 1e12, 1)}
+    roofline["per_gemm"] = per_gemm
+    roof_att["per_launch"] = per_attn
     out = {
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
         "steps": K, "warmup": W, "ms_per_step": round(ms_max / K, 4), "higher_is_better": True,

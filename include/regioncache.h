@@ -286,12 +286,16 @@ rc_status rc_sync(rc_ctx* ctx, rc_stream stream);
  * tensor-core GEMM of a block; RC_PROBE_ATTENTION: every attention launch);
  * which = RC_PROBE_OFF disables it.  rc_probe_read waits for the recorded
  * events and returns the summed device time (ms) and the number of launches
- * recorded, then rearms the ring.  Errors: RC_ERR_INVALID_ARG, RC_ERR_CUDA. */
+ * recorded, then rearms the ring.  rc_probe_read_each does the same but
+ * writes each launch's device time (ms, launch order) to the host array
+ * ms_out[0 .. capacity) (caller-owned; launches beyond capacity are counted
+ * in *launches but not written).  Errors: RC_ERR_INVALID_ARG, RC_ERR_CUDA. */
 #define RC_PROBE_OFF 0
 #define RC_PROBE_GEMM 1
 #define RC_PROBE_ATTENTION 2
 rc_status rc_probe_enable(rc_ctx* ctx, int which, int capacity);
 rc_status rc_probe_read(rc_ctx* ctx, double* total_ms, int* launches);
+rc_status rc_probe_read_each(rc_ctx* ctx, float* ms_out, int capacity, int* launches);
 
 /* Number of kernels this library has launched in the calling process. */
 uint64_t rc_launch_count(void);

@@ -55,16 +55,6 @@ __device__ __forceinline__ int live_count(const int* dcount, int bound, unsigned
   return d;
 }
 
-// Split-reduction ticket: atomic add with acquire-release semantics at GPU
-// scope.  The release half publishes this thread's earlier stores of its
-// partial result; the acquire half lets the last arriver read every other
-// split's partial after the ticket, without separate fences.
-__device__ __forceinline__ int ticket_add(int* p, int v) {
-  int old;
-  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
-  return old;
-}
-
 // Programmatic dependent launch.  Every kernel of this library is launched
 // with programmatic stream serialisation: it may start while its predecessor
 // in the stream is still running, does its private set-up, then waits

@@ -7,18 +7,19 @@
 //
 // C[M][n] = A[M][k] W[n][k]^T, A and W K-major bf16, f32 accumulation.
 // M (the dirty-token count) may live on the device: every CTA reads it and
-// derives a stream-K schedule (equal shares of all tiles' k-blocks, so small
-// and ragged tile counts still fill the GPU).  The gated residual
+// derives the schedule: whole tiles in full waves.  The gated residual
 // (x += gate (C + b)) is written as vector reductions into x, so pieces of a
-// tile simply add up; for the other epilogues the pieces of a split tile
-// reduce into a zeroed f32 workspace tile and a small finish kernel, launched
-// right after, applies the epilogue and zeroes the tile again.
+// tile simply add up: for it a small last wave is instead cut into equal
+// k-block ranges (stream-K) so ragged tile counts still fill the GPU.  The
+// other epilogues always see whole tiles (splitting them would need a
+// workspace round trip that costs more than the idle SMs).
 //
 // CTA = 6 warps: warp 0 issues TMA loads, warp 1 owns TMEM and issues the
 // MMAs (one thread), warps 2..5 drain the accumulator (one TMEM lane = one
-// output row per thread).  Two TMEM accumulators (tiles of 128 x 192, or
-// 128 x 128 when 192 does not divide n) let the epilogue of one tile overlap
-// the main loop of the next.
+// output row per thread, re-staged through shared memory so that global
+// writes are whole row pieces).  Two TMEM accumulators (tiles of 128 x 192,
+// or 128 x 128 when 192 does not divide n) let the epilogue of one tile
+// overlap the main loop of the next.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -39,7 +40,8 @@ constexpr int BM = 128, BK = 64;
 constexpr int THREADS = 192;
 constexpr int STAGE_A = BM * BK * 2;   // bytes
 constexpr int MIN_KB_PER_CTA = 4;
-constexpr int MAX_BN = 192;
+constexpr int STAGING_WARP = 32 * 128;  // epilogue staging: 32 rows of 128 B per warp
+constexpr int STAGING_BYTES = 4 * STAGING_WARP;
 
 // Tile width BN (output features per tile): 192 when it divides n (every
 // PixArt-alpha width: 1152, 2304, 3456, 4608), else 128.
@@ -48,7 +50,8 @@ struct TileCfg {
   static constexpr int STAGE_B = BN * BK * 2;
   static constexpr int STAGES = (200 * 1024) / (STAGE_A + STAGE_B);  // 6 for 128, 5 for 192
   static constexpr int TMEM_COLS = (2 * BN <= 256) ? 256 : 512;     // two accumulators
-  static constexpr size_t SMEM_BYTES = size_t(STAGES) * (STAGE_A + STAGE_B) + 1024 + 256;
+  static constexpr size_t SMEM_BYTES =
+      size_t(STAGES) * (STAGE_A + STAGE_B) + STAGING_BYTES + 1024 + 256;
   // Instruction descriptor, kind::f16: D f32, A and B bf16, both K-major,
   // N >> 3 at bit 17, M >> 4 at bit 24.
   static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
@@ -63,131 +66,199 @@ __device__ __forceinline__ void load32(const float* p, float* v) {
     v[4 * i] = a.x; v[4 * i + 1] = a.y; v[4 * i + 2] = a.z; v[4 * i + 3] = a.w;
   }
 }
-__device__ __forceinline__ void store32_bf16(bf16* p, const float* v) {
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    uint4 u;
-    u.x = pack_bf16x2(v[8 * i + 0], v[8 * i + 1]);
-    u.y = pack_bf16x2(v[8 * i + 2], v[8 * i + 3]);
-    u.z = pack_bf16x2(v[8 * i + 4], v[8 * i + 5]);
-    u.w = pack_bf16x2(v[8 * i + 6], v[8 * i + 7]);
-    reinterpret_cast<uint4*>(p)[i] = u;
-  }
-}
-
 __device__ __forceinline__ void red_add_v4(float* p, float a, float b, float c, float d) {
   asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(p), "f"(a), "f"(b), "f"(c),
                "f"(d)
                : "memory");
 }
 
-// Applies the epilogue to columns c0 .. c0+31 of output row r (r < M).  The
-// bias is added when with_bias (the gated residual adds it from split 0 only:
-// its update is a sum over splits).
-__device__ __forceinline__ void epilogue32(const GemmEpi& ep, int r, int c0, float* v,
-                                           bool with_bias) {
+// Epilogue values of columns c0 .. c0+31 of one output row: bias (when
+// with_bias: a split gated residual adds it with its first piece only, its
+// update being a sum over pieces), tanh-GELU, gate.
+__device__ __forceinline__ void epilogue_values(const GemmEpi& ep, int c0, float* v,
+                                                bool with_bias) {
   if (ep.bias && with_bias) {
     float b[32];
     load32(ep.bias + c0, b);
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] += b[i];
   }
-  switch (ep.mode) {
-    case EPI_F32: {
-      float4* o = reinterpret_cast<float4*>(ep.out_f + size_t(r) * ep.ld_out + c0);
+  if (ep.mode == EPI_GELU_BF16) {
 #pragma unroll
-      for (int i = 0; i < 8; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-      break;
+    for (int i = 0; i < 32; ++i) v[i] = gelu_tanh(v[i]);
+  } else if (ep.mode == EPI_GATE_RES && ep.gate_tab) {
+    float g[32];
+    load32(ep.gate_tab + c0, g);
+    if (ep.gate_tb) {
+      float g2[32];
+      load32(ep.gate_tb + c0, g2);
+#pragma unroll
+      for (int i = 0; i < 32; ++i) g[i] += g2[i];
     }
-    case EPI_BIAS_BF16:
-      store32_bf16(ep.out_bf + size_t(r) * ep.ld_out + c0, v);
-      break;
-    case EPI_GELU_BF16:
 #pragma unroll
-      for (int i = 0; i < 32; ++i) v[i] = gelu_tanh(v[i]);
-      store32_bf16(ep.out_bf + size_t(r) * ep.ld_out + c0, v);
-      break;
-    case EPI_GATE_RES: {
-      // x += gate (acc + b), as vector reductions: no read of x, and the
-      // partial sums of a split K add up in place
-      if (ep.gate_tab) {
-        float g[32];
-        load32(ep.gate_tab + c0, g);
-        if (ep.gate_tb) {
-          float g2[32];
-          load32(ep.gate_tb + c0, g2);
-#pragma unroll
-          for (int i = 0; i < 32; ++i) g[i] += g2[i];
-        }
-#pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] *= g[i];
-      }
-      float* xp = ep.xf + size_t(r) * ep.ld_xf + c0;
-#pragma unroll
-      for (int i = 0; i < 8; ++i) red_add_v4(xp + 4 * i, v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-      break;
-    }
-    case EPI_QKV: {
-      const int part = c0 / ep.dsplit;
-      const int cc = c0 - part * ep.dsplit;
-      if (part == 0) {
-        store32_bf16(ep.out_bf + size_t(r) * ep.ld_out + cc, v);
-      } else {
-        const int tok = ep.idx ? ep.idx[r] : r;
-        if (tok >= 0 && tok < ep.n_tokens)
-          store32_bf16((part == 1 ? ep.kc : ep.vc) + size_t(tok) * ep.ld_kv + cc, v);
-        else
-          atomicOr(ep.err, DEVERR_INDEX);
-      }
-      break;
-    }
+    for (int i = 0; i < 32; ++i) v[i] *= g[i];
   }
 }
 
-// Stream-K schedule: the tiles' k-blocks are laid end to end (tile t =
-// nn * mt + m, m fastest so neighbouring CTAs share weight tiles in L2) and
-// CTA c takes the contiguous range [bound(c), bound(c+1)); a tile cut by a
-// range boundary is "split".  At least MIN_KB_PER_CTA k-blocks per CTA.
+// Destination of columns c0 .. c0+31 of output row r, or null when the row is
+// beyond the live count (or its token index is bad: QKV raises DEVERR_INDEX).
+// tok = idx[r] for the QKV epilogue, loaded once per tile.
+__device__ __forceinline__ char* chunk_dst(const GemmEpi& ep, int r, int M, int tok, int c0) {
+  if (r >= M) return nullptr;
+  switch (ep.mode) {
+    case EPI_F32:
+      return reinterpret_cast<char*>(ep.out_f + size_t(r) * ep.ld_out + c0);
+    case EPI_GATE_RES:
+      return reinterpret_cast<char*>(ep.xf + size_t(r) * ep.ld_xf + c0);
+    case EPI_QKV: {
+      const int part = c0 / ep.dsplit;
+      const int cc = c0 - part * ep.dsplit;
+      if (part == 0) return reinterpret_cast<char*>(ep.out_bf + size_t(r) * ep.ld_out + cc);
+      if (tok < 0 || tok >= ep.n_tokens) {
+        atomicOr(ep.err, DEVERR_INDEX);
+        return nullptr;
+      }
+      return reinterpret_cast<char*>((part == 1 ? ep.kc : ep.vc) + size_t(tok) * ep.ld_kv + cc);
+    }
+    default:
+      return reinterpret_cast<char*>(ep.out_bf + size_t(r) * ep.ld_out + c0);
+  }
+}
+
+// Writes one warp's 32 x 32 chunk (lane = row, v = its 32 columns) to global
+// memory with coalesced accesses: each lane parks its row in the warp's 4 KB
+// staging area, then groups of lanes write whole 128-byte (f32) or 64-byte
+// (bf16) row pieces.  Staging is XOR-swizzled in 16-byte units so that both
+// the row-per-lane writes and the piece-per-lane-group reads are free of bank
+// conflicts.  The gated residual goes out as vector reductions (x += value).
+__device__ __forceinline__ void store_chunk(int mode, uint8_t* stg, int lane, const float* v,
+                                            char* dst) {
+  const uint32_t s0 = saddr(stg);
+  if (mode == EPI_F32 || mode == EPI_GATE_RES) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(
+                       s0 + lane * 128 + 16 * (j ^ (lane & 7))),
+                   "f"(v[4 * j]), "f"(v[4 * j + 1]), "f"(v[4 * j + 2]), "f"(v[4 * j + 3])
+                   : "memory");
+    __syncwarp();
+    const int j = lane & 7;
+#pragma unroll
+    for (int pass = 0; pass < 8; ++pass) {
+      const int row = pass * 4 + (lane >> 3);
+      float4 x;
+      asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                   : "=f"(x.x), "=f"(x.y), "=f"(x.z), "=f"(x.w)
+                   : "r"(s0 + row * 128 + 16 * (j ^ (row & 7)))
+                   : "memory");
+      char* d = reinterpret_cast<char*>(
+          __shfl_sync(0xffffffffu, reinterpret_cast<unsigned long long>(dst), row));
+      if (d) {
+        float* q = reinterpret_cast<float*>(d) + 4 * j;
+        if (mode == EPI_GATE_RES)
+          red_add_v4(q, x.x, x.y, x.z, x.w);
+        else
+          *reinterpret_cast<float4*>(q) = x;
+      }
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                       s0 + lane * 64 + 16 * (j ^ ((lane >> 1) & 3))),
+                   "r"(pack_bf16x2(v[8 * j + 0], v[8 * j + 1])),
+                   "r"(pack_bf16x2(v[8 * j + 2], v[8 * j + 3])),
+                   "r"(pack_bf16x2(v[8 * j + 4], v[8 * j + 5])),
+                   "r"(pack_bf16x2(v[8 * j + 6], v[8 * j + 7]))
+                   : "memory");
+    __syncwarp();
+    const int j = lane & 3;
+#pragma unroll
+    for (int pass = 0; pass < 4; ++pass) {
+      const int row = pass * 8 + (lane >> 2);
+      uint4 x;
+      asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                   : "=r"(x.x), "=r"(x.y), "=r"(x.z), "=r"(x.w)
+                   : "r"(s0 + row * 64 + 16 * (j ^ ((row >> 1) & 3)))
+                   : "memory");
+      char* d = reinterpret_cast<char*>(
+          __shfl_sync(0xffffffffu, reinterpret_cast<unsigned long long>(dst), row));
+      if (d) reinterpret_cast<uint4*>(d)[j] = x;
+    }
+  }
+  __syncwarp();  // the staging area is rewritten by the next chunk
+}
+
+// Schedule.  Tiles (t = nn * mt + m, m fastest so neighbouring CTAs share
+// weight tiles in L2) go whole to CTA t mod G in full waves.  For an additive
+// epilogue, when the last wave would leave more than half the CTAs idle, its
+// R remainder tiles are instead laid end to end by k-block and cut into G_r
+// equal ranges (stream-K, at least MIN_KB_PER_CTA k-blocks each).
 template <int BN>
 struct Sched {
-  int mt, nt, tiles, kbt, G;
-  long long work;
-  __device__ void init(int M, int n, int k, int grid) {
+  int mt, nt, tiles, kbt, G, whole, Gr;
+  long long Wr;
+  __device__ void init(int M, int n, int k, int grid, bool additive) {
     mt = (M + BM - 1) / BM;
     nt = n / BN;
     tiles = mt * nt;
     kbt = k / BK;
-    work = (long long)tiles * kbt;
-    long long g = work / MIN_KB_PER_CTA;
+    G = grid;
+    const int R = tiles % G;
+    const bool split = additive && R > 0 && 2 * R <= G && kbt >= 2 * MIN_KB_PER_CTA;
+    whole = split ? tiles - R : tiles;
+    Wr = split ? (long long)R * kbt : 0;
+    long long g = Wr / MIN_KB_PER_CTA;
     if (g < 1) g = 1;
-    G = int(g < grid ? g : grid);
+    Gr = split ? int(g < G ? g : G) : 0;
   }
-  __device__ long long bound(int c) const { return work * c / G; }
-  // Workspace slot of tile t when a CTA range starts strictly inside it (the
-  // first such CTA index, 1..G-1), else -1.
-  __device__ int split_slot(int t) const {
-    const long long lo = (long long)t * kbt, hi = lo + kbt;
-    long long c = ((lo + 1) * G + work - 1) / work;
-    while (c > 1 && bound(int(c - 1)) > lo) --c;
-    while (c < G && bound(int(c)) <= lo) ++c;
-    return (c < G && bound(int(c)) < hi) ? int(c) : -1;
+  __device__ long long bound(int c) const { return Wr * c / Gr; }
+};
+
+// The segments (tile, k-blocks [kb0, kb1)) of one CTA, in order.
+template <int BN>
+struct Segs {
+  const Sched<BN>* sc;
+  int t_next;
+  long long cur, end;
+  __device__ void init(const Sched<BN>& s, int c) {
+    sc = &s;
+    t_next = c;
+    cur = c < s.Gr ? s.bound(c) : 0;
+    end = c < s.Gr ? s.bound(c + 1) : 0;
+  }
+  __device__ bool next(int& t, int& kb0, int& kb1) {
+    if (t_next < sc->whole) {
+      t = t_next;
+      t_next += sc->G;
+      kb0 = 0;
+      kb1 = sc->kbt;
+      return true;
+    }
+    if (cur >= end) return false;
+    const int tr = int(cur / sc->kbt);
+    kb0 = int(cur - (long long)tr * sc->kbt);
+    kb1 = int(min((long long)sc->kbt, kb0 + (end - cur)));
+    cur += kb1 - kb0;
+    t = sc->whole + tr;
+    return true;
   }
 };
 
 template <int BN>
 __global__ void __launch_bounds__(THREADS, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-               int Mbound, const int* __restrict__ dcount, int n, int k, GemmEpi ep,
-               float* __restrict__ ws, int ws_units) {
+               int Mbound, const int* __restrict__ dcount, int n, int k, GemmEpi ep) {
   using TC = TileCfg<BN>;
   constexpr int STAGES = TC::STAGES, STAGE_B = TC::STAGE_B, TMEM_COLS = TC::TMEM_COLS;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  // 1024-aligned operand stages, then barriers
+  // 1024-aligned operand stages, epilogue staging, then barriers
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + STAGES * STAGE_A;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sB + STAGES * STAGE_B);
+  uint8_t* sStg = sB + STAGES * STAGE_B;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sStg + STAGING_BYTES);
   // bars: full[STAGES], empty[STAGES], tfull[2], tempty[2]
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 4);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -230,20 +301,17 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   pdl_trigger();
   const int M = live_count(dcount, Mbound, ep.err);
   Sched<BN> sc;
-  sc.init(M, n, k, min(int(gridDim.x), ws_units));
-  const long long seg_beg = blockIdx.x < sc.G ? sc.bound(blockIdx.x) : 0;
-  const long long seg_end = blockIdx.x < sc.G ? sc.bound(blockIdx.x + 1) : 0;
+  sc.init(M, n, k, int(gridDim.x), ep.mode == EPI_GATE_RES);
 
   if (warp == 0) {
     // ------------------------------------------------------- TMA producer
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
-      for (long long cur = seg_beg; cur < seg_end;) {
-        const int t = int(cur / sc.kbt);
-        const int kb0 = int(cur - (long long)t * sc.kbt);
-        const int kb1 = int(min((long long)sc.kbt, kb0 + (seg_end - cur)));
-        cur += kb1 - kb0;
+      Segs<BN> sg;
+      sg.init(sc, blockIdx.x);
+      int t, kb0, kb1;
+      while (sg.next(t, kb0, kb1)) {
         const int m = t % sc.mt, nn = t / sc.mt;
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(empty0 + 8 * stage, phase ^ 1, abort_flag)) goto timeout;
@@ -261,11 +329,10 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       uint32_t phase = 0;
       int acc = 0;
       uint32_t acc_phase = 0;
-      for (long long cur = seg_beg; cur < seg_end;) {
-        const int t = int(cur / sc.kbt);
-        const int kb0 = int(cur - (long long)t * sc.kbt);
-        const int kb1 = int(min((long long)sc.kbt, kb0 + (seg_end - cur)));
-        cur += kb1 - kb0;
+      Segs<BN> sg;
+      sg.init(sc, blockIdx.x);
+      int t, kb0, kb1;
+      while (sg.next(t, kb0, kb1)) {
         if (!mbar_wait(tempty0 + 8 * acc, acc_phase ^ 1, abort_flag)) goto timeout;
         tc_fence_after();
         const uint32_t dtm = tmem_base + uint32_t(acc * (TMEM_COLS / 2));
@@ -289,33 +356,26 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     const int sp = warp & 3;  // TMEM lane sub-partition this warp may access
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (long long cur = seg_beg; cur < seg_end;) {
-      const int t = int(cur / sc.kbt);
-      const int kb0 = int(cur - (long long)t * sc.kbt);
-      const int kb1 = int(min((long long)sc.kbt, kb0 + (seg_end - cur)));
-      cur += kb1 - kb0;
+    Segs<BN> sg;
+    sg.init(sc, blockIdx.x);
+    int t, kb0, kb1;
+    while (sg.next(t, kb0, kb1)) {
       const int m = t % sc.mt, nn = t / sc.mt;
       if (!mbar_wait_warp(tfull0 + 8 * acc, acc_phase, abort_flag)) goto timeout;
       tc_fence_after();
       const int row = sp * 32 + lane;
       const int r = m * BM + row;
       const uint32_t tbase = tmem_base + uint32_t(acc * (TMEM_COLS / 2)) + (uint32_t(sp * 32) << 16);
-      // a whole tile, or any piece of a gated residual (its update is a sum),
-      // goes straight to the epilogue; a piece of another epilogue reduces
-      // into the tile's workspace slot and the finish kernel completes it
-      const bool direct = (kb0 == 0 && kb1 == sc.kbt) || ep.mode == EPI_GATE_RES;
-      float* acc_row = direct ? nullptr : ws + size_t(sc.split_slot(t)) * (BM * BN) + size_t(row) * BN;
+      const int tok = (ep.mode == EPI_QKV && r < M) ? (ep.idx ? __ldg(ep.idx + r) : r) : 0;
+      // a piece of a split tile only occurs for the gated residual, whose
+      // update is a sum: the bias goes with the piece that starts at k = 0
 #pragma unroll 1
       for (int ch = 0; ch < BN / 32; ++ch) {
         float v[32];
         tmem_ld32(tbase + uint32_t(ch * 32), v);
-        if (direct) {
-          if (r < M) epilogue32(ep, r, nn * BN + ch * 32, v, kb0 == 0);
-        } else {
-#pragma unroll
-          for (int i = 0; i < 8; ++i)
-            red_add_v4(acc_row + ch * 32 + 4 * i, v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-        }
+        const int c0 = nn * BN + ch * 32;
+        epilogue_values(ep, c0, v, kb0 == 0);
+        store_chunk(ep.mode, sStg + sp * STAGING_WARP, lane, v, chunk_dst(ep, r, M, tok, c0));
       }
       tc_fence_before();
       mbar_arrive(tempty0 + 8 * acc);
@@ -335,41 +395,6 @@ done:
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
                  "r"(TMEM_COLS)
                  : "memory");
-  }
-}
-
-// Completes the split tiles of a non-additive epilogue: reads the reduced
-// f32 tile from its workspace slot, zeroes it, applies the epilogue.  One
-// thread per (slot, row, 32-column chunk), grid-stride.
-template <int BN>
-__global__ void __launch_bounds__(256)
-gemm_finish_kernel(float* __restrict__ ws, int Mbound, const int* __restrict__ dcount, int n,
-                   int k, int grid, GemmEpi ep) {
-  pdl_wait();
-  pdl_trigger();
-  const int M = live_count(dcount, Mbound, ep.err);
-  Sched<BN> sc;
-  sc.init(M, n, k, grid);
-  constexpr int CH = BN / 32;
-  // split tiles = tiles whose first inner CTA boundary is c (c = 1 .. G-1)
-  const int items = (sc.G - 1) * BM * CH;
-  for (int it = blockIdx.x * 256 + threadIdx.x; it < items; it += gridDim.x * 256) {
-    const int c = 1 + it / (BM * CH);
-    const int rem = it - (c - 1) * (BM * CH);
-    const int row = rem / CH, ch = rem - (rem / CH) * CH;
-    const int t = int(sc.bound(c) / sc.kbt);
-    if (sc.split_slot(t) != c) continue;
-    float4* p4 = reinterpret_cast<float4*>(ws + size_t(c) * (BM * BN) + size_t(row) * BN + ch * 32);
-    float v[32];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const float4 a = __ldcg(p4 + i);
-      v[4 * i] = a.x; v[4 * i + 1] = a.y; v[4 * i + 2] = a.z; v[4 * i + 3] = a.w;
-      __stcg(p4 + i, make_float4(0.f, 0.f, 0.f, 0.f));
-    }
-    const int m = t % sc.mt, nn = t / sc.mt;
-    const int r = m * BM + row;
-    if (r < M) epilogue32(ep, r, nn * BN + ch * 32, v, true);
   }
 }
 
@@ -452,16 +477,8 @@ int device_sms() {
 
 }  // namespace
 
-cudaError_t gemm_scratch_shape(int* units, size_t* ws_floats) {
-  const int sms = device_sms();
-  if (!sms) return cudaErrorInvalidDevice;
-  *units = sms;
-  *ws_floats = size_t(sms) * BM * MAX_BN;
-  return cudaSuccess;
-}
-
 cudaError_t launch_gemm(const bf16* A, int lda, const bf16* W, int Mbound, const int* dcount,
-                        int n, int k, const GemmEpi& ep, const GemmScratch& gs, cudaStream_t st) {
+                        int n, int k, const GemmEpi& ep, cudaStream_t st) {
   if (Mbound <= 0) return cudaSuccess;
   if (n % 128 || k % BK) return cudaErrorInvalidValue;
   const int sms = device_sms();
@@ -471,24 +488,14 @@ cudaError_t launch_gemm(const bf16* A, int lda, const bf16* W, int Mbound, const
   CUtensorMap ta, tb;
   if ((e = tensor_map(A, Mbound, k, lda, BM, &ta)) != cudaSuccess) return e;
   if ((e = tensor_map(W, n, k, k, BN, &tb)) != cudaSuccess) return e;
-  // one workspace slot per CTA range boundary
-  const int grid = min(sms, gs.units);
+  const int grid = sms;
   if (BN == 192)
     RC_TRY(launch_k(gemm_tc_kernel<192>, dim3(grid), dim3(THREADS), TileCfg<192>::SMEM_BYTES, st,
-                    ta, tb, Mbound, dcount, n, k, ep, gs.ws, grid));
+                    ta, tb, Mbound, dcount, n, k, ep));
   else
     RC_TRY(launch_k(gemm_tc_kernel<128>, dim3(grid), dim3(THREADS), TileCfg<128>::SMEM_BYTES, st,
-                    ta, tb, Mbound, dcount, n, k, ep, gs.ws, grid));
+                    ta, tb, Mbound, dcount, n, k, ep));
   count_launches(1);
-  if (ep.mode != EPI_GATE_RES) {
-    if (BN == 192)
-      RC_TRY(launch_k(gemm_finish_kernel<192>, dim3(2 * sms), dim3(256), 0, st, gs.ws, Mbound,
-                      dcount, n, k, grid, ep));
-    else
-      RC_TRY(launch_k(gemm_finish_kernel<128>, dim3(2 * sms), dim3(256), 0, st, gs.ws, Mbound,
-                      dcount, n, k, grid, ep));
-    count_launches(1);
-  }
   return cudaSuccess;
 }
 

@@ -86,20 +86,10 @@ struct GemmEpi {
   unsigned* err;
 };
 
-// Stream-K scratch of one context: `units` f32 accumulator tiles (zero
-// between launches), one per CTA range boundary.
-struct GemmScratch {
-  float* ws;
-  int units;
-};
-// Workspace tiles and floats a context should allocate on the current device.
-cudaError_t gemm_scratch_shape(int* units, size_t* ws_floats);
-
 // C[M][n] = A[M][k] W[n][k]^T, epilogue `ep`.  M = *dcount if non-null (bounded
-// by Mbound) else Mbound.  n % 128 == 0, k % 64 == 0.  Launches on one
-// GemmScratch must be stream-ordered.
+// by Mbound) else Mbound.  n % 128 == 0, k % 64 == 0.
 cudaError_t launch_gemm(const bf16* A, int lda, const bf16* W, int Mbound, const int* dcount,
-                        int n, int k, const GemmEpi& ep, const GemmScratch& gs, cudaStream_t st);
+                        int n, int k, const GemmEpi& ep, cudaStream_t st);
 
 
 // ----------------------------------------------------------------- attention

@@ -73,7 +73,6 @@ struct rc_ctx {
   float* tb = nullptr;   // [6d]
   int* iota = nullptr;   // [N] identity row map (dense path)
   unsigned* err = nullptr;
-  rc::GemmScratch gs{};  // stream-K workspace tiles
   rc::AttnScratch as{};  // key-split partial outputs
   // timing probe
   int probe_which = RC_PROBE_OFF;
@@ -147,8 +146,7 @@ void free_ctx(rc_ctx* c) {
   if (!c) return;
   probe_free(c);
   void* ps[] = {c->xf,   c->xb,  c->ob,   c->q,        c->u,         c->fbuf,
-                c->h1,   c->temb, c->tb,  c->iota,     c->err,       c->gs.ws,
-                c->as.part};
+                c->h1,   c->temb, c->tb,  c->iota,     c->err,       c->as.part};
   for (void* p : ps)
     if (p) cudaFree(p);
   delete c;
@@ -211,7 +209,7 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
   {
     Probe pr(c, RC_PROBE_GEMM, st);
     RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_qkv), rw.bound, rw.dcount, 3 * d,
-                            d, e, c->gs, st), "gemm(qkv)");
+                            d, e, st), "gemm(qkv)");
   }
   // dirty queries over all N keys / values of (l, t)
   {
@@ -231,7 +229,7 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
   {
     Probe pr(c, RC_PROBE_GEMM, st);
     RC_CUDA(rc::launch_gemm(c->ob, d, static_cast<const bf16*>(w.W_o), rw.bound, rw.dcount, d, d, e,
-                            c->gs, st), "gemm(out)");
+                            st), "gemm(out)");
   }
   // q' = x W_xq^T + b (on a bf16 copy of x)
   RC_CUDA(rc::launch_cast_rows(c->xf, d, c->xb, d, rw.bound, rw.dcount, d, c->err, st), "cast");
@@ -244,7 +242,7 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
   {
     Probe pr(c, RC_PROBE_GEMM, st);
     RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_xq), rw.bound, rw.dcount, d, d,
-                            e, c->gs, st), "gemm(xq)");
+                            e, st), "gemm(xq)");
   }
   {
     Probe pr(c, RC_PROBE_ATTENTION, st);
@@ -261,7 +259,7 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
   {
     Probe pr(c, RC_PROBE_GEMM, st);
     RC_CUDA(rc::launch_gemm(c->ob, d, static_cast<const bf16*>(w.W_xo), rw.bound, rw.dcount, d, d,
-                            e, c->gs, st), "gemm(xo)");
+                            e, st), "gemm(xo)");
   }
   // MLP
   RC_CUDA(rc::launch_ln_mod(c->xf, d, mv(tab, 3), mv(tbv, 3), mv(tab, 4), mv(tbv, 4), c->xb, d,
@@ -276,7 +274,7 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
   {
     Probe pr(c, RC_PROBE_GEMM, st);
     RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_1), rw.bound, rw.dcount, F, d, e,
-                            c->gs, st), "gemm(fc1)");
+                            st), "gemm(fc1)");
   }
   // x += gate_mlp (u W_2^T + b_2); the caller stores x as the merged H^{l+1}
   e = rc::GemmEpi{};
@@ -290,7 +288,7 @@ rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows&
   {
     Probe pr(c, RC_PROBE_GEMM, st);
     RC_CUDA(rc::launch_gemm(c->u, F, static_cast<const bf16*>(w.W_2), rw.bound, rw.dcount, d, F, e,
-                            c->gs, st), "gemm(fc2)");
+                            st), "gemm(fc2)");
   }
   return RC_OK;
 }
@@ -361,22 +359,10 @@ rc_status rc_create(const rc_dims* dims, rc_ctx** out) {
     free_ctx(c);
     return s;
   }
-  {
-    int units = 0;
-    size_t ws_floats = 0;
-    cudaError_t e0 = rc::gemm_scratch_shape(&units, &ws_floats);
-    if (e0 != cudaSuccess) {
-      free_ctx(c);
-      return cuda_fail(e0, "rc_create: device query");
-    }
-    c->gs.units = units;
-    c->as.part_floats = rc::attention_split_floats(int(N), D.heads, dh);
-    if ((s = dalloc(&c->gs.ws, ws_floats, "gemm workspace")) ||
-        (s = dalloc(&c->as.part, c->as.part_floats, "attn part"))) {
-      free_ctx(c);
-      return s;
-    }
-    cudaMemset(c->gs.ws, 0, sizeof(float) * ws_floats);  // workspace tiles start at zero
+  c->as.part_floats = rc::attention_split_floats(int(N), D.heads, dh);
+  if ((s = dalloc(&c->as.part, c->as.part_floats, "attn part"))) {
+    free_ctx(c);
+    return s;
   }
   iota_kernel<<<int((N + 255) / 256), 256>>>(c->iota, int(N));
   rc::count_launches(1);
@@ -506,7 +492,7 @@ rc_status rc_set_text(rc_ctx* c, rc_cache* k, int s, const void* ctx_bf16, rc_st
     e.err = c->err;
     RC_CUDA(rc::launch_gemm(static_cast<const bf16*>(ctx_bf16), c->d,
                             static_cast<const bf16*>(c->lw[l].W_xkv), c->M, nullptr, 2 * c->d,
-                            c->d, e, c->gs, st), "gemm(text kv)");
+                            c->d, e, st), "gemm(text kv)");
   }
   k->text_set[s] = 1;
   return RC_OK;
@@ -652,7 +638,7 @@ rc_status rc_linear(rc_ctx* c, const void* x, const void* W, const float* b, flo
   e.ld_out = n;
   e.err = c->err;
   RC_CUDA(rc::launch_gemm(static_cast<const bf16*>(x), kdim, static_cast<const bf16*>(W), rows,
-                          nullptr, n, kdim, e, c->gs, static_cast<cudaStream_t>(stream)),
+                          nullptr, n, kdim, e, static_cast<cudaStream_t>(stream)),
           "gemm(linear)");
   return RC_OK;
 }
@@ -690,19 +676,30 @@ rc_status rc_probe_enable(rc_ctx* c, int which, int capacity) {
   return RC_OK;
 }
 
-rc_status rc_probe_read(rc_ctx* c, double* total_ms, int* launches) {
-  if (!c || !total_ms || !launches) return fail(RC_ERR_INVALID_ARG, "rc_probe_read: null");
-  double tot = 0.0;
-  for (int i = 0; i < c->probe_n; ++i) {
+rc_status rc_probe_read_each(rc_ctx* c, float* ms_out, int capacity, int* launches) {
+  if (!c || !launches || (capacity > 0 && !ms_out) || capacity < 0)
+    return fail(RC_ERR_INVALID_ARG, "rc_probe_read_each: null or negative argument");
+  const int n = c->probe_n;
+  for (int i = 0; i < n; ++i) {
     RC_CUDA(cudaEventSynchronize(c->probe_ev[2 * i + 1]), "cudaEventSynchronize");
     float ms = 0.f;
     RC_CUDA(cudaEventElapsedTime(&ms, c->probe_ev[2 * i], c->probe_ev[2 * i + 1]),
             "cudaEventElapsedTime");
-    tot += ms;
+    if (i < capacity) ms_out[i] = ms;
   }
-  *total_ms = tot;
-  *launches = c->probe_n;
+  *launches = n;
   c->probe_n = 0;
+  return RC_OK;
+}
+
+rc_status rc_probe_read(rc_ctx* c, double* total_ms, int* launches) {
+  if (!c || !total_ms || !launches) return fail(RC_ERR_INVALID_ARG, "rc_probe_read: null");
+  std::vector<float> ms(size_t(c->probe_n));
+  rc_status s = rc_probe_read_each(c, ms.data(), int(ms.size()), launches);
+  if (s != RC_OK) return s;
+  double tot = 0.0;
+  for (float v : ms) tot += v;
+  *total_ms = tot;
   return RC_OK;
 }
 

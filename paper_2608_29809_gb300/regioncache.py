@@ -79,6 +79,7 @@ def load_library(path: str = LIB_PATH) -> C.CDLL:
         "rc_sync": (I, [P, P]),
         "rc_probe_enable": (I, [P, I, I]),
         "rc_probe_read": (I, [P, C.POINTER(C.c_double), C.POINTER(I)]),
+        "rc_probe_read_each": (I, [P, C.POINTER(C.c_float), I, C.POINTER(I)]),
         "rc_launch_count": (C.c_uint64, []),
         "rc_status_string": (C.c_char_p, [I]),
         "rc_last_error": (C.c_char_p, []),
@@ -232,6 +233,14 @@ def rc_probe_read(ctx):
     ms, n = C.c_double(), C.c_int()
     _check(_lib.rc_probe_read(ctx, C.byref(ms), C.byref(n)))
     return ms.value, n.value
+
+
+def rc_probe_read_each(ctx, capacity):
+    """Per-launch device times (ms, launch order) of the recorded launches."""
+    buf = (C.c_float * max(1, capacity))()
+    n = C.c_int()
+    _check(_lib.rc_probe_read_each(ctx, buf, capacity, C.byref(n)))
+    return [buf[i] for i in range(min(n.value, capacity))]
 
 
 def rc_launch_count() -> int:
