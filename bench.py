@@ -20,6 +20,7 @@ replica (its own session and cache); value = all ranks' steps / max time.
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import os
 import statistics
@@ -54,6 +55,38 @@ def linear_flops_per_token_block(d: synth.Dims) -> float:
 def attn_flops_per_token_block(d: synth.Dims) -> float:
     """Self-attention (4 N h) plus cross-attention (4 M h) per dirty token and block."""
     return 4.0 * d.tokens * d.hidden + 4.0 * d.text_len * d.hidden
+
+
+KERNEL_SOURCES = {
+    "gemm": ["gemm_tc.cu", "tc_common.cuh", "common.cuh", "kernels.h"],
+    "attention": ["attention_tc.cu", "tc_common.cuh", "common.cuh", "kernels.h"],
+}
+PROFILES = {"gemm": "gemm_tc_kernel_pixart1024_d831.md",
+            "attention": "attn_tc_kernel_pixart1024_d831.md"}
+
+
+def profiled_traffic(kernel: str):
+    """DRAM bytes per launch from the committed ncu summary of `kernel`, or
+    None when the kernel's sources changed since the counters were taken."""
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES[kernel]:
+        with open(os.path.join(ROOT, "paper_2608_29809_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    path = os.path.join(ROOT, "profiles", PROFILES[kernel])
+    if not os.path.exists(path):
+        return None
+    meta = {}
+    with open(path) as fh:
+        for ln in fh:
+            if ":" in ln and not ln.startswith(("|", "#", " ")):
+                k, v = ln.split(":", 1)
+                meta[k.strip()] = v.strip()
+    if meta.get("kernel_source_sha256_16") != h.hexdigest()[:16]:
+        return None
+    try:
+        return int(meta["dram_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
 
 
 def load_peaks():
@@ -307,13 +340,15 @@ def run_ours(args, world, rank, local):
     peak = peaks["bf16_tflops_sustained"]
     att_tflops = (attn_flops_per_token_block(d) * D * d.layers * K) / (att_ms / 1e3) / 1e12
     roofline = {"bound": "tensor", "achieved": round(gemm_tflops, 2), "peak": peak,
-                "unit": "TFLOP/s", "frac": round(gemm_tflops / peak, 4), "traffic": None,
+                "unit": "TFLOP/s", "frac": round(gemm_tflops / peak, 4),
+                "traffic": profiled_traffic("gemm"),
                 "kernel": "gemm (QKV, out, cross-q, cross-out, fc1, fc2 of every block)",
                 "launches": gemm_n, "avg_launch_ms": round(gemm_avg_ms, 5),
                 "timing": "CUDA events around each launch, separate pass of the same K steps",
                 "flops_per_launch": lin_flops_launch,
                 "peak_source": f"{peaks['source']} bf16_tflops_sustained"}
     roof_att = {"bound": "tensor", "achieved": round(att_tflops, 2), "peak": peak,
+                "traffic": profiled_traffic("attention"),
                 "unit": "TFLOP/s", "frac": round(att_tflops / peak, 4), "launches": att_n,
                 "avg_launch_ms": round(att_ms / max(att_n, 1), 5)}
     # per-launch breakdown: launches come in block order (GEMMs: QKV, out,
