@@ -318,3 +318,9 @@ def similarity(seed: int, turn: int) -> float:
     """Seeded prompt-similarity scalar s in [0, 1] for one editing turn."""
     rng = np.random.default_rng(tensor_seed(seed, "similarity", turn))
     return float(rng.uniform(0.0, 1.0))
+
+
+def turn_dirty_fraction(seed: int, turn: int, lo: float = 0.05, hi: float = 0.20) -> float:
+    """Seeded target dirty fraction of one editing turn's mask, U(lo, hi)."""
+    rng = np.random.default_rng(tensor_seed(seed, "turn_fraction", turn))
+    return float(rng.uniform(lo, hi))

@@ -1,0 +1,170 @@
+"""GPU parity at the full sizes of the 1024 px workload (4096 tokens, 28
+blocks) in the launch configuration the benchmark times, and the multi-turn
+editing session (the cache updated in place across turns)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2608_29809_gb300 import synth
+from tests.gpu_cases import LATENT_REL_L2, Problem, block_close, rel_l2
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def R():
+    from paper_2608_29809_gb300 import build as B
+    B.build()
+    from paper_2608_29809_gb300 import regioncache
+    return regioncache
+
+
+def _localize(R, A, ids, d, dil):
+    N = d.tokens
+    ws = torch.empty(R.rc_localize_workspace_size(N, len(ids)), dtype=torch.uint8, device="cuda")
+    mask = torch.zeros(N, dtype=torch.uint8, device="cuda")
+    idx = torch.zeros(N, dtype=torch.int32, device="cuda")
+    cnt = torch.zeros(1, dtype=torch.int32, device="cuda")
+    R.rc_localize_mask(torch.from_numpy(np.ascontiguousarray(A)).cuda(), A.shape[0], N,
+                       A.shape[2], d.grid_h, d.grid_w, ids, 0.5, dil, mask, idx, cnt, ws)
+    return mask, idx, cnt
+
+
+def _eps_from_update(got, x, ab_t, ab_n):
+    c_x = np.sqrt(ab_n / ab_t)
+    c_e = np.sqrt(1 - ab_n) - np.sqrt(ab_n) * np.sqrt(1 - ab_t) / np.sqrt(ab_t)
+    return (got - c_x * x) / c_e
+
+
+# --------------------------------------------- 4096 tokens, benchmark launch
+@pytest.fixture(scope="module")
+def c3_problem(R):
+    p = Problem(R, synth.PIXART_1024, 1234 + 300, ts=(7,))
+    yield p
+    p.close()
+
+
+def test_c3_full_step_bench_configuration(R, c3_problem):
+    """One full 28-block step at 4096 tokens, 20 % dirty ellipse union, the
+    mask made on the device and the dirty count left there (D = -1), exactly
+    as the benchmark runs it; the oracle runs the whole step."""
+    p = c3_problem
+    d = p.d
+    t = 7
+    blobs = synth.ellipse_blobs(d, p.seed, 0.2)
+    A, ids = synth.indicator_scores(d, blobs, p.seed)
+    mask, idx_d, cnt = _localize(R, A, ids, d, 0)
+    _, idx = O.localize_mask(A, ids, d.grid_h, d.grid_w, 0.5, 0)
+    torch.cuda.synchronize()
+    D = int(cnt.item())
+    assert D == len(idx) and abs(D / d.tokens - 0.2) <= 0.006
+    assert np.array_equal(idx_d.cpu().numpy()[:D], idx)
+    lat = synth.make_latent(d, p.seed)
+    latent = lat.clone().cuda()
+    sched = np.full(d.timesteps, O.MODE_SPARSE, np.uint8)
+    R.rc_step(p.model.ctx, p.model.cache, 0, latent, t, sched, idx_d, -1, cnt)
+    R.rc_sync(p.model.ctx)
+    got = latent.cpu().double().numpy()
+    ref, eps, cache = p.oracle_step(O.to64(lat), t, O.MODE_SPARSE, idx)
+    assert rel_l2(got, ref) <= LATENT_REL_L2
+    block_close(_eps_from_update(got, O.to64(lat), float(p.ab[t]), float(p.ab[t + 1])), eps, "eps")
+    clean = np.setdiff1d(np.arange(d.tokens), idx)
+    for l in (0, 9, 18, 27):
+        s = p.read_slot(l, t)
+        for k in ("H", "K", "V"):
+            block_close(s[k][idx], cache[l][k][idx], f"{k} rows, layer {l}")
+            # clean rows are the previous turn's values, untouched
+            assert np.array_equal(s[k][clean], p.cache64[(l, t)][k][clean])
+
+
+def test_c3_dense_step_invariant_full_size(R, c3_problem):
+    """A DENSE step and a SPARSE step with every token dirty compute the same
+    thing (both on the device)."""
+    p = c3_problem
+    d = p.d
+    t = 7
+    lat = synth.make_latent(d, p.seed + 1)
+
+    def run(mode):
+        for l in range(d.layers):
+            H, K, V = synth.make_cache_slice(d, p.seed, 0, l, t)
+            R.rc_cache_fill(p.model.cache, 0, l, t, H.cuda(), K.cuda(), V.cuda())
+        latent = lat.clone().cuda()
+        sched = np.full(d.timesteps, mode, np.uint8)
+        all_idx = torch.arange(d.tokens, dtype=torch.int32, device="cuda")
+        R.rc_step(p.model.ctx, p.model.cache, 0, latent, t, sched, all_idx, d.tokens, None)
+        R.rc_sync(p.model.ctx)
+        return latent.cpu().numpy(), p.read_slot(d.layers - 1, t)["H"]
+
+    dense, h_dense = run(O.MODE_DENSE)
+    sparse_all, h_sparse = run(O.MODE_SPARSE)
+    # equal up to the order of the f32 reductions of split gated-residual
+    # tiles (atomic adds), which the two launches need not share
+    assert rel_l2(sparse_all, dense) <= LATENT_REL_L2
+    block_close(h_sparse, h_dense, "H of the last block, DENSE vs all-dirty SPARSE")
+    for l in range(d.layers):
+        H, K, V = synth.make_cache_slice(d, p.seed, 0, l, t)
+        R.rc_cache_fill(p.model.cache, 0, l, t, H.cuda(), K.cuda(), V.cuda())
+    torch.cuda.synchronize()
+
+
+# ------------------------------------------------- multi-turn editing session
+def test_c4_multi_turn_session(R):
+    """Five editing turns over one session: each turn draws a similarity s
+    (k = 2 (1 + min(3, floor(4 (1 - s)))) leading DENSE steps), new delta
+    tokens and a new ellipse mask (5-20 % dirty), starts from fresh noise and
+    runs all T steps; the cache is updated in place across turns.  Each step
+    is compared with the oracle given the same input latent, and each turn's
+    cache against the oracle's (both sides start every turn from the same
+    bf16 cache).  Reduced to a 16 x 16 grid and 2 blocks so the oracle runs
+    the 100 steps in seconds."""
+    d = synth.Dims(grid_h=16, grid_w=16, layers=2, timesteps=20)
+    seed = 1234 + 300
+    p = Problem(R, d, seed, ts=tuple(range(d.timesteps)))
+    try:
+        cache64 = dict(p.cache64)
+        for turn in range(5):
+            # both sides start the turn from the same bf16 cache
+            for (l, t), c in cache64.items():
+                b = {k: torch.from_numpy(v).to(torch.bfloat16) for k, v in c.items()}
+                R.rc_cache_fill(p.model.cache, 0, l, t, b["H"].cuda(), b["K"].cuda(),
+                                b["V"].cuda())
+                cache64[(l, t)] = {k: O.to64(v) for k, v in b.items()}
+            torch.cuda.synchronize()
+            s = synth.similarity(seed, turn)
+            k = O.k_from_similarity(s)
+            sched = O.schedule_first_k_dense(k, d.timesteps)
+            f = synth.turn_dirty_fraction(seed, turn)
+            blobs = synth.ellipse_blobs(d, seed + turn, f)
+            A, ids = synth.indicator_scores(d, blobs, seed + turn)
+            _, idx_d, cnt = _localize(R, A, ids, d, 0)
+            _, idx = O.localize_mask(A, ids, d.grid_h, d.grid_w, 0.5, 0)
+            torch.cuda.synchronize()
+            assert int(cnt.item()) == len(idx) > 0
+            x = O.to64(synth.make_latent(d, seed + 17 * turn))
+            for t in range(d.timesteps):
+                latent = torch.from_numpy(x.astype(np.float32)).cuda()
+                R.rc_step(p.model.ctx, p.model.cache, 0, latent, t, sched, idx_d, -1, cnt)
+                R.rc_sync(p.model.ctx)
+                got = latent.cpu().double().numpy()
+                cache_t = [cache64[(l, t)] for l in range(d.layers)]
+                ref, eps, new = O.step(p.G64, p.layers64, p.pos64, x, t, int(sched[t]), idx,
+                                       cache_t, p.tkv64, p.tv.astype(np.float64),
+                                       p.ab.astype(np.float64), d.heads, d.grid_h, d.grid_w,
+                                       d.patch, d.in_ch)
+                assert rel_l2(got, ref) <= LATENT_REL_L2, (turn, t)
+                for l in range(d.layers):
+                    cache64[(l, t)] = new[l]
+                x = ref
+            # the turn's cache: DENSE slices entirely, SPARSE slices on the
+            # dirty rows (clean rows were compared bitwise in the C3 test)
+            for t in (0, k - 1, k, d.timesteps - 1):
+                rows = np.arange(d.tokens) if sched[t] == O.MODE_DENSE else idx
+                for l in range(d.layers):
+                    got = p.read_slot(l, t)
+                    for key in ("H", "K", "V"):
+                        block_close(got[key][rows], cache64[(l, t)][key][rows],
+                                    f"turn {turn} t {t} layer {l} {key}")
+    finally:
+        p.close()
