@@ -58,11 +58,15 @@ typedef void* rc_stream; /* cudaStream_t */
 
 /* Model and problem sizes.  PixArt-alpha: hidden 1152, heads 16 (head_dim
  * 72), mlp 4608, layers 28, patch 2, in_ch 4, out_ch 8, text_len 120,
- * freq_dim 256.  N = grid_h * grid_w image tokens. */
+ * freq_dim 256.  N = grid_h * grid_w image tokens.  max_batch = most items
+ * of one rc_step_batched call (1 .. RC_MAX_BATCH; 0 means 1): the context's
+ * row scratch is sized for max_batch * N rows. */
+#define RC_MAX_BATCH 16
 typedef struct rc_dims {
   int hidden, heads, mlp, layers;
   int grid_h, grid_w, patch, in_ch, out_ch;
   int text_len, timesteps, freq_dim;
+  int max_batch;
 } rc_dims;
 
 /* One block's weights (device pointers, borrowed).  W_* bf16 [out][in];
@@ -251,6 +255,35 @@ rc_status rc_block_forward_region(rc_ctx* ctx, rc_cache* cache, int session, int
 rc_status rc_step(rc_ctx* ctx, rc_cache* cache, int session, float* latent, int t,
                   const uint8_t* schedule_host, const int32_t* dirty_idx, int D,
                   const int32_t* dirty_count, rc_stream stream);
+
+/* One item of a batched step: one session's denoising step.
+ *   session      cache session (an item per (session, t) at most per call)
+ *   latent       device f32 [in_ch][grid_h*patch][grid_w*patch], in/out
+ *   t            timestep index in [0, timesteps)
+ *   mode         RC_MODE_DENSE / SPARSE / REUSE for this step
+ *   dirty_idx, D, dirty_count   SPARSE only, as in rc_step */
+typedef struct rc_batch_item {
+  int session;
+  float* latent;
+  int t;
+  int mode;
+  const int32_t* dirty_idx;
+  int D;
+  const int32_t* dirty_count;
+} rc_batch_item;
+
+/* Batched serving (no counterpart in the paper, which serves one request at
+ * a time): one denoising step for each of n_items sessions, each exactly as
+ * rc_step would compute it (Section 3.3 region-level sparse attention per
+ * item: an item's dirty queries attend over its own session's cached and
+ * fresh keys / values at its own timestep, with its own text context).  The
+ * dirty rows of all items are processed together, so every weight matrix is
+ * read once per call.  items: host array; 1 <= n_items <= the context's
+ * max_batch.  Errors: RC_ERR_INVALID_ARG (bad item, two items on the same
+ * (session, t), n_items out of range), RC_ERR_STATE (weights, schedule or a
+ * session's text not set). */
+rc_status rc_step_batched(rc_ctx* ctx, rc_cache* cache, const rc_batch_item* items, int n_items,
+                          rc_stream stream);
 
 /* Full-recompute baseline: rc_step with mode DENSE. */
 rc_status rc_step_dense(rc_ctx* ctx, rc_cache* cache, int session, float* latent, int t,

@@ -81,11 +81,29 @@ struct ACfg {
                                          (uint32_t(16 >> 3) << 17) | (uint32_t(BQ >> 4) << 24);
 };
 
+// Query tile qt of a launch: its item, first compact row and live rows.
+struct TileLoc {
+  int item, row0, rows;
+};
+__device__ __forceinline__ TileLoc locate_tile(const RowMap& rm, int n_items, int D, int qt) {
+  if (!rm.meta) return TileLoc{0, qt * BQ, min(BQ, D - qt * BQ)};
+  int i = 0;
+  while (i + 1 < n_items && __ldg(rm.meta + META_TILE + i + 1) <= qt) ++i;
+  const int j = qt - __ldg(rm.meta + META_TILE + i);
+  return TileLoc{i, __ldg(rm.meta + META_OFF + i) + j * BQ,
+                 min(BQ, __ldg(rm.meta + META_CNT + i) - j * BQ)};
+}
+
+// Query tiles of a launch: 128-row tiles of each item's rows.
+__device__ __forceinline__ int query_tiles(const RowMap& rm, int n_items, int D) {
+  return rm.meta ? __ldg(rm.meta + META_TILE + n_items) : (D + BQ - 1) / BQ;
+}
+
 // Work list of one launch, identical in every thread.
 struct AttnSched {
   int qtiles, pairs, nkb, split, per, units;
-  __device__ void init(int D, int heads, int Nk, int grid, int ws_units) {
-    qtiles = (D + BQ - 1) / BQ;
+  __device__ void init(int tiles, int heads, int Nk, int grid, int ws_units) {
+    qtiles = tiles;
     pairs = qtiles * heads;
     nkb = (Nk + BKV - 1) / BKV;
     split = 1;
@@ -113,9 +131,9 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
 attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmQt,
                const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmKt,
                const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmVt,
-               int Nk, bf16* __restrict__ O, int ldo, int heads, int Dbound,
-               const int* __restrict__ dcount, float scale_log2, unsigned* err,
-               float* __restrict__ part, int ws_units) {
+               const __grid_constant__ AttnItems ai, int Nk, bf16* __restrict__ O, int ldo,
+               int heads, RowMap rm, float scale_log2, unsigned* err, float* __restrict__ part,
+               int ws_units) {
   using C = ACfg<DH>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -172,9 +190,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 
   pdl_wait();
   pdl_trigger();
-  const int D = live_count(dcount, Dbound, err);
+  const int D = live_count(rm.count, rm.bound, err);
   AttnSched sc;
-  sc.init(D, heads, Nk, gridDim.x, ws_units);
+  sc.init(query_tiles(rm, ai.n, D), heads, Nk, gridDim.x, ws_units);
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA
@@ -183,20 +201,23 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
       for (int u = blockIdx.x; u < sc.units; u += gridDim.x, ++uc) {
         int qt, h, sp, kb0, kb1;
         sc.decode(u, qt, h, sp, kb0, kb1);
+        const TileLoc tl = locate_tile(rm, ai.n, D, qt);
+        const int krow = ai.krow[tl.item], vrow = ai.vrow[tl.item];
         if (!mbar_wait(q_empty, (uc + 1) & 1, abort_flag)) goto timeout;
         mbar_expect_tx(q_full, C::Q_BYTES);
-        tma_load_3d(saddr(sQ), &tmQ, q_full, 0, h, qt * BQ);
-        if (C::TAIL) tma_load_3d(saddr(sQ + C::Q128), &tmQt, q_full, 64, h, qt * BQ);
+        tma_load_3d(saddr(sQ), &tmQ, q_full, 0, h, tl.row0);
+        if (C::TAIL) tma_load_3d(saddr(sQ + C::Q128), &tmQt, q_full, 64, h, tl.row0);
         for (int kb = kb0; kb < kb1; ++kb, ++g) {
           const int st = g % KV_STAGES;
           if (!mbar_wait(kv_empty + 8 * st, ((g / KV_STAGES) & 1) ^ 1, abort_flag)) goto timeout;
           mbar_expect_tx(kv_full + 8 * st, C::KV_BYTES);
           uint8_t* base = sKV + st * C::KV_BYTES;
           const uint32_t fb = kv_full + 8 * st;
-          tma_load_3d(saddr(base), &tmK, fb, 0, h, kb * BKV);
-          if (C::TAIL) tma_load_3d(saddr(base + C::K128), &tmKt, fb, 64, h, kb * BKV);
-          tma_load_3d(saddr(base + C::K128 + C::K32), &tmV, fb, 0, h, kb * BKV);
-          if (C::TAIL) tma_load_3d(saddr(base + 2 * C::K128 + C::K32), &tmVt, fb, 64, h, kb * BKV);
+          tma_load_3d(saddr(base), &tmK, fb, 0, h, krow + kb * BKV);
+          if (C::TAIL) tma_load_3d(saddr(base + C::K128), &tmKt, fb, 64, h, krow + kb * BKV);
+          tma_load_3d(saddr(base + C::K128 + C::K32), &tmV, fb, 0, h, vrow + kb * BKV);
+          if (C::TAIL)
+            tma_load_3d(saddr(base + 2 * C::K128 + C::K32), &tmVt, fb, 64, h, vrow + kb * BKV);
         }
       }
     }
@@ -364,9 +385,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
       tmem_wait_ld();
       tc_fence_before();
       mbar_arrive(o_free);
-      const int qrow = qt * BQ + row;
       if (sc.split == 1) {
-        if (qrow < D) {
+        const TileLoc tl = locate_tile(rm, ai.n, D, qt);
+        const int qrow = tl.row0 + row;
+        if (row < tl.rows) {
           const float inv = l > 0.f ? 1.f / l : 0.f;
           uint4* dst = reinterpret_cast<uint4*>(O + size_t(qrow) * ldo + h * DH);
 #pragma unroll
@@ -414,20 +436,20 @@ done:
 template <int DH>
 __global__ void __launch_bounds__(256)
 attn_combine_kernel(const float* __restrict__ part, bf16* __restrict__ O, int ldo, int heads,
-                    int Dbound, const int* __restrict__ dcount, int Nk, int attn_grid,
-                    int ws_units, unsigned* err) {
+                    RowMap rm, int n_items, int Nk, int attn_grid, int ws_units, unsigned* err) {
   pdl_wait();
   pdl_trigger();
-  const int D = live_count(dcount, Dbound, err);
+  const int D = live_count(rm.count, rm.bound, err);
   AttnSched sc;
-  sc.init(D, heads, Nk, attn_grid, ws_units);
+  sc.init(query_tiles(rm, n_items, D), heads, Nk, attn_grid, ws_units);
   if (sc.split == 1) return;
   const int lane = threadIdx.x & 31;
   for (int gw = blockIdx.x * 8 + (threadIdx.x >> 5); gw < sc.pairs * BQ; gw += gridDim.x * 8) {
   const int pair = gw / BQ, row = gw - pair * BQ;
   const int qt = pair % sc.qtiles, h = pair / sc.qtiles;
-  const int qrow = qt * BQ + row;
-  if (qrow >= D) continue;
+  const TileLoc tl = locate_tile(rm, n_items, D, qt);
+  if (row >= tl.rows) continue;
+  const int qrow = tl.row0 + row;
   const float* base = part + size_t(pair) * sc.split * (BQ * PART_STRIDE) + size_t(row) * PART_STRIDE;
   float2 ml = make_float2(-INFINITY, 0.f);
   if (lane < sc.split) ml = __ldcg(reinterpret_cast<const float2*>(base + size_t(lane) * (BQ * PART_STRIDE) + DH));
@@ -548,43 +570,48 @@ size_t attention_split_floats(int Nmax, int heads, int dh) {
 
 
 cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* V, int ldkv,
-                             int Nk, bf16* O, int ldo, int heads, int dh, int Dbound,
-                             const int* dcount, unsigned* err, const AttnScratch& as,
+                             int kv_rows, const AttnItems& ai, int Nk, bf16* O, int ldo, int heads,
+                             int dh, const RowMap& rm, unsigned* err, const AttnScratch& as,
                              cudaStream_t st) {
-  if (Dbound <= 0) return cudaSuccess;
+  if (rm.bound <= 0) return cudaSuccess;
   if (dh != 72 && dh != 64) return cudaErrorInvalidValue;
+  if (ai.n < 1 || ai.n > MAX_ITEMS || (ai.n > 1 && !rm.meta)) return cudaErrorInvalidValue;
+  for (int i = 0; i < ai.n; ++i)
+    if (ai.krow[i] < 0 || ai.vrow[i] < 0 || ai.krow[i] > kv_rows - Nk || ai.vrow[i] > kv_rows - Nk)
+      return cudaErrorInvalidValue;
   const int sms = device_sms_attn();
   if (!sms) return cudaErrorInvalidDevice;
   // a 64-wide 128B-swizzled map and a 16-wide 32B-swizzled tail map per operand
   CUtensorMap tq, tqt, tk, tkt, tv, tvt;
-  RC_TRY(head_map(Q, Dbound, ldq, heads, dh, 64, BQ, &tq));
-  RC_TRY(head_map(K, Nk, ldkv, heads, dh, 64, BKV, &tk));
-  RC_TRY(head_map(V, Nk, ldkv, heads, dh, 64, BKV, &tv));
-  RC_TRY(head_map(Q, Dbound, ldq, heads, dh, 16, BQ, &tqt));
-  RC_TRY(head_map(K, Nk, ldkv, heads, dh, 16, BKV, &tkt));
-  RC_TRY(head_map(V, Nk, ldkv, heads, dh, 16, BKV, &tvt));
+  RC_TRY(head_map(Q, rm.bound, ldq, heads, dh, 64, BQ, &tq));
+  RC_TRY(head_map(K, kv_rows, ldkv, heads, dh, 64, BKV, &tk));
+  RC_TRY(head_map(V, kv_rows, ldkv, heads, dh, 64, BKV, &tv));
+  RC_TRY(head_map(Q, rm.bound, ldq, heads, dh, 16, BQ, &tqt));
+  RC_TRY(head_map(K, kv_rows, ldkv, heads, dh, 16, BKV, &tkt));
+  RC_TRY(head_map(V, kv_rows, ldkv, heads, dh, 16, BKV, &tvt));
   const float scale_log2 = float(1.4426950408889634 / sqrt(double(dh)));
   const int ws_units = int(as.part_floats / (size_t(BQ) * PART_STRIDE));
   const int grid = CTAS_PER_SM * sms;
   if (dh == 72)
     RC_TRY(launch_k(attn_tc_kernel<72>, dim3(grid), dim3(THREADS), ACfg<72>::SMEM, st, tq, tqt,
-                    tk, tkt, tv, tvt, Nk, O, ldo, heads, Dbound, dcount, scale_log2, err, as.part,
+                    tk, tkt, tv, tvt, ai, Nk, O, ldo, heads, rm, scale_log2, err, as.part,
                     ws_units));
   else
     RC_TRY(launch_k(attn_tc_kernel<64>, dim3(grid), dim3(THREADS), ACfg<64>::SMEM, st, tq, tqt,
-                    tk, tkt, tv, tvt, Nk, O, ldo, heads, Dbound, dcount, scale_log2, err, as.part,
+                    tk, tkt, tv, tvt, ai, Nk, O, ldo, heads, rm, scale_log2, err, as.part,
                     ws_units));
   count_launches(1);
   // key splits happen only with at least MIN_KB_PER_SPLIT key blocks per split
   if ((Nk + BKV - 1) / BKV >= 2 * MIN_KB_PER_SPLIT) {
-    const int warps = ((Dbound + BQ - 1) / BQ) * heads * BQ;
+    const int tiles = (rm.bound + BQ - 1) / BQ + ai.n - 1;  // bound of the query tiles
+    const int warps = tiles * heads * BQ;
     const int cgrid = min((warps + 7) / 8, 4 * sms);
     if (dh == 72)
       RC_TRY(launch_k(attn_combine_kernel<72>, dim3(cgrid), dim3(256), 0, st, as.part, O,
-                      ldo, heads, Dbound, dcount, Nk, grid, ws_units, err));
+                      ldo, heads, rm, ai.n, Nk, grid, ws_units, err));
     else
       RC_TRY(launch_k(attn_combine_kernel<64>, dim3(cgrid), dim3(256), 0, st, as.part, O,
-                      ldo, heads, Dbound, dcount, Nk, grid, ws_units, err));
+                      ldo, heads, rm, ai.n, Nk, grid, ws_units, err));
     count_launches(1);
   }
   return cudaSuccess;

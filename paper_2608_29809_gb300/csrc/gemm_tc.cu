@@ -75,7 +75,7 @@ __device__ __forceinline__ void red_add_v4(float* p, float a, float b, float c, 
 // Epilogue values of columns c0 .. c0+31 of one output row: bias (when
 // with_bias: a split gated residual adds it with its first piece only, its
 // update being a sum over pieces), tanh-GELU, gate.
-__device__ __forceinline__ void epilogue_values(const GemmEpi& ep, int c0, float* v,
+__device__ __forceinline__ void epilogue_values(const GemmEpi& ep, int c0, int item, float* v,
                                                 bool with_bias) {
   if (ep.bias && with_bias) {
     float b[32];
@@ -89,9 +89,10 @@ __device__ __forceinline__ void epilogue_values(const GemmEpi& ep, int c0, float
   } else if (ep.mode == EPI_GATE_RES && ep.gate_tab) {
     float g[32];
     load32(ep.gate_tab + c0, g);
-    if (ep.gate_tb) {
+    const float* tb = ep.gate_off >= 0 ? ep.its.tb[item] : nullptr;
+    if (tb) {
       float g2[32];
-      load32(ep.gate_tb + c0, g2);
+      load32(tb + ep.gate_off + c0, g2);
 #pragma unroll
       for (int i = 0; i < 32; ++i) g[i] += g2[i];
     }
@@ -101,9 +102,10 @@ __device__ __forceinline__ void epilogue_values(const GemmEpi& ep, int c0, float
 }
 
 // Destination of columns c0 .. c0+31 of output row r, or null when the row is
-// beyond the live count (or its token index is bad: QKV raises DEVERR_INDEX).
-// tok = idx[r] for the QKV epilogue, loaded once per tile.
-__device__ __forceinline__ char* chunk_dst(const GemmEpi& ep, int r, int M, int tok, int c0) {
+// beyond the live count (or its token / item index is bad: QKV raises
+// DEVERR_INDEX).  tok / item of the row are loaded once per tile.
+__device__ __forceinline__ char* chunk_dst(const GemmEpi& ep, int r, int M, int tok, int item,
+                                           int c0) {
   if (r >= M) return nullptr;
   switch (ep.mode) {
     case EPI_F32:
@@ -114,11 +116,12 @@ __device__ __forceinline__ char* chunk_dst(const GemmEpi& ep, int r, int M, int 
       const int part = c0 / ep.dsplit;
       const int cc = c0 - part * ep.dsplit;
       if (part == 0) return reinterpret_cast<char*>(ep.out_bf + size_t(r) * ep.ld_out + cc);
-      if (tok < 0 || tok >= ep.n_tokens) {
+      if (tok < 0 || tok >= ep.n_tokens || item < 0 || item >= ep.its.n) {
         atomicOr(ep.err, DEVERR_INDEX);
         return nullptr;
       }
-      return reinterpret_cast<char*>((part == 1 ? ep.kc : ep.vc) + size_t(tok) * ep.ld_kv + cc);
+      return reinterpret_cast<char*>(ep.its.slice[item] + (part == 1 ? ep.k_off : ep.v_off) +
+                                     size_t(tok) * ep.dsplit + cc);
     }
     default:
       return reinterpret_cast<char*>(ep.out_bf + size_t(r) * ep.ld_out + c0);
@@ -248,7 +251,8 @@ struct Segs {
 template <int BN>
 __global__ void __launch_bounds__(THREADS, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-               int Mbound, const int* __restrict__ dcount, int n, int k, GemmEpi ep) {
+               int Mbound, const int* __restrict__ dcount, int n, int k,
+               const __grid_constant__ GemmEpi ep) {
   using TC = TileCfg<BN>;
   constexpr int STAGES = TC::STAGES, STAGE_B = TC::STAGE_B, TMEM_COLS = TC::TMEM_COLS;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -366,7 +370,11 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       const int row = sp * 32 + lane;
       const int r = m * BM + row;
       const uint32_t tbase = tmem_base + uint32_t(acc * (TMEM_COLS / 2)) + (uint32_t(sp * 32) << 16);
-      const int tok = (ep.mode == EPI_QKV && r < M) ? (ep.idx ? __ldg(ep.idx + r) : r) : 0;
+      int tok = 0, item = 0;
+      if (r < M) {
+        if (ep.mode == EPI_QKV) tok = ep.tok ? __ldg(ep.tok + r) : r;
+        if (ep.item) item = __ldg(ep.item + r);
+      }
       // a piece of a split tile only occurs for the gated residual, whose
       // update is a sum: the bias goes with the piece that starts at k = 0
 #pragma unroll 1
@@ -374,8 +382,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         float v[32];
         tmem_ld32(tbase + uint32_t(ch * 32), v);
         const int c0 = nn * BN + ch * 32;
-        epilogue_values(ep, c0, v, kb0 == 0);
-        store_chunk(ep.mode, sStg + sp * STAGING_WARP, lane, v, chunk_dst(ep, r, M, tok, c0));
+        epilogue_values(ep, c0, item, v, kb0 == 0);
+        store_chunk(ep.mode, sStg + sp * STAGING_WARP, lane, v, chunk_dst(ep, r, M, tok, item, c0));
       }
       tc_fence_before();
       mbar_arrive(tempty0 + 8 * acc);

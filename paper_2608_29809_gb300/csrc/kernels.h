@@ -25,24 +25,62 @@ cudaError_t launch_localize(const float* A, int S, int N, int M, int gh, int gw,
                             const DeltaIds& ids, float tau, int dilation, uint8_t* mask,
                             int32_t* idx, int32_t* count, void* ws, cudaStream_t st);
 
+// ------------------------------------------------------------- step rows
+// A step processes one or more items (an item = one session's denoising
+// step).  Their dirty rows are concatenated into one compact row space: item
+// i owns rows [off_i, off_i + cnt_i) and row r is token tok[r] of item item[r].
+constexpr int MAX_ITEMS = 16;
+enum {
+  META_TOTAL = 0,                     // rows of all items
+  META_OFF = 1,                       // off[i]
+  META_CNT = 1 + MAX_ITEMS,           // cnt[i]
+  META_TILE = 1 + 2 * MAX_ITEMS,      // first 128-row query tile of item i; [n] = all tiles
+  META_INTS = 2 + 3 * MAX_ITEMS
+};
+struct RowMap {
+  const int* tok;    // [rows] token of row r (null: row r is token r)
+  const int* item;   // [rows] item of row r (null: every row is item 0)
+  const int* meta;   // device META_* table (null: a single item holding every row)
+  int bound;         // host bound of the row count
+  const int* count;  // device row count (null: bound)
+  int n_tokens;      // N; token indices outside [0, N) raise DEVERR_INDEX
+};
+// Per-item addressing (passed by value).
+struct Items {
+  int n;
+  bf16* slice[MAX_ITEMS];      // the item's (session, t) cache slice [L][H,K,V][N][d]
+  const float* tb[MAX_ITEMS];  // modulation [6][d] of the item's timestep (null: none)
+  float* latent[MAX_ITEMS];    // the item's latent (patch embedding input)
+};
+// Builds tok / item / meta of a multi-item step.  Item i contributes cnt_i =
+// min(*count_i, bound_i) rows (count_i null: bound_i) taken from idx_i (null:
+// tokens 0 .. cnt_i - 1).
+struct BatchIn {
+  int n;
+  const int* idx[MAX_ITEMS];
+  const int* count[MAX_ITEMS];
+  int bound[MAX_ITEMS];
+};
+cudaError_t launch_batch_rows(const BatchIn& in, int* tok, int* item, int* meta, int n_tokens,
+                              unsigned* err, cudaStream_t st);
+
 // --------------------------------------------------------------- row kernels
-// out[r] = bf16(LN(x[r]) * (1 + scale) + shift) for r < D; scale = tab_sc (+ tb_sc),
-// shift = tab_sh (+ tb_sh) (the tb_* terms may be null).  With hprev non-null
-// the row itself is also stored as bf16 to hprev[idx[r]] (the previous
-// block's merged hidden state, Section 3.3).
-cudaError_t launch_ln_mod(const float* x, int ldx, const float* tab_sh, const float* tb_sh,
-                          const float* tab_sc, const float* tb_sc, bf16* out, int ldo,
-                          int Dbound, const int* dcount, int d, bf16* hprev, const int* idx,
-                          int n_tokens, unsigned* err, cudaStream_t st);
+// out[r] = bf16(LN(x[r]) (1 + scale) + shift) for live rows r, with
+// shift = tab[k_sh] (+ tb_item[k_sh]), scale = tab[k_sc] (+ tb_item[k_sc])
+// ([6][d] vectors; tab may be null).  With hprev_off >= 0 the row itself is
+// also stored as bf16 to the item's cache slice at element offset
+// hprev_off + tok[r] * d (the previous block's merged hidden state, Section 3.3).
+cudaError_t launch_ln_mod(const float* x, const float* tab, int k_sh, int k_sc, const Items& it,
+                          bf16* out, const RowMap& rm, long long hprev_off, int d, unsigned* err,
+                          cudaStream_t st);
 // out[r] = bf16(x[r]) for r < D.
 cudaError_t launch_cast_rows(const float* x, int ldx, bf16* out, int ldo, int Dbound,
                              const int* dcount, int d, unsigned* err, cudaStream_t st);
 
-// xf[r] = W_e patch(idx[r]) + b_e + pos[idx[r]]  (idx null: identity)
-cudaError_t launch_patch_embed(const float* latent, int gh, int gw, int p, int C,
-                               const bf16* We, const float* be, const float* pos,
-                               const int* idx, int Dbound, const int* dcount, float* xf, int d,
-                               unsigned* err, cudaStream_t st);
+// xf[r] = W_e patch(tok[r]) + b_e + pos[tok[r]], the patch from the row's item latent.
+cudaError_t launch_patch_embed(int gh, int gw, int p, int C, const bf16* We, const float* be,
+                               const float* pos, const Items& it, const RowMap& rm, float* xf,
+                               int d, unsigned* err, cudaStream_t st);
 
 // Timestep embedding chain: f = sinusoid(t_value); h1 = W_t1 f + b; temb = W_t2 silu(h1) + b;
 // tb = W_tb silu(temb) + b.  scratch h1/f are caller buffers.
@@ -60,9 +98,9 @@ cudaError_t launch_final_ddim(const bf16* H, const float* temb, const float* tab
 cudaError_t launch_rows_f32(const float* src, float* dst, const int* idx, int Dbound,
                             const int* dcount, int d, int N, bool scatter, unsigned* err,
                             cudaStream_t st);
-// dst[idx[r]] = bf16(src[r]), f32 rows -> bf16 rows.
-cudaError_t launch_scatter_bf16(const float* src, bf16* dst, const int* idx, int Dbound,
-                                const int* dcount, int d, int N, unsigned* err, cudaStream_t st);
+// item slice + off + tok[r] * d  <-  bf16(src[r]), f32 rows -> bf16 cache rows.
+cudaError_t launch_scatter_bf16(const float* src, const Items& it, long long off,
+                                const RowMap& rm, int d, unsigned* err, cudaStream_t st);
 
 // ---------------------------------------------------------------------- GEMM
 enum EpiMode { EPI_F32 = 0, EPI_BIAS_BF16 = 1, EPI_GELU_BF16 = 2, EPI_GATE_RES = 3, EPI_QKV = 4 };
@@ -75,15 +113,15 @@ struct GemmEpi {
   float* out_f;            // F32
   float* xf;               // GATE_RES residual, f32
   int ld_xf;
-  const float* gate_tab;   // gate = gate_tab[c] (+ gate_tb[c]); null tab = no gate
-  const float* gate_tb;
-  bf16* kc;                // QKV: K rows idx[r] (cache)
-  bf16* vc;                // QKV: V rows idx[r] (cache)
-  int ld_kv;
+  const float* gate_tab;   // gate = gate_tab[c] (+ tb_item[gate_off + c]); null tab = no gate
+  long long gate_off;      // element offset of the gate in the item tb vectors (-1: none)
+  long long k_off, v_off;  // QKV: K / V rows at item slice + k_off / v_off + tok * dsplit
   int dsplit;              // QKV: hidden size (q | k | v boundaries)
-  const int* idx;          // row -> token index (null: identity)
-  int n_tokens;            // bound of idx values
+  const int* tok;          // row -> token (null: identity)
+  const int* item;         // row -> item (null: item 0)
+  int n_tokens;            // bound of token indices
   unsigned* err;
+  Items its;               // per-item cache slices and modulation vectors
 };
 
 // C[M][n] = A[M][k] W[n][k]^T, epilogue `ep`.  M = *dcount if non-null (bounded
@@ -100,11 +138,21 @@ struct AttnScratch {
 };
 size_t attention_split_floats(int Nmax, int heads, int dh);
 
-// O[r][h*dh..] = softmax(Q_r K^T / sqrt(dh)) V per head, over Nk keys.
-// Q/O compact rows (r < D), K/V rows 0..Nk-1 with row stride ldkv.
+// Per-item key / value placement of one attention launch: item i's keys are
+// rows krow[i] .. krow[i] + Nk - 1 of K (values likewise from vrow[i] of V).
+struct AttnItems {
+  int n;
+  int krow[MAX_ITEMS];
+  int vrow[MAX_ITEMS];
+};
+
+// O[r][h*dh..] = softmax(Q_r K_i^T / sqrt(dh)) V_i per head over the Nk keys of
+// row r's item i.  Q and O are compact rows (rm); K / V are row-major with row
+// stride ldkv and kv_rows rows in all.  Keys beyond Nk are masked, but their
+// values must be finite (they are multiplied by zero).
 cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* V, int ldkv,
-                             int Nk, bf16* O, int ldo, int heads, int dh, int Dbound,
-                             const int* dcount, unsigned* err, const AttnScratch& as,
+                             int kv_rows, const AttnItems& ai, int Nk, bf16* O, int ldo, int heads,
+                             int dh, const RowMap& rm, unsigned* err, const AttnScratch& as,
                              cudaStream_t st);
 
 }  // namespace rc

@@ -54,6 +54,7 @@ void set_last_error(const char* msg) { g_last_error = msg; }
 struct rc_ctx {
   rc_dims dims;
   int N, d, F, dh, L, T, M;
+  int max_batch;  // items per batched step; row scratch = max_batch * N rows
   int device;
   std::vector<rc_layer_weights> lw;
   std::vector<char> lw_set;
@@ -61,17 +62,20 @@ struct rc_ctx {
   bool gw_set = false;
   std::vector<float> t_values, alpha_bar;
   bool sched_set = false;
-  // device scratch
-  float* xf = nullptr;   // [N][d] residual rows of the dirty tokens (compact)
-  bf16* xb = nullptr;    // [N][d] GEMM input: modulated rows / residual copy
-  bf16* ob = nullptr;    // [N][d] attention output
-  bf16* q = nullptr;     // [N][d] queries (self, then cross)
-  bf16* u = nullptr;     // [N][F] MLP hidden
+  // device scratch (R = max_batch * N compact rows)
+  float* xf = nullptr;   // [R][d] residual rows of the dirty tokens (compact)
+  bf16* xb = nullptr;    // [R][d] GEMM input: modulated rows / residual copy
+  bf16* ob = nullptr;    // [R][d] attention output
+  bf16* q = nullptr;     // [R][d] queries (self, then cross)
+  bf16* u = nullptr;     // [R][F] MLP hidden
   float* fbuf = nullptr; // [freq_dim]
   float* h1 = nullptr;   // [d]
-  float* temb = nullptr; // [d]
-  float* tb = nullptr;   // [6d]
+  float* temb = nullptr; // [RC_MAX_BATCH][d] timestep embedding per item
+  float* tb = nullptr;   // [RC_MAX_BATCH][6d] t_block modulation per item
   int* iota = nullptr;   // [N] identity row map (dense path)
+  int* b_tok = nullptr;  // [R] token of each compact row (batched steps)
+  int* b_item = nullptr; // [R] item of each compact row (batched steps)
+  int* b_meta = nullptr; // [META_INTS] row offsets / counts / query tiles per item
   unsigned* err = nullptr;
   rc::AttnScratch as{};  // key-split partial outputs
   // timing probe
@@ -88,10 +92,14 @@ struct rc_cache {
   std::vector<char> text_set;
 
   size_t slot_elems() const { return size_t(ctx->N) * ctx->d; }
-  bf16* slot(int s, int l, int t, int which) const {
-    size_t i = ((size_t(s) * ctx->T + t) * ctx->L + l) * 3 + which;
-    return base + i * slot_elems();
+  // index of the [N][d] slot (s, l, t, which) in units of slots
+  size_t slot_index(int s, int l, int t, int which) const {
+    return ((size_t(s) * ctx->T + t) * ctx->L + l) * 3 + which;
   }
+  bf16* slot(int s, int l, int t, int which) const {
+    return base + slot_index(s, l, t, which) * slot_elems();
+  }
+  size_t total_rows() const { return size_t(sessions) * ctx->T * ctx->L * 3 * ctx->N; }
   bf16* text_kv(int s, int l) const {
     return text + (size_t(s) * ctx->L + l) * size_t(ctx->M) * 2 * ctx->d;
   }
@@ -145,8 +153,9 @@ struct Probe {
 void free_ctx(rc_ctx* c) {
   if (!c) return;
   probe_free(c);
-  void* ps[] = {c->xf,   c->xb,  c->ob,   c->q,        c->u,         c->fbuf,
-                c->h1,   c->temb, c->tb,  c->iota,     c->err,       c->as.part};
+  void* ps[] = {c->xf,   c->xb,   c->ob,   c->q,    c->u,      c->fbuf,
+                c->h1,   c->temb, c->tb,   c->iota, c->b_tok,  c->b_item,
+                c->b_meta, c->err, c->as.part};
   for (void* p : ps)
     if (p) cudaFree(p);
   delete c;
@@ -168,127 +177,145 @@ rc_status check_ready(const rc_ctx* c, const rc_cache* cache, int session, bool 
   return RC_OK;
 }
 
-// Row map of a call: the dirty rows (idx, D bound, optional device count).
-struct Rows {
-  const int* idx;
-  int bound;
-  const int* dcount;
+// The items of one step (one for rc_step / rc_block_forward_region): cache
+// slices and modulation vectors for the kernels, key / value rows of every
+// item for the attention launches.
+struct StepItems {
+  rc::Items its{};
+  int session[rc::MAX_ITEMS] = {};
+  int t[rc::MAX_ITEMS] = {};
 };
 
+rc::AttnItems self_kv(const rc_cache* k, const StepItems& si, int l) {
+  rc::AttnItems ai{};
+  ai.n = si.its.n;
+  for (int i = 0; i < ai.n; ++i) {
+    ai.krow[i] = int(k->slot_index(si.session[i], l, si.t[i], 1) * k->ctx->N);
+    ai.vrow[i] = int(k->slot_index(si.session[i], l, si.t[i], 2) * k->ctx->N);
+  }
+  return ai;
+}
+
+rc::AttnItems text_kv_rows(const rc_cache* k, const StepItems& si, int l) {
+  rc::AttnItems ai{};
+  ai.n = si.its.n;
+  for (int i = 0; i < ai.n; ++i)
+    ai.krow[i] = ai.vrow[i] = (si.session[i] * k->ctx->L + l) * k->ctx->M;
+  return ai;
+}
+
 // One region-sparse block on the compact residual rows c->xf (Section 3.3,
-// Region-Level Sparse Attention; Section 3.4, Kernel Fusing).  tab / tbv give
-// the modulation vector as tab (+ tbv), each [6][d] (tbv may be null).
-rc_status run_block(rc_ctx* c, rc_cache* cache, int s, int l, int t, const Rows& rw,
-                    const float* tab, const float* tbv, bf16* hprev, cudaStream_t st) {
+// Region-Level Sparse Attention; Section 3.4, Kernel Fusing).  The modulation
+// vector of a row is tab (+ the row item's tb), each [6][d].  hprev_off >= 0:
+// the block input (the previous block's merged output H^l) is also written to
+// the cache slice at that element offset.
+rc_status run_block(rc_ctx* c, rc_cache* k, int l, const rc::RowMap& rm, const StepItems& si,
+                    const float* tab, long long hprev_off, cudaStream_t st) {
   const int d = c->d, F = c->F, N = c->N;
   const rc_layer_weights& w = c->lw[l];
-  auto mv = [&](const float* base, int k) { return base ? base + size_t(k) * d : nullptr; };
-  bf16* Kc = cache->slot(s, l, t, 1);
-  bf16* Vc = cache->slot(s, l, t, 2);
-  const bf16* tk = cache->text_kv(s, l);
-  const bf16* tv = tk + d;
+  const size_t Nd = size_t(N) * d;
 
   // x_hat = LN(x)(1 + scale_msa) + shift_msa; x itself is the previous
   // block's output H^l of the dirty rows, written to their cache rows here
-  RC_CUDA(rc::launch_ln_mod(c->xf, d, mv(tab, 0), mv(tbv, 0), mv(tab, 1), mv(tbv, 1), c->xb, d,
-                            rw.bound, rw.dcount, d, hprev, rw.idx, N, c->err, st),
+  RC_CUDA(rc::launch_ln_mod(c->xf, tab, 0, 1, si.its, c->xb, rm, hprev_off, d, c->err, st),
           "ln_mod(msa)");
-  // [q | k | v] = x_hat W_qkv^T + b; k, v rows go straight to cache rows idx[r]
+  // [q | k | v] = x_hat W_qkv^T + b; k, v rows go straight to cache rows tok[r]
   rc::GemmEpi e{};
   e.mode = rc::EPI_QKV;
   e.bias = w.b_qkv;
   e.out_bf = c->q;
   e.ld_out = d;
-  e.kc = Kc;
-  e.vc = Vc;
-  e.ld_kv = d;
+  e.k_off = (long long)(size_t(l) * 3 + 1) * Nd;
+  e.v_off = (long long)(size_t(l) * 3 + 2) * Nd;
   e.dsplit = d;
-  e.idx = rw.idx;
+  e.tok = rm.tok;
+  e.item = rm.item;
   e.n_tokens = N;
   e.err = c->err;
+  e.its = si.its;
+  e.gate_off = -1;
   {
     Probe pr(c, RC_PROBE_GEMM, st);
-    RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_qkv), rw.bound, rw.dcount, 3 * d,
-                            d, e, st), "gemm(qkv)");
+    RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_qkv), rm.bound, rm.count,
+                            3 * d, d, e, st), "gemm(qkv)");
   }
-  // dirty queries over all N keys / values of (l, t)
+  // dirty queries over all N keys / values of each item's (session, l, t)
   {
     Probe pr(c, RC_PROBE_ATTENTION, st);
-    RC_CUDA(rc::launch_attention(c->q, d, Kc, Vc, d, N, c->ob, d, c->dims.heads, c->dh, rw.bound,
-                                 rw.dcount, c->err, c->as, st), "attention(self)");
+    RC_CUDA(rc::launch_attention(c->q, d, k->base, k->base, d, int(k->total_rows()),
+                                 self_kv(k, si, l), N, c->ob, d, c->dims.heads, c->dh, rm,
+                                 c->err, c->as, st), "attention(self)");
   }
   // x += gate_msa (o W_o^T + b_o)
-  e = rc::GemmEpi{};
-  e.mode = rc::EPI_GATE_RES;
-  e.bias = w.b_o;
-  e.xf = c->xf;
-  e.ld_xf = d;
-  e.gate_tab = mv(tab, 2);
-  e.gate_tb = mv(tbv, 2);
-  e.err = c->err;
+  auto gated = [&](const float* bias, int gate_k) {
+    rc::GemmEpi g{};
+    g.mode = rc::EPI_GATE_RES;
+    g.bias = bias;
+    g.xf = c->xf;
+    g.ld_xf = d;
+    g.gate_tab = gate_k >= 0 && tab ? tab + size_t(gate_k) * d : nullptr;
+    g.gate_off = gate_k >= 0 ? (long long)gate_k * d : -1;
+    g.item = rm.item;
+    g.n_tokens = N;
+    g.err = c->err;
+    g.its = si.its;
+    return g;
+  };
+  e = gated(w.b_o, 2);
   {
     Probe pr(c, RC_PROBE_GEMM, st);
-    RC_CUDA(rc::launch_gemm(c->ob, d, static_cast<const bf16*>(w.W_o), rw.bound, rw.dcount, d, d, e,
-                            st), "gemm(out)");
+    RC_CUDA(rc::launch_gemm(c->ob, d, static_cast<const bf16*>(w.W_o), rm.bound, rm.count, d, d,
+                            e, st), "gemm(out)");
   }
   // q' = x W_xq^T + b (on a bf16 copy of x)
-  RC_CUDA(rc::launch_cast_rows(c->xf, d, c->xb, d, rw.bound, rw.dcount, d, c->err, st), "cast");
+  RC_CUDA(rc::launch_cast_rows(c->xf, d, c->xb, d, rm.bound, rm.count, d, c->err, st), "cast");
   e = rc::GemmEpi{};
   e.mode = rc::EPI_BIAS_BF16;
   e.bias = w.b_xq;
   e.out_bf = c->q;
   e.ld_out = d;
+  e.gate_off = -1;
   e.err = c->err;
   {
     Probe pr(c, RC_PROBE_GEMM, st);
-    RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_xq), rw.bound, rw.dcount, d, d,
+    RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_xq), rm.bound, rm.count, d, d,
                             e, st), "gemm(xq)");
   }
   {
     Probe pr(c, RC_PROBE_ATTENTION, st);
-    RC_CUDA(rc::launch_attention(c->q, d, tk, tv, 2 * d, c->M, c->ob, d, c->dims.heads, c->dh,
-                                 rw.bound, rw.dcount, c->err, c->as, st), "attention(cross)");
+    RC_CUDA(rc::launch_attention(c->q, d, k->text, k->text + d, 2 * d,
+                                 k->sessions * c->L * c->M, text_kv_rows(k, si, l), c->M, c->ob,
+                                 d, c->dims.heads, c->dh, rm, c->err, c->as, st),
+            "attention(cross)");
   }
-  // x += o' W_xo^T + b
-  e = rc::GemmEpi{};
-  e.mode = rc::EPI_GATE_RES;
-  e.bias = w.b_xo;
-  e.xf = c->xf;
-  e.ld_xf = d;
-  e.err = c->err;
+  // x += o' W_xo^T + b (no gate)
+  e = gated(w.b_xo, -1);
   {
     Probe pr(c, RC_PROBE_GEMM, st);
-    RC_CUDA(rc::launch_gemm(c->ob, d, static_cast<const bf16*>(w.W_xo), rw.bound, rw.dcount, d, d,
+    RC_CUDA(rc::launch_gemm(c->ob, d, static_cast<const bf16*>(w.W_xo), rm.bound, rm.count, d, d,
                             e, st), "gemm(xo)");
   }
   // MLP
-  RC_CUDA(rc::launch_ln_mod(c->xf, d, mv(tab, 3), mv(tbv, 3), mv(tab, 4), mv(tbv, 4), c->xb, d,
-                            rw.bound, rw.dcount, d, nullptr, nullptr, N, c->err, st),
+  RC_CUDA(rc::launch_ln_mod(c->xf, tab, 3, 4, si.its, c->xb, rm, -1, d, c->err, st),
           "ln_mod(mlp)");
   e = rc::GemmEpi{};
   e.mode = rc::EPI_GELU_BF16;
   e.bias = w.b_1;
   e.out_bf = c->u;
   e.ld_out = F;
+  e.gate_off = -1;
   e.err = c->err;
   {
     Probe pr(c, RC_PROBE_GEMM, st);
-    RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_1), rw.bound, rw.dcount, F, d, e,
-                            st), "gemm(fc1)");
+    RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_1), rm.bound, rm.count, F, d,
+                            e, st), "gemm(fc1)");
   }
   // x += gate_mlp (u W_2^T + b_2); the caller stores x as the merged H^{l+1}
-  e = rc::GemmEpi{};
-  e.mode = rc::EPI_GATE_RES;
-  e.bias = w.b_2;
-  e.xf = c->xf;
-  e.ld_xf = d;
-  e.gate_tab = mv(tab, 5);
-  e.gate_tb = mv(tbv, 5);
-  e.err = c->err;
+  e = gated(w.b_2, 5);
   {
     Probe pr(c, RC_PROBE_GEMM, st);
-    RC_CUDA(rc::launch_gemm(c->u, F, static_cast<const bf16*>(w.W_2), rw.bound, rw.dcount, d, F, e,
-                            st), "gemm(fc2)");
+    RC_CUDA(rc::launch_gemm(c->u, F, static_cast<const bf16*>(w.W_2), rm.bound, rm.count, d, F,
+                            e, st), "gemm(fc2)");
   }
   return RC_OK;
 }
@@ -334,6 +361,9 @@ rc_status rc_create(const rc_dims* dims, rc_ctx** out) {
   if (N > 16384) return fail(RC_ERR_SHAPE, "N = %lld tokens > 16384", N);
   if (D.in_ch * D.patch * D.patch > 16 || D.out_ch < D.in_ch)
     return fail(RC_ERR_SHAPE, "in_ch * patch^2 must be <= 16 and out_ch >= in_ch");
+  const int max_batch = D.max_batch <= 0 ? 1 : D.max_batch;
+  if (max_batch > RC_MAX_BATCH)
+    return fail(RC_ERR_INVALID_ARG, "max_batch %d above %d", D.max_batch, RC_MAX_BATCH);
 
   rc_ctx* c = new (std::nothrow) rc_ctx();
   if (!c) return fail(RC_ERR_OOM, "host allocation");
@@ -345,16 +375,22 @@ rc_status rc_create(const rc_dims* dims, rc_ctx** out) {
   c->L = D.layers;
   c->T = D.timesteps;
   c->M = D.text_len;
+  c->max_batch = max_batch;
   cudaGetDevice(&c->device);
   c->lw.resize(c->L);
   c->lw_set.assign(c->L, 0);
   rc_status s = RC_OK;
-  const size_t Nd = size_t(N) * D.hidden;
-  if ((s = dalloc(&c->xf, Nd, "xf")) || (s = dalloc(&c->xb, Nd, "xb")) ||
-      (s = dalloc(&c->ob, Nd, "ob")) || (s = dalloc(&c->q, Nd, "q")) ||
-      (s = dalloc(&c->u, size_t(N) * D.mlp, "u")) || (s = dalloc(&c->fbuf, D.freq_dim, "f")) ||
-      (s = dalloc(&c->h1, D.hidden, "h1")) || (s = dalloc(&c->temb, D.hidden, "temb")) ||
-      (s = dalloc(&c->tb, 6 * size_t(D.hidden), "tb")) || (s = dalloc(&c->iota, N, "iota")) ||
+  const size_t R = size_t(max_batch) * N;  // compact rows of a step
+  const size_t Rd = R * D.hidden;
+  if ((s = dalloc(&c->xf, Rd, "xf")) || (s = dalloc(&c->xb, Rd, "xb")) ||
+      (s = dalloc(&c->ob, Rd, "ob")) || (s = dalloc(&c->q, Rd, "q")) ||
+      (s = dalloc(&c->u, R * D.mlp, "u")) || (s = dalloc(&c->fbuf, D.freq_dim, "f")) ||
+      (s = dalloc(&c->h1, D.hidden, "h1")) ||
+      (s = dalloc(&c->temb, size_t(RC_MAX_BATCH) * D.hidden, "temb")) ||
+      (s = dalloc(&c->tb, size_t(RC_MAX_BATCH) * 6 * D.hidden, "tb")) ||
+      (s = dalloc(&c->iota, N, "iota")) || (s = dalloc(&c->b_tok, R, "batch tok")) ||
+      (s = dalloc(&c->b_item, R, "batch item")) ||
+      (s = dalloc(&c->b_meta, size_t(rc::META_INTS), "batch meta")) ||
       (s = dalloc(&c->err, 1, "err"))) {
     free_ctx(c);
     return s;
@@ -424,11 +460,24 @@ rc_status rc_cache_create(rc_ctx* c, int sessions, rc_cache** out) {
   k->ctx = c;
   k->sessions = sessions;
   k->text_set.assign(sessions, 0);
+  // attention addresses every cache row with a 32-bit tensor coordinate
+  if (k->total_rows() >= (size_t(1) << 31) || size_t(sessions) * c->L * c->M >= (size_t(1) << 31)) {
+    delete k;
+    return fail(RC_ERR_SHAPE, "cache of %d sessions has 2^31 rows or more", sessions);
+  }
   const size_t n = size_t(sessions) * c->T * c->L * 3 * k->slot_elems();
   rc_status s = dalloc(&k->base, n, "cache");
-  if (s == RC_OK) s = dalloc(&k->text, size_t(sessions) * c->L * c->M * 2 * c->d, "text kv");
+  const size_t n_text = size_t(sessions) * c->L * c->M * 2 * c->d;
+  if (s == RC_OK) s = dalloc(&k->text, n_text, "text kv");
+  // zero-filled: the attention reads whole 64-key blocks, and keys past a
+  // slot's end (weighted by zero) come from the next slot, which must be finite
+  if (s == RC_OK && (cudaMemset(k->base, 0, n * sizeof(bf16)) != cudaSuccess ||
+                     cudaMemset(k->text, 0, n_text * sizeof(bf16)) != cudaSuccess ||
+                     cudaDeviceSynchronize() != cudaSuccess))
+    s = fail(RC_ERR_CUDA, "cache zero fill failed");
   if (s != RC_OK) {
     if (k->base) cudaFree(k->base);
+    if (k->text) cudaFree(k->text);
     delete k;
     return s;
   }
@@ -535,15 +584,15 @@ rc_status rc_localize_mask(const float* xattn, int S, int N, int M, int grid_h, 
   return RC_OK;
 }
 
-static rc_status rows_of(const rc_ctx* c, const int32_t* idx, int D, const int32_t* dcount,
-                         Rows* rw) {
+// The dirty rows of one item: host bound and optional device count.
+static rc_status dirty_rows(const rc_ctx* c, const int32_t* idx, int D, const int32_t* dcount,
+                            int* bound) {
   if (D < -1 || D > c->N) return fail(RC_ERR_INVALID_ARG, "D = %d outside [-1, %d]", D, c->N);
   if (D == -1 && !dcount) return fail(RC_ERR_INVALID_ARG, "D = -1 needs a device dirty_count");
-  const int bound = D < 0 ? c->N : D;
-  if (bound > 0 && !idx) return fail(RC_ERR_INVALID_ARG, "dirty_idx is null");
-  rw->idx = idx;
-  rw->bound = bound;
-  rw->dcount = dcount;
+  *bound = D < 0 ? c->N : D;
+  if (*bound > 0 && !idx) return fail(RC_ERR_INVALID_ARG, "dirty_idx is null");
+  if (idx && (reinterpret_cast<uintptr_t>(idx) & 3u))
+    return fail(RC_ERR_INVALID_ARG, "dirty_idx not 4-B aligned");
   return RC_OK;
 }
 
@@ -560,17 +609,104 @@ rc_status rc_block_forward_region(rc_ctx* c, rc_cache* k, int s, int l, int t, f
   if (!aligned16(hidden) || !aligned16(mod6))
     return fail(RC_ERR_INVALID_ARG, "hidden / mod6 not 16-B aligned");
   if ((r = check_ready(c, k, s, false))) return r;
-  Rows rw;
-  if ((r = rows_of(c, dirty_idx, D, dirty_count, &rw))) return r;
-  if (rw.bound == 0) return RC_OK;
+  int bound = 0;
+  if ((r = dirty_rows(c, dirty_idx, D, dirty_count, &bound))) return r;
+  if (bound == 0) return RC_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  RC_CUDA(rc::launch_rows_f32(hidden, c->xf, rw.idx, rw.bound, rw.dcount, c->d, c->N, false,
+  StepItems si;
+  si.its.n = 1;
+  si.its.slice[0] = k->slot(s, 0, t, 0);
+  si.session[0] = s;
+  si.t[0] = t;
+  const rc::RowMap rm{dirty_idx, nullptr, nullptr, bound, dirty_count, c->N};
+  RC_CUDA(rc::launch_rows_f32(hidden, c->xf, dirty_idx, bound, dirty_count, c->d, c->N, false,
                               c->err, st), "gather");
-  if ((r = run_block(c, k, s, l, t, rw, mod6, nullptr, nullptr, st))) return r;
-  RC_CUDA(rc::launch_scatter_bf16(c->xf, k->slot(s, l, t, 0), rw.idx, rw.bound, rw.dcount, c->d,
-                                  c->N, c->err, st), "H scatter");
-  RC_CUDA(rc::launch_rows_f32(c->xf, hidden, rw.idx, rw.bound, rw.dcount, c->d, c->N, true,
+  if ((r = run_block(c, k, l, rm, si, mod6, -1, st))) return r;
+  RC_CUDA(rc::launch_scatter_bf16(c->xf, si.its, (long long)(size_t(l) * 3) * c->N * c->d, rm,
+                                  c->d, c->err, st), "H scatter");
+  RC_CUDA(rc::launch_rows_f32(c->xf, hidden, dirty_idx, bound, dirty_count, c->d, c->N, true,
                               c->err, st), "scatter");
+  return RC_OK;
+}
+
+// Denoising steps of n items (validated by the callers).
+static rc_status step_items(rc_ctx* c, rc_cache* k, const rc_batch_item* items, int n,
+                            cudaStream_t st) {
+  const rc_global_weights& g = c->gw;
+  const int d = c->d, N = c->N;
+  const size_t Nd = size_t(N) * d;
+  StepItems si;
+  si.its.n = n;
+  rc::BatchIn bin{};
+  bin.n = n;
+  long long rows = 0;
+  for (int i = 0; i < n; ++i) {
+    const rc_batch_item& it = items[i];
+    si.session[i] = it.session;
+    si.t[i] = it.t;
+    si.its.slice[i] = k->slot(it.session, 0, it.t, 0);
+    si.its.tb[i] = c->tb + size_t(i) * 6 * d;
+    si.its.latent[i] = it.latent;
+    if (it.mode == RC_MODE_DENSE) {
+      bin.idx[i] = c->iota;
+      bin.bound[i] = N;
+    } else if (it.mode == RC_MODE_SPARSE) {
+      bin.idx[i] = it.dirty_idx;
+      bin.count[i] = it.dirty_count;
+      bin.bound[i] = it.D < 0 ? N : it.D;
+    }
+    rows += bin.bound[i];
+    RC_CUDA(rc::launch_t_embed(c->t_values[it.t], c->dims.freq_dim, d,
+                               static_cast<const bf16*>(g.W_t1), g.b_t1,
+                               static_cast<const bf16*>(g.W_t2), g.b_t2,
+                               static_cast<const bf16*>(g.W_tb), g.b_tb, c->fbuf, c->h1,
+                               c->temb + size_t(i) * d, c->tb + size_t(i) * 6 * d, st),
+            "t_embed");
+  }
+  if (rows > 0) {
+    // compact rows: a single item uses its own index list; several items are
+    // concatenated on the device (their counts may live there)
+    rc::RowMap rm{bin.idx[0], nullptr, nullptr, int(rows), bin.count[0], N};
+    if (n > 1) {
+      RC_CUDA(rc::launch_batch_rows(bin, c->b_tok, c->b_item, c->b_meta, N, c->err, st),
+              "batch rows");
+      rm = rc::RowMap{c->b_tok, c->b_item, c->b_meta, int(rows), c->b_meta + rc::META_TOTAL, N};
+    }
+    RC_CUDA(rc::launch_patch_embed(c->dims.grid_h, c->dims.grid_w, c->dims.patch, c->dims.in_ch,
+                                   static_cast<const bf16*>(g.W_e), g.b_e, g.pos, si.its, rm,
+                                   c->xf, d, c->err, st),
+            "patch_embed");
+    for (int l = 0; l < c->L; ++l) {
+      rc_status r = run_block(c, k, l, rm, si, c->lw[l].table,
+                              l > 0 ? (long long)(size_t(l - 1) * 3) * Nd : -1, st);
+      if (r) return r;
+    }
+    RC_CUDA(rc::launch_scatter_bf16(c->xf, si.its, (long long)(size_t(c->L - 1) * 3) * Nd, rm, d,
+                                    c->err, st), "H scatter");
+  }
+  for (int i = 0; i < n; ++i) {
+    const rc_batch_item& it = items[i];
+    RC_CUDA(rc::launch_final_ddim(k->slot(it.session, c->L - 1, it.t, 0), c->temb + size_t(i) * d,
+                                  g.table_f, static_cast<const bf16*>(g.W_f), g.b_f, it.latent,
+                                  c->dims.grid_h, c->dims.grid_w, c->dims.patch, c->dims.in_ch,
+                                  c->dims.out_ch, d, c->alpha_bar[it.t], c->alpha_bar[it.t + 1],
+                                  st), "final_ddim");
+  }
+  return RC_OK;
+}
+
+static rc_status check_item(rc_ctx* c, rc_cache* k, const rc_batch_item& it) {
+  rc_status r = check_session(k, it.session);
+  if (r) return r;
+  if (it.t < 0 || it.t >= c->T) return fail(RC_ERR_INVALID_ARG, "t %d outside [0, %d)", it.t, c->T);
+  if (!it.latent || !aligned16(it.latent))
+    return fail(RC_ERR_INVALID_ARG, "latent null or not 16-B aligned");
+  if (it.mode != RC_MODE_DENSE && it.mode != RC_MODE_SPARSE && it.mode != RC_MODE_REUSE)
+    return fail(RC_ERR_INVALID_ARG, "mode %d is not a mode", it.mode);
+  if ((r = check_ready(c, k, it.session, true))) return r;
+  int bound = 0;
+  if (it.mode == RC_MODE_SPARSE && (r = dirty_rows(c, it.dirty_idx, it.D, it.dirty_count, &bound)))
+    return r;
   return RC_OK;
 }
 
@@ -580,41 +716,28 @@ rc_status rc_step(rc_ctx* c, rc_cache* k, int s, float* latent, int t,
   if (!c || !k || !latent || !schedule_host)
     return fail(RC_ERR_INVALID_ARG, "rc_step: null argument");
   if (k->ctx != c) return fail(RC_ERR_INVALID_ARG, "cache belongs to another context");
-  rc_status r = check_session(k, s);
-  if (r) return r;
   if (t < 0 || t >= c->T) return fail(RC_ERR_INVALID_ARG, "t %d outside [0, %d)", t, c->T);
-  if (!aligned16(latent)) return fail(RC_ERR_INVALID_ARG, "latent not 16-B aligned");
-  const int mode = schedule_host[t];
-  if (mode != RC_MODE_DENSE && mode != RC_MODE_SPARSE && mode != RC_MODE_REUSE)
-    return fail(RC_ERR_INVALID_ARG, "schedule[%d] = %d is not a mode", t, mode);
-  if ((r = check_ready(c, k, s, true))) return r;
-  Rows rw{c->iota, c->N, nullptr};
-  if (mode == RC_MODE_SPARSE && (r = rows_of(c, dirty_idx, D, dirty_count, &rw))) return r;
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
-  const rc_global_weights& g = c->gw;
-  const int d = c->d;
-  RC_CUDA(rc::launch_t_embed(c->t_values[t], c->dims.freq_dim, d,
-                             static_cast<const bf16*>(g.W_t1), g.b_t1,
-                             static_cast<const bf16*>(g.W_t2), g.b_t2,
-                             static_cast<const bf16*>(g.W_tb), g.b_tb, c->fbuf, c->h1, c->temb,
-                             c->tb, st), "t_embed");
-  if (mode != RC_MODE_REUSE && rw.bound > 0) {
-    RC_CUDA(rc::launch_patch_embed(latent, c->dims.grid_h, c->dims.grid_w, c->dims.patch,
-                                   c->dims.in_ch, static_cast<const bf16*>(g.W_e), g.b_e, g.pos,
-                                   rw.idx, rw.bound, rw.dcount, c->xf, d, c->err, st),
-            "patch_embed");
-    for (int l = 0; l < c->L; ++l)
-      if ((r = run_block(c, k, s, l, t, rw, c->lw[l].table, c->tb,
-                         l > 0 ? k->slot(s, l - 1, t, 0) : nullptr, st)))
-        return r;
-    RC_CUDA(rc::launch_scatter_bf16(c->xf, k->slot(s, c->L - 1, t, 0), rw.idx, rw.bound,
-                                    rw.dcount, d, c->N, c->err, st), "H scatter");
+  rc_batch_item it{s, latent, t, int(schedule_host[t]), dirty_idx, D, dirty_count};
+  rc_status r = check_item(c, k, it);
+  if (r) return r;
+  return step_items(c, k, &it, 1, static_cast<cudaStream_t>(stream));
+}
+
+rc_status rc_step_batched(rc_ctx* c, rc_cache* k, const rc_batch_item* items, int n,
+                          rc_stream stream) {
+  if (!c || !k || !items) return fail(RC_ERR_INVALID_ARG, "rc_step_batched: null argument");
+  if (k->ctx != c) return fail(RC_ERR_INVALID_ARG, "cache belongs to another context");
+  if (n < 1 || n > c->max_batch)
+    return fail(RC_ERR_INVALID_ARG, "n_items %d outside [1, %d]", n, c->max_batch);
+  for (int i = 0; i < n; ++i) {
+    rc_status r = check_item(c, k, items[i]);
+    if (r) return r;
+    for (int j = 0; j < i; ++j)
+      if (items[j].session == items[i].session && items[j].t == items[i].t)
+        return fail(RC_ERR_INVALID_ARG, "items %d and %d share session %d, t %d", j, i,
+                    items[i].session, items[i].t);
   }
-  RC_CUDA(rc::launch_final_ddim(k->slot(s, c->L - 1, t, 0), c->temb, g.table_f,
-                                static_cast<const bf16*>(g.W_f), g.b_f, latent, c->dims.grid_h,
-                                c->dims.grid_w, c->dims.patch, c->dims.in_ch, c->dims.out_ch, d,
-                                c->alpha_bar[t], c->alpha_bar[t + 1], st), "final_ddim");
-  return RC_OK;
+  return step_items(c, k, items, n, static_cast<cudaStream_t>(stream));
 }
 
 rc_status rc_step_dense(rc_ctx* c, rc_cache* k, int s, float* latent, int t, rc_stream stream) {
@@ -654,12 +777,13 @@ rc_status rc_attention(rc_ctx* c, const void* Q, int ldq, const void* K, const v
     return fail(RC_ERR_INVALID_ARG, "rc_attention: pointers must be 16-B aligned");
   if (Nq == 0) return RC_OK;
   if (Nk == 0) return fail(RC_ERR_SHAPE, "rc_attention: Nk = 0 with queries");
-  if ((Nq + 127) / 128 > (c->N + 127) / 128)
-    return fail(RC_ERR_SHAPE, "rc_attention: Nq %d above the context's %d tokens", Nq, c->N);
+  rc::AttnItems ai{};
+  ai.n = 1;
+  const rc::RowMap rm{nullptr, nullptr, nullptr, Nq, nullptr, Nk};
   RC_CUDA(rc::launch_attention(static_cast<const bf16*>(Q), ldq, static_cast<const bf16*>(K),
-                               static_cast<const bf16*>(V), ldkv, Nk, static_cast<bf16*>(O), ldo,
-                               c->dims.heads, c->dh, Nq, nullptr, c->err, c->as,
-                               static_cast<cudaStream_t>(stream)),
+                               static_cast<const bf16*>(V), ldkv, Nk, ai, Nk,
+                               static_cast<bf16*>(O), ldo, c->dims.heads, c->dh, rm, c->err,
+                               c->as, static_cast<cudaStream_t>(stream)),
           "attention");
   return RC_OK;
 }

@@ -215,80 +215,88 @@ cudaError_t launch_localize(const float* A, int S, int N, int M, int gh, int gw,
 constexpr int LN_WARPS = 8;
 constexpr int LN_MAXV = 12;  // float4 per lane
 
+// Token and item of compact row r; false (and DEVERR_INDEX) when either is
+// out of range.
+__device__ __forceinline__ bool row_target(const RowMap& rm, int n_items, int r, int& tok,
+                                           int& item, unsigned* err, int lane) {
+  tok = rm.tok ? __ldg(rm.tok + r) : r;
+  item = rm.item ? __ldg(rm.item + r) : 0;
+  if (tok < 0 || tok >= rm.n_tokens || item < 0 || item >= n_items) {
+    if (lane == 0) atomicOr(err, DEVERR_INDEX);
+    return false;
+  }
+  return true;
+}
+
 __global__ void __launch_bounds__(LN_WARPS * 32)
-ln_mod_kernel(const float* __restrict__ x, int ldx, const float* __restrict__ tab_sh,
-              const float* __restrict__ tb_sh, const float* __restrict__ tab_sc,
-              const float* __restrict__ tb_sc, bf16* __restrict__ out, int ldo, int Dbound,
-              const int* __restrict__ dcount, int d, bf16* __restrict__ hprev,
-              const int* __restrict__ idx, int n_tokens, unsigned* err) {
+ln_mod_kernel(const float* __restrict__ x, const float* __restrict__ tab, int k_sh, int k_sc,
+              const __grid_constant__ Items it, bf16* __restrict__ out, RowMap rm,
+              long long hprev_off, int d, unsigned* err) {
   pdl_wait();
   pdl_trigger();
-  const int D = live_count(dcount, Dbound, err);
+  const int D = live_count(rm.count, rm.bound, err);
   const int lane = threadIdx.x & 31;
   const int nv = d / 128;
   for (int r = blockIdx.x * LN_WARPS + (threadIdx.x >> 5); r < D; r += gridDim.x * LN_WARPS) {
-  const float4* xr = reinterpret_cast<const float4*>(x + size_t(r) * ldx);
-  float4 v[LN_MAXV];
-  float s = 0.f;
+    int tok, item;
+    if (!row_target(rm, it.n, r, tok, item, err, lane)) continue;
+    const float4* xr = reinterpret_cast<const float4*>(x + size_t(r) * d);
+    float4 v[LN_MAXV];
+    float s = 0.f;
 #pragma unroll
-  for (int k = 0; k < LN_MAXV; ++k)
-    if (k < nv) {
-      v[k] = xr[lane + 32 * k];
-      s += (v[k].x + v[k].y) + (v[k].z + v[k].w);
-    }
-  if (hprev) {
-    const int tok = idx ? idx[r] : r;
-    if (tok >= 0 && tok < n_tokens) {
-      uint2* hrow = reinterpret_cast<uint2*>(hprev + size_t(tok) * d);
+    for (int k = 0; k < LN_MAXV; ++k)
+      if (k < nv) {
+        v[k] = xr[lane + 32 * k];
+        s += (v[k].x + v[k].y) + (v[k].z + v[k].w);
+      }
+    if (hprev_off >= 0) {
+      uint2* hrow = reinterpret_cast<uint2*>(it.slice[item] + hprev_off + size_t(tok) * d);
 #pragma unroll
       for (int k = 0; k < LN_MAXV; ++k)
         if (k < nv)
           hrow[lane + 32 * k] = make_uint2(pack_bf16x2(v[k].x, v[k].y), pack_bf16x2(v[k].z, v[k].w));
-    } else if (lane == 0) {
-      atomicOr(err, DEVERR_INDEX);
     }
-  }
-  const float mean = warp_sum(s) / float(d);
-  float q = 0.f;
+    const float mean = warp_sum(s) / float(d);
+    float q = 0.f;
 #pragma unroll
-  for (int k = 0; k < LN_MAXV; ++k)
-    if (k < nv) {
-      float a = v[k].x - mean, b = v[k].y - mean, c = v[k].z - mean, e = v[k].w - mean;
-      q += (a * a + b * b) + (c * c + e * e);
-    }
-  const float rstd = 1.0f / sqrtf(warp_sum(q) / float(d) + 1e-6f);
-  uint2* orow = reinterpret_cast<uint2*>(out + size_t(r) * ldo);
+    for (int k = 0; k < LN_MAXV; ++k)
+      if (k < nv) {
+        float a = v[k].x - mean, b = v[k].y - mean, c = v[k].z - mean, e = v[k].w - mean;
+        q += (a * a + b * b) + (c * c + e * e);
+      }
+    const float rstd = 1.0f / sqrtf(warp_sum(q) / float(d) + 1e-6f);
+    const float* tb = it.tb[item];
+    uint2* orow = reinterpret_cast<uint2*>(out + size_t(r) * d);
 #pragma unroll
-  for (int k = 0; k < LN_MAXV; ++k)
-    if (k < nv) {
-      const int c = 4 * (lane + 32 * k);
-      float4 sh = *reinterpret_cast<const float4*>(tab_sh + c);
-      float4 sc = *reinterpret_cast<const float4*>(tab_sc + c);
-      if (tb_sh) {
-        float4 a = *reinterpret_cast<const float4*>(tb_sh + c);
-        sh.x += a.x; sh.y += a.y; sh.z += a.z; sh.w += a.w;
+    for (int k = 0; k < LN_MAXV; ++k)
+      if (k < nv) {
+        const int c = 4 * (lane + 32 * k);
+        float4 sh = make_float4(0.f, 0.f, 0.f, 0.f), sc = sh;
+        if (tab) {
+          sh = *reinterpret_cast<const float4*>(tab + size_t(k_sh) * d + c);
+          sc = *reinterpret_cast<const float4*>(tab + size_t(k_sc) * d + c);
+        }
+        if (tb) {
+          const float4 a = *reinterpret_cast<const float4*>(tb + size_t(k_sh) * d + c);
+          const float4 b = *reinterpret_cast<const float4*>(tb + size_t(k_sc) * d + c);
+          sh.x += a.x; sh.y += a.y; sh.z += a.z; sh.w += a.w;
+          sc.x += b.x; sc.y += b.y; sc.z += b.z; sc.w += b.w;
+        }
+        float y0 = (v[k].x - mean) * rstd * (1.f + sc.x) + sh.x;
+        float y1 = (v[k].y - mean) * rstd * (1.f + sc.y) + sh.y;
+        float y2 = (v[k].z - mean) * rstd * (1.f + sc.z) + sh.z;
+        float y3 = (v[k].w - mean) * rstd * (1.f + sc.w) + sh.w;
+        orow[lane + 32 * k] = make_uint2(pack_bf16x2(y0, y1), pack_bf16x2(y2, y3));
       }
-      if (tb_sc) {
-        float4 a = *reinterpret_cast<const float4*>(tb_sc + c);
-        sc.x += a.x; sc.y += a.y; sc.z += a.z; sc.w += a.w;
-      }
-      float y0 = (v[k].x - mean) * rstd * (1.f + sc.x) + sh.x;
-      float y1 = (v[k].y - mean) * rstd * (1.f + sc.y) + sh.y;
-      float y2 = (v[k].z - mean) * rstd * (1.f + sc.z) + sh.z;
-      float y3 = (v[k].w - mean) * rstd * (1.f + sc.w) + sh.w;
-      orow[lane + 32 * k] = make_uint2(pack_bf16x2(y0, y1), pack_bf16x2(y2, y3));
-    }
   }
 }
 
-cudaError_t launch_ln_mod(const float* x, int ldx, const float* tab_sh, const float* tb_sh,
-                          const float* tab_sc, const float* tb_sc, bf16* out, int ldo,
-                          int Dbound, const int* dcount, int d, bf16* hprev, const int* idx,
-                          int n_tokens, unsigned* err, cudaStream_t st) {
-  if (Dbound <= 0) return cudaSuccess;
-  RC_TRY(launch_k(ln_mod_kernel, dim3(row_grid(Dbound, LN_WARPS, 4)), dim3(LN_WARPS * 32), 0, st, x, ldx,
-                  tab_sh, tb_sh, tab_sc, tb_sc, out, ldo, Dbound, dcount, d, hprev, idx, n_tokens,
-                  err));
+cudaError_t launch_ln_mod(const float* x, const float* tab, int k_sh, int k_sc, const Items& it,
+                          bf16* out, const RowMap& rm, long long hprev_off, int d, unsigned* err,
+                          cudaStream_t st) {
+  if (rm.bound <= 0) return cudaSuccess;
+  RC_TRY(launch_k(ln_mod_kernel, dim3(row_grid(rm.bound, LN_WARPS, 4)), dim3(LN_WARPS * 32), 0,
+                  st, x, tab, k_sh, k_sc, it, out, rm, hprev_off, d, err));
   count_launches(1);
   return cudaSuccess;
 }
@@ -327,10 +335,10 @@ constexpr int PE_WARPS = 8;
 constexpr int PE_MAXD = 1536;
 
 __global__ void __launch_bounds__(PE_WARPS * 32)
-patch_embed_kernel(const float* __restrict__ latent, int gh, int gw, int p, int C,
-                   const bf16* __restrict__ We, const float* __restrict__ be,
-                   const float* __restrict__ pos, const int* __restrict__ idx, int Dbound,
-                   const int* __restrict__ dcount, float* __restrict__ xf, int d, unsigned* err) {
+patch_embed_kernel(int gh, int gw, int p, int C, const bf16* __restrict__ We,
+                   const float* __restrict__ be, const float* __restrict__ pos,
+                   const __grid_constant__ Items it, RowMap rm, float* __restrict__ xf, int d,
+                   unsigned* err) {
   pdl_wait();
   pdl_trigger();
   extern __shared__ __align__(16) uint8_t pe_smem[];
@@ -341,15 +349,13 @@ patch_embed_kernel(const float* __restrict__ latent, int gh, int gw, int p, int 
     s_w[e] = k < P ? We[size_t(o) * P + k] : f2bf(0.f);
   }
   __syncthreads();
-  const int D = live_count(dcount, Dbound, err);
+  const int D = live_count(rm.count, rm.bound, err);
   const int lane = threadIdx.x & 31;
-  const int N = gh * gw, W = gw * p, H = gh * p;
+  const int W = gw * p, H = gh * p;
   for (int r = blockIdx.x * PE_WARPS + (threadIdx.x >> 5); r < D; r += gridDim.x * PE_WARPS) {
-    const int i = idx ? idx[r] : r;
-    if (i < 0 || i >= N) {
-      if (lane == 0) atomicOr(err, DEVERR_INDEX);
-      continue;
-    }
+    int i, item;
+    if (!row_target(rm, it.n, r, i, item, err, lane)) continue;
+    const float* latent = it.latent[item];
     const int gy = i / gw, gx = i - gy * gw;
     float pv = 0.f;
     if (lane < P) {
@@ -382,15 +388,14 @@ patch_embed_kernel(const float* __restrict__ latent, int gh, int gw, int p, int 
   }
 }
 
-cudaError_t launch_patch_embed(const float* latent, int gh, int gw, int p, int C,
-                               const bf16* We, const float* be, const float* pos,
-                               const int* idx, int Dbound, const int* dcount, float* xf, int d,
-                               unsigned* err, cudaStream_t st) {
-  if (Dbound <= 0) return cudaSuccess;
+cudaError_t launch_patch_embed(int gh, int gw, int p, int C, const bf16* We, const float* be,
+                               const float* pos, const Items& it, const RowMap& rm, float* xf,
+                               int d, unsigned* err, cudaStream_t st) {
+  if (rm.bound <= 0) return cudaSuccess;
   if (d > PE_MAXD || C * p * p > 16) return cudaErrorInvalidValue;
-  RC_TRY(launch_k(patch_embed_kernel, dim3(row_grid(Dbound, PE_WARPS, 1)), dim3(PE_WARPS * 32),
-                  size_t(d) * 16 * sizeof(bf16), st, latent, gh, gw, p, C, We, be, pos, idx, Dbound,
-                  dcount, xf, d, err));
+  RC_TRY(launch_k(patch_embed_kernel, dim3(row_grid(rm.bound, PE_WARPS, 1)), dim3(PE_WARPS * 32),
+                  size_t(d) * 16 * sizeof(bf16), st, gh, gw, p, C, We, be, pos, it, rm, xf, d,
+                  err));
   count_launches(1);
   return cudaSuccess;
 }
@@ -612,26 +617,76 @@ rows_f32_kernel(const float* __restrict__ src, float* __restrict__ dst,
 }
 
 __global__ void __launch_bounds__(RW_WARPS * 32)
-scatter_bf16_kernel(const float* __restrict__ src, bf16* __restrict__ dst,
-                    const int* __restrict__ idx, int Dbound, const int* __restrict__ dcount,
-                    int d, int N, unsigned* err) {
+scatter_bf16_kernel(const float* __restrict__ src, const __grid_constant__ Items it,
+                    long long off, RowMap rm, int d, unsigned* err) {
   pdl_wait();
   pdl_trigger();
-  const int D = live_count(dcount, Dbound, err);
+  const int D = live_count(rm.count, rm.bound, err);
   const int lane = threadIdx.x & 31;
   for (int r = blockIdx.x * RW_WARPS + (threadIdx.x >> 5); r < D; r += gridDim.x * RW_WARPS) {
-    const int i = idx ? idx[r] : r;
-    if (i < 0 || i >= N) {
-      if (lane == 0) atomicOr(err, DEVERR_INDEX);
-      continue;
-    }
+    int i, item;
+    if (!row_target(rm, it.n, r, i, item, err, lane)) continue;
     const float4* s4 = reinterpret_cast<const float4*>(src + size_t(r) * d);
-    uint2* t2 = reinterpret_cast<uint2*>(dst + size_t(i) * d);
+    uint2* t2 = reinterpret_cast<uint2*>(it.slice[item] + off + size_t(i) * d);
     for (int c = lane; c < d / 4; c += 32) {
       const float4 v = s4[c];
       t2[c] = make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
     }
   }
+}
+
+// Concatenated rows of a multi-item step: block (x, i) fills rows of item i.
+__global__ void __launch_bounds__(256)
+batch_rows_kernel(const __grid_constant__ BatchIn in, int* __restrict__ tok,
+                  int* __restrict__ item, int* __restrict__ meta, int n_tokens, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
+  const int i = blockIdx.y;
+  int off = 0, tiles = 0, cnt = 0;
+  for (int j = 0; j <= i; ++j) {
+    int c = in.bound[j];
+    if (in.count[j]) {
+      c = *in.count[j];
+      if (c < 0 || c > in.bound[j]) {
+        if (threadIdx.x == 0 && blockIdx.x == 0) atomicOr(err, DEVERR_COUNT);
+        c = 0;
+      }
+    }
+    if (j < i) {
+      off += c;
+      tiles += (c + 127) / 128;
+    } else {
+      cnt = c;
+    }
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    meta[META_OFF + i] = off;
+    meta[META_CNT + i] = cnt;
+    meta[META_TILE + i] = tiles;
+    if (i == in.n - 1) {
+      meta[META_TOTAL] = off + cnt;
+      meta[META_TILE + in.n] = tiles + (cnt + 127) / 128;
+    }
+  }
+  const int* idx = in.idx[i];
+  for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < cnt; r += gridDim.x * blockDim.x) {
+    const int t = idx ? idx[r] : r;
+    if (t < 0 || t >= n_tokens) atomicOr(err, DEVERR_INDEX);
+    tok[off + r] = t;
+    item[off + r] = i;
+  }
+}
+
+cudaError_t launch_batch_rows(const BatchIn& in, int* tok, int* item, int* meta, int n_tokens,
+                              unsigned* err, cudaStream_t st) {
+  if (in.n <= 0 || in.n > MAX_ITEMS) return cudaErrorInvalidValue;
+  int maxb = 1;
+  for (int j = 0; j < in.n; ++j) maxb = maxb > in.bound[j] ? maxb : in.bound[j];
+  const int gx = cdiv(maxb, 256) < 16 ? cdiv(maxb, 256) : 16;
+  RC_TRY(launch_k(batch_rows_kernel, dim3(gx, in.n), dim3(256), 0, st, in, tok, item, meta,
+                  n_tokens, err));
+  count_launches(1);
+  return cudaSuccess;
 }
 
 cudaError_t launch_rows_f32(const float* src, float* dst, const int* idx, int Dbound,
@@ -644,11 +699,11 @@ cudaError_t launch_rows_f32(const float* src, float* dst, const int* idx, int Db
   return cudaSuccess;
 }
 
-cudaError_t launch_scatter_bf16(const float* src, bf16* dst, const int* idx, int Dbound,
-                                const int* dcount, int d, int N, unsigned* err, cudaStream_t st) {
-  if (Dbound <= 0) return cudaSuccess;
-  RC_TRY(launch_k(scatter_bf16_kernel, dim3(row_grid(Dbound, RW_WARPS, 4)), dim3(RW_WARPS * 32), 0,
-                  st, src, dst, idx, Dbound, dcount, d, N, err));
+cudaError_t launch_scatter_bf16(const float* src, const Items& it, long long off,
+                                const RowMap& rm, int d, unsigned* err, cudaStream_t st) {
+  if (rm.bound <= 0) return cudaSuccess;
+  RC_TRY(launch_k(scatter_bf16_kernel, dim3(row_grid(rm.bound, RW_WARPS, 4)), dim3(RW_WARPS * 32),
+                  0, st, src, it, off, rm, d, err));
   count_launches(1);
   return cudaSuccess;
 }

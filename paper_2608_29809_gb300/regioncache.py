@@ -34,7 +34,15 @@ class RCError(RuntimeError):
 class rc_dims(C.Structure):
     _fields_ = [(n, C.c_int) for n in ("hidden", "heads", "mlp", "layers", "grid_h", "grid_w",
                                        "patch", "in_ch", "out_ch", "text_len", "timesteps",
-                                       "freq_dim")]
+                                       "freq_dim", "max_batch")]
+
+
+RC_MAX_BATCH = 16
+
+
+class rc_batch_item(C.Structure):
+    _fields_ = [("session", C.c_int), ("latent", C.c_void_p), ("t", C.c_int), ("mode", C.c_int),
+                ("dirty_idx", C.c_void_p), ("D", C.c_int), ("dirty_count", C.c_void_p)]
 
 
 LAYER_FIELDS = ("W_qkv", "b_qkv", "W_o", "b_o", "W_xq", "b_xq", "W_xkv", "b_xkv", "W_xo",
@@ -73,6 +81,7 @@ def load_library(path: str = LIB_PATH) -> C.CDLL:
         "rc_localize_mask_noalloc": (I, [P, I, I, I, I, I, P, I, F, I, P, P, P, P]),
         "rc_block_forward_region": (I, [P, P, I, I, I, P, P, I, P, P, P]),
         "rc_step": (I, [P, P, I, P, I, P, P, I, P, P]),
+        "rc_step_batched": (I, [P, P, C.POINTER(rc_batch_item), I, P]),
         "rc_step_dense": (I, [P, P, I, P, I, P]),
         "rc_linear": (I, [P, P, P, P, P, I, I, I, P]),
         "rc_attention": (I, [P, P, I, P, P, I, I, I, P, I, P]),
@@ -205,6 +214,17 @@ def rc_step(ctx, cache, session, latent, t, schedule, dirty_idx, D, dirty_count,
                         D, _ptr(dirty_count), _stream(stream)))
 
 
+def rc_step_batched(ctx, cache, items, stream=None):
+    """items: sequence of dicts with session, latent, t, mode and, for SPARSE,
+    dirty_idx, D (-1: device count) and dirty_count."""
+    arr = (rc_batch_item * max(1, len(items)))()
+    for i, it in enumerate(items):
+        arr[i] = rc_batch_item(it["session"], _ptr(it["latent"]), it["t"], it["mode"],
+                               _ptr(it.get("dirty_idx")), it.get("D", 0),
+                               _ptr(it.get("dirty_count")))
+    _check(_lib.rc_step_batched(ctx, cache, arr, len(items), _stream(stream)))
+
+
 def rc_step_dense(ctx, cache, session, latent, t, stream=None):
     _check(_lib.rc_step_dense(ctx, cache, session, _ptr(latent), t, _stream(stream)))
 
@@ -256,19 +276,19 @@ def rc_last_error() -> str:
 
 
 # ------------------------------------------------------- convenience wrapper
-def dims_struct(d) -> rc_dims:
+def dims_struct(d, max_batch: int = 1) -> rc_dims:
     return rc_dims(d.hidden, d.heads, d.mlp, d.layers, d.grid_h, d.grid_w, d.patch, d.in_ch,
-                   d.out_ch, d.text_len, d.timesteps, d.freq_dim)
+                   d.out_ch, d.text_len, d.timesteps, d.freq_dim, max_batch)
 
 
 class Model:
     """Owns a context, device copies of the weights (kept alive here) and a
     cache; thin sugar over the entry points for tests and the benchmark."""
 
-    def __init__(self, dims, weights, sessions=1, device="cuda"):
+    def __init__(self, dims, weights, sessions=1, device="cuda", max_batch=1):
         self.dims = dims
         self.w = weights.to(device)
-        self.ctx = rc_create(dims_struct(dims))
+        self.ctx = rc_create(dims_struct(dims, max_batch))
         for l, L in enumerate(self.w.layers):
             rc_set_layer_weights(self.ctx, l, L)
         g = dict(self.w.glob)
