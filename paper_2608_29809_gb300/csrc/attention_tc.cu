@@ -5,23 +5,26 @@
 // attention they are the per-layer text keys / values.
 //
 // One work unit = 128 queries of one head over one split of the keys.  CTAs
-// are persistent (one per SM) and warp-specialised:
-//   warp 0     TMA: Q once per unit, then K/V blocks of 64 keys (3 stages).
+// are persistent and warp-specialised:
+//   warp 0     TMA: Q once per unit, then K/V blocks of 64 keys (4 stages).
 //              Every operand comes through 3-D tensor maps (head_dim, head,
 //              row) as a 64-wide 128B-swizzled tile plus a 16-wide 32B-
 //              swizzled tail; the head_dim extent is the true 72, so the pad
 //              to 80 reads as zero and adds nothing to Q K^T.
-//   warp 1     TMEM owner and MMA issuer: S = Q K^T (M=128, N=64, 5 K-steps
-//              of 16) into one of two TMEM S buffers, ahead of O += P V
-//              (M=128, N=64 + 16, K=64; V is an MN-major operand) whenever
-//              the next block's K/V have landed.
+//   warp 1     TMEM owner and MMA issuer, polling its inputs: S = Q K^T
+//              (M=128, N=64, 5 K-steps of 16) into one of two TMEM S buffers
+//              as soon as the block's K/V have landed and the buffer is free,
+//              and O += P V (M=128, N=64 + 16, K=64) as soon as P is ready;
+//              P is read from TMEM (A operand) and V from shared memory
+//              (MN-major B operand).
 //   warps 2-5  softmax, one thread per query row: reads its S row from TMEM,
 //              online softmax in base 2 with lazy rescaling (O in TMEM is
 //              rescaled only when the running max grows by more than 2^8),
-//              writes its P row (bf16) to a 128-byte-swizzled shared buffer,
-//              and at the end normalises O and stores it.
-// Two CTAs share an SM (256 TMEM columns and ~94 KB of shared memory each), so
-// the softmax of one overlaps the MMAs and exponentials of the other.
+//              and writes its P row (bf16 pairs) back into the first 32
+//              columns of the same S buffer; the next block's softmax never
+//              waits for this block's P V.  At the end it normalises O.
+// Two CTAs share an SM (256 TMEM columns and ~100 KB of shared memory each),
+// so the softmax of one overlaps the MMAs and exponentials of the other.
 // Key splits of the same (query tile, head) leave their unnormalised O and
 // row max / sum in a workspace; a small combine kernel, launched right after,
 // merges them (one warp per row, coalesced).
@@ -43,9 +46,8 @@ namespace {
 using namespace rc::tc;
 
 constexpr int BQ = 128, BKV = 64, THREADS = 192;
-constexpr int KV_STAGES = 3;
-constexpr int P_BYTES = BQ * BKV * 2;  // [128][64] bf16, 128-byte swizzle (one buffer)
-constexpr int TMEM_COLS = 256;     // S0 | S1 (64 columns each) | O (<= 128)
+constexpr int KV_STAGES = 4;
+constexpr int TMEM_COLS = 256;     // S0 | S1 (64 columns each; P overwrites the first 32) | O
 constexpr int CTAS_PER_SM = 2;
 constexpr int PART_STRIDE = 76;    // floats per row of a split's partial result
 constexpr float LAZY_RESCALE = 8.f;
@@ -71,7 +73,7 @@ struct ACfg {
   static constexpr int K128 = BKV * 128, K32 = TAIL ? BKV * 32 : 0;
   static constexpr int Q_BYTES = Q128 + Q32;
   static constexpr int KV_BYTES = 2 * (K128 + K32);  // K then V
-  static constexpr size_t SMEM = size_t(Q_BYTES) + KV_STAGES * KV_BYTES + P_BYTES + 1024 + 256;
+  static constexpr size_t SMEM = size_t(Q_BYTES) + KV_STAGES * KV_BYTES + 1024 + 256;
   // kind::f16, D f32, A/B bf16; S: both K-major; PV: B (V) MN-major (bit 16)
   static constexpr uint32_t IDESC_S = (1u << 4) | (1u << 7) | (1u << 10) |
                                       (uint32_t(BKV >> 3) << 17) | (uint32_t(BQ >> 4) << 24);
@@ -140,17 +142,17 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                                              ~uintptr_t(1023));
   uint8_t* sQ = smem;
   uint8_t* sKV = sQ + C::Q_BYTES;
-  uint8_t* sP = sKV + KV_STAGES * C::KV_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + P_BYTES);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 16);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sKV + KV_STAGES * C::KV_BYTES);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 24);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   // barrier addresses
   const uint32_t b0 = saddr(bars);
   const uint32_t q_full = b0, q_empty = b0 + 8;
   const uint32_t kv_full = b0 + 16, kv_empty = kv_full + 8 * KV_STAGES;
-  const uint32_t s_full = kv_empty + 8 * KV_STAGES, s_free = s_full + 16;
-  const uint32_t p_ready = s_free + 16, p_free = p_ready + 8;
-  const uint32_t o_full = p_free + 8, o_free = o_full + 8;
+  const uint32_t s_full = kv_empty + 8 * KV_STAGES;  // [2]: S of a block is in TMEM
+  const uint32_t p_ready = s_full + 16;              // [2]: P of a block is in TMEM
+  const uint32_t pv_done = p_ready + 16;             // one phase per completed P V
+  const uint32_t o_full = pv_done + 8, o_free = o_full + 8;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -162,10 +164,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(s_full + 8 * b, 1);
-      mbar_init(s_free + 8 * b, 128);
+      mbar_init(p_ready + 8 * b, 128);
     }
-    mbar_init(p_ready, 128);
-    mbar_init(p_free, 1);
+    mbar_init(pv_done, 1);
     mbar_init(o_full, 1);
     mbar_init(o_free, 128);
     *abort_flag = 0;
@@ -223,6 +224,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA
+    // Polls its inputs and issues whatever is ready: S of block ns (its K/V
+    // landed; at most two S/P buffers in use) and P V of block np (its P is
+    // in TMEM).  MMAs from this thread run in issue order, so S(j + 2) is
+    // written into the buffer of P(j) only after P(j) V(j) has read it.
     if (lane == 0) {
       int g = 0, uc = 0;
       const uint32_t qb = saddr(sQ);
@@ -232,60 +237,62 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         const int n = kb1 - kb0;
         if (!mbar_wait(q_full, uc & 1, abort_flag)) goto timeout;
         tc_fence_after();
-        int s_issued = 0;
-        // S = Q K^T for block s_issued of the unit.  Non-blocking form: only
-        // if its K/V have landed and its S buffer is free.  Returns false on
-        // timeout.
-        auto issue_S = [&](bool block, bool& done) -> bool {
-          const int gg = g + s_issued;
-          const int st = gg % KV_STAGES;
-          const uint32_t kvp = (gg / KV_STAGES) & 1, sfp = ((gg >> 1) + 1) & 1;
-          if (block) {
-            if (!mbar_wait(kv_full + 8 * st, kvp, abort_flag)) return false;
-            if (!mbar_wait(s_free + 8 * (gg & 1), sfp, abort_flag)) return false;
-          } else if (!mbar_test(kv_full + 8 * st, kvp) || !mbar_test(s_free + 8 * (gg & 1), sfp)) {
-            done = false;
-            return true;
-          }
-          tc_fence_after();
-          const uint32_t kb = saddr(sKV + st * C::KV_BYTES);
-          const uint32_t sd = tS0 + uint32_t(BKV) * uint32_t(gg & 1);
+        int ns = 0, np = 0;
+        bool o_ok = false;
+        unsigned spins = 0;
+        unsigned long long t_idle = 0;
+        while (np < n) {
+          bool progress = false;
+          if (ns < n && ns < np + 2) {
+            const int gs = g + ns;
+            const int st = gs % KV_STAGES;
+            if (mbar_test(kv_full + 8 * st, (gs / KV_STAGES) & 1)) {
+              tc_fence_after();
+              const uint32_t kb = saddr(sKV + st * C::KV_BYTES);
+              const uint32_t sd = tS0 + uint32_t(BKV) * uint32_t(gs & 1);
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            umma_bf16(sd, sw128_desc(qb + 32 * kk), sw128_desc(kb + 32 * kk), C::IDESC_S,
-                      kk > 0 ? 1u : 0u);
-          if (C::TAIL)
-            umma_bf16(sd, sw32_kmajor_desc(qb + C::Q128), sw32_kmajor_desc(kb + C::K128),
-                      C::IDESC_S, 1u);
-          umma_commit(s_full + 8 * (gg & 1));
-          if (++s_issued == n) umma_commit(q_empty);  // last S of the unit issued
-          done = true;
-          return true;
-        };
-        bool done = false;
-        if (!issue_S(true, done)) goto timeout;
-        for (int j = 0; j < n; ++j) {
-          const int gj = g + j;
-          // S of the next block early if its data is already here
-          if (s_issued == j + 1 && j + 1 < n && !issue_S(false, done)) goto timeout;
-          if (j == 0 && !mbar_wait(o_free, (uc + 1) & 1, abort_flag)) goto timeout;
-          if (!mbar_wait(p_ready, gj & 1, abort_flag)) goto timeout;
-          tc_fence_after();
-          const int st = gj % KV_STAGES;
-          const uint32_t vb = saddr(sKV + st * C::KV_BYTES + C::K128 + C::K32);
-          const uint32_t pb = saddr(sP);
-#pragma unroll
-          for (int kk = 0; kk < BKV / 16; ++kk) {
-            const uint32_t acc = (j > 0 || kk > 0) ? 1u : 0u;
-            umma_bf16(tO, sw128_desc(pb + 32 * kk), sw128_mnmajor_desc(vb + kk * 16 * 128),
-                      C::IDESC_PV64, acc);
-            if (C::TAIL)
-              umma_bf16(tO + 64, sw128_desc(pb + 32 * kk),
-                        sw32_mnmajor_desc(vb + C::K128 + kk * 16 * 32, 16), C::IDESC_PV16, acc);
+              for (int kk = 0; kk < 4; ++kk)
+                umma_bf16(sd, sw128_desc(qb + 32 * kk), sw128_desc(kb + 32 * kk), C::IDESC_S,
+                          kk > 0 ? 1u : 0u);
+              if (C::TAIL)
+                umma_bf16(sd, sw32_kmajor_desc(qb + C::Q128), sw32_kmajor_desc(kb + C::K128),
+                          C::IDESC_S, 1u);
+              umma_commit(s_full + 8 * (gs & 1));
+              if (++ns == n) umma_commit(q_empty);  // last S of the unit issued
+              progress = true;
+            }
           }
-          umma_commit(p_free);
-          umma_commit(kv_empty + 8 * st);
-          if (s_issued == j + 1 && j + 1 < n && !issue_S(true, done)) goto timeout;
+          if (np < ns) {
+            const int gp = g + np;
+            if (!o_ok) o_ok = np > 0 || mbar_test(o_free, (uc + 1) & 1);
+            if (o_ok && mbar_test(p_ready + 8 * (gp & 1), (gp >> 1) & 1)) {
+              tc_fence_after();
+              const int st = gp % KV_STAGES;
+              const uint32_t vb = saddr(sKV + st * C::KV_BYTES + C::K128 + C::K32);
+              const uint32_t pa = tS0 + uint32_t(BKV) * uint32_t(gp & 1);
+#pragma unroll
+              for (int kk = 0; kk < BKV / 16; ++kk) {
+                const uint32_t acc = (np > 0 || kk > 0) ? 1u : 0u;
+                umma_bf16_ta(tO, pa + 8 * kk, sw128_mnmajor_desc(vb + kk * 16 * 128),
+                             C::IDESC_PV64, acc);
+                if (C::TAIL)
+                  umma_bf16_ta(tO + 64, pa + 8 * kk,
+                               sw32_mnmajor_desc(vb + C::K128 + kk * 16 * 32, 16), C::IDESC_PV16,
+                               acc);
+              }
+              umma_commit(kv_empty + 8 * st);
+              umma_commit(pv_done);
+              ++np;
+              progress = true;
+            }
+          }
+          if (progress) {
+            spins = 0;
+          } else if ((++spins & 63) == 0) {
+            const unsigned long long now = globaltimer();
+            if (spins == 64) t_idle = now;
+            if (*abort_flag || now - t_idle > WAIT_NS) goto timeout;
+          }
         }
         g += n;
         umma_commit(o_full);
@@ -310,8 +317,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         for (int i = 0; i < BKV / 16; ++i)
           tmem_ld16_nowait(tS0 + uint32_t(BKV) * uint32_t(g & 1) + lane_off + 16u * i, r + 16 * i);
         tmem_wait_ld();
-        tc_fence_before();
-        mbar_arrive(s_free + 8 * (g & 1));
         // raw scores: the running max m is kept in scaled base-2 units; the
         // scale (log2 e / sqrt(dh) > 0) commutes with the max, and
         // p = 2^(s * scale - m) is one FFMA + ex2 per element
@@ -327,13 +332,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         }
         float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
                          fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]))) * scale_log2;
-        // the single P buffer is free once P V of the previous block is done
-        // (that is also when O may be rescaled)
-        if (!mbar_wait_warp(p_free, (g + 1) & 1, abort_flag)) goto timeout;
         if (j == 0) {
           m = mx;
         } else if (__any_sync(0xffffffffu, mx > m + LAZY_RESCALE)) {
           // (warp-uniform branch: the TMEM accesses below are warp-wide)
+          // O may be rescaled once P V of the previous block is done
+          if (!mbar_wait_warp(pv_done, (g - 1) & 1, abort_flag)) goto timeout;
           mx = fmaxf(mx, m);
           tc_fence_after();
           const float alpha = ex2_ftz(m - mx);
@@ -361,20 +365,21 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
           sum8[c & 7] += p;
         }
         l += ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) + ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
-        // P row: 64 keys = one 128-byte row of the 128B-swizzled A tile
-        uint8_t* prow = sP + row * 128;
+        // P row (64 keys as 32 bf16 pairs) into the first 32 columns of the
+        // same S buffer: the A operand of P V
+        const uint32_t tp = tS0 + uint32_t(BKV) * uint32_t(g & 1) + lane_off;
 #pragma unroll
-        for (int ch = 0; ch < BKV / 8; ++ch) {
-          uint4 w;
-          w.x = pack_bf16x2(__uint_as_float(r[8 * ch + 0]), __uint_as_float(r[8 * ch + 1]));
-          w.y = pack_bf16x2(__uint_as_float(r[8 * ch + 2]), __uint_as_float(r[8 * ch + 3]));
-          w.z = pack_bf16x2(__uint_as_float(r[8 * ch + 4]), __uint_as_float(r[8 * ch + 5]));
-          w.w = pack_bf16x2(__uint_as_float(r[8 * ch + 6]), __uint_as_float(r[8 * ch + 7]));
-          *reinterpret_cast<uint4*>(prow + ((ch ^ (row & 7)) << 4)) = w;
+        for (int h2 = 0; h2 < 2; ++h2) {
+          uint32_t w[16];
+#pragma unroll
+          for (int c = 0; c < 16; ++c)
+            w[c] = pack_bf16x2(__uint_as_float(r[32 * h2 + 2 * c]),
+                               __uint_as_float(r[32 * h2 + 2 * c + 1]));
+          tmem_st16(tp + 16u * h2, w);
         }
-        fence_proxy_async_smem();
+        tmem_wait_st();
         tc_fence_before();
-        mbar_arrive(p_ready);
+        mbar_arrive(p_ready + 8 * (g & 1));
       }
       // ---- unit epilogue
       if (!mbar_wait_warp(o_full, uc & 1, abort_flag)) goto timeout;
