@@ -46,13 +46,32 @@ namespace {
 using namespace rc::tc;
 
 constexpr int BQ = 128, BKV = 64, THREADS = 192;
-constexpr int KV_STAGES = 4;
 constexpr int TMEM_COLS = 256;     // S0 | S1 (64 columns each; P overwrites the first 32) | O
 constexpr int CTAS_PER_SM = 2;
 constexpr int PART_STRIDE = 76;    // floats per row of a split's partial result
 constexpr float LAZY_RESCALE = 8.f;
 constexpr int MAX_SPLIT = 16;
 constexpr int MIN_KB_PER_SPLIT = 4;  // key blocks per split, at least
+
+// Packed f32x2 arithmetic (two lanes of f32 per 64-bit register pair).
+__device__ __forceinline__ uint64_t f32x2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void unpack_f32x2(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t fma_f32x2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t add_f32x2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
 
 // 2^x on the special-function unit (flushes subnormal results to zero; the
 // argument is at most 8 here).
@@ -71,16 +90,20 @@ struct ACfg {
   // 32B-swizzled tail
   static constexpr int Q128 = BQ * 128, Q32 = TAIL ? BQ * 32 : 0;
   static constexpr int K128 = BKV * 128, K32 = TAIL ? BKV * 32 : 0;
+  // K: 64-wide SW128 tile + 16-wide SW32 tail (the S MMA reads them as two
+  // K-major operands); V: one SW128 atom per 64 head-dim columns, so that P V
+  // is a single MMA of N = DHP per 16 keys (MN-major B spanning the atoms)
+  static constexpr int K_BYTES = K128 + K32;
+  static constexpr int V_BYTES = TAIL ? 2 * K128 : K128;
+  static constexpr int STAGES = TAIL ? 3 : 4;
   static constexpr int Q_BYTES = Q128 + Q32;
-  static constexpr int KV_BYTES = 2 * (K128 + K32);  // K then V
-  static constexpr size_t SMEM = size_t(Q_BYTES) + KV_STAGES * KV_BYTES + 1024 + 256;
+  static constexpr int KV_BYTES = K_BYTES + V_BYTES;  // K then V
+  static constexpr size_t SMEM = size_t(Q_BYTES) + STAGES * KV_BYTES + 1024 + 256;
   // kind::f16, D f32, A/B bf16; S: both K-major; PV: B (V) MN-major (bit 16)
   static constexpr uint32_t IDESC_S = (1u << 4) | (1u << 7) | (1u << 10) |
                                       (uint32_t(BKV >> 3) << 17) | (uint32_t(BQ >> 4) << 24);
-  static constexpr uint32_t IDESC_PV64 = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) |
-                                         (uint32_t(64 >> 3) << 17) | (uint32_t(BQ >> 4) << 24);
-  static constexpr uint32_t IDESC_PV16 = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) |
-                                         (uint32_t(16 >> 3) << 17) | (uint32_t(BQ >> 4) << 24);
+  static constexpr uint32_t IDESC_PV = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) |
+                                       (uint32_t(DHP >> 3) << 17) | (uint32_t(BQ >> 4) << 24);
 };
 
 // Query tile qt of a launch: its item, first compact row and live rows.
@@ -132,8 +155,7 @@ template <int DH>
 __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
 attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmQt,
                const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmKt,
-               const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmVt,
-               const __grid_constant__ AttnItems ai, int Nk, bf16* __restrict__ O, int ldo,
+               const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnItems ai, int Nk, bf16* __restrict__ O, int ldo,
                int heads, RowMap rm, float scale_log2, unsigned* err, float* __restrict__ part,
                int ws_units) {
   using C = ACfg<DH>;
@@ -142,6 +164,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
                                              ~uintptr_t(1023));
   uint8_t* sQ = smem;
   uint8_t* sKV = sQ + C::Q_BYTES;
+  constexpr int KV_STAGES = C::STAGES;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sKV + KV_STAGES * C::KV_BYTES);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 24);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -180,7 +203,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     if (C::TAIL) {
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmQt)) : "memory");
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmKt)) : "memory");
-      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmVt)) : "memory");
     }
   }
   tc_fence_before();
@@ -216,9 +238,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
           const uint32_t fb = kv_full + 8 * st;
           tma_load_3d(saddr(base), &tmK, fb, 0, h, krow + kb * BKV);
           if (C::TAIL) tma_load_3d(saddr(base + C::K128), &tmKt, fb, 64, h, krow + kb * BKV);
-          tma_load_3d(saddr(base + C::K128 + C::K32), &tmV, fb, 0, h, vrow + kb * BKV);
+          tma_load_3d(saddr(base + C::K_BYTES), &tmV, fb, 0, h, vrow + kb * BKV);
           if (C::TAIL)
-            tma_load_3d(saddr(base + 2 * C::K128 + C::K32), &tmVt, fb, 64, h, vrow + kb * BKV);
+            tma_load_3d(saddr(base + C::K_BYTES + C::K128), &tmV, fb, 64, h, vrow + kb * BKV);
         }
       }
     }
@@ -230,7 +252,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     // written into the buffer of P(j) only after P(j) V(j) has read it.
     if (lane == 0) {
       int g = 0, uc = 0;
-      const uint32_t qb = saddr(sQ);
+      // descriptors of stage 0; a stage's differ only in the start address
+      // field (address >> 4, which never carries out of its 14 bits here)
+      const uint32_t qb = saddr(sQ), kb_0 = saddr(sKV);
+      const uint64_t dq = sw128_desc(qb), dqt = sw32_kmajor_desc(qb + C::Q128);
+      const uint64_t dk = sw128_desc(kb_0), dkt = sw32_kmajor_desc(kb_0 + C::K128);
+      const uint64_t dv = sw128_mnmajor_desc_lbo(kb_0 + C::K_BYTES, C::K128);
       for (int u = blockIdx.x; u < sc.units; u += gridDim.x, ++uc) {
         int qt, h, sp, kb0, kb1;
         sc.decode(u, qt, h, sp, kb0, kb1);
@@ -248,15 +275,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             const int st = gs % KV_STAGES;
             if (mbar_test(kv_full + 8 * st, (gs / KV_STAGES) & 1)) {
               tc_fence_after();
-              const uint32_t kb = saddr(sKV + st * C::KV_BYTES);
+              const uint64_t so = uint64_t(st * (C::KV_BYTES >> 4));
               const uint32_t sd = tS0 + uint32_t(BKV) * uint32_t(gs & 1);
 #pragma unroll
               for (int kk = 0; kk < 4; ++kk)
-                umma_bf16(sd, sw128_desc(qb + 32 * kk), sw128_desc(kb + 32 * kk), C::IDESC_S,
-                          kk > 0 ? 1u : 0u);
-              if (C::TAIL)
-                umma_bf16(sd, sw32_kmajor_desc(qb + C::Q128), sw32_kmajor_desc(kb + C::K128),
-                          C::IDESC_S, 1u);
+                umma_bf16(sd, dq + 2 * kk, dk + so + 2 * kk, C::IDESC_S, kk > 0 ? 1u : 0u);
+              if (C::TAIL) umma_bf16(sd, dqt, dkt + so, C::IDESC_S, 1u);
               umma_commit(s_full + 8 * (gs & 1));
               if (++ns == n) umma_commit(q_empty);  // last S of the unit issued
               progress = true;
@@ -268,18 +292,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
             if (o_ok && mbar_test(p_ready + 8 * (gp & 1), (gp >> 1) & 1)) {
               tc_fence_after();
               const int st = gp % KV_STAGES;
-              const uint32_t vb = saddr(sKV + st * C::KV_BYTES + C::K128 + C::K32);
+              const uint64_t vd = dv + uint64_t(st * (C::KV_BYTES >> 4));
               const uint32_t pa = tS0 + uint32_t(BKV) * uint32_t(gp & 1);
+              // 16 keys per MMA: P columns 8 kk .., V rows 16 kk .. (2 KB)
 #pragma unroll
-              for (int kk = 0; kk < BKV / 16; ++kk) {
-                const uint32_t acc = (np > 0 || kk > 0) ? 1u : 0u;
-                umma_bf16_ta(tO, pa + 8 * kk, sw128_mnmajor_desc(vb + kk * 16 * 128),
-                             C::IDESC_PV64, acc);
-                if (C::TAIL)
-                  umma_bf16_ta(tO + 64, pa + 8 * kk,
-                               sw32_mnmajor_desc(vb + C::K128 + kk * 16 * 32, 16), C::IDESC_PV16,
-                               acc);
-              }
+              for (int kk = 0; kk < BKV / 16; ++kk)
+                umma_bf16_ta(tO, pa + 8 * kk, vd + 128 * kk, C::IDESC_PV,
+                             (np > 0 || kk > 0) ? 1u : 0u);
               umma_commit(kv_empty + 8 * st);
               umma_commit(pv_done);
               ++np;
@@ -321,15 +340,16 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         // scale (log2 e / sqrt(dh) > 0) commutes with the max, and
         // p = 2^(s * scale - m) is one FFMA + ex2 per element
         const int valid = Nk - (kb0 + j) * BKV;
+        if (valid < BKV) {  // the last, partial key block (warp-uniform)
+#pragma unroll
+          for (int c = 0; c < BKV; ++c)
+            if (c >= valid) r[c] = __float_as_uint(-INFINITY);
+        }
         float mx8[8];
 #pragma unroll
-        for (int q = 0; q < 8; ++q) mx8[q] = -INFINITY;
+        for (int q = 0; q < 8; ++q) mx8[q] = __uint_as_float(r[q]);
 #pragma unroll
-        for (int c = 0; c < BKV; ++c) {
-          const float v = c < valid ? __uint_as_float(r[c]) : -INFINITY;
-          r[c] = __float_as_uint(v);
-          mx8[c & 7] = fmaxf(mx8[c & 7], v);
-        }
+        for (int c = 8; c < BKV; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(r[c]));
         float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
                          fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]))) * scale_log2;
         if (j == 0) {
@@ -354,17 +374,29 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
           l *= alpha;
           m = mx;
         }
-        const float negm = -m;
-        float sum8[8];
+        // p = 2^(s scale - m): the scaling FMA and the row sum run two
+        // columns per instruction (packed f32x2)
+        const uint64_t sc2 = f32x2(scale_log2, scale_log2), nm2 = f32x2(-m, -m);
+        uint64_t sum2[4];
 #pragma unroll
-        for (int q = 0; q < 8; ++q) sum8[q] = 0.f;
+        for (int q = 0; q < 4; ++q) sum2[q] = f32x2(0.f, 0.f);
 #pragma unroll
-        for (int c = 0; c < BKV; ++c) {
-          const float p = ex2_ftz(fmaf(__uint_as_float(r[c]), scale_log2, negm));
-          r[c] = __float_as_uint(p);
-          sum8[c & 7] += p;
+        for (int c = 0; c < BKV; c += 2) {
+          float a, b;
+          unpack_f32x2(fma_f32x2(f32x2(__uint_as_float(r[c]), __uint_as_float(r[c + 1])), sc2, nm2),
+                       a, b);
+          a = ex2_ftz(a);
+          b = ex2_ftz(b);
+          r[c] = __float_as_uint(a);
+          r[c + 1] = __float_as_uint(b);
+          sum2[(c >> 1) & 3] = add_f32x2(sum2[(c >> 1) & 3], f32x2(a, b));
         }
-        l += ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) + ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
+        float s0, s1, s2, s3, s4, s5, s6, s7;
+        unpack_f32x2(sum2[0], s0, s1);
+        unpack_f32x2(sum2[1], s2, s3);
+        unpack_f32x2(sum2[2], s4, s5);
+        unpack_f32x2(sum2[3], s6, s7);
+        l += ((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7));
         // P row (64 keys as 32 bf16 pairs) into the first 32 columns of the
         // same S buffer: the A operand of P V
         const uint32_t tp = tS0 + uint32_t(BKV) * uint32_t(g & 1) + lane_off;
@@ -587,23 +619,22 @@ cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* 
   const int sms = device_sms_attn();
   if (!sms) return cudaErrorInvalidDevice;
   // a 64-wide 128B-swizzled map and a 16-wide 32B-swizzled tail map per operand
-  CUtensorMap tq, tqt, tk, tkt, tv, tvt;
+  CUtensorMap tq, tqt, tk, tkt, tv;
   RC_TRY(head_map(Q, rm.bound, ldq, heads, dh, 64, BQ, &tq));
   RC_TRY(head_map(K, kv_rows, ldkv, heads, dh, 64, BKV, &tk));
   RC_TRY(head_map(V, kv_rows, ldkv, heads, dh, 64, BKV, &tv));
   RC_TRY(head_map(Q, rm.bound, ldq, heads, dh, 16, BQ, &tqt));
   RC_TRY(head_map(K, kv_rows, ldkv, heads, dh, 16, BKV, &tkt));
-  RC_TRY(head_map(V, kv_rows, ldkv, heads, dh, 16, BKV, &tvt));
   const float scale_log2 = float(1.4426950408889634 / sqrt(double(dh)));
   const int ws_units = int(as.part_floats / (size_t(BQ) * PART_STRIDE));
   const int grid = CTAS_PER_SM * sms;
   if (dh == 72)
     RC_TRY(launch_k(attn_tc_kernel<72>, dim3(grid), dim3(THREADS), ACfg<72>::SMEM, st, tq, tqt,
-                    tk, tkt, tv, tvt, ai, Nk, O, ldo, heads, rm, scale_log2, err, as.part,
+                    tk, tkt, tv, ai, Nk, O, ldo, heads, rm, scale_log2, err, as.part,
                     ws_units));
   else
     RC_TRY(launch_k(attn_tc_kernel<64>, dim3(grid), dim3(THREADS), ACfg<64>::SMEM, st, tq, tqt,
-                    tk, tkt, tv, tvt, ai, Nk, O, ldo, heads, rm, scale_log2, err, as.part,
+                    tk, tkt, tv, ai, Nk, O, ldo, heads, rm, scale_log2, err, as.part,
                     ws_units));
   count_launches(1);
   // key splits happen only with at least MIN_KB_PER_SPLIT key blocks per split

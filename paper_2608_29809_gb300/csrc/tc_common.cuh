@@ -194,6 +194,18 @@ __device__ __forceinline__ uint64_t sw128_mnmajor_desc(uint32_t addr) {
   return d;
 }
 
+// As sw128_mnmajor_desc for an operand wider than 64 in MN: consecutive
+// 64-element MN atoms `lbo` bytes apart.
+__device__ __forceinline__ uint64_t sw128_mnmajor_desc_lbo(uint32_t addr, uint32_t lbo) {
+  uint64_t d = 0;
+  d |= uint64_t((addr & 0x3FFFFu) >> 4);
+  d |= uint64_t((lbo >> 4) & 0x3FFFu) << 16;
+  d |= uint64_t(1024 >> 4) << 32;
+  d |= uint64_t(1) << 46;
+  d |= uint64_t(2) << 61;
+  return d;
+}
+
 // 16 consecutive f32 columns of this thread's TMEM lane (no wait).
 __device__ __forceinline__ void tmem_ld16_nowait(uint32_t taddr, uint32_t* r) {
   asm volatile(
