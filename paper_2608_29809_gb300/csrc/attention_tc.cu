@@ -11,18 +11,19 @@
 //              row) as a 64-wide 128B-swizzled tile plus a 16-wide 32B-
 //              swizzled tail; the head_dim extent is the true 72, so the pad
 //              to 80 reads as zero and adds nothing to Q K^T.
-//   warp 1     TMEM owner and MMA issuer, polling its inputs: S = Q K^T
-//              (M=128, N=64, 5 K-steps of 16) into one of two TMEM S buffers
-//              as soon as the block's K/V have landed and the buffer is free,
-//              and O += P V (M=128, N=64 + 16, K=64) as soon as P is ready;
-//              P is read from TMEM (A operand) and V from shared memory
-//              (MN-major B operand).
-//   warps 2-5  softmax, one thread per query row: reads its S row from TMEM,
-//              online softmax in base 2 with lazy rescaling (O in TMEM is
-//              rescaled only when the running max grows by more than 2^8),
-//              and writes its P row (bf16 pairs) back into the first 32
-//              columns of the same S buffer; the next block's softmax never
-//              waits for this block's P V.  At the end it normalises O.
+//   warp 1     TMEM owner and MMA issuer, polling its inputs: O += P V
+//              (M=128, N=80, 4 K-steps of 16 keys; P read from TMEM as the A
+//              operand, V from shared memory as an MN-major B operand) as
+//              soon as P is ready, and S = Q K^T (M=128, N=64, 5 K-steps of
+//              16) into one of two TMEM S buffers as soon as the block's K/V
+//              have landed and the softmax has read that buffer's last S
+//              (so S runs up to two blocks ahead of the softmax).
+//   warps 2-5  softmax, one thread per query row: reads its S row from TMEM
+//              (freeing the buffer), online softmax in base 2 with lazy
+//              rescaling (O in TMEM is rescaled only when the running max
+//              grows by more than 2^8), and writes its P row (bf16 pairs) to
+//              the TMEM P buffer once the previous P V has read it.  At the
+//              end it normalises O.
 // Two CTAs share an SM (256 TMEM columns and ~100 KB of shared memory each),
 // so the softmax of one overlaps the MMAs and exponentials of the other.
 // Key splits of the same (query tile, head) leave their unnormalised O and
@@ -46,7 +47,7 @@ namespace {
 using namespace rc::tc;
 
 constexpr int BQ = 128, BKV = 64, THREADS = 192;
-constexpr int TMEM_COLS = 256;     // S0 | S1 (64 columns each; P overwrites the first 32) | O
+constexpr int TMEM_COLS = 256;     // S0 | S1 (64 columns each) | O (80) | P (32)
 constexpr int CTAS_PER_SM = 2;
 constexpr int PART_STRIDE = 76;    // floats per row of a split's partial result
 constexpr float LAZY_RESCALE = 8.f;
@@ -173,8 +174,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
   const uint32_t q_full = b0, q_empty = b0 + 8;
   const uint32_t kv_full = b0 + 16, kv_empty = kv_full + 8 * KV_STAGES;
   const uint32_t s_full = kv_empty + 8 * KV_STAGES;  // [2]: S of a block is in TMEM
-  const uint32_t p_ready = s_full + 16;              // [2]: P of a block is in TMEM
-  const uint32_t pv_done = p_ready + 16;             // one phase per completed P V
+  const uint32_t s_free = s_full + 16;               // [2]: the softmax has read it
+  const uint32_t p_ready = s_free + 16;              // P of the next block is in TMEM
+  const uint32_t pv_done = p_ready + 8;              // one phase per completed P V
   const uint32_t o_full = pv_done + 8, o_free = o_full + 8;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -187,8 +189,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(s_full + 8 * b, 1);
-      mbar_init(p_ready + 8 * b, 128);
+      mbar_init(s_free + 8 * b, 128);
     }
+    mbar_init(p_ready, 128);
     mbar_init(pv_done, 1);
     mbar_init(o_full, 1);
     mbar_init(o_free, 128);
@@ -209,7 +212,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const uint32_t tS0 = tmem_base, tO = tmem_base + 2 * BKV;
+  const uint32_t tS0 = tmem_base, tO = tmem_base + 2 * BKV, tP = tO + 80;
 
   pdl_wait();
   pdl_trigger();
@@ -246,10 +249,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA
-    // Polls its inputs and issues whatever is ready: S of block ns (its K/V
-    // landed; at most two S/P buffers in use) and P V of block np (its P is
-    // in TMEM).  MMAs from this thread run in issue order, so S(j + 2) is
-    // written into the buffer of P(j) only after P(j) V(j) has read it.
+    // Polls its inputs and issues whatever is ready: P V of block np (its
+    // P is in TMEM; first, as the softmax of the next block waits on it),
+    // then S of block ns (its K/V landed and its S buffer was read).
     if (lane == 0) {
       int g = 0, uc = 0;
       // descriptors of stage 0; a stage's differ only in the start address
@@ -270,10 +272,29 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         unsigned long long t_idle = 0;
         while (np < n) {
           bool progress = false;
-          if (ns < n && ns < np + 2) {
+          if (np < ns) {
+            const int gp = g + np;
+            if (!o_ok) o_ok = np > 0 || mbar_test(o_free, (uc + 1) & 1);
+            if (o_ok && mbar_test(p_ready, gp & 1)) {
+              tc_fence_after();
+              const int st = gp % KV_STAGES;
+              const uint64_t vd = dv + uint64_t(st * (C::KV_BYTES >> 4));
+              // 16 keys per MMA: P columns 8 kk .., V rows 16 kk .. (2 KB)
+#pragma unroll
+              for (int kk = 0; kk < BKV / 16; ++kk)
+                umma_bf16_ta(tO, tP + 8 * kk, vd + 128 * kk, C::IDESC_PV,
+                             (np > 0 || kk > 0) ? 1u : 0u);
+              umma_commit(kv_empty + 8 * st);
+              umma_commit(pv_done);
+              ++np;
+              progress = true;
+            }
+          }
+          if (ns < n) {
             const int gs = g + ns;
             const int st = gs % KV_STAGES;
-            if (mbar_test(kv_full + 8 * st, (gs / KV_STAGES) & 1)) {
+            if (mbar_test(kv_full + 8 * st, (gs / KV_STAGES) & 1) &&
+                mbar_test(s_free + 8 * (gs & 1), ((gs >> 1) + 1) & 1)) {
               tc_fence_after();
               const uint64_t so = uint64_t(st * (C::KV_BYTES >> 4));
               const uint32_t sd = tS0 + uint32_t(BKV) * uint32_t(gs & 1);
@@ -283,25 +304,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
               if (C::TAIL) umma_bf16(sd, dqt, dkt + so, C::IDESC_S, 1u);
               umma_commit(s_full + 8 * (gs & 1));
               if (++ns == n) umma_commit(q_empty);  // last S of the unit issued
-              progress = true;
-            }
-          }
-          if (np < ns) {
-            const int gp = g + np;
-            if (!o_ok) o_ok = np > 0 || mbar_test(o_free, (uc + 1) & 1);
-            if (o_ok && mbar_test(p_ready + 8 * (gp & 1), (gp >> 1) & 1)) {
-              tc_fence_after();
-              const int st = gp % KV_STAGES;
-              const uint64_t vd = dv + uint64_t(st * (C::KV_BYTES >> 4));
-              const uint32_t pa = tS0 + uint32_t(BKV) * uint32_t(gp & 1);
-              // 16 keys per MMA: P columns 8 kk .., V rows 16 kk .. (2 KB)
-#pragma unroll
-              for (int kk = 0; kk < BKV / 16; ++kk)
-                umma_bf16_ta(tO, pa + 8 * kk, vd + 128 * kk, C::IDESC_PV,
-                             (np > 0 || kk > 0) ? 1u : 0u);
-              umma_commit(kv_empty + 8 * st);
-              umma_commit(pv_done);
-              ++np;
               progress = true;
             }
           }
@@ -336,6 +338,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         for (int i = 0; i < BKV / 16; ++i)
           tmem_ld16_nowait(tS0 + uint32_t(BKV) * uint32_t(g & 1) + lane_off + 16u * i, r + 16 * i);
         tmem_wait_ld();
+        tc_fence_before();
+        mbar_arrive(s_free + 8 * (g & 1));
         // raw scores: the running max m is kept in scaled base-2 units; the
         // scale (log2 e / sqrt(dh) > 0) commutes with the max, and
         // p = 2^(s * scale - m) is one FFMA + ex2 per element
@@ -352,25 +356,17 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         for (int c = 8; c < BKV; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(r[c]));
         float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
                          fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]))) * scale_log2;
+        // lazy rescale (warp-uniform decision: the TMEM accesses are
+        // warp-wide); O itself is rescaled below, once P V of the previous
+        // block has completed
+        bool rescale = false;
+        float alpha = 1.f;
         if (j == 0) {
           m = mx;
         } else if (__any_sync(0xffffffffu, mx > m + LAZY_RESCALE)) {
-          // (warp-uniform branch: the TMEM accesses below are warp-wide)
-          // O may be rescaled once P V of the previous block is done
-          if (!mbar_wait_warp(pv_done, (g - 1) & 1, abort_flag)) goto timeout;
+          rescale = true;
           mx = fmaxf(mx, m);
-          tc_fence_after();
-          const float alpha = ex2_ftz(m - mx);
-#pragma unroll
-          for (int i = 0; i < C::DHP / 16; ++i) {
-            uint32_t o16[16];
-            tmem_ld16_nowait(tO + lane_off + 16u * i, o16);
-            tmem_wait_ld();
-#pragma unroll
-            for (int e = 0; e < 16; ++e) o16[e] = __float_as_uint(__uint_as_float(o16[e]) * alpha);
-            tmem_st16(tO + lane_off + 16u * i, o16);
-          }
-          tmem_wait_st();
+          alpha = ex2_ftz(m - mx);
           l *= alpha;
           m = mx;
         }
@@ -397,9 +393,22 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         unpack_f32x2(sum2[2], s4, s5);
         unpack_f32x2(sum2[3], s6, s7);
         l += ((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7));
-        // P row (64 keys as 32 bf16 pairs) into the first 32 columns of the
-        // same S buffer: the A operand of P V
-        const uint32_t tp = tS0 + uint32_t(BKV) * uint32_t(g & 1) + lane_off;
+        // the P buffer and O are free once P V of the previous block is done
+        if (g > 0 && !mbar_wait_warp(pv_done, (g - 1) & 1, abort_flag)) goto timeout;
+        tc_fence_after();
+        if (rescale) {
+#pragma unroll
+          for (int i = 0; i < C::DHP / 16; ++i) {
+            uint32_t o16[16];
+            tmem_ld16_nowait(tO + lane_off + 16u * i, o16);
+            tmem_wait_ld();
+#pragma unroll
+            for (int e = 0; e < 16; ++e) o16[e] = __float_as_uint(__uint_as_float(o16[e]) * alpha);
+            tmem_st16(tO + lane_off + 16u * i, o16);
+          }
+        }
+        // P row (64 keys as 32 bf16 pairs): the A operand of P V
+        const uint32_t tp = tP + lane_off;
 #pragma unroll
         for (int h2 = 0; h2 < 2; ++h2) {
           uint32_t w[16];
@@ -411,7 +420,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         }
         tmem_wait_st();
         tc_fence_before();
-        mbar_arrive(p_ready + 8 * (g & 1));
+        mbar_arrive(p_ready);
       }
       // ---- unit epilogue
       if (!mbar_wait_warp(o_full, uc & 1, abort_flag)) goto timeout;
