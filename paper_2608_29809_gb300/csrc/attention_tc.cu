@@ -51,8 +51,7 @@ constexpr int TMEM_COLS = 256;     // S0 | S1 (64 columns each) | O (80) | P (32
 constexpr int CTAS_PER_SM = 2;
 constexpr int PART_STRIDE = 76;    // floats per row of a split's partial result
 constexpr float LAZY_RESCALE = 8.f;
-constexpr int MAX_SPLIT = 16;
-constexpr int MIN_KB_PER_SPLIT = 4;  // key blocks per split, at least
+constexpr int MIN_KB_PER_SPLIT = 4;  // key blocks per CTA range, at least
 
 // Packed f32x2 arithmetic (two lanes of f32 per 64-bit register pair).
 __device__ __forceinline__ uint64_t f32x2(float lo, float hi) {
@@ -125,30 +124,72 @@ __device__ __forceinline__ int query_tiles(const RowMap& rm, int n_items, int D)
   return rm.meta ? __ldg(rm.meta + META_TILE + n_items) : (D + BQ - 1) / BQ;
 }
 
-// Work list of one launch, identical in every thread.
+// Work list of one launch, identical in every thread.  A pair = one query
+// tile of one head (heads outermost).  With at least 2 MIN_KB_PER_SPLIT key
+// blocks (the self-attention) the (pair, key block) sequence is cut into G
+// equal contiguous ranges, one per CTA (stream-K): every CTA does the same
+// number of key blocks, and a pair cut by a range boundary leaves partial
+// results (unnormalised O, row max and sum) that the combine kernel merges.
+// With fewer key blocks (the text cross-attention) every pair is one unit,
+// handed out round-robin.
 struct AttnSched {
-  int qtiles, pairs, nkb, split, per, units;
-  __device__ void init(int tiles, int heads, int Nk, int grid, int ws_units) {
+  int qtiles, pairs, nkb, G, total;
+  bool streamk;
+  __device__ void init(int tiles, int heads, int Nk, int grid) {
     qtiles = tiles;
     pairs = qtiles * heads;
     nkb = (Nk + BKV - 1) / BKV;
-    split = 1;
-    while (split < MAX_SPLIT && pairs * split < 2 * grid && split * 2 * MIN_KB_PER_SPLIT <= nkb &&
-           pairs * split * 2 <= ws_units)
-      split *= 2;
-    per = (nkb + split - 1) / split;
-    split = (nkb + per - 1) / per;  // no empty split
-    units = pairs * split;
+    total = pairs * nkb;
+    streamk = nkb >= 2 * MIN_KB_PER_SPLIT;
+    G = grid;
+    if (streamk) G = max(1, min(grid, total / MIN_KB_PER_SPLIT));
   }
-  // unit -> (query tile, head, split, key blocks [kb0, kb1)); splits of one
-  // (tile, head) are adjacent, heads outermost
-  __device__ void decode(int u, int& qt, int& h, int& sp, int& kb0, int& kb1) const {
-    sp = u % split;
-    const int pair = u / split;
-    qt = pair % qtiles;
-    h = pair / qtiles;
-    kb0 = sp * per;
-    kb1 = min(nkb, kb0 + per);
+  // unsigned 32-bit arithmetic: the launcher checks total * G < 2^32
+  __device__ int bound(int c) const { return int(unsigned(total) * unsigned(c) / unsigned(G)); }
+  // the CTA whose range holds key-block position pos (0 <= pos < total)
+  __device__ int cta_of(int pos) const {
+    int c = int(unsigned(pos) * unsigned(G) / unsigned(total));
+    while (c > 0 && bound(c) > pos) --c;
+    while (c + 1 < G && bound(c + 1) <= pos) ++c;
+    return c;
+  }
+};
+
+// One CTA's segments in order: (pair, key blocks [kb0, kb1), slot), slot -1
+// for a whole pair (its normalised output is written directly), 0 / 1 for
+// the CTA's first / last partial piece (workspace slot 2 c + slot).
+struct AttnSeg {
+  const AttnSched* sc;
+  int cur, end;
+  bool first;
+  __device__ void init(const AttnSched& s, int c) {
+    sc = &s;
+    first = true;
+    if (s.streamk) {
+      cur = c < s.G ? s.bound(c) : 0;
+      end = c < s.G ? s.bound(c + 1) : 0;
+    } else {
+      cur = c;  // next pair
+      end = s.pairs;
+    }
+  }
+  __device__ bool next(int& pair, int& kb0, int& kb1, int& slot) {
+    if (cur >= end) return false;
+    if (!sc->streamk) {
+      pair = cur;
+      kb0 = 0;
+      kb1 = sc->nkb;
+      slot = -1;
+      cur += sc->G;
+      return true;
+    }
+    pair = cur / sc->nkb;
+    kb0 = cur - pair * sc->nkb;
+    kb1 = min(sc->nkb, kb0 + (end - cur));
+    cur += kb1 - kb0;
+    slot = (kb0 == 0 && kb1 == sc->nkb) ? -1 : (first ? 0 : 1);
+    first = false;
+    return true;
   }
 };
 
@@ -157,8 +198,7 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
 attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmQt,
                const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmKt,
                const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnItems ai, int Nk, bf16* __restrict__ O, int ldo,
-               int heads, RowMap rm, float scale_log2, unsigned* err, float* __restrict__ part,
-               int ws_units) {
+               int heads, RowMap rm, float scale_log2, unsigned* err, float* __restrict__ part) {
   using C = ACfg<DH>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -218,15 +258,17 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
   pdl_trigger();
   const int D = live_count(rm.count, rm.bound, err);
   AttnSched sc;
-  sc.init(query_tiles(rm, ai.n, D), heads, Nk, gridDim.x, ws_units);
+  sc.init(query_tiles(rm, ai.n, D), heads, Nk, gridDim.x);
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA
     if (lane == 0) {
       int g = 0, uc = 0;
-      for (int u = blockIdx.x; u < sc.units; u += gridDim.x, ++uc) {
-        int qt, h, sp, kb0, kb1;
-        sc.decode(u, qt, h, sp, kb0, kb1);
+      AttnSeg it;
+      it.init(sc, blockIdx.x);
+      int pair, kb0, kb1, slot;
+      for (; it.next(pair, kb0, kb1, slot); ++uc) {
+        const int qt = pair % sc.qtiles, h = pair / sc.qtiles;
         const TileLoc tl = locate_tile(rm, ai.n, D, qt);
         const int krow = ai.krow[tl.item], vrow = ai.vrow[tl.item];
         if (!mbar_wait(q_empty, (uc + 1) & 1, abort_flag)) goto timeout;
@@ -260,9 +302,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
       const uint64_t dq = sw128_desc(qb), dqt = sw32_kmajor_desc(qb + C::Q128);
       const uint64_t dk = sw128_desc(kb_0), dkt = sw32_kmajor_desc(kb_0 + C::K128);
       const uint64_t dv = sw128_mnmajor_desc_lbo(kb_0 + C::K_BYTES, C::K128);
-      for (int u = blockIdx.x; u < sc.units; u += gridDim.x, ++uc) {
-        int qt, h, sp, kb0, kb1;
-        sc.decode(u, qt, h, sp, kb0, kb1);
+      AttnSeg it;
+      it.init(sc, blockIdx.x);
+      int pair, kb0, kb1, slot;
+      for (; it.next(pair, kb0, kb1, slot); ++uc) {
+        const int qt = pair % sc.qtiles, h = pair / sc.qtiles;
         const int n = kb1 - kb0;
         if (!mbar_wait(q_full, uc & 1, abort_flag)) goto timeout;
         tc_fence_after();
@@ -325,9 +369,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     const int row = sp4 * 32 + lane;
     const uint32_t lane_off = uint32_t(sp4 * 32) << 16;
     int g = 0, uc = 0;
-    for (int u = blockIdx.x; u < sc.units; u += gridDim.x, ++uc) {
-      int qt, h, sp, kb0, kb1;
-      sc.decode(u, qt, h, sp, kb0, kb1);
+    AttnSeg it;
+    it.init(sc, blockIdx.x);
+    int pair, kb0, kb1, slot;
+    for (; it.next(pair, kb0, kb1, slot); ++uc) {
+      const int qt = pair % sc.qtiles, h = pair / sc.qtiles;
       const int n = kb1 - kb0;
       float m = -INFINITY, l = 0.f;
       for (int j = 0; j < n; ++j, ++g) {
@@ -431,7 +477,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
       tmem_wait_ld();
       tc_fence_before();
       mbar_arrive(o_free);
-      if (sc.split == 1) {
+      if (slot < 0) {
         const TileLoc tl = locate_tile(rm, ai.n, D, qt);
         const int qrow = tl.row0 + row;
         if (row < tl.rows) {
@@ -448,10 +494,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
           }
         }
       } else {
-        // split of the keys: unnormalised O with its row max and sum; the
-        // combine kernel merges the splits
-        const int pair = u / sc.split;
-        float* mine = part + (size_t(pair) * sc.split + sp) * (BQ * PART_STRIDE) +
+        // a piece of the pair's keys: unnormalised O with its row max and
+        // sum; the combine kernel merges the pieces
+        float* mine = part + (size_t(blockIdx.x) * 2 + slot) * (BQ * PART_STRIDE) +
                       size_t(row) * PART_STRIDE;
 #pragma unroll
         for (int c4 = 0; c4 < DH / 4; ++c4)
@@ -476,51 +521,108 @@ done:
   }
 }
 
-// Merge of the key splits: one warp per query row; lane q < split reads that
-// split's row max / sum, the warp reduces the max, then every lane
-// accumulates its 4 head-dim columns over the splits.
+// Merge of the pieces of the pairs that stream-K cut: one warp per (pair,
+// query row).  The pieces come from CTAs cta_of(first block) .. cta_of(last
+// block); a CTA's piece is its first (slot 0) when its range starts inside
+// the pair, else its last (slot 1).  Lanes take the pieces' row max / sum in
+// turn, the warp reduces them, then lanes < DH / 4 accumulate 4 head-dim
+// columns each over the pieces.
 template <int DH>
 __global__ void __launch_bounds__(256)
 attn_combine_kernel(const float* __restrict__ part, bf16* __restrict__ O, int ldo, int heads,
-                    RowMap rm, int n_items, int Nk, int attn_grid, int ws_units, unsigned* err) {
+                    RowMap rm, int n_items, int Nk, int attn_grid, unsigned* err) {
   pdl_wait();
   pdl_trigger();
   const int D = live_count(rm.count, rm.bound, err);
   AttnSched sc;
-  sc.init(query_tiles(rm, n_items, D), heads, Nk, attn_grid, ws_units);
-  if (sc.split == 1) return;
+  sc.init(query_tiles(rm, n_items, D), heads, Nk, attn_grid);
+  if (!sc.streamk) return;
   const int lane = threadIdx.x & 31;
   for (int gw = blockIdx.x * 8 + (threadIdx.x >> 5); gw < sc.pairs * BQ; gw += gridDim.x * 8) {
-  const int pair = gw / BQ, row = gw - pair * BQ;
-  const int qt = pair % sc.qtiles, h = pair / sc.qtiles;
-  const TileLoc tl = locate_tile(rm, n_items, D, qt);
-  if (row >= tl.rows) continue;
-  const int qrow = tl.row0 + row;
-  const float* base = part + size_t(pair) * sc.split * (BQ * PART_STRIDE) + size_t(row) * PART_STRIDE;
-  float2 ml = make_float2(-INFINITY, 0.f);
-  if (lane < sc.split) ml = __ldcg(reinterpret_cast<const float2*>(base + size_t(lane) * (BQ * PART_STRIDE) + DH));
-  float M = ml.x;
+    const int pair = gw / BQ, row = gw - pair * BQ;
+    const int lo = pair * sc.nkb;
+    const int c_lo = sc.cta_of(lo), c_hi = sc.cta_of(lo + sc.nkb - 1);
+    if (c_lo == c_hi) continue;  // one CTA held the whole pair
+    const int qt = pair % sc.qtiles, h = pair / sc.qtiles;
+    const TileLoc tl = locate_tile(rm, n_items, D, qt);
+    if (row >= tl.rows) continue;
+    const int np = c_hi - c_lo + 1;
+    // CTAs after c_lo start inside the pair (their first piece); c_lo's
+    // piece is its first only when its range starts exactly at the pair
+    const int slot_lo = sc.bound(c_lo) == lo ? 0 : 1;
+    const float* base = part + size_t(row) * PART_STRIDE;
+    auto piece = [&](int q) {
+      const int c = c_lo + q;
+      return base + (size_t(c) * 2 + (q == 0 ? slot_lo : 0)) * (BQ * PART_STRIDE);
+    };
+    if (np <= 32) {
+      // lane q holds piece q's row max / sum
+      float2 ml = make_float2(-INFINITY, 0.f);
+      if (lane < np) ml = __ldcg(reinterpret_cast<const float2*>(piece(lane) + DH));
+      float M = ml.x;
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-  const float w = lane < sc.split ? ex2_ftz(ml.x - M) : 0.f;
-  float L = w * ml.y;
+      for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+      const float w = lane < np ? ex2_ftz(ml.x - M) : 0.f;
+      float L = w * ml.y;
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-  if (lane < DH / 4) {
-  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 4
-  for (int q = 0; q < sc.split; ++q) {
-    const float wq = __shfl_sync((1u << (DH / 4)) - 1u, w, q);
-    const float4 v = __ldcg(reinterpret_cast<const float4*>(base + size_t(q) * (BQ * PART_STRIDE)) + lane);
-    acc.x += wq * v.x;
-    acc.y += wq * v.y;
-    acc.z += wq * v.z;
-    acc.w += wq * v.w;
-  }
-  const float inv = L > 0.f ? 1.f / L : 0.f;
-  *reinterpret_cast<uint2*>(O + size_t(qrow) * ldo + h * DH + 4 * lane) =
-      make_uint2(pack_bf16x2(acc.x * inv, acc.y * inv), pack_bf16x2(acc.z * inv, acc.w * inv));
-  }
+      for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+      // lanes < DH / 4 accumulate 4 columns each, four pieces' loads in flight
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int q0 = 0; q0 < np; q0 += 4) {
+        float4 v[4];
+        float wq[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          wq[e] = __shfl_sync(0xffffffffu, w, (q0 + e) & 31);
+          v[e] = (q0 + e < np && lane < DH / 4)
+                     ? __ldcg(reinterpret_cast<const float4*>(piece(q0 + e)) + lane)
+                     : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float ww = q0 + e < np ? wq[e] : 0.f;
+          acc.x += ww * v[e].x;
+          acc.y += ww * v[e].y;
+          acc.z += ww * v[e].z;
+          acc.w += ww * v[e].w;
+        }
+      }
+      if (lane < DH / 4) {
+        const float inv = L > 0.f ? 1.f / L : 0.f;
+        const int qrow = tl.row0 + row;
+        *reinterpret_cast<uint2*>(O + size_t(qrow) * ldo + h * DH + 4 * lane) = make_uint2(
+            pack_bf16x2(acc.x * inv, acc.y * inv), pack_bf16x2(acc.z * inv, acc.w * inv));
+      }
+    } else {
+      // many pieces (very long key ranges): plain loops
+      float M = -INFINITY;
+      for (int q = lane; q < np; q += 32) M = fmaxf(M, __ldcg(piece(q) + DH));
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+      float L = 0.f;
+      for (int q = lane; q < np; q += 32) {
+        const float2 ml = __ldcg(reinterpret_cast<const float2*>(piece(q) + DH));
+        L += ex2_ftz(ml.x - M) * ml.y;
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+      if (lane < DH / 4) {
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int q = 0; q < np; ++q) {
+          const float* b = piece(q);
+          const float wq = ex2_ftz(__ldcg(b + DH) - M);
+          const float4 v = __ldcg(reinterpret_cast<const float4*>(b) + lane);
+          acc.x += wq * v.x;
+          acc.y += wq * v.y;
+          acc.z += wq * v.z;
+          acc.w += wq * v.w;
+        }
+        const float inv = L > 0.f ? 1.f / L : 0.f;
+        const int qrow = tl.row0 + row;
+        *reinterpret_cast<uint2*>(O + size_t(qrow) * ldo + h * DH + 4 * lane) = make_uint2(
+            pack_bf16x2(acc.x * inv, acc.y * inv), pack_bf16x2(acc.z * inv, acc.w * inv));
+      }
+    }
   }
 }
 
@@ -635,28 +737,31 @@ cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* 
   RC_TRY(head_map(Q, rm.bound, ldq, heads, dh, 16, BQ, &tqt));
   RC_TRY(head_map(K, kv_rows, ldkv, heads, dh, 16, BKV, &tkt));
   const float scale_log2 = float(1.4426950408889634 / sqrt(double(dh)));
-  const int ws_units = int(as.part_floats / (size_t(BQ) * PART_STRIDE));
   const int grid = CTAS_PER_SM * sms;
+  {
+    const unsigned long long tiles = (rm.bound + BQ - 1) / BQ + ai.n - 1;
+    if (tiles * heads * ((Nk + BKV - 1) / BKV) * grid >= (1ull << 32)) return cudaErrorInvalidValue;
+  }
+  // two partial pieces per CTA at most
+  if (as.part_floats < size_t(2) * grid * BQ * PART_STRIDE) return cudaErrorInvalidValue;
   if (dh == 72)
     RC_TRY(launch_k(attn_tc_kernel<72>, dim3(grid), dim3(THREADS), ACfg<72>::SMEM, st, tq, tqt,
-                    tk, tkt, tv, ai, Nk, O, ldo, heads, rm, scale_log2, err, as.part,
-                    ws_units));
+                    tk, tkt, tv, ai, Nk, O, ldo, heads, rm, scale_log2, err, as.part));
   else
     RC_TRY(launch_k(attn_tc_kernel<64>, dim3(grid), dim3(THREADS), ACfg<64>::SMEM, st, tq, tqt,
-                    tk, tkt, tv, ai, Nk, O, ldo, heads, rm, scale_log2, err, as.part,
-                    ws_units));
+                    tk, tkt, tv, ai, Nk, O, ldo, heads, rm, scale_log2, err, as.part));
   count_launches(1);
-  // key splits happen only with at least MIN_KB_PER_SPLIT key blocks per split
+  // stream-K (and so partial pieces) only with at least 2 MIN_KB_PER_SPLIT key blocks
   if ((Nk + BKV - 1) / BKV >= 2 * MIN_KB_PER_SPLIT) {
     const int tiles = (rm.bound + BQ - 1) / BQ + ai.n - 1;  // bound of the query tiles
     const int warps = tiles * heads * BQ;
     const int cgrid = min((warps + 7) / 8, 4 * sms);
     if (dh == 72)
       RC_TRY(launch_k(attn_combine_kernel<72>, dim3(cgrid), dim3(256), 0, st, as.part, O,
-                      ldo, heads, rm, ai.n, Nk, grid, ws_units, err));
+                      ldo, heads, rm, ai.n, Nk, grid, err));
     else
       RC_TRY(launch_k(attn_combine_kernel<64>, dim3(cgrid), dim3(256), 0, st, as.part, O,
-                      ldo, heads, rm, ai.n, Nk, grid, ws_units, err));
+                      ldo, heads, rm, ai.n, Nk, grid, err));
     count_launches(1);
   }
   return cudaSuccess;
