@@ -7,19 +7,21 @@
 //
 // C[M][n] = A[M][k] W[n][k]^T, A and W K-major bf16, f32 accumulation.
 // M (the dirty-token count) may live on the device: every CTA reads it and
-// derives the schedule: whole tiles in full waves.  The gated residual
-// (x += gate (C + b)) is written as vector reductions into x, so pieces of a
-// tile simply add up: for it a small last wave is instead cut into equal
-// k-block ranges (stream-K) so ragged tile counts still fill the GPU.  The
-// other epilogues always see whole tiles (splitting them would need a
-// workspace round trip that costs more than the idle SMs).
+// derives the same schedule.  The tile is 128 x BN with BN in {64, 128, 192,
+// 256}, chosen per launch from M by a cost model (the main loop streams
+// (128 + BN) x 64 bf16 operands per k-block from L2 at a fixed per-SM rate,
+// and only the last tile's epilogue is exposed), so that ragged row counts
+// still spread over the GPU.  Whole tiles go out in waves.  The gated
+// residual (x += gate (C + b)) is written as vector reductions into x, so
+// pieces of a tile simply add up: for it a small last wave is instead cut
+// into equal k-block ranges (stream-K).  Its casting variant (x += ..., then
+// xb = bf16(x), read-modify-write) and the other epilogues see whole tiles.
 //
 // CTA = 6 warps: warp 0 issues TMA loads, warp 1 owns TMEM and issues the
 // MMAs (one thread), warps 2..5 drain the accumulator (one TMEM lane = one
 // output row per thread, re-staged through shared memory so that global
-// writes are whole row pieces).  Two TMEM accumulators (tiles of 128 x 192,
-// or 128 x 128 when 192 does not divide n) let the epilogue of one tile
-// overlap the main loop of the next.
+// writes are whole row pieces).  Two TMEM accumulators of up to 256 columns
+// let the epilogue of one tile overlap the main loop of the next.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -43,19 +45,19 @@ constexpr int MIN_KB_PER_CTA = 4;
 constexpr int STAGING_WARP = 32 * 128;  // epilogue staging: 32 rows of 128 B per warp
 constexpr int STAGING_BYTES = 4 * STAGING_WARP;
 
-// Tile width BN (output features per tile): 192 when it divides n (every
-// PixArt-alpha width: 1152, 2304, 3456, 4608), else 128.
-template <int BN>
-struct TileCfg {
-  static constexpr int STAGE_B = BN * BK * 2;
-  static constexpr int STAGES = (200 * 1024) / (STAGE_A + STAGE_B);  // 6 for 128, 5 for 192
-  static constexpr int TMEM_COLS = (2 * BN <= 256) ? 256 : 512;     // two accumulators
-  static constexpr size_t SMEM_BYTES =
-      size_t(STAGES) * (STAGE_A + STAGE_B) + STAGING_BYTES + 1024 + 256;
-  // Instruction descriptor, kind::f16: D f32, A and B bf16, both K-major,
-  // N >> 3 at bit 17, M >> 4 at bit 24.
-  static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
-                                    (uint32_t(BN >> 3) << 17) | (uint32_t(BM >> 4) << 24);
+// Operand ring: stages of A (16 KB) + B (BN x 128 B), as many as fit.
+constexpr int RING_BYTES = 200 * 1024;
+constexpr int MAX_STAGES = 8;
+constexpr int TMEM_COLS = 512;  // two accumulators of up to 256 columns
+constexpr size_t SMEM_BYTES = size_t(RING_BYTES) + STAGING_BYTES + 1024 + 256;
+// Instruction descriptor, kind::f16: D f32, A and B bf16, both K-major,
+// M >> 4 at bit 24; N >> 3 goes to bit 17 at run time.
+constexpr uint32_t IDESC_BASE = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(BM >> 4) << 24);
+// The tile width chosen on the host for 1 .. BN_TABLE row tiles (in units of
+// 64 columns), passed by value; larger row counts choose on the device.
+constexpr int BN_TABLE = 64;
+struct BnTable {
+  uint8_t w64[BN_TABLE];
 };
 
 // ---------------------------------------------------------------- epilogue
@@ -86,7 +88,7 @@ __device__ __forceinline__ void epilogue_values(const GemmEpi& ep, int c0, int i
   if (ep.mode == EPI_GELU_BF16) {
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] = gelu_tanh(v[i]);
-  } else if (ep.mode == EPI_GATE_RES && ep.gate_tab) {
+  } else if ((ep.mode == EPI_GATE_RES || ep.mode == EPI_GATE_RES_CAST) && ep.gate_tab) {
     float g[32];
     load32(ep.gate_tab + c0, g);
     const float* tb = ep.gate_off >= 0 ? ep.its.tb[item] : nullptr;
@@ -111,6 +113,7 @@ __device__ __forceinline__ char* chunk_dst(const GemmEpi& ep, int r, int M, int 
     case EPI_F32:
       return reinterpret_cast<char*>(ep.out_f + size_t(r) * ep.ld_out + c0);
     case EPI_GATE_RES:
+    case EPI_GATE_RES_CAST:
       return reinterpret_cast<char*>(ep.xf + size_t(r) * ep.ld_xf + c0);
     case EPI_QKV: {
       const int part = c0 / ep.dsplit;
@@ -133,11 +136,13 @@ __device__ __forceinline__ char* chunk_dst(const GemmEpi& ep, int r, int M, int 
 // staging area, then groups of lanes write whole 128-byte (f32) or 64-byte
 // (bf16) row pieces.  Staging is XOR-swizzled in 16-byte units so that both
 // the row-per-lane writes and the piece-per-lane-group reads are free of bank
-// conflicts.  The gated residual goes out as vector reductions (x += value).
+// conflicts.  The gated residual goes out as vector reductions (x += value);
+// its casting variant reads x, adds, and writes x and bf16(x) (xb_row: the
+// row's bf16 copy, columns c0 ..).
 __device__ __forceinline__ void store_chunk(int mode, uint8_t* stg, int lane, const float* v,
-                                            char* dst) {
+                                            char* dst, bf16* xb_row) {
   const uint32_t s0 = saddr(stg);
-  if (mode == EPI_F32 || mode == EPI_GATE_RES) {
+  if (mode == EPI_F32 || mode == EPI_GATE_RES || mode == EPI_GATE_RES_CAST) {
 #pragma unroll
     for (int j = 0; j < 8; ++j)
       asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(
@@ -145,23 +150,39 @@ __device__ __forceinline__ void store_chunk(int mode, uint8_t* stg, int lane, co
                    "f"(v[4 * j]), "f"(v[4 * j + 1]), "f"(v[4 * j + 2]), "f"(v[4 * j + 3])
                    : "memory");
     __syncwarp();
+    // all row pointers and pieces first (independent, so they overlap),
+    // then the global writes
     const int j = lane & 7;
+    char* d[8];
+    bf16* xb[8];
+    float4 x[8];
 #pragma unroll
     for (int pass = 0; pass < 8; ++pass) {
       const int row = pass * 4 + (lane >> 3);
-      float4 x;
-      asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
-                   : "=f"(x.x), "=f"(x.y), "=f"(x.z), "=f"(x.w)
-                   : "r"(s0 + row * 128 + 16 * (j ^ (row & 7)))
-                   : "memory");
-      char* d = reinterpret_cast<char*>(
+      d[pass] = reinterpret_cast<char*>(
           __shfl_sync(0xffffffffu, reinterpret_cast<unsigned long long>(dst), row));
-      if (d) {
-        float* q = reinterpret_cast<float*>(d) + 4 * j;
-        if (mode == EPI_GATE_RES)
-          red_add_v4(q, x.x, x.y, x.z, x.w);
-        else
-          *reinterpret_cast<float4*>(q) = x;
+      xb[pass] = mode == EPI_GATE_RES_CAST
+                     ? reinterpret_cast<bf16*>(__shfl_sync(
+                           0xffffffffu, reinterpret_cast<unsigned long long>(xb_row), row))
+                     : nullptr;
+      x[pass] = *reinterpret_cast<const float4*>(stg + row * 128 + 16 * (j ^ (row & 7)));
+    }
+#pragma unroll
+    for (int pass = 0; pass < 8; ++pass) {
+      if (!d[pass]) continue;
+      float* q = reinterpret_cast<float*>(d[pass]) + 4 * j;
+      float4 y = x[pass];
+      if (mode == EPI_GATE_RES) {
+        red_add_v4(q, y.x, y.y, y.z, y.w);
+      } else if (mode == EPI_GATE_RES_CAST) {
+        const float4 o = __ldcg(reinterpret_cast<const float4*>(q));
+        y.x += o.x; y.y += o.y; y.z += o.z; y.w += o.w;
+        *reinterpret_cast<float4*>(q) = y;
+        if (xb[pass])
+          *reinterpret_cast<uint2*>(xb[pass] + 4 * j) =
+              make_uint2(pack_bf16x2(y.x, y.y), pack_bf16x2(y.z, y.w));
+      } else {
+        *reinterpret_cast<float4*>(q) = y;
       }
     }
   } else {
@@ -176,32 +197,34 @@ __device__ __forceinline__ void store_chunk(int mode, uint8_t* stg, int lane, co
                    : "memory");
     __syncwarp();
     const int j = lane & 3;
+    char* d[4];
+    uint4 x[4];
 #pragma unroll
     for (int pass = 0; pass < 4; ++pass) {
       const int row = pass * 8 + (lane >> 2);
-      uint4 x;
-      asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
-                   : "=r"(x.x), "=r"(x.y), "=r"(x.z), "=r"(x.w)
-                   : "r"(s0 + row * 64 + 16 * (j ^ ((row >> 1) & 3)))
-                   : "memory");
-      char* d = reinterpret_cast<char*>(
+      d[pass] = reinterpret_cast<char*>(
           __shfl_sync(0xffffffffu, reinterpret_cast<unsigned long long>(dst), row));
-      if (d) reinterpret_cast<uint4*>(d)[j] = x;
+      x[pass] = *reinterpret_cast<const uint4*>(stg + row * 64 + 16 * (j ^ ((row >> 1) & 3)));
     }
+#pragma unroll
+    for (int pass = 0; pass < 4; ++pass)
+      if (d[pass]) reinterpret_cast<uint4*>(d[pass])[j] = x[pass];
   }
   __syncwarp();  // the staging area is rewritten by the next chunk
 }
 
-// Schedule.  Tiles (t = nn * mt + m, m fastest so neighbouring CTAs share
-// weight tiles in L2) go whole to CTA t mod G in full waves.  For an additive
-// epilogue, when the last wave would leave more than half the CTAs idle, its
-// R remainder tiles are instead laid end to end by k-block and cut into G_r
-// equal ranges (stream-K, at least MIN_KB_PER_CTA k-blocks each).
-template <int BN>
+// Schedule, identical in every thread.  Tiles t = nn * mt + m (m fastest, so
+// CTAs in flight share weight tiles in L2) go whole to CTA t mod G in waves.
+// For the (non-casting) gated residual, when the last wave would leave more
+// than half the CTAs idle, its R remainder tiles are laid end to end by
+// k-block and cut into Gr equal ranges (stream-K, at least MIN_KB_PER_CTA
+// k-blocks each).
 struct Sched {
-  int mt, nt, tiles, kbt, G, whole, Gr;
+  int BN, stages, mt, nt, tiles, kbt, G, whole, Gr;
   long long Wr;
-  __device__ void init(int M, int n, int k, int grid, bool additive) {
+  __host__ __device__ void plan(int M, int bn, int n, int k, int grid, bool additive) {
+    BN = bn;
+    stages = stages_for(bn);
     mt = (M + BM - 1) / BM;
     nt = n / BN;
     tiles = mt * nt;
@@ -215,16 +238,56 @@ struct Sched {
     if (g < 1) g = 1;
     Gr = split ? int(g < G ? g : G) : 0;
   }
+  __host__ __device__ static int stages_for(int bn) {
+    const int s = RING_BYTES / (STAGE_A + bn * BK * 2);
+    return s < MAX_STAGES ? s : MAX_STAGES;
+  }
+  // Estimated duration (SM cycles): waves x k-blocks x per-k-block time (L2
+  // rate of ~60 B/clk per SM) plus the exposed epilogue (~26 B/clk per SM).
+  __host__ __device__ float cost(int out_bytes) const {
+    const float ckb = float(STAGE_A + BN * BK * 2) * (1.f / 60.f);
+    const float cep = float(BM * BN * out_bytes) * (1.f / 26.f);
+    const int waves = (whole + G - 1) / G;
+    float c = float(waves) * float(kbt) * ckb + cep;
+    if (Gr > 0) c += float((Wr + Gr - 1) / Gr) * ckb + cep;
+    return c;
+  }
+  // Picks BN (n % BN == 0) with the lowest estimate; ties go to wider tiles.
+  __host__ __device__ static int pick_bn(int M, int n, int k, int grid, int mode) {
+    Sched s;
+    const bool additive = mode == EPI_GATE_RES;
+    const int out_bytes = mode == EPI_GATE_RES_CAST ? 10
+                          : (mode == EPI_F32 || mode == EPI_GATE_RES) ? 4 : 2;
+    const int cand[4] = {256, 192, 128, 64};
+    float best = 3.4e38f;
+    int pick = 64;
+    for (int i = 0; i < 4; ++i) {
+      if (n % cand[i]) continue;
+      s.plan(M, cand[i], n, k, grid, additive);
+      const float c = s.cost(out_bytes);
+      if (c < best * 0.999f) {
+        best = c;
+        pick = cand[i];
+      }
+    }
+    return pick;
+  }
+  // table: the host's pick for 1 .. BN_TABLE row tiles (0 = not tabulated)
+  __device__ void init(int M, int n, int k, int grid, int mode, const uint8_t* table) {
+    const int m_tiles = (M + BM - 1) / BM;
+    int bn = m_tiles >= 1 && m_tiles <= BN_TABLE ? 64 * int(table[m_tiles - 1]) : 0;
+    if (bn == 0) bn = pick_bn(M, n, k, grid, mode);
+    plan(M, bn, n, k, grid, mode == EPI_GATE_RES);
+  }
   __device__ long long bound(int c) const { return Wr * c / Gr; }
 };
 
 // The segments (tile, k-blocks [kb0, kb1)) of one CTA, in order.
-template <int BN>
 struct Segs {
-  const Sched<BN>* sc;
+  const Sched* sc;
   int t_next;
   long long cur, end;
-  __device__ void init(const Sched<BN>& s, int c) {
+  __device__ void init(const Sched& s, int c) {
     sc = &s;
     t_next = c;
     cur = c < s.Gr ? s.bound(c) : 0;
@@ -248,31 +311,29 @@ struct Segs {
   }
 };
 
-template <int BN>
 __global__ void __launch_bounds__(THREADS, 1)
-gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-               int Mbound, const int* __restrict__ dcount, int n, int k,
-               const __grid_constant__ GemmEpi ep) {
-  using TC = TileCfg<BN>;
-  constexpr int STAGES = TC::STAGES, STAGE_B = TC::STAGE_B, TMEM_COLS = TC::TMEM_COLS;
+gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB64,
+               const __grid_constant__ CUtensorMap tmB128,
+               const __grid_constant__ CUtensorMap tmB192,
+               const __grid_constant__ CUtensorMap tmB256, int Mbound,
+               const int* __restrict__ dcount, int n, int k, const __grid_constant__ GemmEpi ep,
+               const __grid_constant__ BnTable bt) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  // 1024-aligned operand stages, epilogue staging, then barriers
+  // 1024-aligned operand ring, epilogue staging, then barriers
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  uint8_t* sA = smem;
-  uint8_t* sB = smem + STAGES * STAGE_A;
-  uint8_t* sStg = sB + STAGES * STAGE_B;
+  uint8_t* sStg = smem + RING_BYTES;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sStg + STAGING_BYTES);
-  // bars: full[STAGES], empty[STAGES], tfull[2], tempty[2]
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 4);
+  // bars: full[MAX_STAGES], empty[MAX_STAGES], tfull[2], tempty[2]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * MAX_STAGES + 4);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t full0 = saddr(bars), empty0 = saddr(bars + STAGES);
-  const uint32_t tfull0 = saddr(bars + 2 * STAGES), tempty0 = saddr(bars + 2 * STAGES + 2);
+  const uint32_t full0 = saddr(bars), empty0 = saddr(bars + MAX_STAGES);
+  const uint32_t tfull0 = saddr(bars + 2 * MAX_STAGES), tempty0 = saddr(bars + 2 * MAX_STAGES + 2);
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
+    for (int s = 0; s < MAX_STAGES; ++s) {
       mbar_init(full0 + 8 * s, 1);
       mbar_init(empty0 + 8 * s, 1);
     }
@@ -283,16 +344,10 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                     saddr(tmem_slot)),
-                 "r"(TMEM_COLS)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-  }
+  if (warp == 1) tmem_alloc(saddr(tmem_slot), TMEM_COLS);
   if (warp == 0 && lane == 0) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB64)) : "memory");
   }
   tc_fence_before();
   __syncthreads();
@@ -304,24 +359,31 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   pdl_wait();
   pdl_trigger();
   const int M = live_count(dcount, Mbound, ep.err);
-  Sched<BN> sc;
-  sc.init(M, n, k, int(gridDim.x), ep.mode == EPI_GATE_RES);
+  Sched sc;
+  sc.init(M, n, k, int(gridDim.x), ep.mode, bt.w64);
+  const int BN = sc.BN, STAGES = sc.stages;
+  const int STAGE = STAGE_A + BN * BK * 2;
 
   if (warp == 0) {
     // ------------------------------------------------------- TMA producer
     if (lane == 0) {
+      // B as one box of BN rows (maps for the widths that divide n)
+      const CUtensorMap* tmB = BN == 256 ? &tmB256 : BN == 192 ? &tmB192 : BN == 128 ? &tmB128 : &tmB64;
+      if (BN != 64)
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tmB)) : "memory");
       int stage = 0;
       uint32_t phase = 0;
-      Segs<BN> sg;
+      Segs sg;
       sg.init(sc, blockIdx.x);
       int t, kb0, kb1;
       while (sg.next(t, kb0, kb1)) {
         const int m = t % sc.mt, nn = t / sc.mt;
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(empty0 + 8 * stage, phase ^ 1, abort_flag)) goto timeout;
-          mbar_expect_tx(full0 + 8 * stage, STAGE_A + STAGE_B);
-          tma_load_2d(saddr(sA + stage * STAGE_A), &tmA, full0 + 8 * stage, kb * BK, m * BM);
-          tma_load_2d(saddr(sB + stage * STAGE_B), &tmB, full0 + 8 * stage, kb * BK, nn * BN);
+          uint8_t* st = smem + stage * STAGE;
+          mbar_expect_tx(full0 + 8 * stage, STAGE);
+          tma_load_2d(saddr(st), &tmA, full0 + 8 * stage, kb * BK, m * BM);
+          tma_load_2d(saddr(st + STAGE_A), tmB, full0 + 8 * stage, kb * BK, nn * BN);
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
         }
       }
@@ -329,24 +391,28 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   } else if (warp == 1) {
     // ------------------------------------------------------- MMA issuer
     if (lane == 0) {
+      const uint32_t idesc = IDESC_BASE | (uint32_t(BN >> 3) << 17);
+      const uint64_t da = sw128_desc(saddr(smem)), db = sw128_desc(saddr(smem + STAGE_A));
       int stage = 0;
       uint32_t phase = 0;
       int acc = 0;
       uint32_t acc_phase = 0;
-      Segs<BN> sg;
+      Segs sg;
       sg.init(sc, blockIdx.x);
       int t, kb0, kb1;
       while (sg.next(t, kb0, kb1)) {
         if (!mbar_wait(tempty0 + 8 * acc, acc_phase ^ 1, abort_flag)) goto timeout;
         tc_fence_after();
-        const uint32_t dtm = tmem_base + uint32_t(acc * (TMEM_COLS / 2));
+        const uint32_t dtm = tmem_base + uint32_t(acc * 256);
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(full0 + 8 * stage, phase, abort_flag)) goto timeout;
           tc_fence_after();
-          const uint32_t a0 = saddr(sA + stage * STAGE_A), b0 = saddr(sB + stage * STAGE_B);
+          // stage descriptors differ only in the start address field
+          // (address >> 4; no carry out of its 14 bits below 256 KB)
+          const uint64_t so = uint64_t((stage * STAGE) >> 4);
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk)
-            umma_bf16(dtm, sw128_desc(a0 + 32 * kk), sw128_desc(b0 + 32 * kk), TC::IDESC,
+            umma_bf16(dtm, da + so + 2 * kk, db + so + 2 * kk, idesc,
                       (kb > kb0 || kk > 0) ? 1u : 0u);
           umma_commit(empty0 + 8 * stage);
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
@@ -360,7 +426,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     const int sp = warp & 3;  // TMEM lane sub-partition this warp may access
     int acc = 0;
     uint32_t acc_phase = 0;
-    Segs<BN> sg;
+    Segs sg;
     sg.init(sc, blockIdx.x);
     int t, kb0, kb1;
     while (sg.next(t, kb0, kb1)) {
@@ -369,7 +435,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       tc_fence_after();
       const int row = sp * 32 + lane;
       const int r = m * BM + row;
-      const uint32_t tbase = tmem_base + uint32_t(acc * (TMEM_COLS / 2)) + (uint32_t(sp * 32) << 16);
+      const uint32_t tbase = tmem_base + uint32_t(acc * 256) + (uint32_t(sp * 32) << 16);
       int tok = 0, item = 0;
       if (r < M) {
         if (ep.mode == EPI_QKV) tok = ep.tok ? __ldg(ep.tok + r) : r;
@@ -383,7 +449,10 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         tmem_ld32(tbase + uint32_t(ch * 32), v);
         const int c0 = nn * BN + ch * 32;
         epilogue_values(ep, c0, item, v, kb0 == 0);
-        store_chunk(ep.mode, sStg + sp * STAGING_WARP, lane, v, chunk_dst(ep, r, M, tok, item, c0));
+        bf16* xb_row = (ep.mode == EPI_GATE_RES_CAST && r < M)
+                           ? ep.out_bf + size_t(r) * ep.ld_out + c0 : nullptr;
+        store_chunk(ep.mode, sStg + sp * STAGING_WARP, lane, v, chunk_dst(ep, r, M, tok, item, c0),
+                    xb_row);
       }
       tc_fence_before();
       mbar_arrive(tempty0 + 8 * acc);
@@ -400,9 +469,7 @@ done:
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
-                 "r"(TMEM_COLS)
-                 : "memory");
+    tmem_dealloc(tmem_base, TMEM_COLS);
   }
 }
 
@@ -466,6 +533,29 @@ cudaError_t tensor_map(const bf16* p, int rows, int cols, int ld, int box_rows, 
   return cudaSuccess;
 }
 
+// Tile-width table of a GEMM shape, cached (the cost model runs 4 x 64 plans).
+BnTable bn_table(int n, int k, int sms, int mode, int mt_bound) {
+  static std::mutex mu;
+  static std::unordered_map<uint64_t, BnTable> cache;
+  const int mtb = mt_bound < BN_TABLE ? mt_bound : BN_TABLE;
+  // bits: mtb 0-6, mode 7-10, sms 11-18, k 19-40, n 41-63 (n, k < 2^22: checked)
+  const uint64_t full_key = uint64_t(mtb) | (uint64_t(mode & 15) << 7) |
+                            (uint64_t(sms & 255) << 11) | (uint64_t(k & 0x3FFFFF) << 19) |
+                            (uint64_t(n) << 41);
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    auto it = cache.find(full_key);
+    if (it != cache.end()) return it->second;
+  }
+  BnTable bt{};
+  for (int mt = 1; mt <= mtb; ++mt)
+    bt.w64[mt - 1] = uint8_t(Sched::pick_bn(mt * BM, n, k, sms, mode) / 64);
+  std::lock_guard<std::mutex> lock(mu);
+  if (cache.size() > 4096) cache.clear();
+  cache.emplace(full_key, bt);
+  return bt;
+}
+
 int device_sms() {
   static int sms[64] = {};
   int dev = 0;
@@ -473,10 +563,8 @@ int device_sms() {
   if (!sms[dev]) {
     int v = 0;
     if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-    if (cudaFuncSetAttribute(gemm_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             int(TileCfg<128>::SMEM_BYTES)) != cudaSuccess ||
-        cudaFuncSetAttribute(gemm_tc_kernel<192>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             int(TileCfg<192>::SMEM_BYTES)) != cudaSuccess)
+    if (cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             int(SMEM_BYTES)) != cudaSuccess)
       return 0;
     sms[dev] = v;
   }
@@ -488,21 +576,22 @@ int device_sms() {
 cudaError_t launch_gemm(const bf16* A, int lda, const bf16* W, int Mbound, const int* dcount,
                         int n, int k, const GemmEpi& ep, cudaStream_t st) {
   if (Mbound <= 0) return cudaSuccess;
-  if (n % 128 || k % BK) return cudaErrorInvalidValue;
+  if (n % 64 || k % BK || n >= (1 << 22) || k >= (1 << 22)) return cudaErrorInvalidValue;
   const int sms = device_sms();
   if (!sms) return cudaErrorInvalidDevice;
-  const int BN = (n % 192 == 0) ? 192 : 128;
   cudaError_t e;
-  CUtensorMap ta, tb;
+  CUtensorMap ta, tb[4];
   if ((e = tensor_map(A, Mbound, k, lda, BM, &ta)) != cudaSuccess) return e;
-  if ((e = tensor_map(W, n, k, k, BN, &tb)) != cudaSuccess) return e;
-  const int grid = sms;
-  if (BN == 192)
-    RC_TRY(launch_k(gemm_tc_kernel<192>, dim3(grid), dim3(THREADS), TileCfg<192>::SMEM_BYTES, st,
-                    ta, tb, Mbound, dcount, n, k, ep));
-  else
-    RC_TRY(launch_k(gemm_tc_kernel<128>, dim3(grid), dim3(THREADS), TileCfg<128>::SMEM_BYTES, st,
-                    ta, tb, Mbound, dcount, n, k, ep));
+  // one B map per tile width that divides n (the kernel picks the width);
+  // the others repeat the 64-row map and are never used
+  const int widths[4] = {64, 128, 192, 256};
+  for (int i = 0; i < 4; ++i) {
+    const int w = n % widths[i] == 0 ? widths[i] : 64;
+    if ((e = tensor_map(W, n, k, k, w, &tb[i])) != cudaSuccess) return e;
+  }
+  const BnTable bt = bn_table(n, k, sms, ep.mode, (Mbound + BM - 1) / BM);
+  RC_TRY(launch_k(gemm_tc_kernel, dim3(sms), dim3(THREADS), SMEM_BYTES, st, ta, tb[0], tb[1],
+                  tb[2], tb[3], Mbound, dcount, n, k, ep, bt));
   count_launches(1);
   return cudaSuccess;
 }

@@ -73,9 +73,6 @@ cudaError_t launch_batch_rows(const BatchIn& in, int* tok, int* item, int* meta,
 cudaError_t launch_ln_mod(const float* x, const float* tab, int k_sh, int k_sc, const Items& it,
                           bf16* out, const RowMap& rm, long long hprev_off, int d, unsigned* err,
                           cudaStream_t st);
-// out[r] = bf16(x[r]) for r < D.
-cudaError_t launch_cast_rows(const float* x, int ldx, bf16* out, int ldo, int Dbound,
-                             const int* dcount, int d, unsigned* err, cudaStream_t st);
 
 // xf[r] = W_e patch(tok[r]) + b_e + pos[tok[r]], the patch from the row's item latent.
 cudaError_t launch_patch_embed(int gh, int gw, int p, int C, const bf16* We, const float* be,
@@ -103,7 +100,16 @@ cudaError_t launch_scatter_bf16(const float* src, const Items& it, long long off
                                 const RowMap& rm, int d, unsigned* err, cudaStream_t st);
 
 // ---------------------------------------------------------------------- GEMM
-enum EpiMode { EPI_F32 = 0, EPI_BIAS_BF16 = 1, EPI_GELU_BF16 = 2, EPI_GATE_RES = 3, EPI_QKV = 4 };
+// EPI_GATE_RES: xf += gate (acc + b) as reductions (tiles may be split);
+// EPI_GATE_RES_CAST: the same on whole tiles, then out_bf = bf16(xf).
+enum EpiMode {
+  EPI_F32 = 0,
+  EPI_BIAS_BF16 = 1,
+  EPI_GELU_BF16 = 2,
+  EPI_GATE_RES = 3,
+  EPI_QKV = 4,
+  EPI_GATE_RES_CAST = 5
+};
 
 struct GemmEpi {
   int mode;
@@ -125,7 +131,7 @@ struct GemmEpi {
 };
 
 // C[M][n] = A[M][k] W[n][k]^T, epilogue `ep`.  M = *dcount if non-null (bounded
-// by Mbound) else Mbound.  n % 128 == 0, k % 64 == 0.
+// by Mbound) else Mbound.  n % 64 == 0, k % 64 == 0.
 cudaError_t launch_gemm(const bf16* A, int lda, const bf16* W, int Mbound, const int* dcount,
                         int n, int k, const GemmEpi& ep, cudaStream_t st);
 

@@ -261,14 +261,18 @@ rc_status run_block(rc_ctx* c, rc_cache* k, int l, const rc::RowMap& rm, const S
     g.its = si.its;
     return g;
   };
+  // (whole tiles, read-modify-write, also leaving xb = bf16(x) for the
+  // cross-attention query projection)
   e = gated(w.b_o, 2);
+  e.mode = rc::EPI_GATE_RES_CAST;
+  e.out_bf = c->xb;
+  e.ld_out = d;
   {
     Probe pr(c, RC_PROBE_GEMM, st);
     RC_CUDA(rc::launch_gemm(c->ob, d, static_cast<const bf16*>(w.W_o), rm.bound, rm.count, d, d,
                             e, st), "gemm(out)");
   }
-  // q' = x W_xq^T + b (on a bf16 copy of x)
-  RC_CUDA(rc::launch_cast_rows(c->xf, d, c->xb, d, rm.bound, rm.count, d, c->err, st), "cast");
+  // q' = x W_xq^T + b (on the bf16 copy of x)
   e = rc::GemmEpi{};
   e.mode = rc::EPI_BIAS_BF16;
   e.bias = w.b_xq;

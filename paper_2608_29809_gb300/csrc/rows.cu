@@ -301,31 +301,6 @@ cudaError_t launch_ln_mod(const float* x, const float* tab, int k_sh, int k_sc, 
   return cudaSuccess;
 }
 
-// out[r] = bf16(x[r]); one warp per row, 16-byte loads.
-__global__ void __launch_bounds__(LN_WARPS * 32)
-cast_rows_kernel(const float* __restrict__ x, int ldx, bf16* __restrict__ out, int ldo,
-                 int Dbound, const int* __restrict__ dcount, int d, unsigned* err) {
-  pdl_wait();
-  pdl_trigger();
-  const int D = live_count(dcount, Dbound, err);
-  for (int r = blockIdx.x * LN_WARPS + (threadIdx.x >> 5); r < D; r += gridDim.x * LN_WARPS) {
-    const float4* xr = reinterpret_cast<const float4*>(x + size_t(r) * ldx);
-    uint2* orow = reinterpret_cast<uint2*>(out + size_t(r) * ldo);
-    for (int c = threadIdx.x & 31; c < d / 4; c += 32) {
-      const float4 v = xr[c];
-      orow[c] = make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
-    }
-  }
-}
-
-cudaError_t launch_cast_rows(const float* x, int ldx, bf16* out, int ldo, int Dbound,
-                             const int* dcount, int d, unsigned* err, cudaStream_t st) {
-  if (Dbound <= 0) return cudaSuccess;
-  RC_TRY(launch_k(cast_rows_kernel, dim3(row_grid(Dbound, LN_WARPS, 4)), dim3(LN_WARPS * 32), 0, st, x,
-                  ldx, out, ldo, Dbound, dcount, d, err));
-  count_launches(1);
-  return cudaSuccess;
-}
 
 // ============================================================ patch embed
 // x_r = W_e patch(idx[r]) + b_e + pos[idx[r]], the patch vector ordered
