@@ -53,8 +53,8 @@ constexpr size_t SMEM_BYTES = size_t(RING_BYTES) + STAGING_BYTES + 1024 + 256;
 // Instruction descriptor, kind::f16: D f32, A and B bf16, both K-major,
 // M >> 4 at bit 24; N >> 3 goes to bit 17 at run time.
 constexpr uint32_t IDESC_BASE = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(BM >> 4) << 24);
-// The tile width chosen on the host for 1 .. BN_TABLE row tiles (in units of
-// 64 columns), passed by value; larger row counts choose on the device.
+// The tile width and split chosen on the host for 1 .. BN_TABLE row tiles
+// (BN / 64 + 8 S), passed by value; larger row counts choose on the device.
 constexpr int BN_TABLE = 64;
 struct BnTable {
   uint8_t w64[BN_TABLE];
@@ -215,14 +215,16 @@ __device__ __forceinline__ void store_chunk(int mode, uint8_t* stg, int lane, co
 
 // Schedule, identical in every thread.  Tiles t = nn * mt + m (m fastest, so
 // CTAs in flight share weight tiles in L2) go whole to CTA t mod G in waves.
-// For the (non-casting) gated residual, when the last wave would leave more
-// than half the CTAs idle, its R remainder tiles are laid end to end by
-// k-block and cut into Gr equal ranges (stream-K, at least MIN_KB_PER_CTA
-// k-blocks each).
+// The (non-casting) gated residual, whose pieces add up, may instead cut
+// its k range: into S equal parts when tiles x S fit one wave (one piece per
+// CTA), or, when the last wave would leave more than half the CTAs idle, by
+// laying the R remainder tiles end to end by k-block and cutting them into
+// Gr equal ranges (stream-K, at least MIN_KB_PER_CTA k-blocks each).
 struct Sched {
-  int BN, stages, mt, nt, tiles, kbt, G, whole, Gr;
+  int BN, stages, mt, nt, tiles, kbt, G, whole, Gr, S;
   long long Wr;
-  __host__ __device__ void plan(int M, int bn, int n, int k, int grid, bool additive) {
+  // S > 0: split-S (requires tiles * S <= grid); S == 0: waves (+ stream-K)
+  __host__ __device__ void plan(int M, int bn, int n, int k, int grid, bool additive, int s) {
     BN = bn;
     stages = stages_for(bn);
     mt = (M + BM - 1) / BM;
@@ -230,6 +232,13 @@ struct Sched {
     tiles = mt * nt;
     kbt = k / BK;
     G = grid;
+    S = s;
+    if (S > 0) {
+      whole = 0;
+      Wr = 0;
+      Gr = 0;
+      return;
+    }
     const int R = tiles % G;
     const bool split = additive && R > 0 && 2 * R <= G && kbt >= 2 * MIN_KB_PER_CTA;
     whole = split ? tiles - R : tiles;
@@ -242,42 +251,50 @@ struct Sched {
     const int s = RING_BYTES / (STAGE_A + bn * BK * 2);
     return s < MAX_STAGES ? s : MAX_STAGES;
   }
-  // Estimated duration (SM cycles): waves x k-blocks x per-k-block time (L2
-  // rate of ~60 B/clk per SM) plus the exposed epilogue (~26 B/clk per SM).
+  // Estimated duration (SM cycles): k-blocks on the busiest CTA x per-k-block
+  // time (operands from L2 at ~60 B/clk per SM) plus its exposed epilogues
+  // (~12 B/clk per SM, measured); a stream-K CTA holds two pieces.
   __host__ __device__ float cost(int out_bytes) const {
     const float ckb = float(STAGE_A + BN * BK * 2) * (1.f / 60.f);
-    const float cep = float(BM * BN * out_bytes) * (1.f / 26.f);
+    const float cep = float(BM * BN * out_bytes) * (1.f / 12.f);
+    if (S > 0) return float((kbt + S - 1) / S) * ckb + cep;
     const int waves = (whole + G - 1) / G;
-    float c = float(waves) * float(kbt) * ckb + cep;
-    if (Gr > 0) c += float((Wr + Gr - 1) / Gr) * ckb + cep;
+    float c = float(waves) * float(kbt) * ckb + (waves > 0 ? cep : 0.f);
+    if (Gr > 0) c += float((Wr + Gr - 1) / Gr) * ckb + 2.f * cep;
     return c;
   }
-  // Picks BN (n % BN == 0) with the lowest estimate; ties go to wider tiles.
-  __host__ __device__ static int pick_bn(int M, int n, int k, int grid, int mode) {
+  // Picks BN (n % BN == 0) and, for the additive gated residual, a split,
+  // with the lowest estimate; ties go to wider tiles and fewer pieces.
+  // Returns BN / 64 + 8 S.
+  __host__ __device__ static int pick(int M, int n, int k, int grid, int mode) {
     Sched s;
     const bool additive = mode == EPI_GATE_RES;
     const int out_bytes = mode == EPI_GATE_RES_CAST ? 10
                           : (mode == EPI_F32 || mode == EPI_GATE_RES) ? 4 : 2;
     const int cand[4] = {256, 192, 128, 64};
     float best = 3.4e38f;
-    int pick = 64;
+    int code = 1;
     for (int i = 0; i < 4; ++i) {
       if (n % cand[i]) continue;
-      s.plan(M, cand[i], n, k, grid, additive);
-      const float c = s.cost(out_bytes);
-      if (c < best * 0.999f) {
-        best = c;
-        pick = cand[i];
+      for (int sp = 0; sp <= (additive ? 4 : 0); ++sp) {
+        if (sp == 1) continue;
+        s.plan(M, cand[i], n, k, grid, additive, sp);
+        if (sp > 0 && (s.tiles * sp > grid || s.kbt < sp * MIN_KB_PER_CTA)) continue;
+        const float c = s.cost(out_bytes);
+        if (c < best * 0.999f) {
+          best = c;
+          code = cand[i] / 64 + 8 * sp;
+        }
       }
     }
-    return pick;
+    return code;
   }
   // table: the host's pick for 1 .. BN_TABLE row tiles (0 = not tabulated)
   __device__ void init(int M, int n, int k, int grid, int mode, const uint8_t* table) {
     const int m_tiles = (M + BM - 1) / BM;
-    int bn = m_tiles >= 1 && m_tiles <= BN_TABLE ? 64 * int(table[m_tiles - 1]) : 0;
-    if (bn == 0) bn = pick_bn(M, n, k, grid, mode);
-    plan(M, bn, n, k, grid, mode == EPI_GATE_RES);
+    int code = m_tiles >= 1 && m_tiles <= BN_TABLE ? int(table[m_tiles - 1]) : 0;
+    if (code == 0) code = pick(M, n, k, grid, mode);
+    plan(M, 64 * (code & 7), n, k, grid, mode == EPI_GATE_RES, code >> 3);
   }
   __device__ long long bound(int c) const { return Wr * c / Gr; }
 };
@@ -292,8 +309,21 @@ struct Segs {
     t_next = c;
     cur = c < s.Gr ? s.bound(c) : 0;
     end = c < s.Gr ? s.bound(c + 1) : 0;
+    if (s.S > 0) {  // split-S: CTA c < tiles * S holds piece c / tiles of tile c % tiles
+      cur = 0;
+      end = c < s.tiles * s.S ? 1 : 0;
+    }
   }
   __device__ bool next(int& t, int& kb0, int& kb1) {
+    if (sc->S > 0) {
+      if (cur >= end) return false;
+      ++cur;
+      const int p = t_next / sc->tiles;
+      t = t_next - p * sc->tiles;
+      kb0 = p * sc->kbt / sc->S;
+      kb1 = (p + 1) * sc->kbt / sc->S;
+      return true;
+    }
     if (t_next < sc->whole) {
       t = t_next;
       t_next += sc->G;
@@ -548,8 +578,7 @@ BnTable bn_table(int n, int k, int sms, int mode, int mt_bound) {
     if (it != cache.end()) return it->second;
   }
   BnTable bt{};
-  for (int mt = 1; mt <= mtb; ++mt)
-    bt.w64[mt - 1] = uint8_t(Sched::pick_bn(mt * BM, n, k, sms, mode) / 64);
+  for (int mt = 1; mt <= mtb; ++mt) bt.w64[mt - 1] = uint8_t(Sched::pick(mt * BM, n, k, sms, mode));
   std::lock_guard<std::mutex> lock(mu);
   if (cache.size() > 4096) cache.clear();
   cache.emplace(full_key, bt);
