@@ -167,22 +167,33 @@ __device__ __forceinline__ void store_chunk(int mode, uint8_t* stg, int lane, co
                      : nullptr;
       x[pass] = *reinterpret_cast<const float4*>(stg + row * 128 + 16 * (j ^ (row & 7)));
     }
+    if (mode == EPI_GATE_RES_CAST) {
+      // read-modify-write: all eight reads in flight before the writes
+      float4 o[8];
 #pragma unroll
-    for (int pass = 0; pass < 8; ++pass) {
-      if (!d[pass]) continue;
-      float* q = reinterpret_cast<float*>(d[pass]) + 4 * j;
-      float4 y = x[pass];
-      if (mode == EPI_GATE_RES) {
-        red_add_v4(q, y.x, y.y, y.z, y.w);
-      } else if (mode == EPI_GATE_RES_CAST) {
-        const float4 o = __ldcg(reinterpret_cast<const float4*>(q));
-        y.x += o.x; y.y += o.y; y.z += o.z; y.w += o.w;
-        *reinterpret_cast<float4*>(q) = y;
+      for (int pass = 0; pass < 8; ++pass)
+        o[pass] = d[pass] ? __ldcg(reinterpret_cast<const float4*>(d[pass]) + j)
+                          : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int pass = 0; pass < 8; ++pass) {
+        if (!d[pass]) continue;
+        float4 y = x[pass];
+        y.x += o[pass].x; y.y += o[pass].y; y.z += o[pass].z; y.w += o[pass].w;
+        reinterpret_cast<float4*>(d[pass])[j] = y;
         if (xb[pass])
           *reinterpret_cast<uint2*>(xb[pass] + 4 * j) =
               make_uint2(pack_bf16x2(y.x, y.y), pack_bf16x2(y.z, y.w));
-      } else {
-        *reinterpret_cast<float4*>(q) = y;
+      }
+    } else {
+#pragma unroll
+      for (int pass = 0; pass < 8; ++pass) {
+        if (!d[pass]) continue;
+        float* q = reinterpret_cast<float*>(d[pass]) + 4 * j;
+        const float4 y = x[pass];
+        if (mode == EPI_GATE_RES)
+          red_add_v4(q, y.x, y.y, y.z, y.w);
+        else
+          *reinterpret_cast<float4*>(q) = y;
       }
     }
   } else {

@@ -295,7 +295,7 @@ cudaError_t launch_ln_mod(const float* x, const float* tab, int k_sh, int k_sc, 
                           bf16* out, const RowMap& rm, long long hprev_off, int d, unsigned* err,
                           cudaStream_t st) {
   if (rm.bound <= 0) return cudaSuccess;
-  RC_TRY(launch_k(ln_mod_kernel, dim3(row_grid(rm.bound, LN_WARPS, 4)), dim3(LN_WARPS * 32), 0,
+  RC_TRY(launch_k(ln_mod_kernel, dim3(row_grid(rm.bound, LN_WARPS, 1)), dim3(LN_WARPS * 32), 0,
                   st, x, tab, k_sh, k_sc, it, out, rm, hprev_off, d, err));
   count_launches(1);
   return cudaSuccess;
@@ -677,7 +677,7 @@ cudaError_t launch_rows_f32(const float* src, float* dst, const int* idx, int Db
 cudaError_t launch_scatter_bf16(const float* src, const Items& it, long long off,
                                 const RowMap& rm, int d, unsigned* err, cudaStream_t st) {
   if (rm.bound <= 0) return cudaSuccess;
-  RC_TRY(launch_k(scatter_bf16_kernel, dim3(row_grid(rm.bound, RW_WARPS, 4)), dim3(RW_WARPS * 32),
+  RC_TRY(launch_k(scatter_bf16_kernel, dim3(row_grid(rm.bound, RW_WARPS, 1)), dim3(RW_WARPS * 32),
                   0, st, src, it, off, rm, d, err));
   count_launches(1);
   return cudaSuccess;
