@@ -115,6 +115,19 @@ def cross_attention(x, tk, tv, Lw, heads):
     return linear(multihead_attention(q, tk, tv, heads), Lw["W_xo"], Lw["b_xo"])
 
 
+def cross_attention_maps(x, tk, Lw, heads):
+    """The cross-attention matrices of one block, one per head (Section 3.2:
+    A in R^{N x M} links image tokens to text tokens): softmax over the M text
+    tokens of q'_h k_h^T / sqrt(dh), q' = x W_xq^T + b.  Returns [heads][N][M]."""
+    q = linear(x, Lw["W_xq"], Lw["b_xq"])
+    dh = q.shape[1] // heads
+    out = np.empty((heads, q.shape[0], tk.shape[0]))
+    for h in range(heads):
+        c = slice(h * dh, (h + 1) * dh)
+        out[h] = softmax((q[:, c] @ tk[:, c].T) / math.sqrt(dh))
+    return out
+
+
 def mlp_branch(x, Lw, shift, scale):
     a = modulate(layer_norm(x), shift, scale)
     return linear(gelu_tanh(linear(a, Lw["W_1"], Lw["b_1"])), Lw["W_2"], Lw["b_2"])
@@ -128,16 +141,18 @@ def qkv_rows(x, Lw, shift, scale):
 
 
 # ---------------------------------------------------------------- the blocks
-def dense_block(x, Lw, m6, tkv, heads):
+def dense_block(x, Lw, m6, tkv, heads, want_maps=False):
     """Full recompute of one DiT block over all N tokens (the backbone block,
-    Section 4.1 reading).  Returns (x_out, K, V), K/V post-bias [N][hidden]."""
+    Section 4.1 reading).  Returns (x_out, K, V), K/V post-bias [N][hidden],
+    and with want_maps also the block's cross-attention matrices [heads][N][M]."""
     sh1, sc1, g1, sh2, sc2, g2 = split6(m6)
     q, k, v = qkv_rows(x, Lw, sh1, sc1)
     o = multihead_attention(q, k, v, heads)
     x = x + g1 * linear(o, Lw["W_o"], Lw["b_o"])
+    maps = cross_attention_maps(x, tkv[0], Lw, heads) if want_maps else None
     x = x + cross_attention(x, tkv[0], tkv[1], Lw, heads)
     x = x + g2 * mlp_branch(x, Lw, sh2, sc2)
-    return x, k, v
+    return (x, k, v, maps) if want_maps else (x, k, v)
 
 
 def region_block(x_dirty, idx, cache, Lw, m6, tkv, heads):
@@ -299,6 +314,31 @@ def step(G, layers, pos, latent, t, mode, idx, cache_t, tkv_layers, t_values, al
     eps = final_layer(H_last, temb, G, grid_h, grid_w, patch, in_ch)
     x_next = ddim_update(latent, eps, float(alpha_bar[t]), float(alpha_bar[t + 1]))
     return x_next, eps, new_cache
+
+
+def step_capture(G, layers, pos, latent, t, cache_t, tkv_layers, t_values, alpha_bar, heads,
+                 grid_h, grid_w, patch, in_ch, delta_ids, M):
+    """A DENSE step that also returns the localisation scores of Section 3.2:
+    for each delta (new or modified) text token j, its cross-attention scores
+    aggregated over heads and layers, a_j = mean_{l,h} A^{l,h}[:, j].
+    Returns (latent_next, eps, cache_t_new, scores [N][M]) with the delta
+    columns filled and every other column zero (the layout the localisation
+    takes with S = 1)."""
+    N = grid_h * grid_w
+    temb = t_embed(t_values[t], G)
+    tb = t_block(temb, G)
+    new_cache = []
+    scores = np.zeros((N, M))
+    ids = np.asarray(delta_ids, dtype=np.int64)
+    x = patch_embed(latent, np.arange(N), G, pos, patch)
+    for l, Lw in enumerate(layers):
+        x, K, V, maps = dense_block(x, Lw, Lw["table"] + tb, tkv_layers[l], heads, want_maps=True)
+        new_cache.append({"H": x.copy(), "K": K, "V": V})
+        scores[:, ids] += maps[:, :, ids].sum(axis=0)
+    scores[:, ids] /= len(layers) * heads
+    eps = final_layer(new_cache[-1]["H"], temb, G, grid_h, grid_w, patch, in_ch)
+    x_next = ddim_update(latent, eps, float(alpha_bar[t]), float(alpha_bar[t + 1]))
+    return x_next, eps, new_cache, scores
 
 
 # ------------------------------------------------------------------ schedules
