@@ -231,6 +231,18 @@ class Workload:
             self.latent.copy_(self.latent0)
         self.R.rc_step_dense(self.model.ctx, self.model.cache, 0, self.latent, t)
 
+    def step_capture(self, i):
+        """A DENSE step that also captures the localisation scores of the
+        headline mask's delta tokens (the first step of an editing turn)."""
+        t = i % self.d.timesteps
+        if t == 0:
+            self.latent.copy_(self.latent0)
+        if not hasattr(self, "cap_scores"):
+            self.cap_scores = torch.empty(self.d.tokens, self.d.text_len, device=self.dev)
+        ids = self.scores[HEADLINE][1]
+        self.R.rc_step_capture(self.model.ctx, self.model.cache, 0, self.latent, t, ids,
+                               self.cap_scores)
+
 
 def timed(fn, K, W, world):
     for i in range(W):
@@ -303,6 +315,8 @@ def run_ours(args, world, rank, local):
         dirty[f"{f:.2f}"] = int(wl.cnt.item())
     m = timed(wl.step_dense, max(2, K // 2), min(W, 3), world)
     dense = max(2, K // 2) * world / (max_over_ranks(m, world) / 1e3)
+    m = timed(wl.step_capture, max(2, K // 2), min(W, 3), world)
+    capture = max(2, K // 2) * world / (max_over_ranks(m, world) / 1e3)
     R.rc_sync(wl.model.ctx)
 
     # end to end through the C ABI with host buffers: per step the score map
@@ -382,6 +396,7 @@ def run_ours(args, world, rank, local):
                    "l2": L2_NOTE, "step": "rc_localize_mask + rc_step(SPARSE)"},
         "sweep_steps_per_s": sweep, "sweep_dirty_tokens": dirty,
         "dense_steps_per_s": round(dense, 3),
+        "dense_capture_steps_per_s": round(capture, 3),
         "speedup_vs_dense": {k: round(v / dense, 3) for k, v in sweep.items()},
         "roofline": roofline, "roofline_attention": roof_att,
         "e2e": e2e, "gpu_launches": int(launches), "clocks": clk,

@@ -285,6 +285,21 @@ typedef struct rc_batch_item {
 rc_status rc_step_batched(rc_ctx* ctx, rc_cache* cache, const rc_batch_item* items, int n_items,
                           rc_stream stream);
 
+/* A DENSE step (as rc_step with mode DENSE) that also produces the
+ * localisation scores of Section 3.2 for the next sparse steps: for each of
+ * the n_delta (1..8) newly introduced or modified text tokens j in
+ * delta_ids_host (host array, values in [0, text_len)), the cross-attention
+ * probabilities of j, aggregated (averaged) over the heads and layers of
+ * the step:  scores[i][j] = mean_{l,h} softmax_j'(q'_{l,h,i} k_{l,h,j'} /
+ * sqrt(head_dim))[j], for every image token i.
+ *   scores  device f32 [N][text_len] (caller-owned, 16-B aligned): zeroed,
+ *           then the delta columns written; it is the [S = 1][N][M] score map
+ *           rc_localize_mask takes.
+ * Errors: as rc_step; RC_ERR_INVALID_ARG for bad ids or n_delta. */
+rc_status rc_step_capture(rc_ctx* ctx, rc_cache* cache, int session, float* latent, int t,
+                          const int32_t* delta_ids_host, int n_delta, float* scores,
+                          rc_stream stream);
+
 /* Full-recompute baseline: rc_step with mode DENSE. */
 rc_status rc_step_dense(rc_ctx* ctx, rc_cache* cache, int session, float* latent, int t,
                         rc_stream stream);

@@ -198,7 +198,8 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
 attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmQt,
                const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmKt,
                const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnItems ai, int Nk, bf16* __restrict__ O, int ldo,
-               int heads, RowMap rm, float scale_log2, unsigned* err, float* __restrict__ part) {
+               int heads, RowMap rm, float scale_log2, unsigned* err, float* __restrict__ part,
+               const __grid_constant__ AttnCapture cap) {
   using C = ACfg<DH>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -376,6 +377,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
       const int qt = pair % sc.qtiles, h = pair / sc.qtiles;
       const int n = kb1 - kb0;
       float m = -INFINITY, l = 0.f;
+      float cap_s[8];  // scaled scores of the captured key columns
+#pragma unroll
+      for (int q = 0; q < 8; ++q) cap_s[q] = -INFINITY;
       for (int j = 0; j < n; ++j, ++g) {
         if (!mbar_wait_warp(s_full + 8 * (g & 1), (g >> 1) & 1, abort_flag)) goto timeout;
         tc_fence_after();
@@ -384,6 +388,15 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         for (int i = 0; i < BKV / 16; ++i)
           tmem_ld16_nowait(tS0 + uint32_t(BKV) * uint32_t(g & 1) + lane_off + 16u * i, r + 16 * i);
         tmem_wait_ld();
+        if (cap.n) {  // (warp-uniform) the captured columns that fall in this block
+#pragma unroll
+          for (int q = 0; q < 8; ++q)
+            if (q < cap.n && cap.id[q] / BKV == kb0 + j)
+              cap_s[q] = __uint_as_float(tmem_ld1_nowait(tS0 + uint32_t(BKV) * uint32_t(g & 1) +
+                                                         lane_off + uint32_t(cap.id[q] % BKV))) *
+                         scale_log2;
+          tmem_wait_ld();
+        }
         tc_fence_before();
         mbar_arrive(s_free + 8 * (g & 1));
         // raw scores: the running max m is kept in scaled base-2 units; the
@@ -480,6 +493,15 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
       if (slot < 0) {
         const TileLoc tl = locate_tile(rm, ai.n, D, qt);
         const int qrow = tl.row0 + row;
+        if (cap.n && row < tl.rows) {
+          const int tok = rm.tok ? __ldg(rm.tok + qrow) : qrow;
+          const float inv_l = l > 0.f ? 1.f / l : 0.f;
+#pragma unroll
+          for (int q = 0; q < 8; ++q)
+            if (q < cap.n)
+              atomicAdd(cap.out + size_t(tok) * cap.ldo + cap.id[q],
+                        cap.w * ex2_ftz(cap_s[q] - m) * inv_l);
+        }
         if (row < tl.rows) {
           const float inv = l > 0.f ? 1.f / l : 0.f;
           uint4* dst = reinterpret_cast<uint4*>(O + size_t(qrow) * ldo + h * DH);
@@ -720,7 +742,7 @@ size_t attention_split_floats(int Nmax, int heads, int dh) {
 cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* V, int ldkv,
                              int kv_rows, const AttnItems& ai, int Nk, bf16* O, int ldo, int heads,
                              int dh, const RowMap& rm, unsigned* err, const AttnScratch& as,
-                             cudaStream_t st) {
+                             cudaStream_t st, const AttnCapture* capture) {
   if (rm.bound <= 0) return cudaSuccess;
   if (dh != 72 && dh != 64) return cudaErrorInvalidValue;
   if (ai.n < 1 || ai.n > MAX_ITEMS || (ai.n > 1 && !rm.meta)) return cudaErrorInvalidValue;
@@ -737,6 +759,16 @@ cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* 
   RC_TRY(head_map(Q, rm.bound, ldq, heads, dh, 16, BQ, &tqt));
   RC_TRY(head_map(K, kv_rows, ldkv, heads, dh, 16, BKV, &tkt));
   const float scale_log2 = float(1.4426950408889634 / sqrt(double(dh)));
+  AttnCapture cap{};
+  if (capture && capture->n > 0) {
+    // every key must sit in the one unit of its (query tile, head)
+    if (capture->n > 8 || !capture->out || (Nk + BKV - 1) / BKV >= 2 * MIN_KB_PER_SPLIT)
+      return cudaErrorInvalidValue;
+    for (int q = 0; q < capture->n; ++q)
+      if (capture->id[q] < 0 || capture->id[q] >= Nk || capture->id[q] >= capture->ldo)
+        return cudaErrorInvalidValue;
+    cap = *capture;
+  }
   const int grid = CTAS_PER_SM * sms;
   {
     const unsigned long long tiles = (rm.bound + BQ - 1) / BQ + ai.n - 1;
@@ -746,10 +778,10 @@ cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* 
   if (as.part_floats < size_t(2) * grid * BQ * PART_STRIDE) return cudaErrorInvalidValue;
   if (dh == 72)
     RC_TRY(launch_k(attn_tc_kernel<72>, dim3(grid), dim3(THREADS), ACfg<72>::SMEM, st, tq, tqt,
-                    tk, tkt, tv, ai, Nk, O, ldo, heads, rm, scale_log2, err, as.part));
+                    tk, tkt, tv, ai, Nk, O, ldo, heads, rm, scale_log2, err, as.part, cap));
   else
     RC_TRY(launch_k(attn_tc_kernel<64>, dim3(grid), dim3(THREADS), ACfg<64>::SMEM, st, tq, tqt,
-                    tk, tkt, tv, ai, Nk, O, ldo, heads, rm, scale_log2, err, as.part));
+                    tk, tkt, tv, ai, Nk, O, ldo, heads, rm, scale_log2, err, as.part, cap));
   count_launches(1);
   // stream-K (and so partial pieces) only with at least 2 MIN_KB_PER_SPLIT key blocks
   if ((Nk + BKV - 1) / BKV >= 2 * MIN_KB_PER_SPLIT) {

@@ -152,6 +152,19 @@ struct AttnItems {
   int vrow[MAX_ITEMS];
 };
 
+// Capture of attention probabilities (the localisation scores of Section
+// 3.2): for each listed key column id[q], out[tok(r)][id[q]] += w * P[r][id[q]]
+// over every head of the launch (P the softmax probability of that key for
+// query row r).  Needs all keys in one unit per (query tile, head), i.e. the
+// short text cross-attention.
+struct AttnCapture {
+  int n;         // listed columns, 0 .. 8 (0: no capture)
+  int id[8];
+  float* out;    // [tokens][ldo]
+  int ldo;
+  float w;
+};
+
 // O[r][h*dh..] = softmax(Q_r K_i^T / sqrt(dh)) V_i per head over the Nk keys of
 // row r's item i.  Q and O are compact rows (rm); K / V are row-major with row
 // stride ldkv and kv_rows rows in all.  Keys beyond Nk are masked, but their
@@ -159,6 +172,6 @@ struct AttnItems {
 cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* V, int ldkv,
                              int kv_rows, const AttnItems& ai, int Nk, bf16* O, int ldo, int heads,
                              int dh, const RowMap& rm, unsigned* err, const AttnScratch& as,
-                             cudaStream_t st);
+                             cudaStream_t st, const AttnCapture* cap = nullptr);
 
 }  // namespace rc

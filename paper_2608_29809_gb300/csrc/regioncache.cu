@@ -210,7 +210,8 @@ rc::AttnItems text_kv_rows(const rc_cache* k, const StepItems& si, int l) {
 // the block input (the previous block's merged output H^l) is also written to
 // the cache slice at that element offset.
 rc_status run_block(rc_ctx* c, rc_cache* k, int l, const rc::RowMap& rm, const StepItems& si,
-                    const float* tab, long long hprev_off, cudaStream_t st) {
+                    const float* tab, long long hprev_off, cudaStream_t st,
+                    const rc::AttnCapture* cap = nullptr) {
   const int d = c->d, F = c->F, N = c->N;
   const rc_layer_weights& w = c->lw[l];
   const size_t Nd = size_t(N) * d;
@@ -289,7 +290,7 @@ rc_status run_block(rc_ctx* c, rc_cache* k, int l, const rc::RowMap& rm, const S
     Probe pr(c, RC_PROBE_ATTENTION, st);
     RC_CUDA(rc::launch_attention(c->q, d, k->text, k->text + d, 2 * d,
                                  k->sessions * c->L * c->M, text_kv_rows(k, si, l), c->M, c->ob,
-                                 d, c->dims.heads, c->dh, rm, c->err, c->as, st),
+                                 d, c->dims.heads, c->dh, rm, c->err, c->as, st, cap),
             "attention(cross)");
   }
   // x += o' W_xo^T + b (no gate)
@@ -633,9 +634,10 @@ rc_status rc_block_forward_region(rc_ctx* c, rc_cache* k, int s, int l, int t, f
   return RC_OK;
 }
 
-// Denoising steps of n items (validated by the callers).
+// Denoising steps of n items (validated by the callers); cap (DENSE single
+// item only) captures cross-attention probabilities of listed text tokens.
 static rc_status step_items(rc_ctx* c, rc_cache* k, const rc_batch_item* items, int n,
-                            cudaStream_t st) {
+                            cudaStream_t st, const rc::AttnCapture* cap = nullptr) {
   const rc_global_weights& g = c->gw;
   const int d = c->d, N = c->N;
   const size_t Nd = size_t(N) * d;
@@ -682,7 +684,7 @@ static rc_status step_items(rc_ctx* c, rc_cache* k, const rc_batch_item* items, 
             "patch_embed");
     for (int l = 0; l < c->L; ++l) {
       rc_status r = run_block(c, k, l, rm, si, c->lw[l].table,
-                              l > 0 ? (long long)(size_t(l - 1) * 3) * Nd : -1, st);
+                              l > 0 ? (long long)(size_t(l - 1) * 3) * Nd : -1, st, cap);
       if (r) return r;
     }
     RC_CUDA(rc::launch_scatter_bf16(c->xf, si.its, (long long)(size_t(c->L - 1) * 3) * Nd, rm, d,
@@ -742,6 +744,34 @@ rc_status rc_step_batched(rc_ctx* c, rc_cache* k, const rc_batch_item* items, in
                     items[i].session, items[i].t);
   }
   return step_items(c, k, items, n, static_cast<cudaStream_t>(stream));
+}
+
+rc_status rc_step_capture(rc_ctx* c, rc_cache* k, int s, float* latent, int t,
+                          const int32_t* delta_ids_host, int n_delta, float* scores,
+                          rc_stream stream) {
+  if (!c || !k || !latent || !delta_ids_host || !scores)
+    return fail(RC_ERR_INVALID_ARG, "rc_step_capture: null argument");
+  if (k->ctx != c) return fail(RC_ERR_INVALID_ARG, "cache belongs to another context");
+  if (t < 0 || t >= c->T) return fail(RC_ERR_INVALID_ARG, "t %d outside [0, %d)", t, c->T);
+  if (n_delta < 1 || n_delta > 8)
+    return fail(RC_ERR_INVALID_ARG, "n_delta %d not in 1..8", n_delta);
+  if (!aligned16(scores)) return fail(RC_ERR_INVALID_ARG, "scores not 16-B aligned");
+  rc::AttnCapture cap{};
+  cap.n = n_delta;
+  for (int q = 0; q < n_delta; ++q) {
+    if (delta_ids_host[q] < 0 || delta_ids_host[q] >= c->M)
+      return fail(RC_ERR_INVALID_ARG, "delta id %d outside [0, %d)", delta_ids_host[q], c->M);
+    cap.id[q] = delta_ids_host[q];
+  }
+  cap.out = scores;
+  cap.ldo = c->M;
+  cap.w = 1.f / float(c->L * c->dims.heads);
+  rc_batch_item it{s, latent, t, RC_MODE_DENSE, nullptr, 0, nullptr};
+  rc_status r = check_item(c, k, it);
+  if (r) return r;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  RC_CUDA(cudaMemsetAsync(scores, 0, sizeof(float) * size_t(c->N) * c->M, st), "scores reset");
+  return step_items(c, k, &it, 1, st, &cap);
 }
 
 rc_status rc_step_dense(rc_ctx* c, rc_cache* k, int s, float* latent, int t, rc_stream stream) {

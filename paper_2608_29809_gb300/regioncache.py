@@ -82,6 +82,7 @@ def load_library(path: str = LIB_PATH) -> C.CDLL:
         "rc_block_forward_region": (I, [P, P, I, I, I, P, P, I, P, P, P]),
         "rc_step": (I, [P, P, I, P, I, P, P, I, P, P]),
         "rc_step_batched": (I, [P, P, C.POINTER(rc_batch_item), I, P]),
+        "rc_step_capture": (I, [P, P, I, P, I, P, I, P, P]),
         "rc_step_dense": (I, [P, P, I, P, I, P]),
         "rc_linear": (I, [P, P, P, P, P, I, I, I, P]),
         "rc_attention": (I, [P, P, I, P, P, I, I, I, P, I, P]),
@@ -223,6 +224,12 @@ def rc_step_batched(ctx, cache, items, stream=None):
                                _ptr(it.get("dirty_idx")), it.get("D", 0),
                                _ptr(it.get("dirty_count")))
     _check(_lib.rc_step_batched(ctx, cache, arr, len(items), _stream(stream)))
+
+
+def rc_step_capture(ctx, cache, session, latent, t, delta_ids, scores, stream=None):
+    ids = np.ascontiguousarray(delta_ids, np.int32)
+    _check(_lib.rc_step_capture(ctx, cache, session, _ptr(latent), t, ids.ctypes.data, len(ids),
+                                _ptr(scores), _stream(stream)))
 
 
 def rc_step_dense(ctx, cache, session, latent, t, stream=None):
