@@ -300,6 +300,18 @@ rc_status rc_step_capture(rc_ctx* ctx, rc_cache* cache, int session, float* late
                           const int32_t* delta_ids_host, int n_delta, float* scores,
                           rc_stream stream);
 
+/* Semantic-aware adaptive reuse scheduling (Section 3.3), host-only.
+ * rc_prompt_similarity: Eq. 1, s = cos(e(tau-), e(tau+)) of two token
+ *   embeddings (host arrays of dim floats), accumulated in double.
+ * rc_reuse_schedule: Eq. 2, T_reuse = T if s >= tau_s else floor(rho T), and
+ *   the per-step modes of an edited region for rc_step: RC_MODE_REUSE for
+ *   t < T_reuse, RC_MODE_SPARSE after (modes_out: host array of T).  The
+ *   paper sets rho = 0.2.
+ * Errors: RC_ERR_INVALID_ARG (null, dim or T <= 0, zero embedding, rho
+ * outside [0, 1], NaN). */
+rc_status rc_prompt_similarity(const float* e_minus, const float* e_plus, int dim, float* s_out);
+rc_status rc_reuse_schedule(float s, float tau_s, float rho, int T, uint8_t* modes_out);
+
 /* Full-recompute baseline: rc_step with mode DENSE. */
 rc_status rc_step_dense(rc_ctx* ctx, rc_cache* cache, int session, float* latent, int t,
                         rc_stream stream);

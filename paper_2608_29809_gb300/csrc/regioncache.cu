@@ -6,6 +6,7 @@
 #include <string.h>
 
 #include <atomic>
+#include <cmath>
 #include <new>
 #include <string>
 #include <vector>
@@ -772,6 +773,30 @@ rc_status rc_step_capture(rc_ctx* c, rc_cache* k, int s, float* latent, int t,
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   RC_CUDA(cudaMemsetAsync(scores, 0, sizeof(float) * size_t(c->N) * c->M, st), "scores reset");
   return step_items(c, k, &it, 1, st, &cap);
+}
+
+rc_status rc_prompt_similarity(const float* e_minus, const float* e_plus, int dim, float* s_out) {
+  if (!e_minus || !e_plus || !s_out || dim <= 0)
+    return fail(RC_ERR_INVALID_ARG, "rc_prompt_similarity: null argument or dim <= 0");
+  double dot = 0.0, na = 0.0, nb = 0.0;
+  for (int i = 0; i < dim; ++i) {
+    dot += double(e_minus[i]) * e_plus[i];
+    na += double(e_minus[i]) * e_minus[i];
+    nb += double(e_plus[i]) * e_plus[i];
+  }
+  if (!(na > 0.0) || !(nb > 0.0))
+    return fail(RC_ERR_INVALID_ARG, "rc_prompt_similarity: zero embedding");
+  *s_out = float(dot / (std::sqrt(na) * std::sqrt(nb)));
+  return RC_OK;
+}
+
+rc_status rc_reuse_schedule(float s, float tau_s, float rho, int T, uint8_t* modes_out) {
+  if (!modes_out || T <= 0) return fail(RC_ERR_INVALID_ARG, "rc_reuse_schedule: T or output");
+  if (!(rho >= 0.f && rho <= 1.f) || s != s || tau_s != tau_s)
+    return fail(RC_ERR_INVALID_ARG, "rc_reuse_schedule: rho outside [0, 1] or NaN input");
+  const int t_reuse = s >= tau_s ? T : int(std::floor(double(rho) * T));
+  for (int t = 0; t < T; ++t) modes_out[t] = uint8_t(t < t_reuse ? RC_MODE_REUSE : RC_MODE_SPARSE);
+  return RC_OK;
 }
 
 rc_status rc_step_dense(rc_ctx* c, rc_cache* k, int s, float* latent, int t, rc_stream stream) {

@@ -83,6 +83,8 @@ def load_library(path: str = LIB_PATH) -> C.CDLL:
         "rc_step": (I, [P, P, I, P, I, P, P, I, P, P]),
         "rc_step_batched": (I, [P, P, C.POINTER(rc_batch_item), I, P]),
         "rc_step_capture": (I, [P, P, I, P, I, P, I, P, P]),
+        "rc_prompt_similarity": (I, [P, P, I, C.POINTER(F)]),
+        "rc_reuse_schedule": (I, [F, F, F, I, P]),
         "rc_step_dense": (I, [P, P, I, P, I, P]),
         "rc_linear": (I, [P, P, P, P, P, I, I, I, P]),
         "rc_attention": (I, [P, P, I, P, P, I, I, I, P, I, P]),
@@ -230,6 +232,22 @@ def rc_step_capture(ctx, cache, session, latent, t, delta_ids, scores, stream=No
     ids = np.ascontiguousarray(delta_ids, np.int32)
     _check(_lib.rc_step_capture(ctx, cache, session, _ptr(latent), t, ids.ctypes.data, len(ids),
                                 _ptr(scores), _stream(stream)))
+
+
+def rc_prompt_similarity(e_minus, e_plus):
+    a = np.ascontiguousarray(e_minus, np.float32)
+    b = np.ascontiguousarray(e_plus, np.float32)
+    if a.shape != b.shape:
+        raise ValueError("embeddings of different sizes")
+    out = C.c_float()
+    _check(_lib.rc_prompt_similarity(a.ctypes.data, b.ctypes.data, a.size, C.byref(out)))
+    return out.value
+
+
+def rc_reuse_schedule(s, tau_s, T, rho=0.2):
+    modes = np.zeros(T, np.uint8)
+    _check(_lib.rc_reuse_schedule(s, tau_s, rho, T, modes.ctypes.data))
+    return modes
 
 
 def rc_step_dense(ctx, cache, session, latent, t, stream=None):

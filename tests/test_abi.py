@@ -75,3 +75,36 @@ def test_null_handles_are_rejected(R):
     assert lib.rc_block_forward_region(None, None, 0, 0, 0, None, None, 0, None, None, None) == 1
     assert lib.rc_sync(None, None) == 1
     assert lib.rc_linear(None, None, None, None, None, 1, 128, 64, None) == 1
+
+
+# --------------------------------------------- Eq. 1 / Eq. 2 (host-only entry points)
+def test_reuse_schedule_matches_eq2_golden_and_oracle(R):
+    import os
+    import oracle as O
+    golden = os.path.join(os.path.dirname(__file__), "golden", "eq2_reuse_cutoff.txt")
+    for ln in open(golden):
+        if ln.startswith("#") or not ln.strip():
+            continue
+        T, s, tau, tr = ln.split()
+        modes = R.rc_reuse_schedule(float(s), float(tau), int(T))
+        assert int((modes == R.RC_MODE_REUSE).sum()) == int(tr)
+        assert np.array_equal(modes, O.schedule_eq2(float(s), float(tau), int(T)))
+        assert np.all(modes[:int(tr)] == R.RC_MODE_REUSE) and np.all(modes[int(tr):] == R.RC_MODE_SPARSE)
+    with pytest.raises(R.RCError):
+        R.rc_reuse_schedule(0.1, 0.5, 0)
+    with pytest.raises(R.RCError):
+        R.rc_reuse_schedule(0.1, 0.5, 20, rho=1.5)
+
+
+def test_prompt_similarity_eq1(R):
+    import oracle as O
+    g = np.random.default_rng(5)
+    for dim in (1, 7, 4096):
+        a = g.standard_normal(dim).astype(np.float32)
+        b = g.standard_normal(dim).astype(np.float32)
+        s = R.rc_prompt_similarity(a, b)
+        assert abs(s - O.cosine_similarity(a, b)) <= 1e-6
+        assert abs(R.rc_prompt_similarity(a, a) - 1.0) <= 1e-6
+        assert abs(R.rc_prompt_similarity(a, -a) + 1.0) <= 1e-6
+    with pytest.raises(R.RCError):
+        R.rc_prompt_similarity(np.zeros(4, np.float32), np.ones(4, np.float32))
