@@ -244,6 +244,39 @@ class Workload:
                                self.cap_scores)
 
 
+    def host_tier_rate(self, K, W, world, seed=SEED):
+        R, d, dev = self.R, self.d, self.dev
+        hc = R.rc_cache_create_host(self.model.ctx, 1)
+        try:
+            for t in range(d.timesteps):
+                for l in range(d.layers):
+                    H, K_, V = synth.make_cache_slice(d, seed, 0, l, t, device=dev)
+                    R.rc_cache_fill(hc, 0, l, t, H, K_, V)
+            R.rc_set_text(self.model.ctx, hc, 0, self.text)
+            torch.cuda.synchronize()
+
+            def step(i):
+                t = i % d.timesteps
+                if t == 0:
+                    self.latent.copy_(self.latent0)
+                self.localize(HEADLINE)
+                R.rc_step(self.model.ctx, hc, 0, self.latent, t, self.sparse, self.idx, -1,
+                          self.cnt)
+
+            m = timed(step, K, W, world)
+            R.rc_sync(self.model.ctx)
+        finally:
+            R.rc_cache_destroy(hc)
+        slot = d.tokens * d.hidden * 2
+        h2d = (2 * (d.layers - 1) + 3) * slot
+        return {"steps_per_s": round(K * world / (max_over_ranks(m, world) / 1e3), 3),
+                "pool_bytes": d.timesteps * d.layers * 3 * slot,
+                "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": 3 * int(self.cnt.item()) * d.hidden * 2 * d.layers,
+                "h2d_gbs_over_step": round(h2d / (m / K / 1e3) / 1e9, 1),
+                "step": "rc_localize_mask + rc_step(SPARSE) on rc_cache_create_host"}
+
+
 def timed(fn, K, W, world):
     for i in range(W):
         fn(i)
@@ -318,6 +351,12 @@ def run_ours(args, world, rank, local):
     m = timed(wl.step_capture, max(2, K // 2), min(W, 3), world)
     capture = max(2, K // 2) * world / (max_over_ranks(m, world) / 1e3)
     R.rc_sync(wl.model.ctx)
+
+    # the same headline steps on a host-tier cache (pinned host pool, each
+    # layer's K, V streamed into HBM windows while the previous layer runs)
+    host_tier = None
+    if not args.no_host_tier:
+        host_tier = wl.host_tier_rate(K, W, world)
 
     # end to end through the C ABI with host buffers: per step the score map
     # and the latent go host -> device, the updated latent comes back
@@ -397,6 +436,7 @@ def run_ours(args, world, rank, local):
         "sweep_steps_per_s": sweep, "sweep_dirty_tokens": dirty,
         "dense_steps_per_s": round(dense, 3),
         "dense_capture_steps_per_s": round(capture, 3),
+        "host_tier": host_tier,
         "speedup_vs_dense": {k: round(v / dense, 3) for k, v in sweep.items()},
         "roofline": roofline, "roofline_attention": roof_att,
         "e2e": e2e, "gpu_launches": int(launches), "clocks": clk,
@@ -511,6 +551,8 @@ def main():
     ap.add_argument("--cpu-layers", type=int, default=2)
     ap.add_argument("--quick", action="store_true",
                     help="headline only: no attention probe, sweep, dense, e2e or cpu baseline")
+    ap.add_argument("--no-host-tier", action="store_true",
+                    help="skip the host-tier cache measurement (a pinned host pool)")
     ap.add_argument("--resident-steps", type=int, default=20,
                     help="timesteps held in the cache (1 keeps a profiling run to ~2 GB)")
     args = ap.parse_args()

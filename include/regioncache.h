@@ -132,6 +132,19 @@ rc_status rc_set_schedule(rc_ctx* ctx, const float* t_values_host, const float* 
  * sessions * timesteps * layers * 3 * N * hidden * 2 bytes (15.85 GB for one
  * PixArt-alpha session at 4096 tokens and 20 steps). */
 rc_status rc_cache_create(rc_ctx* ctx, int sessions, rc_cache** out);
+
+/* The same pool in pinned, device-mapped host memory (Section 3.4, Pipelined
+ * Execution): for pools larger than HBM.  The text keys/values and two HBM
+ * windows of 3 * N * hidden bf16 stay on the device.  rc_step and
+ * rc_step_capture on such a cache load each layer's cached K, V (plus H for the
+ * last layer) into a window on a library-owned copy stream while the previous
+ * layer computes, then write the dirty rows' H, K, V back to host memory; the
+ * results equal those of a device-tier cache.  rc_step_batched takes one item
+ * and rc_block_forward_region is refused (RC_ERR_INVALID_ARG).  Steps on one
+ * host-tier cache must be issued from one host thread.  rc_cache_fill /
+ * rc_cache_read work as for a device-tier cache.  Errors: RC_ERR_OOM when the
+ * pinned allocation or a window fails. */
+rc_status rc_cache_create_host(rc_ctx* ctx, int sessions, rc_cache** out);
 void rc_cache_destroy(rc_cache* cache);
 
 /* Copies caller bf16 [N][hidden] device buffers into / out of the (session,

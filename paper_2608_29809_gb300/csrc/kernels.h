@@ -52,6 +52,11 @@ struct Items {
   const float* tb[MAX_ITEMS];  // modulation [6][d] of the item's timestep (null: none)
   float* latent[MAX_ITEMS];    // the item's latent (patch embedding input)
 };
+// Host-tier write-back of a layer: rows tok[r] of the HBM window [H,K,V][N][d]
+// go to the same rows of the host slice (device-mapped).
+cudaError_t launch_writeback(const bf16* win, bf16* host, const RowMap& rm, int d, unsigned* err,
+                             cudaStream_t st);
+
 // Builds tok / item / meta of a multi-item step.  Item i contributes cnt_i =
 // min(*count_i, bound_i) rows (count_i null: bound_i) taken from idx_i (null:
 // tokens 0 .. cnt_i - 1).

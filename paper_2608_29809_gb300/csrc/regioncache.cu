@@ -88,9 +88,24 @@ struct rc_ctx {
 struct rc_cache {
   rc_ctx* ctx;
   int sessions;
-  bf16* base = nullptr;  // [sessions][T][L][3 (H,K,V)][N][d]
-  bf16* text = nullptr;  // [sessions][L][M][2d]
+  bf16* base = nullptr;  // [sessions][T][L][3 (H,K,V)][N][d] (device-addressable)
+  bf16* text = nullptr;  // [sessions][L][M][2d], always in HBM
   std::vector<char> text_set;
+  // host tier (Section 3.4, Pipelined Execution): the slots live in pinned,
+  // mapped host memory (base is its device address).  A step runs layer l on
+  // HBM window l % 3: the copy stream loads layer l + 2's cached K, V into
+  // its window while layer l computes, and the write-back stream sends layer
+  // l - 1's dirty H, K, V rows back to host memory
+  static constexpr int WINDOWS = 3;
+  bool host_tier = false;
+  void* host_mem = nullptr;
+  bf16* window = nullptr;  // [WINDOWS][3][N][d]
+  cudaStream_t copy_st = nullptr, wb_st = nullptr;
+  cudaEvent_t begin = nullptr;                // step start on the compute stream
+  cudaEvent_t h_ready = nullptr;              // a layer's H rows are in its window
+  cudaEvent_t wb_done = nullptr;              // the last write-back of a step
+  cudaEvent_t loaded[WINDOWS] = {};           // window filled
+  cudaEvent_t consumed[WINDOWS] = {};         // window no longer read
 
   size_t slot_elems() const { return size_t(ctx->N) * ctx->d; }
   // index of the [N][d] slot (s, l, t, which) in units of slots
@@ -185,11 +200,17 @@ struct StepItems {
   rc::Items its{};
   int session[rc::MAX_ITEMS] = {};
   int t[rc::MAX_ITEMS] = {};
+  const bf16* win = nullptr;  // host tier: the layer's HBM window [H,K,V][N][d] (one item)
 };
 
 rc::AttnItems self_kv(const rc_cache* k, const StepItems& si, int l) {
   rc::AttnItems ai{};
   ai.n = si.its.n;
+  if (si.win) {
+    ai.krow[0] = k->ctx->N;
+    ai.vrow[0] = 2 * k->ctx->N;
+    return ai;
+  }
   for (int i = 0; i < ai.n; ++i) {
     ai.krow[i] = int(k->slot_index(si.session[i], l, si.t[i], 1) * k->ctx->N);
     ai.vrow[i] = int(k->slot_index(si.session[i], l, si.t[i], 2) * k->ctx->N);
@@ -209,10 +230,11 @@ rc::AttnItems text_kv_rows(const rc_cache* k, const StepItems& si, int l) {
 // Region-Level Sparse Attention; Section 3.4, Kernel Fusing).  The modulation
 // vector of a row is tab (+ the row item's tb), each [6][d].  hprev_off >= 0:
 // the block input (the previous block's merged output H^l) is also written to
-// the cache slice at that element offset.
+// the cache slice at that element offset, and h_stored (if any) is recorded
+// on st once it is there.
 rc_status run_block(rc_ctx* c, rc_cache* k, int l, const rc::RowMap& rm, const StepItems& si,
                     const float* tab, long long hprev_off, cudaStream_t st,
-                    const rc::AttnCapture* cap = nullptr) {
+                    const rc::AttnCapture* cap = nullptr, cudaEvent_t h_stored = nullptr) {
   const int d = c->d, F = c->F, N = c->N;
   const rc_layer_weights& w = c->lw[l];
   const size_t Nd = size_t(N) * d;
@@ -221,6 +243,7 @@ rc_status run_block(rc_ctx* c, rc_cache* k, int l, const rc::RowMap& rm, const S
   // block's output H^l of the dirty rows, written to their cache rows here
   RC_CUDA(rc::launch_ln_mod(c->xf, tab, 0, 1, si.its, c->xb, rm, hprev_off, d, c->err, st),
           "ln_mod(msa)");
+  if (h_stored) RC_CUDA(cudaEventRecord(h_stored, st), "H stored");
   // [q | k | v] = x_hat W_qkv^T + b; k, v rows go straight to cache rows tok[r]
   rc::GemmEpi e{};
   e.mode = rc::EPI_QKV;
@@ -244,9 +267,11 @@ rc_status run_block(rc_ctx* c, rc_cache* k, int l, const rc::RowMap& rm, const S
   // dirty queries over all N keys / values of each item's (session, l, t)
   {
     Probe pr(c, RC_PROBE_ATTENTION, st);
-    RC_CUDA(rc::launch_attention(c->q, d, k->base, k->base, d, int(k->total_rows()),
-                                 self_kv(k, si, l), N, c->ob, d, c->dims.heads, c->dh, rm,
-                                 c->err, c->as, st), "attention(self)");
+    const bf16* kv = si.win ? si.win : k->base;
+    const int kv_rows = si.win ? 3 * N : int(k->total_rows());
+    RC_CUDA(rc::launch_attention(c->q, d, kv, kv, d, kv_rows, self_kv(k, si, l), N, c->ob, d,
+                                 c->dims.heads, c->dh, rm, c->err, c->as, st),
+            "attention(self)");
   }
   // x += gate_msa (o W_o^T + b_o)
   auto gated = [&](const float* bias, int gate_k) {
@@ -493,9 +518,74 @@ rc_status rc_cache_create(rc_ctx* c, int sessions, rc_cache** out) {
 
 void rc_cache_destroy(rc_cache* k) {
   if (!k) return;
-  if (k->base) cudaFree(k->base);
+  if (k->host_tier) {
+    for (cudaStream_t q : {k->copy_st, k->wb_st})
+      if (q) cudaStreamSynchronize(q);
+    if (k->host_mem) cudaFreeHost(k->host_mem);
+    if (k->window) cudaFree(k->window);
+    for (cudaEvent_t e : {k->begin, k->h_ready, k->wb_done}) if (e) cudaEventDestroy(e);
+    for (int i = 0; i < rc_cache::WINDOWS; ++i) {
+      if (k->loaded[i]) cudaEventDestroy(k->loaded[i]);
+      if (k->consumed[i]) cudaEventDestroy(k->consumed[i]);
+    }
+    for (cudaStream_t q : {k->copy_st, k->wb_st})
+      if (q) cudaStreamDestroy(q);
+  } else if (k->base) {
+    cudaFree(k->base);
+  }
   if (k->text) cudaFree(k->text);
   delete k;
+}
+
+rc_status rc_cache_create_host(rc_ctx* c, int sessions, rc_cache** out) {
+  if (!c || !out) return fail(RC_ERR_INVALID_ARG, "rc_cache_create_host: null argument");
+  *out = nullptr;
+  if (sessions <= 0) return fail(RC_ERR_INVALID_ARG, "sessions = %d", sessions);
+  rc_cache* k = new (std::nothrow) rc_cache();
+  if (!k) return fail(RC_ERR_OOM, "host allocation");
+  k->ctx = c;
+  k->sessions = sessions;
+  k->text_set.assign(sessions, 0);
+  k->host_tier = true;
+  const size_t n = size_t(sessions) * c->T * c->L * 3 * k->slot_elems();
+  const size_t n_text = size_t(sessions) * c->L * c->M * 2 * c->d;
+  rc_status s = RC_OK;
+  if (cudaHostAlloc(&k->host_mem, n * sizeof(bf16), cudaHostAllocMapped | cudaHostAllocPortable) !=
+      cudaSuccess) {
+    cudaGetLastError();
+    k->host_mem = nullptr;
+    s = fail(RC_ERR_OOM, "pinned host cache of %zu bytes", n * sizeof(bf16));
+  }
+  void* dev = nullptr;
+  if (s == RC_OK && cudaHostGetDevicePointer(&dev, k->host_mem, 0) != cudaSuccess)
+    s = fail(RC_ERR_CUDA, "no device address for the host cache");
+  if (s == RC_OK) {
+    k->base = static_cast<bf16*>(dev);
+    memset(k->host_mem, 0, n * sizeof(bf16));
+    s = dalloc(&k->window, rc_cache::WINDOWS * 3 * k->slot_elems(), "cache window");
+  }
+  if (s == RC_OK) s = dalloc(&k->text, n_text, "text kv");
+  if (s == RC_OK &&
+      (cudaMemset(k->window, 0, rc_cache::WINDOWS * 3 * k->slot_elems() * sizeof(bf16)) !=
+           cudaSuccess ||
+       cudaMemset(k->text, 0, n_text * sizeof(bf16)) != cudaSuccess ||
+       cudaStreamCreateWithFlags(&k->copy_st, cudaStreamNonBlocking) != cudaSuccess ||
+       cudaStreamCreateWithFlags(&k->wb_st, cudaStreamNonBlocking) != cudaSuccess))
+    s = fail(RC_ERR_CUDA, "host cache set-up failed");
+  cudaEvent_t* evs[] = {&k->begin,       &k->h_ready,     &k->wb_done,     &k->loaded[0],
+                        &k->loaded[1],   &k->loaded[2],   &k->consumed[0], &k->consumed[1],
+                        &k->consumed[2]};
+  for (cudaEvent_t* e : evs)
+    if (s == RC_OK && cudaEventCreateWithFlags(e, cudaEventDisableTiming) != cudaSuccess)
+      s = fail(RC_ERR_CUDA, "host cache events");
+  if (s == RC_OK && cudaDeviceSynchronize() != cudaSuccess)
+    s = fail(RC_ERR_CUDA, "host cache set-up failed");
+  if (s != RC_OK) {
+    rc_cache_destroy(k);
+    return s;
+  }
+  *out = k;
+  return RC_OK;
 }
 
 static rc_status cache_copy(rc_cache* k, int s, int l, int t, void* H, void* K, void* V,
@@ -512,7 +602,7 @@ static rc_status cache_copy(rc_cache* k, int s, int l, int t, void* H, void* K, 
     bf16* slot = k->slot(s, l, t, w);
     RC_CUDA(cudaMemcpyAsync(fill ? static_cast<void*>(slot) : ps[w],
                             fill ? static_cast<const void*>(ps[w]) : slot, bytes,
-                            cudaMemcpyDeviceToDevice, st),
+                            cudaMemcpyDefault, st),
             "cache copy");
   }
   return RC_OK;
@@ -608,6 +698,8 @@ rc_status rc_block_forward_region(rc_ctx* c, rc_cache* k, int s, int l, int t, f
   if (!c || !k || !hidden || !mod6)
     return fail(RC_ERR_INVALID_ARG, "rc_block_forward_region: null argument");
   if (k->ctx != c) return fail(RC_ERR_INVALID_ARG, "cache belongs to another context");
+  if (k->host_tier)
+    return fail(RC_ERR_INVALID_ARG, "rc_block_forward_region needs a device-tier cache");
   rc_status r = check_session(k, s);
   if (r) return r;
   if (l < 0 || l >= c->L || t < 0 || t >= c->T)
@@ -635,8 +727,40 @@ rc_status rc_block_forward_region(rc_ctx* c, rc_cache* k, int s, int l, int t, f
   return RC_OK;
 }
 
+// Host tier: window l % 3 receives layer l's cached K, V of item (s, t) (and
+// H for the last layer, which the final layer reads over all tokens) on the
+// copy stream, once the window's previous readers are done.
+static rc_status host_load(rc_cache* k, int s, int t, int l) {
+  const size_t Nd = k->slot_elems();
+  const int first = l == k->ctx->L - 1 ? 0 : 1, w = l % rc_cache::WINDOWS;
+  RC_CUDA(cudaStreamWaitEvent(k->copy_st, k->consumed[w], 0), "window wait");
+  RC_CUDA(cudaMemcpyAsync(k->window + (size_t(w) * 3 + first) * Nd, k->slot(s, l, t, first),
+                          (3 - first) * Nd * sizeof(bf16), cudaMemcpyDefault, k->copy_st),
+          "window load");
+  RC_CUDA(cudaEventRecord(k->loaded[w], k->copy_st), "window event");
+  return RC_OK;
+}
+
+// Host tier: once layer l's H rows are in window l % 3 (h_ready, recorded on
+// st by the next block after its first LN, or here for the last layer), the
+// write-back stream sends its dirty H, K, V rows to the host slice.
+static rc_status host_writeback(rc_ctx* c, rc_cache* k, int s, int t, int l,
+                                const rc::RowMap& rm, cudaStream_t st, bool last) {
+  const int w = l % rc_cache::WINDOWS;
+  if (last) RC_CUDA(cudaEventRecord(k->h_ready, st), "write-back event");
+  RC_CUDA(cudaStreamWaitEvent(k->wb_st, k->h_ready, 0), "write-back wait");
+  RC_CUDA(rc::launch_writeback(k->window + size_t(w) * 3 * k->slot_elems(), k->slot(s, l, t, 0),
+                               rm, c->d, c->err, k->wb_st),
+          "write-back");
+  RC_CUDA(cudaEventRecord(k->consumed[w], k->wb_st), "window event");
+  if (last) RC_CUDA(cudaEventRecord(k->wb_done, k->wb_st), "write-back event");
+  return RC_OK;
+}
+
 // Denoising steps of n items (validated by the callers); cap (DENSE single
 // item only) captures cross-attention probabilities of listed text tokens.
+// On a host-tier cache (one item) the layers run on HBM windows while the
+// copy stream loads the layers ahead (Section 3.4, Pipelined Execution).
 static rc_status step_items(rc_ctx* c, rc_cache* k, const rc_batch_item* items, int n,
                             cudaStream_t st, const rc::AttnCapture* cap = nullptr) {
   const rc_global_weights& g = c->gw;
@@ -670,6 +794,19 @@ static rc_status step_items(rc_ctx* c, rc_cache* k, const rc_batch_item* items, 
                                c->temb + size_t(i) * d, c->tb + size_t(i) * 6 * d, st),
             "t_embed");
   }
+  const bool host = k->host_tier;
+  const int s0 = items[0].session, t0 = items[0].t, L = c->L;
+  const size_t wstride = 3 * Nd;  // elements per window
+  bf16* const win_last =
+      host ? k->window + size_t((L - 1) % rc_cache::WINDOWS) * wstride : nullptr;
+  if (host) {
+    if (n != 1) return fail(RC_ERR_INVALID_ARG, "a host-tier cache steps one item at a time");
+    RC_CUDA(cudaEventRecord(k->begin, st), "step event");
+    RC_CUDA(cudaStreamWaitEvent(k->copy_st, k->begin, 0), "step wait");
+    rc_status r = host_load(k, s0, t0, rows > 0 ? 0 : L - 1);
+    if (r == RC_OK && rows > 0 && L > 1) r = host_load(k, s0, t0, 1);
+    if (r) return r;
+  }
   if (rows > 0) {
     // compact rows: a single item uses its own index list; several items are
     // concatenated on the device (their counts may live there)
@@ -683,21 +820,56 @@ static rc_status step_items(rc_ctx* c, rc_cache* k, const rc_batch_item* items, 
                                    static_cast<const bf16*>(g.W_e), g.b_e, g.pos, si.its, rm,
                                    c->xf, d, c->err, st),
             "patch_embed");
-    for (int l = 0; l < c->L; ++l) {
-      rc_status r = run_block(c, k, l, rm, si, c->lw[l].table,
-                              l > 0 ? (long long)(size_t(l - 1) * 3) * Nd : -1, st, cap);
+    for (int l = 0; l < L; ++l) {
+      if (!host) {
+        rc_status r = run_block(c, k, l, rm, si, c->lw[l].table,
+                                l > 0 ? (long long)(size_t(l - 1) * 3) * Nd : -1, st, cap);
+        if (r) return r;
+        continue;
+      }
+      // the window stands in for the slice: its K, V rows take the QKV
+      // epilogue's writes and feed the self-attention, and the block's first
+      // LN stores its input (layer l - 1's output H) into window (l - 1) % 3,
+      // after which the write-back stream sends layer l - 1's rows home
+      const int w = l % rc_cache::WINDOWS, wp = (l + rc_cache::WINDOWS - 1) % rc_cache::WINDOWS;
+      bf16* win = k->window + size_t(w) * wstride;
+      si.win = win;
+      si.its.slice[0] = reinterpret_cast<bf16*>(reinterpret_cast<uintptr_t>(win) -
+                                                size_t(l) * wstride * sizeof(bf16));
+      const long long hprev =
+          l > 0 ? (long long)(size_t(wp) * wstride + size_t(l) * wstride) - (long long)(w * wstride)
+                : -1;
+      RC_CUDA(cudaStreamWaitEvent(st, k->loaded[w], 0), "window ready");
+      rc_status r = run_block(c, k, l, rm, si, c->lw[l].table, hprev, st, cap,
+                              l > 0 ? k->h_ready : nullptr);
+      if (r) return r;
+      if (l > 0 && (r = host_writeback(c, k, s0, t0, l - 1, rm, st, false))) return r;
+      if (l + 2 < L && (r = host_load(k, s0, t0, l + 2))) return r;
+    }
+    RC_CUDA(rc::launch_scatter_bf16(c->xf, si.its, (long long)(size_t(L - 1) * 3) * Nd, rm, d,
+                                    c->err, st), "H scatter");
+    if (host) {
+      rc_status r = host_writeback(c, k, s0, t0, L - 1, rm, st, true);
       if (r) return r;
     }
-    RC_CUDA(rc::launch_scatter_bf16(c->xf, si.its, (long long)(size_t(c->L - 1) * 3) * Nd, rm, d,
-                                    c->err, st), "H scatter");
+  } else if (host) {
+    RC_CUDA(cudaStreamWaitEvent(st, k->loaded[(L - 1) % rc_cache::WINDOWS], 0), "window ready");
   }
   for (int i = 0; i < n; ++i) {
     const rc_batch_item& it = items[i];
-    RC_CUDA(rc::launch_final_ddim(k->slot(it.session, c->L - 1, it.t, 0), c->temb + size_t(i) * d,
+    RC_CUDA(rc::launch_final_ddim(host ? win_last : k->slot(it.session, L - 1, it.t, 0),
+                                  c->temb + size_t(i) * d,
                                   g.table_f, static_cast<const bf16*>(g.W_f), g.b_f, it.latent,
                                   c->dims.grid_h, c->dims.grid_w, c->dims.patch, c->dims.in_ch,
                                   c->dims.out_ch, d, c->alpha_bar[it.t], c->alpha_bar[it.t + 1],
                                   st), "final_ddim");
+  }
+  if (host) {
+    // the step ends when its write-backs have landed; the next step's loads
+    // also wait for the final layer's reads
+    if (rows > 0) RC_CUDA(cudaStreamWaitEvent(st, k->wb_done, 0), "write-back done");
+    for (int i = 0; i < rc_cache::WINDOWS; ++i)
+      RC_CUDA(cudaEventRecord(k->consumed[i], st), "window event");
   }
   return RC_OK;
 }
@@ -736,6 +908,8 @@ rc_status rc_step_batched(rc_ctx* c, rc_cache* k, const rc_batch_item* items, in
   if (k->ctx != c) return fail(RC_ERR_INVALID_ARG, "cache belongs to another context");
   if (n < 1 || n > c->max_batch)
     return fail(RC_ERR_INVALID_ARG, "n_items %d outside [1, %d]", n, c->max_batch);
+  if (k->host_tier && n != 1)
+    return fail(RC_ERR_INVALID_ARG, "a host-tier cache steps one item at a time");
   for (int i = 0; i < n; ++i) {
     rc_status r = check_item(c, k, items[i]);
     if (r) return r;

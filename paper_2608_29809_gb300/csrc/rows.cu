@@ -610,6 +610,39 @@ scatter_bf16_kernel(const float* __restrict__ src, const __grid_constant__ Items
   }
 }
 
+// Host-tier write-back of one layer: the dirty rows tok[r] of the HBM window
+// [H,K,V][N][d] go to the same rows of the host slice (device-mapped
+// addresses); one warp per row, 16-byte accesses.
+__global__ void __launch_bounds__(RW_WARPS * 32)
+writeback_kernel(const bf16* __restrict__ win, bf16* host, RowMap rm, int d, unsigned* err) {
+  pdl_wait();
+  pdl_trigger();
+  const int D = live_count(rm.count, rm.bound, err);
+  const int lane = threadIdx.x & 31;
+  const size_t Nd = size_t(rm.n_tokens) * d;
+  for (int r = blockIdx.x * RW_WARPS + (threadIdx.x >> 5); r < D; r += gridDim.x * RW_WARPS) {
+    const int i = rm.tok ? __ldg(rm.tok + r) : r;
+    if (i < 0 || i >= rm.n_tokens) {
+      if (lane == 0) atomicOr(err, DEVERR_INDEX);
+      continue;
+    }
+    for (int part = 0; part < 3; ++part) {
+      const uint4* src = reinterpret_cast<const uint4*>(win + part * Nd + size_t(i) * d);
+      uint4* dst = reinterpret_cast<uint4*>(host + part * Nd + size_t(i) * d);
+      for (int c = lane; c < d / 8; c += 32) dst[c] = src[c];
+    }
+  }
+}
+
+cudaError_t launch_writeback(const bf16* win, bf16* host, const RowMap& rm, int d, unsigned* err,
+                             cudaStream_t st) {
+  if (rm.bound <= 0) return cudaSuccess;
+  RC_TRY(launch_k(writeback_kernel, dim3(row_grid(rm.bound, RW_WARPS, 1)), dim3(RW_WARPS * 32), 0,
+                  st, win, host, rm, d, err));
+  count_launches(1);
+  return cudaSuccess;
+}
+
 // Concatenated rows of a multi-item step: block (x, i) fills rows of item i.
 __global__ void __launch_bounds__(256)
 batch_rows_kernel(const __grid_constant__ BatchIn in, int* __restrict__ tok,

@@ -72,6 +72,7 @@ def load_library(path: str = LIB_PATH) -> C.CDLL:
         "rc_set_global_weights": (I, [P, C.POINTER(rc_global_weights)]),
         "rc_set_schedule": (I, [P, P, P]),
         "rc_cache_create": (I, [P, I, C.POINTER(P)]),
+        "rc_cache_create_host": (I, [P, I, C.POINTER(P)]),
         "rc_cache_destroy": (None, [P]),
         "rc_cache_fill": (I, [P, I, I, I, P, P, P, P]),
         "rc_cache_read": (I, [P, I, I, I, P, P, P, P]),
@@ -161,6 +162,12 @@ def rc_set_schedule(ctx, t_values, alpha_bar):
 def rc_cache_create(ctx, sessions) -> int:
     h = C.c_void_p()
     _check(_lib.rc_cache_create(ctx, sessions, C.byref(h)))
+    return h.value
+
+
+def rc_cache_create_host(ctx, sessions) -> int:
+    h = C.c_void_p()
+    _check(_lib.rc_cache_create_host(ctx, sessions, C.byref(h)))
     return h.value
 
 
@@ -310,7 +317,7 @@ class Model:
     """Owns a context, device copies of the weights (kept alive here) and a
     cache; thin sugar over the entry points for tests and the benchmark."""
 
-    def __init__(self, dims, weights, sessions=1, device="cuda", max_batch=1):
+    def __init__(self, dims, weights, sessions=1, device="cuda", max_batch=1, host_cache=False):
         self.dims = dims
         self.w = weights.to(device)
         self.ctx = rc_create(dims_struct(dims, max_batch))
@@ -319,7 +326,7 @@ class Model:
         g = dict(self.w.glob)
         g["pos"] = self.w.pos
         rc_set_global_weights(self.ctx, g)
-        self.cache = rc_cache_create(self.ctx, sessions)
+        self.cache = (rc_cache_create_host if host_cache else rc_cache_create)(self.ctx, sessions)
 
     def close(self):
         if self.cache:
