@@ -9,9 +9,11 @@ union of 1-3 seeded ellipses covering 5 / 10 / 20 / 40 % of the tokens,
 presented to the localisation kernel as a cross-attention score map.
 
 One step = localisation mask (rc_localize_mask) + one region-sparse
-denoising step (rc_step, mode SPARSE) at timestep t = step mod 20; the
-headline value is steps/s at 20 % dirty.  The library's own dense path
-(rc_step_dense) and every sweep point are reported beside it.
+denoising step at timestep t = step mod 20, replayed from the CUDA graph of
+rc_step (mode SPARSE) for that timestep, which reads the dirty list from the
+localisation buffers; the headline value is steps/s at 20 % dirty.  The same
+steps issued launch by launch (rc_step), the library's own dense path and
+every sweep point are reported beside it.
 
 Usage: python bench.py [--gpus N --steps K --warmup W] [--impl reference]
 For N > 1 launch with torch.distributed.run: every rank runs an independent
@@ -225,6 +227,36 @@ class Workload:
         self.R.rc_step(self.model.ctx, self.model.cache, 0, self.latent, t, self.sparse, self.idx,
                        -1, self.cnt)
 
+    def make_graphs(self):
+        """One CUDA graph of rc_step per timestep, SPARSE over the localisation
+        buffers (their contents are read at each replay), and one DENSE."""
+        R, d = self.R, self.d
+        dense = np.full(d.timesteps, R.RC_MODE_DENSE, np.uint8)
+        self.graphs = [R.rc_step_graph_create(self.model.ctx, self.model.cache, 0, self.latent,
+                                              t, self.sparse, self.idx, -1, self.cnt)
+                       for t in range(d.timesteps)]
+        self.dense_graphs = [R.rc_step_graph_create(self.model.ctx, self.model.cache, 0,
+                                                    self.latent, t, dense, None, 0, None)
+                             for t in range(d.timesteps)]
+
+    def free_graphs(self):
+        for g in self.graphs + self.dense_graphs:
+            self.R.rc_graph_destroy(g)
+        self.graphs, self.dense_graphs = [], []
+
+    def gstep(self, i, f):
+        t = i % self.d.timesteps
+        if t == 0:
+            self.latent.copy_(self.latent0)
+        self.localize(f)
+        self.R.rc_graph_launch(self.graphs[t])
+
+    def gstep_dense(self, i):
+        t = i % self.d.timesteps
+        if t == 0:
+            self.latent.copy_(self.latent0)
+        self.R.rc_graph_launch(self.dense_graphs[t])
+
     def step_dense(self, i):
         t = i % self.d.timesteps
         if t == 0:
@@ -303,25 +335,32 @@ def run_ours(args, world, rank, local):
     wl = Workload(R, d, SEED + rank, dev)
     peaks = load_peaks()
 
-    # headline: 20 % dirty, clock sampler running; no probe events in this pass
+    # headline: 20 % dirty, each step = localisation + the CUDA graph of
+    # rc_step for the timestep; clock sampler running, no probe events
+    wl.make_graphs()
     for i in range(W):
-        wl.step(i, HEADLINE)
+        wl.gstep(i, HEADLINE)
     torch.cuda.synchronize()
     clocks = ClockSampler(local)
     clocks.start()
     n0 = R.rc_launch_count()
-    ms = timed(lambda i: wl.step(i, HEADLINE), K, 0, world)
+    ms = timed(lambda i: wl.gstep(i, HEADLINE), K, 0, world)
     launches = R.rc_launch_count() - n0
     clk = clocks.stop()
     R.rc_sync(wl.model.ctx)
     D = int(wl.cnt.item())
     ms_max = max_over_ranks(ms, world)
     value = K * world / (ms_max / 1e3)
+    # the same steps issued launch by launch (rc_step)
+    m = timed(lambda i: wl.step(i, HEADLINE), K, W, world)
+    direct = K * world / (max_over_ranks(m, world) / 1e3)
     if args.quick:
         if rank == 0:
             print(json.dumps({"metric": METRIC, "value": round(value, 3), "unit": UNIT,
                               "quick": True, "ms_per_step": round(ms_max / K, 4),
+                              "direct_steps_per_s": round(direct, 3),
                               "dirty_tokens": D, "gpu_launches": int(launches)}), flush=True)
+        wl.free_graphs()
         wl.model.close()
         return
 
@@ -340,13 +379,13 @@ def run_ours(args, world, rank, local):
     gemm_ms, gemm_n, gemm_each = probe(R.RC_PROBE_GEMM, 6)
     att_ms, att_n, att_each = probe(R.RC_PROBE_ATTENTION, 2)
 
-    # sweep and dense baseline
+    # sweep and dense baseline (graphs, like the headline)
     sweep, dirty = {}, {}
     for f in FRACS:
-        m = timed(lambda i, f=f: wl.step(i, f), K, W, world)
+        m = timed(lambda i, f=f: wl.gstep(i, f), K, W, world)
         sweep[f"{f:.2f}"] = round(K * world / (max_over_ranks(m, world) / 1e3), 3)
         dirty[f"{f:.2f}"] = int(wl.cnt.item())
-    m = timed(wl.step_dense, max(2, K // 2), min(W, 3), world)
+    m = timed(wl.gstep_dense, max(2, K // 2), min(W, 3), world)
     dense = max(2, K // 2) * world / (max_over_ranks(m, world) / 1e3)
     m = timed(wl.step_capture, max(2, K // 2), min(W, 3), world)
     capture = max(2, K // 2) * world / (max_over_ranks(m, world) / 1e3)
@@ -371,7 +410,7 @@ def run_ours(args, world, rank, local):
         A_dev.copy_(A_host, non_blocking=True)
         wl.latent.copy_(lat_host, non_blocking=True)
         wl.localize(HEADLINE, A_dev)
-        R.rc_step(wl.model.ctx, wl.model.cache, 0, wl.latent, t, wl.sparse, wl.idx, -1, wl.cnt)
+        R.rc_graph_launch(wl.graphs[t])
         lat_host.copy_(wl.latent, non_blocking=True)
         torch.cuda.current_stream().synchronize()
 
@@ -432,11 +471,14 @@ def run_ours(args, world, rank, local):
         "config": {"workload": WORKLOAD, "tokens": d.tokens, "dirty_frac": HEADLINE,
                    "dirty_tokens": D, "layers": d.layers, "timesteps": d.timesteps,
                    "sessions_per_gpu": 1, "parallelism": "replicas" if world > 1 else "single",
-                   "l2": L2_NOTE, "step": "rc_localize_mask + rc_step(SPARSE)"},
+                   "l2": L2_NOTE,
+                   "step": "rc_localize_mask + rc_graph_launch (CUDA graph of rc_step SPARSE, "
+                           "dirty list read from the localisation buffers)"},
         "sweep_steps_per_s": sweep, "sweep_dirty_tokens": dirty,
         "dense_steps_per_s": round(dense, 3),
         "dense_capture_steps_per_s": round(capture, 3),
         "host_tier": host_tier,
+        "direct_steps_per_s": round(direct, 3),
         "speedup_vs_dense": {k: round(v / dense, 3) for k, v in sweep.items()},
         "roofline": roofline, "roofline_attention": roof_att,
         "e2e": e2e, "gpu_launches": int(launches), "clocks": clk,
@@ -445,6 +487,7 @@ def run_ours(args, world, rank, local):
         out["cpu_baseline"] = cpu_baseline(d, SEED, HEADLINE, layers_sample=args.cpu_layers)
     if rank == 0:
         print(json.dumps(out), flush=True)
+    wl.free_graphs()
     wl.model.close()
 
 

@@ -325,6 +325,26 @@ rc_status rc_step_capture(rc_ctx* ctx, rc_cache* cache, int session, float* late
 rc_status rc_prompt_similarity(const float* e_minus, const float* e_plus, int dim, float* s_out);
 rc_status rc_reuse_schedule(float s, float tau_s, float rho, int T, uint8_t* modes_out);
 
+/* CUDA Graph of one rc_step (no counterpart in the paper; serving
+ * plumbing): the step's ~320 kernel launches for fixed arguments are
+ * recorded once and replayed with one launch call.  The arguments are those
+ * of rc_step; the graph keeps the device pointers (latent, dirty_idx,
+ * dirty_count, the cache slots of (session, t)) and reads and writes their
+ * CONTENTS at each replay, so a new edit region only needs new dirty_idx /
+ * dirty_count contents (use D = -1 with a device count whose bound is N).
+ * Mode schedule_host[t] and the host bound D are fixed at creation.  The
+ * graph reuses the context's scratch: replays of graphs of one context are
+ * serialised on one stream, like its steps.  Creation enqueues nothing.
+ * Errors: as rc_step; RC_ERR_INVALID_ARG for a host-tier cache or while a
+ * timing probe is enabled; RC_ERR_CUDA when capture or instantiation fails. */
+typedef struct rc_graph rc_graph;
+rc_status rc_step_graph_create(rc_ctx* ctx, rc_cache* cache, int session, float* latent, int t,
+                               const uint8_t* schedule_host, const int32_t* dirty_idx, int D,
+                               const int32_t* dirty_count, rc_graph** out);
+/* Replays the graph on `stream`. */
+rc_status rc_graph_launch(rc_graph* graph, rc_stream stream);
+void rc_graph_destroy(rc_graph* graph);
+
 /* Full-recompute baseline: rc_step with mode DENSE. */
 rc_status rc_step_dense(rc_ctx* ctx, rc_cache* cache, int session, float* latent, int t,
                         rc_stream stream);

@@ -272,13 +272,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         const int qt = pair % sc.qtiles, h = pair / sc.qtiles;
         const TileLoc tl = locate_tile(rm, ai.n, D, qt);
         const int krow = ai.krow[tl.item], vrow = ai.vrow[tl.item];
-        if (!mbar_wait(q_empty, (uc + 1) & 1, abort_flag)) goto timeout;
+        if (!mbar_sleep(q_empty, (uc + 1) & 1, abort_flag)) goto timeout;
         mbar_expect_tx(q_full, C::Q_BYTES);
         tma_load_3d(saddr(sQ), &tmQ, q_full, 0, h, tl.row0);
         if (C::TAIL) tma_load_3d(saddr(sQ + C::Q128), &tmQt, q_full, 64, h, tl.row0);
         for (int kb = kb0; kb < kb1; ++kb, ++g) {
           const int st = g % KV_STAGES;
-          if (!mbar_wait(kv_empty + 8 * st, ((g / KV_STAGES) & 1) ^ 1, abort_flag)) goto timeout;
+          if (!mbar_sleep(kv_empty + 8 * st, ((g / KV_STAGES) & 1) ^ 1, abort_flag)) goto timeout;
           mbar_expect_tx(kv_full + 8 * st, C::KV_BYTES);
           uint8_t* base = sKV + st * C::KV_BYTES;
           const uint32_t fb = kv_full + 8 * st;
@@ -292,9 +292,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA
-    // Polls its inputs and issues whatever is ready: P V of block np (its
-    // P is in TMEM; first, as the softmax of the next block waits on it),
-    // then S of block ns (its K/V landed and its S buffer was read).
+    // In a fixed order, sleeping on each input: S of the unit's first two
+    // blocks, then per block j: P V of block j (once its P is in TMEM), then
+    // S of block j + 2 into the S buffer the softmax of block j has read.
+    // S(j + 2) is first needed after the softmax of block j + 1, so issuing it
+    // after P V(j) costs nothing, and no warp spins.
     if (lane == 0) {
       int g = 0, uc = 0;
       // descriptors of stage 0; a stage's differ only in the start address
@@ -307,58 +309,43 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
       it.init(sc, blockIdx.x);
       int pair, kb0, kb1, slot;
       for (; it.next(pair, kb0, kb1, slot); ++uc) {
-        const int qt = pair % sc.qtiles, h = pair / sc.qtiles;
         const int n = kb1 - kb0;
-        if (!mbar_wait(q_full, uc & 1, abort_flag)) goto timeout;
+        if (!mbar_sleep(q_full, uc & 1, abort_flag)) goto timeout;
         tc_fence_after();
-        int ns = 0, np = 0;
-        bool o_ok = false;
-        unsigned spins = 0;
-        unsigned long long t_idle = 0;
-        while (np < n) {
-          bool progress = false;
-          if (np < ns) {
-            const int gp = g + np;
-            if (!o_ok) o_ok = np > 0 || mbar_test(o_free, (uc + 1) & 1);
-            if (o_ok && mbar_test(p_ready, gp & 1)) {
-              tc_fence_after();
-              const int st = gp % KV_STAGES;
-              const uint64_t vd = dv + uint64_t(st * (C::KV_BYTES >> 4));
-              // 16 keys per MMA: P columns 8 kk .., V rows 16 kk .. (2 KB)
+        // S of block ns of the unit
+        auto issue_s = [&](int ns) -> bool {
+          const int gs = g + ns;
+          const int st = gs % KV_STAGES;
+          if (!mbar_sleep(kv_full + 8 * st, (gs / KV_STAGES) & 1, abort_flag) ||
+              !mbar_sleep(s_free + 8 * (gs & 1), ((gs >> 1) + 1) & 1, abort_flag))
+            return false;
+          tc_fence_after();
+          const uint64_t so = uint64_t(st * (C::KV_BYTES >> 4));
+          const uint32_t sd = tS0 + uint32_t(BKV) * uint32_t(gs & 1);
 #pragma unroll
-              for (int kk = 0; kk < BKV / 16; ++kk)
-                umma_bf16_ta(tO, tP + 8 * kk, vd + 128 * kk, C::IDESC_PV,
-                             (np > 0 || kk > 0) ? 1u : 0u);
-              umma_commit(kv_empty + 8 * st);
-              umma_commit(pv_done);
-              ++np;
-              progress = true;
-            }
-          }
-          if (ns < n) {
-            const int gs = g + ns;
-            const int st = gs % KV_STAGES;
-            if (mbar_test(kv_full + 8 * st, (gs / KV_STAGES) & 1) &&
-                mbar_test(s_free + 8 * (gs & 1), ((gs >> 1) + 1) & 1)) {
-              tc_fence_after();
-              const uint64_t so = uint64_t(st * (C::KV_BYTES >> 4));
-              const uint32_t sd = tS0 + uint32_t(BKV) * uint32_t(gs & 1);
+          for (int kk = 0; kk < 4; ++kk)
+            umma_bf16(sd, dq + 2 * kk, dk + so + 2 * kk, C::IDESC_S, kk > 0 ? 1u : 0u);
+          if (C::TAIL) umma_bf16(sd, dqt, dkt + so, C::IDESC_S, 1u);
+          umma_commit(s_full + 8 * (gs & 1));
+          if (ns == n - 1) umma_commit(q_empty);  // last S of the unit issued
+          return true;
+        };
+        if (!issue_s(0) || (n > 1 && !issue_s(1))) goto timeout;
+        for (int np = 0; np < n; ++np) {
+          const int gp = g + np;
+          if (np == 0 && !mbar_sleep(o_free, (uc + 1) & 1, abort_flag)) goto timeout;
+          if (!mbar_sleep(p_ready, gp & 1, abort_flag)) goto timeout;
+          tc_fence_after();
+          const int st = gp % KV_STAGES;
+          const uint64_t vd = dv + uint64_t(st * (C::KV_BYTES >> 4));
+          // 16 keys per MMA: P columns 8 kk .., V rows 16 kk .. (2 KB)
 #pragma unroll
-              for (int kk = 0; kk < 4; ++kk)
-                umma_bf16(sd, dq + 2 * kk, dk + so + 2 * kk, C::IDESC_S, kk > 0 ? 1u : 0u);
-              if (C::TAIL) umma_bf16(sd, dqt, dkt + so, C::IDESC_S, 1u);
-              umma_commit(s_full + 8 * (gs & 1));
-              if (++ns == n) umma_commit(q_empty);  // last S of the unit issued
-              progress = true;
-            }
-          }
-          if (progress) {
-            spins = 0;
-          } else if ((++spins & 63) == 0) {
-            const unsigned long long now = globaltimer();
-            if (spins == 64) t_idle = now;
-            if (*abort_flag || now - t_idle > WAIT_NS) goto timeout;
-          }
+          for (int kk = 0; kk < BKV / 16; ++kk)
+            umma_bf16_ta(tO, tP + 8 * kk, vd + 128 * kk, C::IDESC_PV,
+                         (np > 0 || kk > 0) ? 1u : 0u);
+          umma_commit(kv_empty + 8 * st);
+          umma_commit(pv_done);
+          if (np + 2 < n && !issue_s(np + 2)) goto timeout;
         }
         g += n;
         umma_commit(o_full);
@@ -381,7 +368,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
 #pragma unroll
       for (int q = 0; q < 8; ++q) cap_s[q] = -INFINITY;
       for (int j = 0; j < n; ++j, ++g) {
-        if (!mbar_wait_warp(s_full + 8 * (g & 1), (g >> 1) & 1, abort_flag)) goto timeout;
+        if (!mbar_sleep_warp(s_full + 8 * (g & 1), (g >> 1) & 1, abort_flag)) goto timeout;
         tc_fence_after();
         uint32_t r[BKV];
 #pragma unroll
@@ -453,7 +440,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         unpack_f32x2(sum2[3], s6, s7);
         l += ((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7));
         // the P buffer and O are free once P V of the previous block is done
-        if (g > 0 && !mbar_wait_warp(pv_done, (g - 1) & 1, abort_flag)) goto timeout;
+        if (g > 0 && !mbar_sleep_warp(pv_done, (g - 1) & 1, abort_flag)) goto timeout;
         tc_fence_after();
         if (rescale) {
 #pragma unroll
@@ -482,7 +469,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         mbar_arrive(p_ready);
       }
       // ---- unit epilogue
-      if (!mbar_wait_warp(o_full, uc & 1, abort_flag)) goto timeout;
+      if (!mbar_sleep_warp(o_full, uc & 1, abort_flag)) goto timeout;
       tc_fence_after();
       uint32_t o[C::DHP];
 #pragma unroll

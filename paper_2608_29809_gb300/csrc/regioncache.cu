@@ -902,6 +902,72 @@ rc_status rc_step(rc_ctx* c, rc_cache* k, int s, float* latent, int t,
   return step_items(c, k, &it, 1, static_cast<cudaStream_t>(stream));
 }
 
+struct rc_graph {
+  rc_ctx* ctx = nullptr;
+  cudaGraph_t graph = nullptr;
+  cudaGraphExec_t exec = nullptr;
+  uint64_t launches = 0;  // kernels per replay
+};
+
+void rc_graph_destroy(rc_graph* gr) {
+  if (!gr) return;
+  if (gr->exec) cudaGraphExecDestroy(gr->exec);
+  if (gr->graph) cudaGraphDestroy(gr->graph);
+  delete gr;
+}
+
+rc_status rc_step_graph_create(rc_ctx* c, rc_cache* k, int s, float* latent, int t,
+                               const uint8_t* schedule_host, const int32_t* dirty_idx, int D,
+                               const int32_t* dirty_count, rc_graph** out) {
+  if (!c || !k || !latent || !schedule_host || !out)
+    return fail(RC_ERR_INVALID_ARG, "rc_step_graph_create: null argument");
+  *out = nullptr;
+  if (k->ctx != c) return fail(RC_ERR_INVALID_ARG, "cache belongs to another context");
+  if (k->host_tier) return fail(RC_ERR_INVALID_ARG, "no graphs of host-tier cache steps");
+  if (c->probe_which != RC_PROBE_OFF)
+    return fail(RC_ERR_INVALID_ARG, "a timing probe is enabled");
+  if (t < 0 || t >= c->T) return fail(RC_ERR_INVALID_ARG, "t %d outside [0, %d)", t, c->T);
+  rc_batch_item it{s, latent, t, int(schedule_host[t]), dirty_idx, D, dirty_count};
+  rc_status r = check_item(c, k, it);
+  if (r) return r;
+  rc_graph* gr = new (std::nothrow) rc_graph();
+  if (!gr) return fail(RC_ERR_OOM, "host allocation");
+  gr->ctx = c;
+  cudaStream_t cs = nullptr;
+  cudaError_t e = cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking);
+  if (e != cudaSuccess) {
+    delete gr;
+    return cuda_fail(e, "capture stream");
+  }
+  const uint64_t n0 = rc_launch_count();
+  e = cudaStreamBeginCapture(cs, cudaStreamCaptureModeRelaxed);
+  if (e == cudaSuccess) {
+    r = step_items(c, k, &it, 1, cs);
+    e = cudaStreamEndCapture(cs, &gr->graph);  // ends the capture whatever happened
+  }
+  const uint64_t n = rc_launch_count() - n0;
+  g_launches.fetch_sub(n, std::memory_order_relaxed);  // counted when replayed
+  cudaStreamDestroy(cs);
+  if (r == RC_OK && e != cudaSuccess) r = cuda_fail(e, "stream capture");
+  if (r == RC_OK && (e = cudaGraphInstantiate(&gr->exec, gr->graph, 0)) != cudaSuccess)
+    r = cuda_fail(e, "graph instantiation");
+  if (r != RC_OK) {
+    cudaGetLastError();
+    rc_graph_destroy(gr);
+    return r;
+  }
+  gr->launches = n;
+  *out = gr;
+  return RC_OK;
+}
+
+rc_status rc_graph_launch(rc_graph* gr, rc_stream stream) {
+  if (!gr || !gr->exec) return fail(RC_ERR_INVALID_ARG, "rc_graph_launch: null graph");
+  RC_CUDA(cudaGraphLaunch(gr->exec, static_cast<cudaStream_t>(stream)), "graph launch");
+  rc::count_launches(int(gr->launches));
+  return RC_OK;
+}
+
 rc_status rc_step_batched(rc_ctx* c, rc_cache* k, const rc_batch_item* items, int n,
                           rc_stream stream) {
   if (!c || !k || !items) return fail(RC_ERR_INVALID_ARG, "rc_step_batched: null argument");

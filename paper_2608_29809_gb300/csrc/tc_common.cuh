@@ -66,6 +66,28 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
   }
 }
 
+// The same wait with mbarrier.try_wait, which suspends the thread in hardware
+// until the phase completes (or a system time limit passes) instead of
+// spinning: a waiting warp takes no issue slots from the warps sharing its
+// scheduler.
+__device__ __forceinline__ bool mbar_sleep(uint32_t bar, uint32_t parity,
+                                           volatile int* abort_flag) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const unsigned long long t0 = globaltimer();
+  for (unsigned n = 1;; ++n) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((n & 7) == 0) {
+      if (*abort_flag) return false;
+      if (globaltimer() - t0 > WAIT_NS) return false;
+    }
+  }
+}
+__device__ __forceinline__ bool mbar_sleep_warp(uint32_t bar, uint32_t parity,
+                                                volatile int* abort_flag) {
+  const bool ok = mbar_sleep(bar, parity, abort_flag);
+  return __all_sync(0xffffffffu, ok);
+}
+
 // mbar_wait taken by every lane of a warp; the outcome is made warp-uniform
 // so that a timeout never leaves part of a warp at a warp-wide instruction.
 __device__ __forceinline__ bool mbar_wait_warp(uint32_t bar, uint32_t parity,

@@ -73,6 +73,9 @@ def load_library(path: str = LIB_PATH) -> C.CDLL:
         "rc_set_schedule": (I, [P, P, P]),
         "rc_cache_create": (I, [P, I, C.POINTER(P)]),
         "rc_cache_create_host": (I, [P, I, C.POINTER(P)]),
+        "rc_step_graph_create": (I, [P, P, I, P, I, P, P, I, P, C.POINTER(P)]),
+        "rc_graph_launch": (I, [P, P]),
+        "rc_graph_destroy": (None, [P]),
         "rc_cache_destroy": (None, [P]),
         "rc_cache_fill": (I, [P, I, I, I, P, P, P, P]),
         "rc_cache_read": (I, [P, I, I, I, P, P, P, P]),
@@ -222,6 +225,23 @@ def rc_step(ctx, cache, session, latent, t, schedule, dirty_idx, D, dirty_count,
     sch = np.ascontiguousarray(schedule, np.uint8)
     _check(_lib.rc_step(ctx, cache, session, _ptr(latent), t, sch.ctypes.data, _ptr(dirty_idx),
                         D, _ptr(dirty_count), _stream(stream)))
+
+
+def rc_step_graph_create(ctx, cache, session, latent, t, schedule, dirty_idx, D,
+                         dirty_count) -> int:
+    sch = np.ascontiguousarray(schedule, np.uint8)
+    h = C.c_void_p()
+    _check(_lib.rc_step_graph_create(ctx, cache, session, _ptr(latent), t, sch.ctypes.data,
+                                     _ptr(dirty_idx), D, _ptr(dirty_count), C.byref(h)))
+    return h.value
+
+
+def rc_graph_launch(graph, stream=None):
+    _check(_lib.rc_graph_launch(graph, _stream(stream)))
+
+
+def rc_graph_destroy(graph):
+    _lib.rc_graph_destroy(graph)
 
 
 def rc_step_batched(ctx, cache, items, stream=None):
