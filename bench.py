@@ -309,6 +309,47 @@ class Workload:
                 "step": "rc_localize_mask + rc_step(SPARSE) on rc_cache_create_host"}
 
 
+def kernel_rooflines(d, D, gemm_each, att_each, peak):
+    """GEMM and attention rooflines of one probe pass: algorithmic FLOPs of
+    D dirty rows per launch over the CUDA-event launch durations."""
+    gemm_ms, gemm_n = sum(gemm_each), len(gemm_each)
+    att_ms, att_n = sum(att_each), len(att_each)
+    steps = gemm_n / (6 * d.layers)
+    lin_flops_launch = linear_flops_per_token_block(d) * D / 6
+    gemm_tflops = linear_flops_per_token_block(d) * D * d.layers * steps / (gemm_ms / 1e3) / 1e12
+    att_tflops = attn_flops_per_token_block(d) * D * d.layers * steps / (att_ms / 1e3) / 1e12
+    roofline = {"bound": "tensor", "achieved": round(gemm_tflops, 2), "peak": peak,
+                "unit": "TFLOP/s", "frac": round(gemm_tflops / peak, 4),
+                "traffic": profiled_traffic("gemm"),
+                "kernel": "gemm (QKV, out, cross-q, cross-out, fc1, fc2 of every block)",
+                "launches": gemm_n, "avg_launch_ms": round(gemm_ms / max(gemm_n, 1), 5),
+                "flops_per_launch": lin_flops_launch}
+    roof_att = {"bound": "tensor", "achieved": round(att_tflops, 2), "peak": peak,
+                "traffic": profiled_traffic("attention"),
+                "unit": "TFLOP/s", "frac": round(att_tflops / peak, 4), "launches": att_n,
+                "avg_launch_ms": round(att_ms / max(att_n, 1), 5)}
+    # per-launch breakdown: launches come in block order (GEMMs: QKV, out,
+    # cross-q, cross-out, fc1, fc2; attention: self, cross)
+    h, F = d.hidden, d.mlp
+    gemm_shapes = [("qkv", 3 * h, h), ("out", h, h), ("cross_q", h, h), ("cross_out", h, h),
+                   ("fc1", F, h), ("fc2", h, F)]
+    per_gemm = {}
+    for j, (name, n_, k_) in enumerate(gemm_shapes):
+        ts = gemm_each[j::6]
+        us = 1e3 * sum(ts) / max(len(ts), 1)
+        per_gemm[name] = {"shape": [D, n_, k_], "avg_us": round(us, 2),
+                          "tflops": round(2.0 * D * n_ * k_ / (us * 1e-6) / 1e12, 1)}
+    per_attn = {}
+    for j, (name, nk) in enumerate([("self", d.tokens), ("cross", d.text_len)]):
+        ts = att_each[j::2]
+        us = 1e3 * sum(ts) / max(len(ts), 1)
+        per_attn[name] = {"queries": D, "keys": nk, "avg_us": round(us, 2),
+                          "tflops": round(4.0 * D * nk * h / (us * 1e-6) / 1e12, 1)}
+    roofline["per_gemm"] = per_gemm
+    roof_att["per_launch"] = per_attn
+    return roofline, roof_att
+
+
 def timed(fn, K, W, world):
     for i in range(W):
         fn(i)
@@ -368,16 +409,20 @@ def run_ours(args, world, rank, local):
     # every GEMM launch and once around every attention launch (events on the
     # launching stream; they serialise the launches they bracket, so these
     # passes are kept out of the headline)
-    def probe(which, per_step):
-        cap = K * d.layers * per_step
+    def probe(which, per_step, fn, nsteps):
+        cap = nsteps * d.layers * per_step
         R.rc_probe_enable(wl.model.ctx, which, cap)
-        timed(lambda i: wl.step(i, HEADLINE), K, 0, 1)
+        timed(fn, nsteps, 0, 1)
         each = R.rc_probe_read_each(wl.model.ctx, cap)
         R.rc_probe_enable(wl.model.ctx, R.RC_PROBE_OFF, 0)
-        return sum(each), len(each), each
+        return each
 
-    gemm_ms, gemm_n, gemm_each = probe(R.RC_PROBE_GEMM, 6)
-    att_ms, att_n, att_each = probe(R.RC_PROBE_ATTENTION, 2)
+    gemm_each = probe(R.RC_PROBE_GEMM, 6, lambda i: wl.step(i, HEADLINE), K)
+    att_each = probe(R.RC_PROBE_ATTENTION, 2, lambda i: wl.step(i, HEADLINE), K)
+    # the same kernels on all 4096 rows (the dense step)
+    Kd = max(2, K // 4)
+    gemm_each_d = probe(R.RC_PROBE_GEMM, 6, wl.step_dense, Kd)
+    att_each_d = probe(R.RC_PROBE_ATTENTION, 2, wl.step_dense, Kd)
 
     # sweep and dense baseline (graphs, like the headline)
     sweep, dirty = {}, {}
@@ -426,42 +471,12 @@ def run_ours(args, world, rank, local):
            "h2d_bytes_per_step": int(A_host.numel() * 4 + lat_host.numel() * 4),
            "d2h_bytes_per_step": int(lat_host.numel() * 4)}
 
-    lin_flops_launch = linear_flops_per_token_block(d) * D * d.layers / (6 * d.layers)
-    gemm_avg_ms = gemm_ms / max(gemm_n, 1)
-    gemm_tflops = linear_flops_per_token_block(d) * D * d.layers * K / (gemm_ms / 1e3) / 1e12
     peak = peaks["bf16_tflops_sustained"]
-    att_tflops = (attn_flops_per_token_block(d) * D * d.layers * K) / (att_ms / 1e3) / 1e12
-    roofline = {"bound": "tensor", "achieved": round(gemm_tflops, 2), "peak": peak,
-                "unit": "TFLOP/s", "frac": round(gemm_tflops / peak, 4),
-                "traffic": profiled_traffic("gemm"),
-                "kernel": "gemm (QKV, out, cross-q, cross-out, fc1, fc2 of every block)",
-                "launches": gemm_n, "avg_launch_ms": round(gemm_avg_ms, 5),
-                "timing": "CUDA events around each launch, separate pass of the same K steps",
-                "flops_per_launch": lin_flops_launch,
-                "peak_source": f"{peaks['source']} bf16_tflops_sustained"}
-    roof_att = {"bound": "tensor", "achieved": round(att_tflops, 2), "peak": peak,
-                "traffic": profiled_traffic("attention"),
-                "unit": "TFLOP/s", "frac": round(att_tflops / peak, 4), "launches": att_n,
-                "avg_launch_ms": round(att_ms / max(att_n, 1), 5)}
-    # per-launch breakdown: launches come in block order (GEMMs: QKV, out,
-    # cross-q, cross-out, fc1, fc2; attention: self, cross)
-    h, F = d.hidden, d.mlp
-    gemm_shapes = [("qkv", 3 * h, h), ("out", h, h), ("cross_q", h, h), ("cross_out", h, h),
-                   ("fc1", F, h), ("fc2", h, F)]
-    per_gemm = {}
-    for j, (name, n_, k_) in enumerate(gemm_shapes):
-        ts = gemm_each[j::6]
-        us = 1e3 * sum(ts) / max(len(ts), 1)
-        per_gemm[name] = {"shape": [D, n_, k_], "avg_us": round(us, 2),
-                          "tflops": round(2.0 * D * n_ * k_ / (us * 1e-6) / 1e12, 1)}
-    per_attn = {}
-    for j, (name, nk) in enumerate([("self", d.tokens), ("cross", d.text_len)]):
-        ts = att_each[j::2]
-        us = 1e3 * sum(ts) / max(len(ts), 1)
-        per_attn[name] = {"queries": D, "keys": nk, "avg_us": round(us, 2),
-                          "tflops": round(4.0 * D * nk * h / (us * 1e-6) / 1e12, 1)}
-    roofline["per_gemm"] = per_gemm
-    roof_att["per_launch"] = per_attn
+    roofline, roof_att = kernel_rooflines(d, D, gemm_each, att_each, peak)
+    roofline.update({"timing": "CUDA events around each launch, separate pass of the same "
+                               "K steps",
+                     "peak_source": f"{peaks['source']} bf16_tflops_sustained"})
+    roof_dense, roof_att_dense = kernel_rooflines(d, d.tokens, gemm_each_d, att_each_d, peak)
     out = {
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
         "steps": K, "warmup": W, "ms_per_step": round(ms_max / K, 4), "higher_is_better": True,
@@ -481,6 +496,7 @@ def run_ours(args, world, rank, local):
         "direct_steps_per_s": round(direct, 3),
         "speedup_vs_dense": {k: round(v / dense, 3) for k, v in sweep.items()},
         "roofline": roofline, "roofline_attention": roof_att,
+        "roofline_dense": {"rows": d.tokens, "gemm": roof_dense, "attention": roof_att_dense},
         "e2e": e2e, "gpu_launches": int(launches), "clocks": clk,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
