@@ -17,10 +17,11 @@
 // into equal k-block ranges (stream-K).  Its casting variant (x += ..., then
 // xb = bf16(x), read-modify-write) and the other epilogues see whole tiles.
 //
-// CTA = 6 warps: warp 0 issues TMA loads, warp 1 owns TMEM and issues the
-// MMAs (one thread), warps 2..5 drain the accumulator (one TMEM lane = one
-// output row per thread, re-staged through shared memory so that global
-// writes are whole row pieces).  Two TMEM accumulators of up to 256 columns
+// CTA = 10 warps: warp 0 issues TMA loads, warp 1 owns TMEM and issues the
+// MMAs (one thread), warps 2..9 drain the accumulator (one TMEM lane = one
+// output row per thread; two warps per TMEM lane quarter take alternate
+// 32-column chunks; re-staged through shared memory so that global writes
+// are whole row pieces).  Two TMEM accumulators of up to 256 columns
 // let the epilogue of one tile overlap the main loop of the next.
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -39,14 +40,14 @@ namespace {
 using namespace rc::tc;
 
 constexpr int BM = 128, BK = 64;
-constexpr int THREADS = 192;
+constexpr int THREADS = 320;  // TMA warp, MMA warp, 8 epilogue warps
 constexpr int STAGE_A = BM * BK * 2;   // bytes
 constexpr int MIN_KB_PER_CTA = 4;
 constexpr int STAGING_WARP = 32 * 128;  // epilogue staging: 32 rows of 128 B per warp
-constexpr int STAGING_BYTES = 4 * STAGING_WARP;
+constexpr int STAGING_BYTES = 8 * STAGING_WARP;
 
 // Operand ring: stages of A (16 KB) + B (BN x 128 B), as many as fit.
-constexpr int RING_BYTES = 200 * 1024;
+constexpr int RING_BYTES = 184 * 1024;
 constexpr int MAX_STAGES = 8;
 constexpr int TMEM_COLS = 512;  // two accumulators of up to 256 columns
 constexpr size_t SMEM_BYTES = size_t(RING_BYTES) + STAGING_BYTES + 1024 + 256;
@@ -380,7 +381,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(tfull0 + 8 * a, 1);
-      mbar_init(tempty0 + 8 * a, 128);
+      mbar_init(tempty0 + 8 * a, 256);
     }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -463,7 +464,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
     }
   } else {
-    // ------------------------------------------------------- epilogue (warps 2..5)
+    // ------------------------------------------------------- epilogue (warps 2..9)
     const int sp = warp & 3;  // TMEM lane sub-partition this warp may access
     int acc = 0;
     uint32_t acc_phase = 0;
@@ -485,14 +486,14 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       // a piece of a split tile only occurs for the gated residual, whose
       // update is a sum: the bias goes with the piece that starts at k = 0
 #pragma unroll 1
-      for (int ch = 0; ch < BN / 32; ++ch) {
+      for (int ch = (warp - 2) >> 2; ch < BN / 32; ch += 2) {
         float v[32];
         tmem_ld32(tbase + uint32_t(ch * 32), v);
         const int c0 = nn * BN + ch * 32;
         epilogue_values(ep, c0, item, v, kb0 == 0);
         bf16* xb_row = (ep.mode == EPI_GATE_RES_CAST && r < M)
                            ? ep.out_bf + size_t(r) * ep.ld_out + c0 : nullptr;
-        store_chunk(ep.mode, sStg + sp * STAGING_WARP, lane, v, chunk_dst(ep, r, M, tok, item, c0),
+        store_chunk(ep.mode, sStg + (warp - 2) * STAGING_WARP, lane, v, chunk_dst(ep, r, M, tok, item, c0),
                     xb_row);
       }
       tc_fence_before();
