@@ -17,11 +17,12 @@
 // into equal k-block ranges (stream-K).  Its casting variant (x += ..., then
 // xb = bf16(x), read-modify-write) and the other epilogues see whole tiles.
 //
-// CTA = 10 warps: warp 0 issues TMA loads, warp 1 owns TMEM and issues the
-// MMAs (one thread), warps 2..9 drain the accumulator (one TMEM lane = one
-// output row per thread; two warps per TMEM lane quarter take alternate
-// 32-column chunks; re-staged through shared memory so that global writes
-// are whole row pieces).  Two TMEM accumulators of up to 256 columns
+// CTA = 14 warps: warp 0 issues TMA loads, warp 1 owns TMEM and issues the
+// MMAs (one thread), warps 2..13 drain the accumulator (one TMEM lane = one
+// output row per thread; three warps per TMEM lane quarter take every third
+// 32-column chunk; re-staged through shared memory so that global writes
+// are whole row pieces).  The epilogue is latency-bound (a CTA holds one
+// tile at small row counts), so its width is worth more than a deeper ring.  Two TMEM accumulators of up to 256 columns
 // let the epilogue of one tile overlap the main loop of the next.
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -40,14 +41,14 @@ namespace {
 using namespace rc::tc;
 
 constexpr int BM = 128, BK = 64;
-constexpr int THREADS = 320;  // TMA warp, MMA warp, 8 epilogue warps
+constexpr int THREADS = 448;  // TMA warp, MMA warp, 12 epilogue warps
 constexpr int STAGE_A = BM * BK * 2;   // bytes
 constexpr int MIN_KB_PER_CTA = 4;
 constexpr int STAGING_WARP = 32 * 128;  // epilogue staging: 32 rows of 128 B per warp
-constexpr int STAGING_BYTES = 8 * STAGING_WARP;
+constexpr int STAGING_BYTES = 12 * STAGING_WARP;
 
 // Operand ring: stages of A (16 KB) + B (BN x 128 B), as many as fit.
-constexpr int RING_BYTES = 184 * 1024;
+constexpr int RING_BYTES = 168 * 1024;
 constexpr int MAX_STAGES = 8;
 constexpr int TMEM_COLS = 512;  // two accumulators of up to 256 columns
 constexpr size_t SMEM_BYTES = size_t(RING_BYTES) + STAGING_BYTES + 1024 + 256;
@@ -264,11 +265,12 @@ struct Sched {
     return s < MAX_STAGES ? s : MAX_STAGES;
   }
   // Estimated duration (SM cycles): k-blocks on the busiest CTA x per-k-block
-  // time (operands from L2 at ~60 B/clk per SM) plus its exposed epilogues
-  // (~12 B/clk per SM, measured); a stream-K CTA holds two pieces.
+  // time (operands at ~60 B/clk per SM) plus its exposed epilogues (~20 B/clk
+  // per SM with twelve epilogue warps; both rates measured); a stream-K CTA
+  // holds two pieces.
   __host__ __device__ float cost(int out_bytes) const {
     const float ckb = float(STAGE_A + BN * BK * 2) * (1.f / 60.f);
-    const float cep = float(BM * BN * out_bytes) * (1.f / 12.f);
+    const float cep = float(BM * BN * out_bytes) * (1.f / 20.f);
     if (S > 0) return float((kbt + S - 1) / S) * ckb + cep;
     const int waves = (whole + G - 1) / G;
     float c = float(waves) * float(kbt) * ckb + (waves > 0 ? cep : 0.f);
@@ -381,7 +383,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(tfull0 + 8 * a, 1);
-      mbar_init(tempty0 + 8 * a, 256);
+      mbar_init(tempty0 + 8 * a, 384);
     }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -464,7 +466,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
     }
   } else {
-    // ------------------------------------------------------- epilogue (warps 2..9)
+    // ------------------------------------------------------- epilogue (warps 2..13)
     const int sp = warp & 3;  // TMEM lane sub-partition this warp may access
     int acc = 0;
     uint32_t acc_phase = 0;
@@ -486,7 +488,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       // a piece of a split tile only occurs for the gated residual, whose
       // update is a sum: the bias goes with the piece that starts at k = 0
 #pragma unroll 1
-      for (int ch = (warp - 2) >> 2; ch < BN / 32; ch += 2) {
+      for (int ch = (warp - 2) >> 2; ch < BN / 32; ch += 3) {
         float v[32];
         tmem_ld32(tbase + uint32_t(ch * 32), v);
         const int c0 = nn * BN + ch * 32;
