@@ -565,9 +565,16 @@ attn_combine_kernel(const float* __restrict__ part, bf16* __restrict__ O, int ld
       return base + (size_t(c) * 2 + (q == 0 ? slot_lo : 0)) * (BQ * PART_STRIDE);
     };
     if (np <= 32) {
-      // lane q holds piece q's row max / sum
+      // lane q holds piece q's row max / sum; the first four pieces' columns
+      // are requested in the same round
       float2 ml = make_float2(-INFINITY, 0.f);
       if (lane < np) ml = __ldcg(reinterpret_cast<const float2*>(piece(lane) + DH));
+      float4 v0[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+        v0[e] = (e < np && lane < DH / 4)
+                    ? __ldcg(reinterpret_cast<const float4*>(piece(e)) + lane)
+                    : make_float4(0.f, 0.f, 0.f, 0.f);
       float M = ml.x;
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
@@ -583,7 +590,8 @@ attn_combine_kernel(const float* __restrict__ part, bf16* __restrict__ O, int ld
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           wq[e] = __shfl_sync(0xffffffffu, w, (q0 + e) & 31);
-          v[e] = (q0 + e < np && lane < DH / 4)
+          v[e] = q0 == 0 ? v0[e]
+                 : (q0 + e < np && lane < DH / 4)
                      ? __ldcg(reinterpret_cast<const float4*>(piece(q0 + e)) + lane)
                      : make_float4(0.f, 0.f, 0.f, 0.f);
         }

@@ -240,6 +240,27 @@ ln_mod_kernel(const float* __restrict__ x, const float* __restrict__ tab, int k_
   for (int r = blockIdx.x * LN_WARPS + (threadIdx.x >> 5); r < D; r += gridDim.x * LN_WARPS) {
     int tok, item;
     if (!row_target(rm, it.n, r, tok, item, err, lane)) continue;
+    // the modulation vectors first: their loads overlap the row's and the
+    // reductions instead of following them
+    const float* tb = it.tb[item];
+    float4 sh[LN_MAXV], sc[LN_MAXV];
+#pragma unroll
+    for (int k = 0; k < LN_MAXV; ++k)
+      if (k < nv) {
+        const int c = 4 * (lane + 32 * k);
+        sh[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+        sc[k] = sh[k];
+        if (tab) {
+          sh[k] = __ldg(reinterpret_cast<const float4*>(tab + size_t(k_sh) * d + c));
+          sc[k] = __ldg(reinterpret_cast<const float4*>(tab + size_t(k_sc) * d + c));
+        }
+        if (tb) {
+          const float4 a = *reinterpret_cast<const float4*>(tb + size_t(k_sh) * d + c);
+          const float4 b = *reinterpret_cast<const float4*>(tb + size_t(k_sc) * d + c);
+          sh[k].x += a.x; sh[k].y += a.y; sh[k].z += a.z; sh[k].w += a.w;
+          sc[k].x += b.x; sc[k].y += b.y; sc[k].z += b.z; sc[k].w += b.w;
+        }
+      }
     const float4* xr = reinterpret_cast<const float4*>(x + size_t(r) * d);
     float4 v[LN_MAXV];
     float s = 0.f;
@@ -265,27 +286,14 @@ ln_mod_kernel(const float* __restrict__ x, const float* __restrict__ tab, int k_
         q += (a * a + b * b) + (c * c + e * e);
       }
     const float rstd = 1.0f / sqrtf(warp_sum(q) / float(d) + 1e-6f);
-    const float* tb = it.tb[item];
     uint2* orow = reinterpret_cast<uint2*>(out + size_t(r) * d);
 #pragma unroll
     for (int k = 0; k < LN_MAXV; ++k)
       if (k < nv) {
-        const int c = 4 * (lane + 32 * k);
-        float4 sh = make_float4(0.f, 0.f, 0.f, 0.f), sc = sh;
-        if (tab) {
-          sh = *reinterpret_cast<const float4*>(tab + size_t(k_sh) * d + c);
-          sc = *reinterpret_cast<const float4*>(tab + size_t(k_sc) * d + c);
-        }
-        if (tb) {
-          const float4 a = *reinterpret_cast<const float4*>(tb + size_t(k_sh) * d + c);
-          const float4 b = *reinterpret_cast<const float4*>(tb + size_t(k_sc) * d + c);
-          sh.x += a.x; sh.y += a.y; sh.z += a.z; sh.w += a.w;
-          sc.x += b.x; sc.y += b.y; sc.z += b.z; sc.w += b.w;
-        }
-        float y0 = (v[k].x - mean) * rstd * (1.f + sc.x) + sh.x;
-        float y1 = (v[k].y - mean) * rstd * (1.f + sc.y) + sh.y;
-        float y2 = (v[k].z - mean) * rstd * (1.f + sc.z) + sh.z;
-        float y3 = (v[k].w - mean) * rstd * (1.f + sc.w) + sh.w;
+        float y0 = (v[k].x - mean) * rstd * (1.f + sc[k].x) + sh[k].x;
+        float y1 = (v[k].y - mean) * rstd * (1.f + sc[k].y) + sh[k].y;
+        float y2 = (v[k].z - mean) * rstd * (1.f + sc[k].z) + sh[k].z;
+        float y3 = (v[k].w - mean) * rstd * (1.f + sc[k].w) + sh[k].w;
         orow[lane + 32 * k] = make_uint2(pack_bf16x2(y0, y1), pack_bf16x2(y2, y3));
       }
   }
