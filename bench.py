@@ -185,7 +185,7 @@ def max_over_ranks(x: float, world: int) -> float:
 
 # ------------------------------------------------------------------ our arm
 class Workload:
-    def __init__(self, R, d: synth.Dims, seed: int, dev: str):
+    def __init__(self, R, d: synth.Dims, seed: int, dev: str, fracs=FRACS):
         self.R, self.d, self.dev = R, d, dev
         w = synth.make_weights(d, seed, device=dev)
         self.model = R.Model(d, w, sessions=1, device=dev)
@@ -208,7 +208,7 @@ class Workload:
         self.ws = torch.empty(R.rc_localize_workspace_size(N, 8), dtype=torch.uint8, device=dev)
         self.sparse = np.full(d.timesteps, R.RC_MODE_SPARSE, np.uint8)
         self.scores = {}
-        for f in FRACS:
+        for f in fracs:
             blobs = synth.ellipse_blobs(d, seed, f)
             A, ids = synth.indicator_scores(d, blobs, seed)
             self.scores[f] = (torch.from_numpy(A).to(dev), ids, A)
@@ -307,6 +307,31 @@ class Workload:
                 "d2h_bytes_per_step": 3 * int(self.cnt.item()) * d.hidden * 2 * d.layers,
                 "h2d_gbs_over_step": round(h2d / (m / K / 1e3) / 1e9, 1),
                 "step": "rc_localize_mask + rc_step(SPARSE) on rc_cache_create_host"}
+
+
+def rate_2048(R, args, world, dev, K, W):
+    """Headline-style steps (20 % dirty, graphs) and dense steps of the 2048 px
+    model (128 x 128 = 16 384 tokens, all 20 timesteps resident)."""
+    from dataclasses import replace
+    d = replace(synth.PIXART_2048, timesteps=args.resident_steps)
+    wl = Workload(R, d, SEED + 7, dev, fracs=(HEADLINE,))
+    try:
+        wl.make_graphs()
+        k = max(2, K // 4)
+        m = timed(lambda i: wl.gstep(i, HEADLINE), k, W, world)
+        sparse = k * world / (max_over_ranks(m, world) / 1e3)
+        D = int(wl.cnt.item())
+        m = timed(wl.gstep_dense, k, min(W, 3), world)
+        dense = k * world / (max_over_ranks(m, world) / 1e3)
+        R.rc_sync(wl.model.ctx)
+        wl.free_graphs()
+    finally:
+        wl.model.close()
+    return {"workload": f"pixart-alpha-2048px: {d.tokens} tokens, {d.layers} blocks, "
+                        f"{d.timesteps} timesteps, batch 1",
+            "dirty_frac": HEADLINE, "dirty_tokens": D, "steps_per_s": round(sparse, 3),
+            "dense_steps_per_s": round(dense, 3), "speedup_vs_dense": round(sparse / dense, 3),
+            "cache_bytes": d.timesteps * d.layers * 3 * d.tokens * d.hidden * 2}
 
 
 def kernel_rooflines(d, D, gemm_each, att_each, peak):
@@ -436,6 +461,11 @@ def run_ours(args, world, rank, local):
     capture = max(2, K // 2) * world / (max_over_ranks(m, world) / 1e3)
     R.rc_sync(wl.model.ctx)
 
+    # the same step at 2048 px (16 384 tokens, 63.4 GB cache resident)
+    big = None
+    if not args.no_2048:
+        big = rate_2048(R, args, world, dev, K, W)
+
     # the same headline steps on a host-tier cache (pinned host pool, each
     # layer's K, V streamed into HBM windows while the previous layer runs)
     host_tier = None
@@ -493,6 +523,7 @@ def run_ours(args, world, rank, local):
         "dense_steps_per_s": round(dense, 3),
         "dense_capture_steps_per_s": round(capture, 3),
         "host_tier": host_tier,
+        "pixart2048": big,
         "direct_steps_per_s": round(direct, 3),
         "speedup_vs_dense": {k: round(v / dense, 3) for k, v in sweep.items()},
         "roofline": roofline, "roofline_attention": roof_att,
@@ -610,6 +641,8 @@ def main():
     ap.add_argument("--cpu-layers", type=int, default=2)
     ap.add_argument("--quick", action="store_true",
                     help="headline only: no attention probe, sweep, dense, e2e or cpu baseline")
+    ap.add_argument("--no-2048", action="store_true",
+                    help="skip the 2048 px (16 384-token, 63 GB cache) measurement")
     ap.add_argument("--no-host-tier", action="store_true",
                     help="skip the host-tier cache measurement (a pinned host pool)")
     ap.add_argument("--resident-steps", type=int, default=20,

@@ -48,6 +48,7 @@ typedef int rc_status;
 #define RC_ERR_TIMEOUT 5       /* a bounded device wait gave up               */
 #define RC_ERR_DEVICE_ASSERT 6 /* a kernel found a bad index / count          */
 #define RC_ERR_STATE 7         /* call order violated (e.g. no weights set)   */
+#define RC_ERR_IO 8            /* a file could not be opened, read or written */
 
 /* Per-step modes of a reuse schedule (Section 3.3, Eq. 2). */
 #define RC_MODE_DENSE 0  /* every token recomputed; cache rows overwritten    */
@@ -153,6 +154,19 @@ rc_status rc_cache_fill(rc_cache* cache, int session, int layer, int t,
                         const void* H, const void* K, const void* V, rc_stream stream);
 rc_status rc_cache_read(rc_cache* cache, int session, int layer, int t,
                         void* H, void* K, void* V, rc_stream stream);
+
+/* One session's whole cache to / from a file, so that an editing session
+ * outlives the process (the paper keeps the pool in host memory between
+ * turns, Section 3.4): every (t, layer) H, K, V slot and the text
+ * keys/values, after a header with N, hidden, layers, timesteps and
+ * text_len.  Synchronous (the device is synchronised first); the file is
+ * raw little-endian bf16, about timesteps * layers * 3 * N * hidden * 2
+ * bytes.  Import requires a header equal to the cache's dimensions
+ * (RC_ERR_SHAPE otherwise) and marks the session's text as set when the
+ * exported session had it.  Errors: RC_ERR_INVALID_ARG, RC_ERR_IO (open,
+ * short read / write, bad magic), RC_ERR_SHAPE, RC_ERR_CUDA. */
+rc_status rc_cache_export(rc_cache* cache, int session, const char* path);
+rc_status rc_cache_import(rc_cache* cache, int session, const char* path);
 
 /* Text conditioning of one session for an editing turn: ctx_bf16 is the
  * text context, bf16 [text_len][hidden].  Computes every layer's

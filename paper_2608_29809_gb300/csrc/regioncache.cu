@@ -619,6 +619,81 @@ rc_status rc_cache_read(rc_cache* k, int s, int l, int t, void* H, void* K, void
   return cache_copy(k, s, l, t, H, K, V, false, static_cast<cudaStream_t>(st));
 }
 
+// Session file: magic, then int32 version, N, hidden, layers, timesteps,
+// text_len, text_set; then the session's slots in cache order
+// ([t][layer][H,K,V][N][hidden]) and its text keys / values
+// ([layer][text_len][2 hidden]), bf16.
+static const char kCacheMagic[8] = {'R', 'C', 'C', 'A', 'C', 'H', 'E', '1'};
+
+// Copies `elems` bf16 between device-addressable `dev` and the file through a
+// pinned staging buffer.
+static rc_status session_io(bf16* dev, size_t elems, FILE* f, bool write, void* stage,
+                            size_t stage_bytes) {
+  const size_t per = stage_bytes / sizeof(bf16);
+  for (size_t off = 0; off < elems; off += per) {
+    const size_t n = elems - off < per ? elems - off : per;
+    if (write) {
+      RC_CUDA(cudaMemcpy(stage, dev + off, n * sizeof(bf16), cudaMemcpyDefault), "export copy");
+      if (fwrite(stage, sizeof(bf16), n, f) != n) return fail(RC_ERR_IO, "short write");
+    } else {
+      if (fread(stage, sizeof(bf16), n, f) != n) return fail(RC_ERR_IO, "short read");
+      RC_CUDA(cudaMemcpy(dev + off, stage, n * sizeof(bf16), cudaMemcpyDefault), "import copy");
+    }
+  }
+  return RC_OK;
+}
+
+static rc_status session_file(rc_cache* k, int s, const char* path, bool write) {
+  if (!k || !path) return fail(RC_ERR_INVALID_ARG, "null cache or path");
+  rc_status r = check_session(k, s);
+  if (r) return r;
+  const rc_ctx* c = k->ctx;
+  RC_CUDA(cudaDeviceSynchronize(), "synchronise");
+  FILE* f = fopen(path, write ? "wb" : "rb");
+  if (!f) return fail(RC_ERR_IO, "cannot open %s", path);
+  int32_t hdr[7] = {1, c->N, c->d, c->L, c->T, c->M, write ? int32_t(k->text_set[s]) : 0};
+  if (write) {
+    if (fwrite(kCacheMagic, 1, 8, f) != 8 || fwrite(hdr, sizeof(int32_t), 7, f) != 7)
+      r = fail(RC_ERR_IO, "short write");
+  } else {
+    char magic[8];
+    int32_t got[7];
+    if (fread(magic, 1, 8, f) != 8 || memcmp(magic, kCacheMagic, 8) != 0)
+      r = fail(RC_ERR_IO, "%s is not a cache file", path);
+    else if (fread(got, sizeof(int32_t), 7, f) != 7)
+      r = fail(RC_ERR_IO, "short read");
+    else if (got[0] != 1 || memcmp(got + 1, hdr + 1, 5 * sizeof(int32_t)) != 0)
+      r = fail(RC_ERR_SHAPE, "file dims N %d hidden %d layers %d T %d text %d differ", got[1],
+               got[2], got[3], got[4], got[5]);
+    else
+      hdr[6] = got[6];
+  }
+  void* stage = nullptr;
+  const size_t stage_bytes = size_t(64) << 20;
+  if (r == RC_OK && cudaMallocHost(&stage, stage_bytes) != cudaSuccess) {
+    cudaGetLastError();
+    stage = nullptr;
+    r = fail(RC_ERR_OOM, "pinned staging buffer");
+  }
+  if (r == RC_OK)
+    r = session_io(k->slot(s, 0, 0, 0), size_t(c->T) * c->L * 3 * k->slot_elems(), f, write,
+                   stage, stage_bytes);
+  if (r == RC_OK)
+    r = session_io(k->text_kv(s, 0), size_t(c->L) * c->M * 2 * c->d, f, write, stage,
+                   stage_bytes);
+  if (stage) cudaFreeHost(stage);
+  if (fclose(f) != 0 && r == RC_OK) r = fail(RC_ERR_IO, "closing %s", path);
+  if (r == RC_OK && !write) k->text_set[s] = char(hdr[6] != 0);
+  return r;
+}
+
+rc_status rc_cache_export(rc_cache* k, int s, const char* path) {
+  return session_file(k, s, path, true);
+}
+rc_status rc_cache_import(rc_cache* k, int s, const char* path) {
+  return session_file(k, s, path, false);
+}
+
 rc_status rc_set_text(rc_ctx* c, rc_cache* k, int s, const void* ctx_bf16, rc_stream stream) {
   if (!c || !k || !ctx_bf16) return fail(RC_ERR_INVALID_ARG, "rc_set_text: null argument");
   if (k->ctx != c) return fail(RC_ERR_INVALID_ARG, "cache belongs to another context");

@@ -22,7 +22,8 @@ HEADER = os.path.join(os.path.dirname(HERE), "include", "regioncache.h")
 RC_OK = 0
 RC_MODE_DENSE, RC_MODE_SPARSE, RC_MODE_REUSE = 0, 1, 2
 STATUS = {0: "RC_OK", 1: "RC_ERR_INVALID_ARG", 2: "RC_ERR_SHAPE", 3: "RC_ERR_OOM",
-          4: "RC_ERR_CUDA", 5: "RC_ERR_TIMEOUT", 6: "RC_ERR_DEVICE_ASSERT", 7: "RC_ERR_STATE"}
+          4: "RC_ERR_CUDA", 5: "RC_ERR_TIMEOUT", 6: "RC_ERR_DEVICE_ASSERT", 7: "RC_ERR_STATE",
+          8: "RC_ERR_IO"}
 
 
 class RCError(RuntimeError):
@@ -73,6 +74,8 @@ def load_library(path: str = LIB_PATH) -> C.CDLL:
         "rc_set_schedule": (I, [P, P, P]),
         "rc_cache_create": (I, [P, I, C.POINTER(P)]),
         "rc_cache_create_host": (I, [P, I, C.POINTER(P)]),
+        "rc_cache_export": (I, [P, I, C.c_char_p]),
+        "rc_cache_import": (I, [P, I, C.c_char_p]),
         "rc_step_graph_create": (I, [P, P, I, P, I, P, P, I, P, C.POINTER(P)]),
         "rc_graph_launch": (I, [P, P]),
         "rc_graph_destroy": (None, [P]),
@@ -172,6 +175,14 @@ def rc_cache_create_host(ctx, sessions) -> int:
     h = C.c_void_p()
     _check(_lib.rc_cache_create_host(ctx, sessions, C.byref(h)))
     return h.value
+
+
+def rc_cache_export(cache, session, path):
+    _check(_lib.rc_cache_export(cache, session, os.fsencode(path)))
+
+
+def rc_cache_import(cache, session, path):
+    _check(_lib.rc_cache_import(cache, session, os.fsencode(path)))
 
 
 def rc_cache_destroy(cache):

@@ -65,6 +65,7 @@ class Dims:
 
 PIXART_512 = Dims(grid_h=32, grid_w=32)
 PIXART_1024 = Dims(grid_h=64, grid_w=64)
+PIXART_2048 = Dims(grid_h=128, grid_w=128)
 ONE_BLOCK_256 = Dims(grid_h=16, grid_w=16, layers=1)
 TINY = Dims(hidden=64, heads=4, mlp=256, layers=2, grid_h=4, grid_w=4, text_len=8,
             timesteps=4, freq_dim=32)
