@@ -45,13 +45,18 @@ def c3_problem(R):
     p.close()
 
 
-def test_c3_full_step_bench_configuration(R, c3_problem):
+@pytest.mark.parametrize("launch", ["graph", "direct"])
+def test_c3_full_step_bench_configuration(R, c3_problem, launch):
     """One full 28-block step at 4096 tokens, 20 % dirty ellipse union, the
     mask made on the device and the dirty count left there (D = -1), exactly
-    as the benchmark runs it; the oracle runs the whole step."""
+    as the benchmark runs it (replayed from the CUDA graph of the timestep,
+    and launch by launch); the oracle runs the whole step."""
     p = c3_problem
     d = p.d
     t = 7
+    for l in range(d.layers):  # the previous turn's cache, whatever ran before
+        H, K, V = synth.make_cache_slice(d, p.seed, 0, l, t)
+        R.rc_cache_fill(p.model.cache, 0, l, t, H.cuda(), K.cuda(), V.cuda())
     blobs = synth.ellipse_blobs(d, p.seed, 0.2)
     A, ids = synth.indicator_scores(d, blobs, p.seed)
     mask, idx_d, cnt = _localize(R, A, ids, d, 0)
@@ -63,10 +68,21 @@ def test_c3_full_step_bench_configuration(R, c3_problem):
     lat = synth.make_latent(d, p.seed)
     latent = lat.clone().cuda()
     sched = np.full(d.timesteps, O.MODE_SPARSE, np.uint8)
-    R.rc_step(p.model.ctx, p.model.cache, 0, latent, t, sched, idx_d, -1, cnt)
-    R.rc_sync(p.model.ctx)
+    if launch == "graph":
+        g = R.rc_step_graph_create(p.model.ctx, p.model.cache, 0, latent, t, sched, idx_d, -1,
+                                   cnt)
+        try:
+            R.rc_graph_launch(g)
+            R.rc_sync(p.model.ctx)
+        finally:
+            R.rc_graph_destroy(g)
+    else:
+        R.rc_step(p.model.ctx, p.model.cache, 0, latent, t, sched, idx_d, -1, cnt)
+        R.rc_sync(p.model.ctx)
     got = latent.cpu().double().numpy()
-    ref, eps, cache = p.oracle_step(O.to64(lat), t, O.MODE_SPARSE, idx)
+    if not hasattr(p, "c3_oracle"):  # the same inputs for both launch modes
+        p.c3_oracle = p.oracle_step(O.to64(lat), t, O.MODE_SPARSE, idx)
+    ref, eps, cache = p.c3_oracle
     assert rel_l2(got, ref) <= LATENT_REL_L2
     block_close(_eps_from_update(got, O.to64(lat), float(p.ab[t]), float(p.ab[t + 1])), eps, "eps")
     clean = np.setdiff1d(np.arange(d.tokens), idx)
