@@ -55,12 +55,23 @@ constexpr size_t SMEM_BYTES = size_t(RING_BYTES) + STAGING_BYTES + 1024 + 256;
 // Instruction descriptor, kind::f16: D f32, A and B bf16, both K-major,
 // M >> 4 at bit 24; N >> 3 goes to bit 17 at run time.
 constexpr uint32_t IDESC_BASE = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(BM >> 4) << 24);
+// the same for the M = 256 MMA of a CTA pair
+constexpr uint32_t IDESC_PAIR = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(256 >> 4) << 24);
 // The tile width and split chosen on the host for 1 .. BN_TABLE row tiles
 // (BN / 64 + 8 S), passed by value; larger row counts choose on the device.
 constexpr int BN_TABLE = 64;
 struct BnTable {
   uint8_t w64[BN_TABLE];
 };
+// W tensor maps by box height 32, 64, 96, 128, 192, 256 rows (a CTA of a
+// pair loads half a tile width)
+constexpr int N_BMAPS = 6;
+struct BMaps {
+  CUtensorMap m[N_BMAPS];
+};
+__host__ __device__ constexpr int bmap_index(int rows) {
+  return rows == 32 ? 0 : rows == 64 ? 1 : rows == 96 ? 2 : rows == 128 ? 3 : rows == 192 ? 4 : 5;
+}
 
 // ---------------------------------------------------------------- epilogue
 __device__ __forceinline__ void load32(const float* p, float* v) {
@@ -233,18 +244,25 @@ __device__ __forceinline__ void store_chunk(int mode, uint8_t* stg, int lane, co
 // CTA), or, when the last wave would leave more than half the CTAs idle, by
 // laying the R remainder tiles end to end by k-block and cutting them into
 // Gr equal ranges (stream-K, at least MIN_KB_PER_CTA k-blocks each).
+//
+// Pairs (two CTAs of a cluster sharing one M = 256 MMA): the same, with a
+// "tile" of two row tiles (2p, 2p + 1) and G the number of pairs.
 struct Sched {
   int BN, stages, mt, nt, tiles, kbt, G, whole, Gr, S;
+  bool pair;
   long long Wr;
   // S > 0: split-S (requires tiles * S <= grid); S == 0: waves (+ stream-K)
-  __host__ __device__ void plan(int M, int bn, int n, int k, int grid, bool additive, int s) {
+  __host__ __device__ void plan(int M, int bn, int n, int k, int grid, bool additive, int s,
+                                bool pr) {
     BN = bn;
-    stages = stages_for(bn);
-    mt = (M + BM - 1) / BM;
+    pair = pr;
+    stages = stages_for(bn, pr);
+    const int mt_rows = (M + BM - 1) / BM;
+    mt = pair ? (mt_rows + 1) / 2 : mt_rows;
     nt = n / BN;
     tiles = mt * nt;
     kbt = k / BK;
-    G = grid;
+    G = pair ? grid / 2 : grid;
     S = s;
     if (S > 0) {
       whole = 0;
@@ -260,8 +278,13 @@ struct Sched {
     if (g < 1) g = 1;
     Gr = split ? int(g < G ? g : G) : 0;
   }
-  __host__ __device__ static int stages_for(int bn) {
-    const int s = RING_BYTES / (STAGE_A + bn * BK * 2);
+  // bytes of one stage in one CTA: A (128 x 64) and B (BN x 64, half of it
+  // in each CTA of a pair)
+  __host__ __device__ static int stage_bytes(int bn, bool pr) {
+    return STAGE_A + (pr ? bn * BK : bn * BK * 2);
+  }
+  __host__ __device__ static int stages_for(int bn, bool pr) {
+    const int s = RING_BYTES / stage_bytes(bn, pr);
     return s < MAX_STAGES ? s : MAX_STAGES;
   }
   // Estimated duration (SM cycles): k-blocks on the busiest CTA x per-k-block
@@ -269,7 +292,7 @@ struct Sched {
   // per SM with twelve epilogue warps; both rates measured); a stream-K CTA
   // holds two pieces.
   __host__ __device__ float cost(int out_bytes) const {
-    const float ckb = float(STAGE_A + BN * BK * 2) * (1.f / 60.f);
+    const float ckb = float(stage_bytes(BN, pair)) * (1.f / 60.f);
     const float cep = float(BM * BN * out_bytes) * (1.f / 20.f);
     if (S > 0) return float((kbt + S - 1) / S) * ckb + cep;
     const int waves = (whole + G - 1) / G;
@@ -280,7 +303,7 @@ struct Sched {
   // Picks BN (n % BN == 0) and, for the additive gated residual, a split,
   // with the lowest estimate; ties go to wider tiles and fewer pieces.
   // Returns BN / 64 + 8 S.
-  __host__ __device__ static int pick(int M, int n, int k, int grid, int mode) {
+  __host__ __device__ static int pick(int M, int n, int k, int grid, int mode, bool pr) {
     Sched s;
     const bool additive = mode == EPI_GATE_RES;
     const int out_bytes = mode == EPI_GATE_RES_CAST ? 10
@@ -292,8 +315,8 @@ struct Sched {
       if (n % cand[i]) continue;
       for (int sp = 0; sp <= (additive ? 4 : 0); ++sp) {
         if (sp == 1) continue;
-        s.plan(M, cand[i], n, k, grid, additive, sp);
-        if (sp > 0 && (s.tiles * sp > grid || s.kbt < sp * MIN_KB_PER_CTA)) continue;
+        s.plan(M, cand[i], n, k, grid, additive, sp, pr);
+        if (sp > 0 && (s.tiles * sp > s.G || s.kbt < sp * MIN_KB_PER_CTA)) continue;
         const float c = s.cost(out_bytes);
         if (c < best * 0.999f) {
           best = c;
@@ -304,11 +327,11 @@ struct Sched {
     return code;
   }
   // table: the host's pick for 1 .. BN_TABLE row tiles (0 = not tabulated)
-  __device__ void init(int M, int n, int k, int grid, int mode, const uint8_t* table) {
+  __device__ void init(int M, int n, int k, int grid, int mode, const uint8_t* table, bool pr) {
     const int m_tiles = (M + BM - 1) / BM;
     int code = m_tiles >= 1 && m_tiles <= BN_TABLE ? int(table[m_tiles - 1]) : 0;
-    if (code == 0) code = pick(M, n, k, grid, mode);
-    plan(M, 64 * (code & 7), n, k, grid, mode == EPI_GATE_RES, code >> 3);
+    if (code == 0) code = pick(M, n, k, grid, mode, pr);
+    plan(M, 64 * (code & 7), n, k, grid, mode == EPI_GATE_RES, code >> 3, pr);
   }
   __device__ long long bound(int c) const { return Wr * c / Gr; }
 };
@@ -355,13 +378,18 @@ struct Segs {
   }
 };
 
+// PAIR: launched in clusters of two CTAs that share every MMA (cta_group::2,
+// M = 256): each CTA loads its own 128 rows of A and half of the W tile, and
+// the even CTA's MMA thread multiplies the pair's operands into both CTAs'
+// tensor memory.  Per k-block a CTA then holds (and pulls from L2)
+// 16 KB + BN x 64 B instead of 16 KB + BN x 128 B, so the ring keeps more
+// k-blocks in flight -- the main loop is bound by k-blocks in flight per SM
+// over the load latency.
+template <bool PAIR>
 __global__ void __launch_bounds__(THREADS, 1)
-gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB64,
-               const __grid_constant__ CUtensorMap tmB128,
-               const __grid_constant__ CUtensorMap tmB192,
-               const __grid_constant__ CUtensorMap tmB256, int Mbound,
-               const int* __restrict__ dcount, int n, int k, const __grid_constant__ GemmEpi ep,
-               const __grid_constant__ BnTable bt) {
+gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ BMaps tmB,
+               int Mbound, const int* __restrict__ dcount, int n, int k,
+               const __grid_constant__ GemmEpi ep, const __grid_constant__ BnTable bt) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 1024-aligned operand ring, epilogue staging, then barriers
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -376,6 +404,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   const uint32_t full0 = saddr(bars), empty0 = saddr(bars + MAX_STAGES);
   const uint32_t tfull0 = saddr(bars + 2 * MAX_STAGES), tempty0 = saddr(bars + 2 * MAX_STAGES + 2);
 
+  // rank 0 of a pair issues the MMAs; its barriers count the pair's loads
+  // (full), and both CTAs' epilogue warps (tempty: one arrival per warp)
+  const uint32_t rank = PAIR ? cluster_ctarank() : 0;
   if (threadIdx.x == 0) {
     for (int s = 0; s < MAX_STAGES; ++s) {
       mbar_init(full0 + 8 * s, 1);
@@ -383,20 +414,26 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(tfull0 + 8 * a, 1);
-      mbar_init(tempty0 + 8 * a, 384);
+      mbar_init(tempty0 + 8 * a, PAIR ? 24 : 12);
     }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 1) tmem_alloc(saddr(tmem_slot), TMEM_COLS);
-  if (warp == 0 && lane == 0) {
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB64)) : "memory");
+  if (warp == 1) {
+    if (PAIR)
+      tmem_alloc_pair(saddr(tmem_slot), TMEM_COLS);
+    else
+      tmem_alloc(saddr(tmem_slot), TMEM_COLS);
   }
+  if (warp == 0 && lane == 0)
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  // the peer's barriers are initialised before any of its loads, commits or
+  // arrivals can reach them
+  if (PAIR) cluster_sync();
 
   // everything above is private set-up; inputs written by earlier kernels
   // are read only after the predecessor has completed
@@ -404,45 +441,57 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   pdl_trigger();
   const int M = live_count(dcount, Mbound, ep.err);
   Sched sc;
-  sc.init(M, n, k, int(gridDim.x), ep.mode, bt.w64);
+  sc.init(M, n, k, int(gridDim.x), ep.mode, bt.w64, PAIR);
   const int BN = sc.BN, STAGES = sc.stages;
-  const int STAGE = STAGE_A + BN * BK * 2;
+  const int STAGE = Sched::stage_bytes(BN, PAIR);
+  // schedule position: the pair (its row tiles 2p + rank) or the CTA
+  const int pos = PAIR ? int(blockIdx.x) >> 1 : int(blockIdx.x);
 
   if (warp == 0) {
     // ------------------------------------------------------- TMA producer
     if (lane == 0) {
-      // B as one box of BN rows (maps for the widths that divide n)
-      const CUtensorMap* tmB = BN == 256 ? &tmB256 : BN == 192 ? &tmB192 : BN == 128 ? &tmB128 : &tmB64;
-      if (BN != 64)
-        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tmB)) : "memory");
+      // W as one box of BN rows, or BN / 2 rows per CTA of a pair (maps for
+      // the heights that divide n)
+      const int brows = PAIR ? BN / 2 : BN;
+      const CUtensorMap* tmW = &tmB.m[bmap_index(brows)];
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tmW)) : "memory");
       int stage = 0;
       uint32_t phase = 0;
       Segs sg;
-      sg.init(sc, blockIdx.x);
+      sg.init(sc, pos);
       int t, kb0, kb1;
       while (sg.next(t, kb0, kb1)) {
-        const int m = t % sc.mt, nn = t / sc.mt;
+        const int mq = t % sc.mt, nn = t / sc.mt;
+        const int m = PAIR ? 2 * mq + int(rank) : mq;
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(empty0 + 8 * stage, phase ^ 1, abort_flag)) goto timeout;
           uint8_t* st = smem + stage * STAGE;
-          mbar_expect_tx(full0 + 8 * stage, STAGE);
-          tma_load_2d(saddr(st), &tmA, full0 + 8 * stage, kb * BK, m * BM);
-          tma_load_2d(saddr(st + STAGE_A), tmB, full0 + 8 * stage, kb * BK, nn * BN);
+          if (PAIR) {
+            // both CTAs' bytes land on rank 0's barrier, which expects them
+            const uint32_t fb = mapa_shared(full0 + 8 * stage, 0);
+            if (rank == 0) mbar_expect_tx(full0 + 8 * stage, 2 * STAGE);
+            tma_load_2d_pair(saddr(st), &tmA, fb, kb * BK, m * BM);
+            tma_load_2d_pair(saddr(st + STAGE_A), tmW, fb, kb * BK, nn * BN + int(rank) * brows);
+          } else {
+            mbar_expect_tx(full0 + 8 * stage, STAGE);
+            tma_load_2d(saddr(st), &tmA, full0 + 8 * stage, kb * BK, m * BM);
+            tma_load_2d(saddr(st + STAGE_A), tmW, full0 + 8 * stage, kb * BK, nn * BN);
+          }
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
         }
       }
     }
   } else if (warp == 1) {
     // ------------------------------------------------------- MMA issuer
-    if (lane == 0) {
-      const uint32_t idesc = IDESC_BASE | (uint32_t(BN >> 3) << 17);
+    if (lane == 0 && rank == 0) {
+      const uint32_t idesc = (PAIR ? IDESC_PAIR : IDESC_BASE) | (uint32_t(BN >> 3) << 17);
       const uint64_t da = sw128_desc(saddr(smem)), db = sw128_desc(saddr(smem + STAGE_A));
       int stage = 0;
       uint32_t phase = 0;
       int acc = 0;
       uint32_t acc_phase = 0;
       Segs sg;
-      sg.init(sc, blockIdx.x);
+      sg.init(sc, pos);
       int t, kb0, kb1;
       while (sg.next(t, kb0, kb1)) {
         if (!mbar_wait(tempty0 + 8 * acc, acc_phase ^ 1, abort_flag)) goto timeout;
@@ -454,14 +503,25 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           // stage descriptors differ only in the start address field
           // (address >> 4; no carry out of its 14 bits below 256 KB)
           const uint64_t so = uint64_t((stage * STAGE) >> 4);
+          if (PAIR) {
 #pragma unroll
-          for (int kk = 0; kk < BK / 16; ++kk)
-            umma_bf16(dtm, da + so + 2 * kk, db + so + 2 * kk, idesc,
-                      (kb > kb0 || kk > 0) ? 1u : 0u);
-          umma_commit(empty0 + 8 * stage);
+            for (int kk = 0; kk < BK / 16; ++kk)
+              umma_bf16_pair(dtm, da + so + 2 * kk, db + so + 2 * kk, idesc,
+                             (kb > kb0 || kk > 0) ? 1u : 0u);
+            umma_commit_pair(empty0 + 8 * stage);  // frees the stage in both CTAs
+          } else {
+#pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk)
+              umma_bf16(dtm, da + so + 2 * kk, db + so + 2 * kk, idesc,
+                        (kb > kb0 || kk > 0) ? 1u : 0u);
+            umma_commit(empty0 + 8 * stage);
+          }
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
         }
-        umma_commit(tfull0 + 8 * acc);
+        if (PAIR)
+          umma_commit_pair(tfull0 + 8 * acc);
+        else
+          umma_commit(tfull0 + 8 * acc);
         if (++acc == 2) { acc = 0; acc_phase ^= 1; }
       }
     }
@@ -471,10 +531,14 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     int acc = 0;
     uint32_t acc_phase = 0;
     Segs sg;
-    sg.init(sc, blockIdx.x);
+    sg.init(sc, pos);
     int t, kb0, kb1;
+    // the accumulator is drained once every epilogue warp of the pair (or
+    // CTA) has arrived on rank 0's barrier
+    const uint32_t tempty_r0 = PAIR ? mapa_shared(tempty0, 0) : tempty0;
     while (sg.next(t, kb0, kb1)) {
-      const int m = t % sc.mt, nn = t / sc.mt;
+      const int mq = t % sc.mt, nn = t / sc.mt;
+      const int m = PAIR ? 2 * mq + int(rank) : mq;
       if (!mbar_wait_warp(tfull0 + 8 * acc, acc_phase, abort_flag)) goto timeout;
       tc_fence_after();
       const int row = sp * 32 + lane;
@@ -499,7 +563,13 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                     xb_row);
       }
       tc_fence_before();
-      mbar_arrive(tempty0 + 8 * acc);
+      __syncwarp();
+      if (lane == 0) {
+        if (PAIR)
+          mbar_arrive_cluster(tempty_r0 + 8 * acc);
+        else
+          mbar_arrive(tempty0 + 8 * acc);
+      }
       if (++acc == 2) { acc = 0; acc_phase ^= 1; }
     }
   }
@@ -510,10 +580,16 @@ timeout:
 done:
   tc_fence_before();
   __syncthreads();
+  // no CTA leaves (or frees its tensor memory) while its peer may still
+  // load, commit or arrive into it
+  if (PAIR) cluster_sync();
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tmem_base, TMEM_COLS);
+    if (PAIR)
+      tmem_dealloc_pair(tmem_base, TMEM_COLS);
+    else
+      tmem_dealloc(tmem_base, TMEM_COLS);
   }
 }
 
@@ -577,41 +653,81 @@ cudaError_t tensor_map(const bf16* p, int rows, int cols, int ld, int box_rows, 
   return cudaSuccess;
 }
 
-// Tile-width table of a GEMM shape, cached (the cost model runs 4 x 64 plans).
-BnTable bn_table(int n, int k, int sms, int mode, int mt_bound) {
+// Tile-width table of a GEMM shape, cached (the cost model runs up to 4 x 5
+// plans per row-tile count).
+BnTable bn_table(int n, int k, int grid, int mode, int mt_bound, bool pair) {
   static std::mutex mu;
   static std::unordered_map<uint64_t, BnTable> cache;
   const int mtb = mt_bound < BN_TABLE ? mt_bound : BN_TABLE;
-  // bits: mtb 0-6, mode 7-10, sms 11-18, k 19-40, n 41-63 (n, k < 2^22: checked)
-  const uint64_t full_key = uint64_t(mtb) | (uint64_t(mode & 15) << 7) |
-                            (uint64_t(sms & 255) << 11) | (uint64_t(k & 0x3FFFFF) << 19) |
-                            (uint64_t(n) << 41);
+  // bits: mtb 0-6, mode 7-9, pair 10, grid 11-18, k 19-40, n 41-63
+  // (mode < 8, grid < 256, n, k < 2^22: checked by the launcher)
+  const uint64_t full_key = uint64_t(mtb) | (uint64_t(mode & 7) << 7) |
+                            (uint64_t(pair ? 1 : 0) << 10) | (uint64_t(grid & 255) << 11) |
+                            (uint64_t(k & 0x3FFFFF) << 19) | (uint64_t(n) << 41);
   {
     std::lock_guard<std::mutex> lock(mu);
     auto it = cache.find(full_key);
     if (it != cache.end()) return it->second;
   }
   BnTable bt{};
-  for (int mt = 1; mt <= mtb; ++mt) bt.w64[mt - 1] = uint8_t(Sched::pick(mt * BM, n, k, sms, mode));
+  for (int mt = 1; mt <= mtb; ++mt)
+    bt.w64[mt - 1] = uint8_t(Sched::pick(mt * BM, n, k, grid, mode, pair));
   std::lock_guard<std::mutex> lock(mu);
   if (cache.size() > 4096) cache.clear();
   cache.emplace(full_key, bt);
   return bt;
 }
 
+// Launch shape of the current device: CTA pairs (clusters of two, one CTA
+// per SM) when every SM can hold one, else one CTA per SM unpaired.
+// grid 0: no device.
+struct GemmShape {
+  int grid;
+  bool pair;
+};
+constexpr int PAIR_MIN_ROWS = 2048;
 int device_sms() {
   static int sms[64] = {};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
-  if (!sms[dev]) {
-    int v = 0;
-    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-    if (cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             int(SMEM_BYTES)) != cudaSuccess)
-      return 0;
-    sms[dev] = v;
-  }
+  if (!sms[dev] && cudaDeviceGetAttribute(&sms[dev], cudaDevAttrMultiProcessorCount, dev) !=
+                       cudaSuccess)
+    return 0;
   return sms[dev];
+}
+GemmShape device_shape() {
+  static GemmShape shp[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return GemmShape{0, false};
+  if (!shp[dev].grid) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        v >= 256)
+      return GemmShape{0, false};
+    if (cudaFuncSetAttribute(gemm_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             int(SMEM_BYTES)) != cudaSuccess ||
+        cudaFuncSetAttribute(gemm_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             int(SMEM_BYTES)) != cudaSuccess)
+      return GemmShape{0, false};
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(v & ~1);
+    cfg.blockDim = dim3(THREADS);
+    cfg.dynamicSmemBytes = SMEM_BYTES;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int nc = 0;
+    if (cudaOccupancyMaxActiveClusters(&nc, gemm_tc_kernel<true>, &cfg) != cudaSuccess) {
+      cudaGetLastError();
+      nc = 0;
+    }
+    shp[dev] = nc > 0 && 2 * nc == (v & ~1) ? GemmShape{2 * nc, true} : GemmShape{v, false};
+  }
+  return shp[dev];
 }
 
 }  // namespace
@@ -619,22 +735,34 @@ int device_sms() {
 cudaError_t launch_gemm(const bf16* A, int lda, const bf16* W, int Mbound, const int* dcount,
                         int n, int k, const GemmEpi& ep, cudaStream_t st) {
   if (Mbound <= 0) return cudaSuccess;
-  if (n % 64 || k % BK || n >= (1 << 22) || k >= (1 << 22)) return cudaErrorInvalidValue;
-  const int sms = device_sms();
-  if (!sms) return cudaErrorInvalidDevice;
+  if (n % 64 || k % BK || n >= (1 << 22) || k >= (1 << 22) || ep.mode < 0 || ep.mode > 7)
+    return cudaErrorInvalidValue;
+  const GemmShape shp = device_shape();
+  if (!shp.grid) return cudaErrorInvalidDevice;
   cudaError_t e;
-  CUtensorMap ta, tb[4];
+  CUtensorMap ta;
+  BMaps tb;
   if ((e = tensor_map(A, Mbound, k, lda, BM, &ta)) != cudaSuccess) return e;
-  // one B map per tile width that divides n (the kernel picks the width);
-  // the others repeat the 64-row map and are never used
-  const int widths[4] = {64, 128, 192, 256};
-  for (int i = 0; i < 4; ++i) {
-    const int w = n % widths[i] == 0 ? widths[i] : 64;
-    if ((e = tensor_map(W, n, k, k, w, &tb[i])) != cudaSuccess) return e;
+  // one W map per box height that divides n (the kernel picks the one its
+  // tile width needs); the others repeat the 32-row map and are never used
+  const int heights[N_BMAPS] = {32, 64, 96, 128, 192, 256};
+  for (int i = 0; i < N_BMAPS; ++i) {
+    const int h = n % heights[i] == 0 ? heights[i] : 32;
+    if ((e = tensor_map(W, n, k, k, h, &tb.m[i])) != cudaSuccess) return e;
   }
-  const BnTable bt = bn_table(n, k, sms, ep.mode, (Mbound + BM - 1) / BM);
-  RC_TRY(launch_k(gemm_tc_kernel, dim3(sms), dim3(THREADS), SMEM_BYTES, st, ta, tb[0], tb[1],
-                  tb[2], tb[3], Mbound, dcount, n, k, ep, bt));
+  // pairs pay for their coupling and the cluster launch only with many row
+  // tiles per CTA: measured faster at 4096 rows (QKV 37 -> 36, fc1 52 -> 48,
+  // fc2 56 -> 47 us) and slower at 831 (cross-q 14.3 -> 16.4 us).  The row
+  // count must be known here: a device-side count keeps CTAs unpaired.
+  const bool pair = shp.pair && !dcount && Mbound >= PAIR_MIN_ROWS;
+  const int grid = pair ? shp.grid : device_sms();
+  const BnTable bt = bn_table(n, k, grid, ep.mode, (Mbound + BM - 1) / BM, pair);
+  if (pair)
+    RC_TRY(launch_k_cluster(gemm_tc_kernel<true>, dim3(shp.grid), dim3(THREADS), SMEM_BYTES, 2,
+                            st, ta, tb, Mbound, dcount, n, k, ep, bt));
+  else
+    RC_TRY(launch_k(gemm_tc_kernel<false>, dim3(grid), dim3(THREADS), SMEM_BYTES, st, ta, tb,
+                    Mbound, dcount, n, k, ep, bt));
   count_launches(1);
   return cudaSuccess;
 }
