@@ -327,9 +327,15 @@ patch_embed_kernel(int gh, int gw, int p, int C, const bf16* __restrict__ We,
   extern __shared__ __align__(16) uint8_t pe_smem[];
   bf16* s_w = reinterpret_cast<bf16*>(pe_smem);  // [d][16], zero beyond P
   const int P = C * p * p;                         // <= 16
-  for (int e = threadIdx.x; e < d * 16; e += blockDim.x) {
-    const int o = e >> 4, k = e & 15;
-    s_w[e] = k < P ? We[size_t(o) * P + k] : f2bf(0.f);
+  if (P == 16 && (reinterpret_cast<uintptr_t>(We) & 15u) == 0) {
+    // rows of 16 weights are 32 bytes: a straight 16-byte copy
+    for (int v = threadIdx.x; v < d * 2; v += blockDim.x)
+      reinterpret_cast<uint4*>(s_w)[v] = __ldg(reinterpret_cast<const uint4*>(We) + v);
+  } else {
+    for (int e = threadIdx.x; e < d * 16; e += blockDim.x) {
+      const int o = e >> 4, k = e & 15;
+      s_w[e] = k < P ? We[size_t(o) * P + k] : f2bf(0.f);
+    }
   }
   __syncthreads();
   const int D = live_count(rm.count, rm.bound, err);
@@ -473,10 +479,13 @@ final_ddim_kernel(const bf16* __restrict__ H, const float* __restrict__ temb,
     s_shift[c] = table_f[c] + temb[c];
     s_scale[c] = table_f[d + c] + temb[c];
   }
-  for (int e = 0; e < n_eps; ++e) {
+  // the eps rows of W_f, 16 bytes per thread and step (d % 8 == 0)
+  const int d8 = d / 8;
+  for (int v = threadIdx.x; v < n_eps * d8; v += blockDim.x) {
+    const int e = v / d8, c8 = v - e * d8;
     const int sub = e / c_in, ch = e - sub * c_in;
-    const bf16* src = Wf + size_t(sub * c_out + ch) * d;
-    for (int c = threadIdx.x; c < d; c += blockDim.x) s_w[size_t(e) * d + c] = src[c];
+    reinterpret_cast<uint4*>(s_w + size_t(e) * d)[c8] =
+        __ldg(reinterpret_cast<const uint4*>(Wf + size_t(sub * c_out + ch) * d) + c8);
   }
   __syncthreads();
   const int N = gh * gw;
@@ -567,8 +576,10 @@ cudaError_t launch_final_ddim(const bf16* H, const float* temb, const float* tab
     attr_set = true;
   }
   const int N = gh * gw;
-  int grid = cdiv(N, FIN_WARPS * 4);
-  if (grid > 1024) grid = 1024;
+  // a warp per token: the per-token reductions are latency-bound chains
+  int grid = cdiv(N, FIN_WARPS);
+  const int cap = 8 * device_sm_count();
+  if (grid > cap) grid = cap;
   RC_TRY(launch_k(final_ddim_kernel, dim3(grid), dim3(FIN_WARPS * 32), smem, st, H, temb, table_f,
                   Wf, bf, latent, gh, gw, p, c_in, c_out, d, ab_t, ab_next));
   count_launches(1);
