@@ -234,68 +234,79 @@ ln_mod_kernel(const float* __restrict__ x, const float* __restrict__ tab, int k_
               long long hprev_off, int d, unsigned* err) {
   pdl_wait();
   pdl_trigger();
+  // shift and scale staged once per CTA: tab (+ the item's tb when the
+  // launch has one item; otherwise each row adds its item's tb)
+  extern __shared__ __align__(16) float s_mod[];  // [2][d]
   const int D = live_count(rm.count, rm.bound, err);
   const int lane = threadIdx.x & 31;
   const int nv = d / 128;
-  for (int r = blockIdx.x * LN_WARPS + (threadIdx.x >> 5); r < D; r += gridDim.x * LN_WARPS) {
+  const float* tb0 = it.n == 1 ? it.tb[0] : nullptr;
+  int r = blockIdx.x * LN_WARPS + (threadIdx.x >> 5);
+  float4 v[LN_MAXV];
+  auto load_row = [&](int rr) {
+    const float4* xr = reinterpret_cast<const float4*>(x + size_t(rr) * d);
+#pragma unroll
+    for (int k = 0; k < LN_MAXV; ++k)
+      if (k < nv) v[k] = xr[lane + 32 * k];
+  };
+  if (r < D) load_row(r);  // requested before the staging barrier
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    float a = tab ? tab[size_t(k_sh) * d + c] : 0.f, b = tab ? tab[size_t(k_sc) * d + c] : 0.f;
+    if (tb0) {
+      a += tb0[size_t(k_sh) * d + c];
+      b += tb0[size_t(k_sc) * d + c];
+    }
+    s_mod[c] = a;
+    s_mod[d + c] = b;
+  }
+  __syncthreads();
+  while (r < D) {
     int tok, item;
-    if (!row_target(rm, it.n, r, tok, item, err, lane)) continue;
-    // the modulation vectors first: their loads overlap the row's and the
-    // reductions instead of following them
-    const float* tb = it.tb[item];
-    float4 sh[LN_MAXV], sc[LN_MAXV];
-#pragma unroll
-    for (int k = 0; k < LN_MAXV; ++k)
-      if (k < nv) {
-        const int c = 4 * (lane + 32 * k);
-        sh[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-        sc[k] = sh[k];
-        if (tab) {
-          sh[k] = __ldg(reinterpret_cast<const float4*>(tab + size_t(k_sh) * d + c));
-          sc[k] = __ldg(reinterpret_cast<const float4*>(tab + size_t(k_sc) * d + c));
-        }
-        if (tb) {
-          const float4 a = *reinterpret_cast<const float4*>(tb + size_t(k_sh) * d + c);
-          const float4 b = *reinterpret_cast<const float4*>(tb + size_t(k_sc) * d + c);
-          sh[k].x += a.x; sh[k].y += a.y; sh[k].z += a.z; sh[k].w += a.w;
-          sc[k].x += b.x; sc[k].y += b.y; sc[k].z += b.z; sc[k].w += b.w;
-        }
-      }
-    const float4* xr = reinterpret_cast<const float4*>(x + size_t(r) * d);
-    float4 v[LN_MAXV];
-    float s = 0.f;
-#pragma unroll
-    for (int k = 0; k < LN_MAXV; ++k)
-      if (k < nv) {
-        v[k] = xr[lane + 32 * k];
-        s += (v[k].x + v[k].y) + (v[k].z + v[k].w);
-      }
-    if (hprev_off >= 0) {
-      uint2* hrow = reinterpret_cast<uint2*>(it.slice[item] + hprev_off + size_t(tok) * d);
+    if (row_target(rm, it.n, r, tok, item, err, lane)) {
+      float s = 0.f;
 #pragma unroll
       for (int k = 0; k < LN_MAXV; ++k)
-        if (k < nv)
-          hrow[lane + 32 * k] = make_uint2(pack_bf16x2(v[k].x, v[k].y), pack_bf16x2(v[k].z, v[k].w));
+        if (k < nv) s += (v[k].x + v[k].y) + (v[k].z + v[k].w);
+      if (hprev_off >= 0) {
+        uint2* hrow = reinterpret_cast<uint2*>(it.slice[item] + hprev_off + size_t(tok) * d);
+#pragma unroll
+        for (int k = 0; k < LN_MAXV; ++k)
+          if (k < nv)
+            hrow[lane + 32 * k] =
+                make_uint2(pack_bf16x2(v[k].x, v[k].y), pack_bf16x2(v[k].z, v[k].w));
+      }
+      const float mean = warp_sum(s) / float(d);
+      float q = 0.f;
+#pragma unroll
+      for (int k = 0; k < LN_MAXV; ++k)
+        if (k < nv) {
+          float a = v[k].x - mean, b = v[k].y - mean, c = v[k].z - mean, e = v[k].w - mean;
+          q += (a * a + b * b) + (c * c + e * e);
+        }
+      const float rstd = 1.0f / sqrtf(warp_sum(q) / float(d) + 1e-6f);
+      const float* tb = tb0 ? nullptr : it.tb[item];
+      uint2* orow = reinterpret_cast<uint2*>(out + size_t(r) * d);
+#pragma unroll
+      for (int k = 0; k < LN_MAXV; ++k)
+        if (k < nv) {
+          const int c = 4 * (lane + 32 * k);
+          float4 sh = *reinterpret_cast<const float4*>(s_mod + c);
+          float4 sc = *reinterpret_cast<const float4*>(s_mod + d + c);
+          if (tb) {
+            const float4 a = *reinterpret_cast<const float4*>(tb + size_t(k_sh) * d + c);
+            const float4 b = *reinterpret_cast<const float4*>(tb + size_t(k_sc) * d + c);
+            sh.x += a.x; sh.y += a.y; sh.z += a.z; sh.w += a.w;
+            sc.x += b.x; sc.y += b.y; sc.z += b.z; sc.w += b.w;
+          }
+          float y0 = (v[k].x - mean) * rstd * (1.f + sc.x) + sh.x;
+          float y1 = (v[k].y - mean) * rstd * (1.f + sc.y) + sh.y;
+          float y2 = (v[k].z - mean) * rstd * (1.f + sc.z) + sh.z;
+          float y3 = (v[k].w - mean) * rstd * (1.f + sc.w) + sh.w;
+          orow[lane + 32 * k] = make_uint2(pack_bf16x2(y0, y1), pack_bf16x2(y2, y3));
+        }
     }
-    const float mean = warp_sum(s) / float(d);
-    float q = 0.f;
-#pragma unroll
-    for (int k = 0; k < LN_MAXV; ++k)
-      if (k < nv) {
-        float a = v[k].x - mean, b = v[k].y - mean, c = v[k].z - mean, e = v[k].w - mean;
-        q += (a * a + b * b) + (c * c + e * e);
-      }
-    const float rstd = 1.0f / sqrtf(warp_sum(q) / float(d) + 1e-6f);
-    uint2* orow = reinterpret_cast<uint2*>(out + size_t(r) * d);
-#pragma unroll
-    for (int k = 0; k < LN_MAXV; ++k)
-      if (k < nv) {
-        float y0 = (v[k].x - mean) * rstd * (1.f + sc[k].x) + sh[k].x;
-        float y1 = (v[k].y - mean) * rstd * (1.f + sc[k].y) + sh[k].y;
-        float y2 = (v[k].z - mean) * rstd * (1.f + sc[k].z) + sh[k].z;
-        float y3 = (v[k].w - mean) * rstd * (1.f + sc[k].w) + sh[k].w;
-        orow[lane + 32 * k] = make_uint2(pack_bf16x2(y0, y1), pack_bf16x2(y2, y3));
-      }
+    r += gridDim.x * LN_WARPS;
+    if (r < D) load_row(r);
   }
 }
 
@@ -303,8 +314,10 @@ cudaError_t launch_ln_mod(const float* x, const float* tab, int k_sh, int k_sc, 
                           bf16* out, const RowMap& rm, long long hprev_off, int d, unsigned* err,
                           cudaStream_t st) {
   if (rm.bound <= 0) return cudaSuccess;
-  RC_TRY(launch_k(ln_mod_kernel, dim3(row_grid(rm.bound, LN_WARPS, 1)), dim3(LN_WARPS * 32), 0,
-                  st, x, tab, k_sh, k_sc, it, out, rm, hprev_off, d, err));
+  if (d % 128 || d > 128 * LN_MAXV) return cudaErrorInvalidValue;
+  RC_TRY(launch_k(ln_mod_kernel, dim3(row_grid(rm.bound, LN_WARPS, 1)), dim3(LN_WARPS * 32),
+                  size_t(2) * d * sizeof(float), st, x, tab, k_sh, k_sc, it, out, rm, hprev_off,
+                  d, err));
   count_launches(1);
   return cudaSuccess;
 }
