@@ -644,15 +644,17 @@ scatter_bf16_kernel(const float* __restrict__ src, const __grid_constant__ Items
 
 // Host-tier write-back of one layer: the dirty rows tok[r] of the HBM window
 // [H,K,V][N][d] go to the same rows of the host slice (device-mapped
-// addresses); one warp per row, 16-byte accesses.
-__global__ void __launch_bounds__(RW_WARPS * 32)
+// addresses); one warp per row, 16-byte accesses.  It runs beside the next
+// layer's kernels, which fill the SMs' registers, so its CTAs are single
+// warps that still fit next to them.
+__global__ void __launch_bounds__(32)
 writeback_kernel(const bf16* __restrict__ win, bf16* host, RowMap rm, int d, unsigned* err) {
   pdl_wait();
   pdl_trigger();
   const int D = live_count(rm.count, rm.bound, err);
   const int lane = threadIdx.x & 31;
   const size_t Nd = size_t(rm.n_tokens) * d;
-  for (int r = blockIdx.x * RW_WARPS + (threadIdx.x >> 5); r < D; r += gridDim.x * RW_WARPS) {
+  for (int r = blockIdx.x; r < D; r += gridDim.x) {
     const int i = rm.tok ? __ldg(rm.tok + r) : r;
     if (i < 0 || i >= rm.n_tokens) {
       if (lane == 0) atomicOr(err, DEVERR_INDEX);
@@ -669,8 +671,8 @@ writeback_kernel(const bf16* __restrict__ win, bf16* host, RowMap rm, int d, uns
 cudaError_t launch_writeback(const bf16* win, bf16* host, const RowMap& rm, int d, unsigned* err,
                              cudaStream_t st) {
   if (rm.bound <= 0) return cudaSuccess;
-  RC_TRY(launch_k(writeback_kernel, dim3(row_grid(rm.bound, RW_WARPS, 1)), dim3(RW_WARPS * 32), 0,
-                  st, win, host, rm, d, err));
+  const int grid = rm.bound < 4 * device_sm_count() ? rm.bound : 4 * device_sm_count();
+  RC_TRY(launch_k(writeback_kernel, dim3(grid), dim3(32), 0, st, win, host, rm, d, err));
   count_launches(1);
   return cudaSuccess;
 }
