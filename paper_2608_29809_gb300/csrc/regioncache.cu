@@ -4,6 +4,7 @@
 #include <stdarg.h>
 #include <stdio.h>
 #include <string.h>
+#include <sys/mman.h>
 
 #include <atomic>
 #include <cmath>
@@ -98,13 +99,16 @@ struct rc_cache {
   // l - 1's dirty H, K, V rows back to host memory
   static constexpr int WINDOWS = 3;
   bool host_tier = false;
-  void* host_mem = nullptr;
+  void* host_mem = nullptr;    // the pool: an anonymous mapping, page-locked
+  void* host_map = nullptr;    // the mapping as made (host_mem is aligned inside)
+  size_t host_map_bytes = 0;
   bf16* window = nullptr;  // [WINDOWS][3][N][d]
-  cudaStream_t copy_st = nullptr, wb_st = nullptr;
+  cudaStream_t copy_st = nullptr, copy_st2 = nullptr, wb_st = nullptr;
   cudaEvent_t begin = nullptr;                // step start on the compute stream
   cudaEvent_t h_ready = nullptr;              // a layer's H rows are in its window
   cudaEvent_t wb_done = nullptr;              // the last write-back of a step
-  cudaEvent_t loaded[WINDOWS] = {};           // window filled
+  cudaEvent_t loaded[WINDOWS] = {};           // window filled (H, K part)
+  cudaEvent_t loaded2[WINDOWS] = {};          // window filled (V part)
   cudaEvent_t consumed[WINDOWS] = {};         // window no longer read
 
   size_t slot_elems() const { return size_t(ctx->N) * ctx->d; }
@@ -519,16 +523,18 @@ rc_status rc_cache_create(rc_ctx* c, int sessions, rc_cache** out) {
 void rc_cache_destroy(rc_cache* k) {
   if (!k) return;
   if (k->host_tier) {
-    for (cudaStream_t q : {k->copy_st, k->wb_st})
+    for (cudaStream_t q : {k->copy_st, k->copy_st2, k->wb_st})
       if (q) cudaStreamSynchronize(q);
-    if (k->host_mem) cudaFreeHost(k->host_mem);
+    if (k->host_mem) cudaHostUnregister(k->host_mem);
+    if (k->host_map) munmap(k->host_map, k->host_map_bytes);
     if (k->window) cudaFree(k->window);
     for (cudaEvent_t e : {k->begin, k->h_ready, k->wb_done}) if (e) cudaEventDestroy(e);
     for (int i = 0; i < rc_cache::WINDOWS; ++i) {
       if (k->loaded[i]) cudaEventDestroy(k->loaded[i]);
+      if (k->loaded2[i]) cudaEventDestroy(k->loaded2[i]);
       if (k->consumed[i]) cudaEventDestroy(k->consumed[i]);
     }
-    for (cudaStream_t q : {k->copy_st, k->wb_st})
+    for (cudaStream_t q : {k->copy_st, k->copy_st2, k->wb_st})
       if (q) cudaStreamDestroy(q);
   } else if (k->base) {
     cudaFree(k->base);
@@ -550,18 +556,34 @@ rc_status rc_cache_create_host(rc_ctx* c, int sessions, rc_cache** out) {
   const size_t n = size_t(sessions) * c->T * c->L * 3 * k->slot_elems();
   const size_t n_text = size_t(sessions) * c->L * c->M * 2 * c->d;
   rc_status s = RC_OK;
-  if (cudaHostAlloc(&k->host_mem, n * sizeof(bf16), cudaHostAllocMapped | cudaHostAllocPortable) !=
-      cudaSuccess) {
-    cudaGetLastError();
-    k->host_mem = nullptr;
-    s = fail(RC_ERR_OOM, "pinned host cache of %zu bytes", n * sizeof(bf16));
+  // an anonymous mapping aligned to 512 MB and advised for transparent huge
+  // pages (fewer translations for the copy engines and the write-back),
+  // zero-filled, then page-locked and mapped for the device
+  const size_t bytes = n * sizeof(bf16), huge = size_t(512) << 20;
+  k->host_map_bytes = bytes + huge;
+  void* m = mmap(nullptr, k->host_map_bytes, PROT_READ | PROT_WRITE, MAP_PRIVATE | MAP_ANONYMOUS,
+                 -1, 0);
+  if (m == MAP_FAILED) {
+    k->host_map_bytes = 0;
+    s = fail(RC_ERR_OOM, "host cache mapping of %zu bytes", bytes);
+  } else {
+    k->host_map = m;
+    void* a = reinterpret_cast<void*>((reinterpret_cast<uintptr_t>(m) + huge - 1) & ~(huge - 1));
+    madvise(a, bytes, MADV_HUGEPAGE);  // advice only: small pages work too
+    memset(a, 0, bytes);
+    if (cudaHostRegister(a, bytes, cudaHostRegisterMapped | cudaHostRegisterPortable) !=
+        cudaSuccess) {
+      cudaGetLastError();
+      s = fail(RC_ERR_OOM, "page-locking a host cache of %zu bytes", bytes);
+    } else {
+      k->host_mem = a;
+    }
   }
   void* dev = nullptr;
   if (s == RC_OK && cudaHostGetDevicePointer(&dev, k->host_mem, 0) != cudaSuccess)
     s = fail(RC_ERR_CUDA, "no device address for the host cache");
   if (s == RC_OK) {
     k->base = static_cast<bf16*>(dev);
-    memset(k->host_mem, 0, n * sizeof(bf16));
     s = dalloc(&k->window, rc_cache::WINDOWS * 3 * k->slot_elems(), "cache window");
   }
   if (s == RC_OK) s = dalloc(&k->text, n_text, "text kv");
@@ -570,11 +592,12 @@ rc_status rc_cache_create_host(rc_ctx* c, int sessions, rc_cache** out) {
            cudaSuccess ||
        cudaMemset(k->text, 0, n_text * sizeof(bf16)) != cudaSuccess ||
        cudaStreamCreateWithFlags(&k->copy_st, cudaStreamNonBlocking) != cudaSuccess ||
+       cudaStreamCreateWithFlags(&k->copy_st2, cudaStreamNonBlocking) != cudaSuccess ||
        cudaStreamCreateWithFlags(&k->wb_st, cudaStreamNonBlocking) != cudaSuccess))
     s = fail(RC_ERR_CUDA, "host cache set-up failed");
-  cudaEvent_t* evs[] = {&k->begin,       &k->h_ready,     &k->wb_done,     &k->loaded[0],
-                        &k->loaded[1],   &k->loaded[2],   &k->consumed[0], &k->consumed[1],
-                        &k->consumed[2]};
+  cudaEvent_t* evs[] = {&k->begin,      &k->h_ready,    &k->wb_done,    &k->loaded[0],
+                        &k->loaded[1],  &k->loaded[2],  &k->loaded2[0], &k->loaded2[1],
+                        &k->loaded2[2], &k->consumed[0], &k->consumed[1], &k->consumed[2]};
   for (cudaEvent_t* e : evs)
     if (s == RC_OK && cudaEventCreateWithFlags(e, cudaEventDisableTiming) != cudaSuccess)
       s = fail(RC_ERR_CUDA, "host cache events");
@@ -808,11 +831,18 @@ rc_status rc_block_forward_region(rc_ctx* c, rc_cache* k, int s, int l, int t, f
 static rc_status host_load(rc_cache* k, int s, int t, int l) {
   const size_t Nd = k->slot_elems();
   const int first = l == k->ctx->L - 1 ? 0 : 1, w = l % rc_cache::WINDOWS;
+  // V on a second copy stream (a second copy engine): H (last layer) and K
+  // on the first
   RC_CUDA(cudaStreamWaitEvent(k->copy_st, k->consumed[w], 0), "window wait");
+  RC_CUDA(cudaStreamWaitEvent(k->copy_st2, k->consumed[w], 0), "window wait");
   RC_CUDA(cudaMemcpyAsync(k->window + (size_t(w) * 3 + first) * Nd, k->slot(s, l, t, first),
-                          (3 - first) * Nd * sizeof(bf16), cudaMemcpyDefault, k->copy_st),
+                          (2 - first) * Nd * sizeof(bf16), cudaMemcpyDefault, k->copy_st),
+          "window load");
+  RC_CUDA(cudaMemcpyAsync(k->window + (size_t(w) * 3 + 2) * Nd, k->slot(s, l, t, 2),
+                          Nd * sizeof(bf16), cudaMemcpyDefault, k->copy_st2),
           "window load");
   RC_CUDA(cudaEventRecord(k->loaded[w], k->copy_st), "window event");
+  RC_CUDA(cudaEventRecord(k->loaded2[w], k->copy_st2), "window event");
   return RC_OK;
 }
 
@@ -878,6 +908,7 @@ static rc_status step_items(rc_ctx* c, rc_cache* k, const rc_batch_item* items, 
     if (n != 1) return fail(RC_ERR_INVALID_ARG, "a host-tier cache steps one item at a time");
     RC_CUDA(cudaEventRecord(k->begin, st), "step event");
     RC_CUDA(cudaStreamWaitEvent(k->copy_st, k->begin, 0), "step wait");
+    RC_CUDA(cudaStreamWaitEvent(k->copy_st2, k->begin, 0), "step wait");
     rc_status r = host_load(k, s0, t0, rows > 0 ? 0 : L - 1);
     if (r == RC_OK && rows > 0 && L > 1) r = host_load(k, s0, t0, 1);
     if (r) return r;
@@ -915,6 +946,7 @@ static rc_status step_items(rc_ctx* c, rc_cache* k, const rc_batch_item* items, 
           l > 0 ? (long long)(size_t(wp) * wstride + size_t(l) * wstride) - (long long)(w * wstride)
                 : -1;
       RC_CUDA(cudaStreamWaitEvent(st, k->loaded[w], 0), "window ready");
+      RC_CUDA(cudaStreamWaitEvent(st, k->loaded2[w], 0), "window ready");
       rc_status r = run_block(c, k, l, rm, si, c->lw[l].table, hprev, st, cap,
                               l > 0 ? k->h_ready : nullptr);
       if (r) return r;
@@ -929,6 +961,7 @@ static rc_status step_items(rc_ctx* c, rc_cache* k, const rc_batch_item* items, 
     }
   } else if (host) {
     RC_CUDA(cudaStreamWaitEvent(st, k->loaded[(L - 1) % rc_cache::WINDOWS], 0), "window ready");
+    RC_CUDA(cudaStreamWaitEvent(st, k->loaded2[(L - 1) % rc_cache::WINDOWS], 0), "window ready");
   }
   for (int i = 0; i < n; ++i) {
     const rc_batch_item& it = items[i];
