@@ -444,6 +444,7 @@ def run_ours(args, world, rank, local):
 
     gemm_each = probe(R.RC_PROBE_GEMM, 6, lambda i: wl.step(i, HEADLINE), K)
     att_each = probe(R.RC_PROBE_ATTENTION, 2, lambda i: wl.step(i, HEADLINE), K)
+    ln_each = probe(R.RC_PROBE_LN, 2, lambda i: wl.step(i, HEADLINE), K)
     # the same kernels on all 4096 rows (the dense step)
     Kd = max(2, K // 4)
     gemm_each_d = probe(R.RC_PROBE_GEMM, 6, wl.step_dense, Kd)
@@ -507,6 +508,19 @@ def run_ours(args, world, rank, local):
                                "K steps",
                      "peak_source": f"{peaks['source']} bf16_tflops_sustained"})
     roof_dense, roof_att_dense = kernel_rooflines(d, d.tokens, gemm_each_d, att_each_d, peak)
+    # LayerNorm-modulation launches (HBM-bound class): bytes per launch are
+    # the D rows read as f32 and written as bf16, plus the bf16 H rows the
+    # first LN of a block stores into the cache
+    ln_msa, ln_mlp = ln_each[0::2], ln_each[1::2]
+    ln_bytes = {"msa": 8.0 * D * d.hidden, "mlp": 6.0 * D * d.hidden}
+    ln_us = {"msa": 1e3 * sum(ln_msa) / max(len(ln_msa), 1),
+             "mlp": 1e3 * sum(ln_mlp) / max(len(ln_mlp), 1)}
+    ln_gbs = (ln_bytes["msa"] * len(ln_msa) + ln_bytes["mlp"] * len(ln_mlp)) / (
+        sum(ln_each) / 1e3) / 1e9
+    roof_ln = {"bound": "hbm", "achieved": round(ln_gbs, 1), "peak": peaks["hbm_gbs"],
+               "unit": "GB/s", "frac": round(ln_gbs / peaks["hbm_gbs"], 4), "traffic": None,
+               "launches": len(ln_each), "avg_us": {k: round(v, 2) for k, v in ln_us.items()},
+               "bytes_per_launch": ln_bytes}
     out = {
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
         "steps": K, "warmup": W, "ms_per_step": round(ms_max / K, 4), "higher_is_better": True,
@@ -528,6 +542,7 @@ def run_ours(args, world, rank, local):
         "speedup_vs_dense": {k: round(v / dense, 3) for k, v in sweep.items()},
         "roofline": roofline, "roofline_attention": roof_att,
         "roofline_dense": {"rows": d.tokens, "gemm": roof_dense, "attention": roof_att_dense},
+        "roofline_ln": roof_ln,
         "e2e": e2e, "gpu_launches": int(launches), "clocks": clk,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -390,7 +390,8 @@ rc_status rc_sync(rc_ctx* ctx, rc_stream stream);
 /* Timing probe.  rc_probe_enable(ctx, which, capacity) makes the context
  * record a pair of CUDA events on the launching stream around each of the
  * next `capacity` launches of kernel class `which` (RC_PROBE_GEMM: every
- * tensor-core GEMM of a block; RC_PROBE_ATTENTION: every attention launch);
+ * tensor-core GEMM of a block; RC_PROBE_ATTENTION: every attention launch;
+ * RC_PROBE_LN: both LayerNorm-modulation launches of a block);
  * which = RC_PROBE_OFF disables it.  rc_probe_read waits for the recorded
  * events and returns the summed device time (ms) and the number of launches
  * recorded, then rearms the ring.  rc_probe_read_each does the same but
@@ -400,6 +401,7 @@ rc_status rc_sync(rc_ctx* ctx, rc_stream stream);
 #define RC_PROBE_OFF 0
 #define RC_PROBE_GEMM 1
 #define RC_PROBE_ATTENTION 2
+#define RC_PROBE_LN 3
 rc_status rc_probe_enable(rc_ctx* ctx, int which, int capacity);
 rc_status rc_probe_read(rc_ctx* ctx, double* total_ms, int* launches);
 rc_status rc_probe_read_each(rc_ctx* ctx, float* ms_out, int capacity, int* launches);

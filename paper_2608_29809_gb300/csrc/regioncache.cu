@@ -245,8 +245,11 @@ rc_status run_block(rc_ctx* c, rc_cache* k, int l, const rc::RowMap& rm, const S
 
   // x_hat = LN(x)(1 + scale_msa) + shift_msa; x itself is the previous
   // block's output H^l of the dirty rows, written to their cache rows here
-  RC_CUDA(rc::launch_ln_mod(c->xf, tab, 0, 1, si.its, c->xb, rm, hprev_off, d, c->err, st),
-          "ln_mod(msa)");
+  {
+    Probe pr(c, RC_PROBE_LN, st);
+    RC_CUDA(rc::launch_ln_mod(c->xf, tab, 0, 1, si.its, c->xb, rm, hprev_off, d, c->err, st),
+            "ln_mod(msa)");
+  }
   if (h_stored) RC_CUDA(cudaEventRecord(h_stored, st), "H stored");
   // [q | k | v] = x_hat W_qkv^T + b; k, v rows go straight to cache rows tok[r]
   rc::GemmEpi e{};
@@ -331,8 +334,11 @@ rc_status run_block(rc_ctx* c, rc_cache* k, int l, const rc::RowMap& rm, const S
                             e, st), "gemm(xo)");
   }
   // MLP
-  RC_CUDA(rc::launch_ln_mod(c->xf, tab, 3, 4, si.its, c->xb, rm, -1, d, c->err, st),
-          "ln_mod(mlp)");
+  {
+    Probe pr(c, RC_PROBE_LN, st);
+    RC_CUDA(rc::launch_ln_mod(c->xf, tab, 3, 4, si.its, c->xb, rm, -1, d, c->err, st),
+            "ln_mod(mlp)");
+  }
   e = rc::GemmEpi{};
   e.mode = rc::EPI_GELU_BF16;
   e.bias = w.b_1;
@@ -1197,7 +1203,7 @@ rc_status rc_attention(rc_ctx* c, const void* Q, int ldq, const void* K, const v
 
 rc_status rc_probe_enable(rc_ctx* c, int which, int capacity) {
   if (!c) return fail(RC_ERR_INVALID_ARG, "rc_probe_enable: null context");
-  if (which < RC_PROBE_OFF || which > RC_PROBE_ATTENTION || capacity < 0 || capacity > 1 << 20)
+  if (which < RC_PROBE_OFF || which > RC_PROBE_LN || capacity < 0 || capacity > 1 << 20)
     return fail(RC_ERR_INVALID_ARG, "rc_probe_enable: which %d capacity %d", which, capacity);
   probe_free(c);
   if (which == RC_PROBE_OFF) return RC_OK;

@@ -305,7 +305,7 @@ def rc_sync(ctx, stream=None):
     _check(_lib.rc_sync(ctx, _stream(stream)))
 
 
-RC_PROBE_OFF, RC_PROBE_GEMM, RC_PROBE_ATTENTION = 0, 1, 2
+RC_PROBE_OFF, RC_PROBE_GEMM, RC_PROBE_ATTENTION, RC_PROBE_LN = 0, 1, 2, 3
 
 
 def rc_probe_enable(ctx, which, capacity):
