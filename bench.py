@@ -309,6 +309,78 @@ class Workload:
                 "step": "rc_localize_mask + rc_step(SPARSE) on rc_cache_create_host"}
 
 
+def rate_batched(R, args, world, dev, K, W, n=8):
+    """Batched serving: n concurrent 512 px sessions (1024 tokens, 28 blocks),
+    each at its own timestep with its own text and a ragged dirty fraction
+    from U(2 %, 35 %); one rc_step_batched per step against n rc_step calls."""
+    from dataclasses import replace
+    d = replace(synth.PIXART_512, timesteps=args.resident_steps)
+    seed = SEED + 11
+    w = synth.make_weights(d, seed, device=dev)
+    model = R.Model(d, w, sessions=n, device=dev, max_batch=n)
+    try:
+        for s in range(n):
+            R.rc_set_text(model.ctx, model.cache, s, synth.make_text(d, seed + s, dev))
+            for t in range(d.timesteps):
+                for l in range(d.layers):
+                    H, K_, V = synth.make_cache_slice(d, seed, s, l, t, device=dev)
+                    R.rc_cache_fill(model.cache, s, l, t, H, K_, V)
+        tv, ab = synth.ddim_tables(d.timesteps)
+        R.rc_set_schedule(model.ctx, tv, ab)
+        rng = np.random.default_rng(seed)
+        fracs = rng.uniform(0.02, 0.35, size=n)
+        N = d.tokens
+        idx, cnt, lat0, lat = [], [], [], []
+        for s in range(n):
+            blobs = synth.ellipse_blobs(d, seed + s, float(fracs[s]))
+            A, ids = synth.indicator_scores(d, blobs, seed + s)
+            ws = torch.empty(R.rc_localize_workspace_size(N, len(ids)), dtype=torch.uint8,
+                             device=dev)
+            mask = torch.zeros(N, dtype=torch.uint8, device=dev)
+            idx.append(torch.zeros(N, dtype=torch.int32, device=dev))
+            cnt.append(torch.zeros(1, dtype=torch.int32, device=dev))
+            R.rc_localize_mask(torch.from_numpy(A).to(dev), A.shape[0], N, A.shape[2], d.grid_h,
+                               d.grid_w, ids, 0.5, 0, mask, idx[s], cnt[s], ws)
+            lat0.append(synth.make_latent(d, seed + s, dev))
+            lat.append(lat0[s].clone())
+        torch.cuda.synchronize()
+        dirty = [int(c.item()) for c in cnt]
+        sparse = np.full(d.timesteps, R.RC_MODE_SPARSE, np.uint8)
+
+        def items(i):
+            out = []
+            for s in range(n):
+                t = (i + 3 * s) % d.timesteps
+                if t == 0:
+                    lat[s].copy_(lat0[s])
+                out.append(dict(session=s, latent=lat[s], t=t, mode=R.RC_MODE_SPARSE,
+                                dirty_idx=idx[s], D=-1, dirty_count=cnt[s]))
+            return out
+
+        def batched(i):
+            R.rc_step_batched(model.ctx, model.cache, items(i))
+
+        def one_by_one(i):
+            for it in items(i):
+                R.rc_step(model.ctx, model.cache, it["session"], it["latent"], it["t"], sparse,
+                          it["dirty_idx"], -1, it["dirty_count"])
+
+        k = max(2, K // 2)
+        m = timed(batched, k, W, world)
+        rate_b = n * k * world / (max_over_ranks(m, world) / 1e3)
+        m = timed(one_by_one, k, W, world)
+        rate_1 = n * k * world / (max_over_ranks(m, world) / 1e3)
+        R.rc_sync(model.ctx)
+    finally:
+        model.close()
+    return {"workload": f"batched serving: {n} sessions x pixart-alpha-512px ({d.tokens} tokens, "
+                        f"{d.layers} blocks, {d.timesteps} timesteps)",
+            "dirty_tokens": dirty, "session_steps_per_s": round(rate_b, 3),
+            "session_steps_per_s_one_by_one": round(rate_1, 3),
+            "speedup_of_batching": round(rate_b / rate_1, 3),
+            "step": "rc_step_batched over all sessions (vs one rc_step per session)"}
+
+
 def rate_2048(R, args, world, dev, K, W):
     """Headline-style steps (20 % dirty, graphs) and dense steps of the 2048 px
     model (128 x 128 = 16 384 tokens, all 20 timesteps resident)."""
@@ -462,6 +534,11 @@ def run_ours(args, world, rank, local):
     capture = max(2, K // 2) * world / (max_over_ranks(m, world) / 1e3)
     R.rc_sync(wl.model.ctx)
 
+    # batched serving of 8 concurrent 512 px sessions
+    batch = None
+    if not args.no_batched:
+        batch = rate_batched(R, args, world, dev, K, W)
+
     # the same step at 2048 px (16 384 tokens, 63.4 GB cache resident)
     big = None
     if not args.no_2048:
@@ -538,6 +615,7 @@ def run_ours(args, world, rank, local):
         "dense_capture_steps_per_s": round(capture, 3),
         "host_tier": host_tier,
         "pixart2048": big,
+        "batched_serving": batch,
         "direct_steps_per_s": round(direct, 3),
         "speedup_vs_dense": {k: round(v / dense, 3) for k, v in sweep.items()},
         "roofline": roofline, "roofline_attention": roof_att,
@@ -656,6 +734,8 @@ def main():
     ap.add_argument("--cpu-layers", type=int, default=2)
     ap.add_argument("--quick", action="store_true",
                     help="headline only: no attention probe, sweep, dense, e2e or cpu baseline")
+    ap.add_argument("--no-batched", action="store_true",
+                    help="skip the batched-serving measurement (8 x 512 px sessions, 32 GB)")
     ap.add_argument("--no-2048", action="store_true",
                     help="skip the 2048 px (16 384-token, 63 GB cache) measurement")
     ap.add_argument("--no-host-tier", action="store_true",
