@@ -530,6 +530,209 @@ done:
   }
 }
 
+// ------------------------------------------------- short keys (text cross-attention)
+// All Nk <= 128 keys of a (query tile, head) in one pass, one CTA per pair:
+// S = Q K^T (M = 128, N = 128) in TMEM, an exact softmax per row (no running
+// max, no rescaling), P (bf16) written over S, O = P V (N = DHP, 8 MMAs of 16
+// keys, P read from TMEM as the A operand), O normalised and stored.  The
+// text cross-attention of a block has 120 keys: the general kernel's two
+// dependent 64-key rounds become one.
+constexpr int XK = 128;  // keys per pass
+template <int DH>
+struct XCfg {
+  using C = ACfg<DH>;
+  static constexpr int K128 = XK * 128, K32 = C::TAIL ? XK * 32 : 0;
+  static constexpr int V_ATOM = XK * 128;  // one MN-major SW128 atom of 64 head-dim columns
+  static constexpr int V_BYTES = C::TAIL ? 2 * V_ATOM : V_ATOM;
+  static constexpr int BYTES = C::Q_BYTES + K128 + K32 + V_BYTES;
+  // rounded up so that at most two CTAs share an SM (2 x 256 TMEM columns)
+  static constexpr size_t SMEM = 100 * 1024;
+  static_assert(size_t(BYTES) + 1024 + 64 <= SMEM, "cross-attention tiles exceed the request");
+  static constexpr uint32_t IDESC_S = (1u << 4) | (1u << 7) | (1u << 10) |
+                                      (uint32_t(XK >> 3) << 17) | (uint32_t(BQ >> 4) << 24);
+};
+
+template <int DH, bool CAP>
+__global__ void __launch_bounds__(128, 2)
+xattn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmQt,
+                const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmKt,
+                const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnItems ai,
+                int Nk, bf16* __restrict__ O, int ldo, int heads, RowMap rm, float scale_log2,
+                unsigned* err, const __grid_constant__ AttnCapture cap) {
+  using C = ACfg<DH>;
+  using X = XCfg<DH>;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint8_t* sQ = smem;
+  uint8_t* sK = sQ + C::Q_BYTES;
+  uint8_t* sV = sK + X::K128 + X::K32;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sV + X::V_BYTES);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const uint32_t load_bar = saddr(bars), mma_bar = saddr(bars + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    mbar_init(load_bar, 1);
+    mbar_init(mma_bar, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmQ)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+  }
+  if (warp == 0) tmem_alloc(saddr(tmem_slot), 256);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const uint32_t tS = tmem_base, tO = tmem_base + XK;  // P is written over S
+
+  pdl_wait();
+  pdl_trigger();
+  const int D = live_count(rm.count, rm.bound, err);
+  const int qtiles = query_tiles(rm, ai.n, D);
+  const int qt = int(blockIdx.x) / heads, h = int(blockIdx.x) - (int(blockIdx.x) / heads) * heads;
+  bool ok = qt < qtiles;
+  TileLoc tl{0, 0, 0};
+  if (ok) tl = locate_tile(rm, ai.n, D, qt);
+  const int row = warp * 32 + lane;
+  const uint32_t lane_off = uint32_t(warp * 32) << 16;
+  if (ok && threadIdx.x == 0) {
+    // ---- loads: Q (128 rows of the tile), K and V (128 keys of the item)
+    const int krow = ai.krow[tl.item], vrow = ai.vrow[tl.item];
+    mbar_expect_tx(load_bar, X::BYTES);
+    tma_load_3d(saddr(sQ), &tmQ, load_bar, 0, h, tl.row0);
+    if (C::TAIL) tma_load_3d(saddr(sQ + C::Q128), &tmQt, load_bar, 64, h, tl.row0);
+    tma_load_3d(saddr(sK), &tmK, load_bar, 0, h, krow);
+    if (C::TAIL) tma_load_3d(saddr(sK + X::K128), &tmKt, load_bar, 64, h, krow);
+    tma_load_3d(saddr(sV), &tmV, load_bar, 0, h, vrow);
+    if (C::TAIL) tma_load_3d(saddr(sV + X::V_ATOM), &tmV, load_bar, 64, h, vrow);
+    // ---- S = Q K^T over the 80 (72 + zero) head dims
+    if (mbar_sleep(load_bar, 0, abort_flag)) {
+      tc_fence_after();
+      const uint64_t dq = sw128_desc(saddr(sQ)), dk = sw128_desc(saddr(sK));
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk)
+        umma_bf16(tS, dq + 2 * kk, dk + 2 * kk, X::IDESC_S, kk > 0 ? 1u : 0u);
+      if (C::TAIL)
+        umma_bf16(tS, sw32_kmajor_desc(saddr(sQ + C::Q128)), sw32_kmajor_desc(saddr(sK + X::K128)),
+                  X::IDESC_S, 1u);
+      umma_commit(mma_bar);
+    } else {
+      *abort_flag = 1;
+    }
+  }
+  // ---- exact softmax of this thread's row
+  if (ok) ok = mbar_sleep_warp(mma_bar, 0, abort_flag);
+  float l = 0.f;
+  if (ok) {
+    tc_fence_after();
+    uint32_t r[XK];
+#pragma unroll
+    for (int i = 0; i < XK / 16; ++i) tmem_ld16_nowait(tS + lane_off + 16u * i, r + 16 * i);
+    tmem_wait_ld();
+#pragma unroll
+    for (int c = 0; c < XK; ++c)
+      if (c >= Nk) r[c] = __float_as_uint(-INFINITY);
+    float mx8[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) mx8[q] = __uint_as_float(r[q]);
+#pragma unroll
+    for (int c = 8; c < XK; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(r[c]));
+    const float m = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                          fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]))) * scale_log2;
+    const uint64_t sc2 = f32x2(scale_log2, scale_log2), nm2 = f32x2(-m, -m);
+    uint64_t sum2[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) sum2[q] = f32x2(0.f, 0.f);
+#pragma unroll
+    for (int c = 0; c < XK; c += 2) {
+      float a, b;
+      unpack_f32x2(fma_f32x2(f32x2(__uint_as_float(r[c]), __uint_as_float(r[c + 1])), sc2, nm2),
+                   a, b);
+      a = ex2_ftz(a);
+      b = ex2_ftz(b);
+      r[c] = __float_as_uint(a);
+      r[c + 1] = __float_as_uint(b);
+      sum2[(c >> 1) & 3] = add_f32x2(sum2[(c >> 1) & 3], f32x2(a, b));
+    }
+    float s0, s1, s2, s3, s4, s5, s6, s7;
+    unpack_f32x2(sum2[0], s0, s1);
+    unpack_f32x2(sum2[1], s2, s3);
+    unpack_f32x2(sum2[2], s4, s5);
+    unpack_f32x2(sum2[3], s6, s7);
+    l = ((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7));
+    if (CAP && cap.n && row < tl.rows) {  // the localisation scores of the listed keys
+      const int qrow = tl.row0 + row;
+      const int tok = rm.tok ? __ldg(rm.tok + qrow) : qrow;
+      const float inv_l = l > 0.f ? 1.f / l : 0.f;
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        if (q < cap.n) {
+          float pq = 0.f;
+#pragma unroll
+          for (int c = 0; c < XK; ++c)
+            if (c == cap.id[q]) pq = __uint_as_float(r[c]);
+          atomicAdd(cap.out + size_t(tok) * cap.ldo + cap.id[q], cap.w * pq * inv_l);
+        }
+    }
+    // P (bf16 pairs) over the first 64 columns of S: the A operand of P V
+#pragma unroll
+    for (int h2 = 0; h2 < XK / 32; ++h2) {
+      uint32_t w[16];
+#pragma unroll
+      for (int c = 0; c < 16; ++c)
+        w[c] = pack_bf16x2(__uint_as_float(r[32 * h2 + 2 * c]),
+                           __uint_as_float(r[32 * h2 + 2 * c + 1]));
+      tmem_st16(tS + lane_off + 16u * h2, w);
+    }
+    tmem_wait_st();
+  }
+  tc_fence_before();
+  __syncthreads();  // every row's P is in TMEM
+  if (ok && threadIdx.x == 0) {
+    tc_fence_after();
+    const uint64_t dv = C::TAIL ? sw128_mnmajor_desc_lbo(saddr(sV), X::V_ATOM)
+                                : sw128_mnmajor_desc(saddr(sV));
+#pragma unroll
+    for (int kk = 0; kk < XK / 16; ++kk)
+      umma_bf16_ta(tO, tS + 8 * kk, dv + 128 * kk, C::IDESC_PV, kk > 0 ? 1u : 0u);
+    umma_commit(mma_bar);
+  }
+  if (ok) ok = mbar_sleep_warp(mma_bar, 1, abort_flag);
+  if (ok) {
+    tc_fence_after();
+    uint32_t o[C::DHP];
+#pragma unroll
+    for (int i = 0; i < C::DHP / 16; ++i) tmem_ld16_nowait(tO + lane_off + 16u * i, o + 16 * i);
+    tmem_wait_ld();
+    if (row < tl.rows) {
+      const float inv = l > 0.f ? 1.f / l : 0.f;
+      uint4* dst = reinterpret_cast<uint4*>(O + size_t(tl.row0 + row) * ldo + h * DH);
+#pragma unroll
+      for (int c8 = 0; c8 < DH / 8; ++c8) {
+        uint4 w;
+        w.x = pack_bf16x2(__uint_as_float(o[8 * c8 + 0]) * inv, __uint_as_float(o[8 * c8 + 1]) * inv);
+        w.y = pack_bf16x2(__uint_as_float(o[8 * c8 + 2]) * inv, __uint_as_float(o[8 * c8 + 3]) * inv);
+        w.z = pack_bf16x2(__uint_as_float(o[8 * c8 + 4]) * inv, __uint_as_float(o[8 * c8 + 5]) * inv);
+        w.w = pack_bf16x2(__uint_as_float(o[8 * c8 + 6]) * inv, __uint_as_float(o[8 * c8 + 7]) * inv);
+        dst[c8] = w;
+      }
+    }
+  }
+  if (qt < qtiles && (!ok || *abort_flag)) {
+    if (threadIdx.x == 0) atomicOr(err, DEVERR_TIMEOUT);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, 256);
+  }
+}
+
 // Merge of the pieces of the pairs that stream-K cut: one warp per (pair,
 // query row).  The pieces come from CTAs cta_of(first block) .. cta_of(last
 // block); a CTA's piece is its first (slot 0) when its range starts inside
@@ -716,7 +919,19 @@ int device_sms_attn() {
     if (cudaFuncSetAttribute(attn_tc_kernel<72>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              int(ACfg<72>::SMEM)) != cudaSuccess ||
         cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             int(ACfg<64>::SMEM)) != cudaSuccess)
+                             int(ACfg<64>::SMEM)) != cudaSuccess ||
+        cudaFuncSetAttribute(xattn_tc_kernel<72, false>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, int(XCfg<72>::SMEM)) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(xattn_tc_kernel<72, true>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, int(XCfg<72>::SMEM)) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(xattn_tc_kernel<64, false>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, int(XCfg<64>::SMEM)) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(xattn_tc_kernel<64, true>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, int(XCfg<64>::SMEM)) !=
+            cudaSuccess)
       return 0;
     sms[dev] = v;
   }
@@ -763,6 +978,23 @@ cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* 
       if (capture->id[q] < 0 || capture->id[q] >= Nk || capture->id[q] >= capture->ldo)
         return cudaErrorInvalidValue;
     cap = *capture;
+  }
+  if (Nk <= XK) {
+    // short key sets (the text cross-attention): one pass per (query tile,
+    // head), a CTA each; tiles beyond the live count exit at once
+    CUtensorMap xk, xkt, xv;
+    RC_TRY(head_map(K, kv_rows, ldkv, heads, dh, 64, XK, &xk));
+    RC_TRY(head_map(K, kv_rows, ldkv, heads, dh, 16, XK, &xkt));
+    RC_TRY(head_map(V, kv_rows, ldkv, heads, dh, 64, XK, &xv));
+    const long long xgrid = ((long long)(rm.bound + BQ - 1) / BQ + ai.n - 1) * heads;
+    if (xgrid >= (1ll << 31)) return cudaErrorInvalidValue;
+    auto xk_fn = dh == 72 ? (cap.n ? xattn_tc_kernel<72, true> : xattn_tc_kernel<72, false>)
+                          : (cap.n ? xattn_tc_kernel<64, true> : xattn_tc_kernel<64, false>);
+    RC_TRY(launch_k(xk_fn, dim3(unsigned(xgrid)), dim3(128),
+                    dh == 72 ? XCfg<72>::SMEM : XCfg<64>::SMEM, st, tq, tqt, xk, xkt, xv, ai, Nk,
+                    O, ldo, heads, rm, scale_log2, err, cap));
+    count_launches(1);
+    return cudaSuccess;
   }
   const int grid = CTAS_PER_SM * sms;
   {
