@@ -49,14 +49,17 @@ L2_NOTE = ("inputs larger than L2: each step streams 1.04 GB of weights and a di
 
 
 def linear_flops_per_token_block(d: synth.Dims) -> float:
-    """2 x (3h^2 + h^2 + h^2 + h^2 + hF + Fh) multiply-adds per dirty token and block."""
+    """2 x (3h^2 + h^2 + h^2 + hF + Fh) per dirty token and block: the GEMM
+    launches (QKV, out, cross-out, fc1, fc2).  The cross-query projection
+    (2 h^2) runs inside the cross-attention kernel, folded into the text keys."""
     h, F = d.hidden, d.mlp
-    return 2.0 * (6 * h * h + 2 * h * F)
+    return 2.0 * (5 * h * h + 2 * h * F)
 
 
 def attn_flops_per_token_block(d: synth.Dims) -> float:
-    """Self-attention (4 N h) plus cross-attention (4 M h) per dirty token and block."""
-    return 4.0 * d.tokens * d.hidden + 4.0 * d.text_len * d.hidden
+    """Self-attention (4 N h) plus cross-attention with its query projection
+    (4 M h + 2 h^2) per dirty token and block."""
+    return 4.0 * d.tokens * d.hidden + 4.0 * d.text_len * d.hidden + 2.0 * d.hidden * d.hidden
 
 
 KERNEL_SOURCES = {
@@ -411,14 +414,14 @@ def kernel_rooflines(d, D, gemm_each, att_each, peak):
     D dirty rows per launch over the CUDA-event launch durations."""
     gemm_ms, gemm_n = sum(gemm_each), len(gemm_each)
     att_ms, att_n = sum(att_each), len(att_each)
-    steps = gemm_n / (6 * d.layers)
-    lin_flops_launch = linear_flops_per_token_block(d) * D / 6
+    steps = gemm_n / (5 * d.layers)
+    lin_flops_launch = linear_flops_per_token_block(d) * D / 5
     gemm_tflops = linear_flops_per_token_block(d) * D * d.layers * steps / (gemm_ms / 1e3) / 1e12
     att_tflops = attn_flops_per_token_block(d) * D * d.layers * steps / (att_ms / 1e3) / 1e12
     roofline = {"bound": "tensor", "achieved": round(gemm_tflops, 2), "peak": peak,
                 "unit": "TFLOP/s", "frac": round(gemm_tflops / peak, 4),
                 "traffic": profiled_traffic("gemm"),
-                "kernel": "gemm (QKV, out, cross-q, cross-out, fc1, fc2 of every block)",
+                "kernel": "gemm (QKV, out, cross-out, fc1, fc2 of every block)",
                 "launches": gemm_n, "avg_launch_ms": round(gemm_ms / max(gemm_n, 1), 5),
                 "flops_per_launch": lin_flops_launch}
     roof_att = {"bound": "tensor", "achieved": round(att_tflops, 2), "peak": peak,
@@ -428,11 +431,11 @@ def kernel_rooflines(d, D, gemm_each, att_each, peak):
     # per-launch breakdown: launches come in block order (GEMMs: QKV, out,
     # cross-q, cross-out, fc1, fc2; attention: self, cross)
     h, F = d.hidden, d.mlp
-    gemm_shapes = [("qkv", 3 * h, h), ("out", h, h), ("cross_q", h, h), ("cross_out", h, h),
-                   ("fc1", F, h), ("fc2", h, F)]
+    gemm_shapes = [("qkv", 3 * h, h), ("out", h, h), ("cross_out", h, h), ("fc1", F, h),
+                   ("fc2", h, F)]
     per_gemm = {}
     for j, (name, n_, k_) in enumerate(gemm_shapes):
-        ts = gemm_each[j::6]
+        ts = gemm_each[j::5]
         us = 1e3 * sum(ts) / max(len(ts), 1)
         per_gemm[name] = {"shape": [D, n_, k_], "avg_us": round(us, 2),
                           "tflops": round(2.0 * D * n_ * k_ / (us * 1e-6) / 1e12, 1)}
@@ -440,8 +443,9 @@ def kernel_rooflines(d, D, gemm_each, att_each, peak):
     for j, (name, nk) in enumerate([("self", d.tokens), ("cross", d.text_len)]):
         ts = att_each[j::2]
         us = 1e3 * sum(ts) / max(len(ts), 1)
+        fl = 4.0 * D * nk * h + (2.0 * D * h * h if name == "cross" else 0.0)
         per_attn[name] = {"queries": D, "keys": nk, "avg_us": round(us, 2),
-                          "tflops": round(4.0 * D * nk * h / (us * 1e-6) / 1e12, 1)}
+                          "tflops": round(fl / (us * 1e-6) / 1e12, 1)}
     roofline["per_gemm"] = per_gemm
     roof_att["per_launch"] = per_attn
     return roofline, roof_att
@@ -514,12 +518,12 @@ def run_ours(args, world, rank, local):
         R.rc_probe_enable(wl.model.ctx, R.RC_PROBE_OFF, 0)
         return each
 
-    gemm_each = probe(R.RC_PROBE_GEMM, 6, lambda i: wl.step(i, HEADLINE), K)
+    gemm_each = probe(R.RC_PROBE_GEMM, 5, lambda i: wl.step(i, HEADLINE), K)
     att_each = probe(R.RC_PROBE_ATTENTION, 2, lambda i: wl.step(i, HEADLINE), K)
     ln_each = probe(R.RC_PROBE_LN, 2, lambda i: wl.step(i, HEADLINE), K)
     # the same kernels on all 4096 rows (the dense step)
     Kd = max(2, K // 4)
-    gemm_each_d = probe(R.RC_PROBE_GEMM, 6, wl.step_dense, Kd)
+    gemm_each_d = probe(R.RC_PROBE_GEMM, 5, wl.step_dense, Kd)
     att_each_d = probe(R.RC_PROBE_ATTENTION, 2, wl.step_dense, Kd)
 
     # sweep and dense baseline (graphs, like the headline)

@@ -733,6 +733,284 @@ xattn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__
   }
 }
 
+// ------------------------------------ cross-attention with the query folded in
+// The text keys and W_xq are fixed for a turn, so the query projection can be
+// folded into the keys once per turn: q'_h K_h^T = (xb W_xq,h^T + b_h) K_h^T =
+// xb G_h^T + kb_h, G_h = K_h W_xq,h, kb_h = K_h b_h (a reassociation of the
+// same products).  The cross-query GEMM then disappears from the block.
+
+// G and kb of one (session, layer): block (h, 8-key group), thread = 9
+// columns of G, 8 keys each, f32 accumulation over the head's dh dims.
+constexpr int FOLD_KEYS = 8, FOLD_THREADS = 128, FOLD_COLS = 12;  // d <= 128 * 12
+__global__ void __launch_bounds__(FOLD_THREADS)
+xq_fold_kernel(const bf16* __restrict__ Kt, int ldk, const bf16* __restrict__ Wq,
+               const float* __restrict__ bq, int M, int dh, int d, bf16* __restrict__ G,
+               float* __restrict__ kb) {
+  pdl_wait();
+  pdl_trigger();
+  __shared__ float sk[FOLD_KEYS][80];
+  const int h = blockIdx.x, r0 = blockIdx.y * FOLD_KEYS;
+  for (int e = threadIdx.x; e < FOLD_KEYS * dh; e += FOLD_THREADS) {
+    const int r = e / dh, j = e - (e / dh) * dh;
+    sk[r][j] = r0 + r < M ? __bfloat162float(Kt[size_t(r0 + r) * ldk + h * dh + j]) : 0.f;
+  }
+  __syncthreads();
+  const int nc = d / FOLD_THREADS;
+  float acc[FOLD_KEYS][FOLD_COLS];
+#pragma unroll
+  for (int r = 0; r < FOLD_KEYS; ++r)
+#pragma unroll
+    for (int i = 0; i < FOLD_COLS; ++i) acc[r][i] = 0.f;
+  for (int j = 0; j < dh; ++j) {
+    const bf16* wrow = Wq + size_t(h * dh + j) * d;
+    float w[FOLD_COLS];
+#pragma unroll
+    for (int i = 0; i < FOLD_COLS; ++i)
+      w[i] = i < nc ? __bfloat162float(wrow[threadIdx.x + FOLD_THREADS * i]) : 0.f;
+#pragma unroll
+    for (int r = 0; r < FOLD_KEYS; ++r)
+#pragma unroll
+      for (int i = 0; i < FOLD_COLS; ++i) acc[r][i] = fmaf(sk[r][j], w[i], acc[r][i]);
+  }
+#pragma unroll
+  for (int r = 0; r < FOLD_KEYS; ++r) {
+    if (r0 + r >= M) break;
+    bf16* grow = G + (size_t(h) * XQ_KEYS + r0 + r) * d;
+#pragma unroll
+    for (int i = 0; i < FOLD_COLS; ++i)
+      if (i < nc) grow[threadIdx.x + FOLD_THREADS * i] = __float2bfloat16_rn(acc[r][i]);
+  }
+  if (threadIdx.x < FOLD_KEYS && r0 + int(threadIdx.x) < M) {
+    float a = 0.f;
+    for (int j = 0; j < dh; ++j) a = fmaf(sk[threadIdx.x][j], bq[h * dh + j], a);
+    kb[size_t(h) * XQ_KEYS + r0 + threadIdx.x] = a;
+  }
+}
+
+// One (query tile, head) per CTA: S = xb_tile G_h^T accumulated over d in
+// 64-column k-blocks (TMA ring, M = 128, N = 128), then the softmax of
+// (S + kb) / sqrt(dh) per row, P over S in TMEM, O = P V, O / l stored.
+constexpr int XF_STAGES = 4;
+template <int DH>
+struct XFCfg {
+  using C = ACfg<DH>;
+  static constexpr int STAGE_A = BQ * 128, STAGE_G = XK * 128;
+  static constexpr int STAGE = STAGE_A + STAGE_G;
+  static constexpr int V_ATOM = XK * 128;
+  static constexpr int V_BYTES = C::TAIL ? 2 * V_ATOM : V_ATOM;
+  static constexpr size_t SMEM =
+      size_t(XF_STAGES) * STAGE + V_BYTES + XK * 4 + 1024 + 256;
+  static constexpr uint32_t IDESC_S = (1u << 4) | (1u << 7) | (1u << 10) |
+                                      (uint32_t(XK >> 3) << 17) | (uint32_t(BQ >> 4) << 24);
+};
+
+template <int DH, bool CAP>
+__global__ void __launch_bounds__(192, 1)
+xfused_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmG,
+                 const __grid_constant__ CUtensorMap tmV, const float* __restrict__ kb,
+                 const __grid_constant__ XqItems xi, int Nk, int d, bf16* __restrict__ O,
+                 int ldo, int heads, RowMap rm, float scale_log2, unsigned* err,
+                 const __grid_constant__ AttnCapture cap) {
+  using C = ACfg<DH>;
+  using X = XFCfg<DH>;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint8_t* sV = smem + XF_STAGES * X::STAGE;
+  float* s_kb = reinterpret_cast<float*>(sV + X::V_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_kb + XK);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * XF_STAGES + 5);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const uint32_t full0 = saddr(bars), empty0 = saddr(bars + XF_STAGES);
+  const uint32_t v_full = saddr(bars + 2 * XF_STAGES), s_full = v_full + 8, p_ready = v_full + 16,
+                 o_full = v_full + 24, kb_ready = v_full + 32;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < XF_STAGES; ++i) {
+      mbar_init(full0 + 8 * i, 1);
+      mbar_init(empty0 + 8 * i, 1);
+    }
+    mbar_init(v_full, 1);
+    mbar_init(s_full, 1);
+    mbar_init(p_ready, 128);
+    mbar_init(o_full, 1);
+    mbar_init(kb_ready, 128);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  pdl_wait();
+  pdl_trigger();
+  const int D = live_count(rm.count, rm.bound, err);
+  const int qtiles = query_tiles(rm, xi.n, D);
+  const int qt = int(blockIdx.x) / heads, h = int(blockIdx.x) - (int(blockIdx.x) / heads) * heads;
+  // the grid covers the bound of the query tiles: CTAs past the live ones
+  // leave before taking tensor memory
+  if (qt >= qtiles) return;
+  const bool live = true;
+  const TileLoc tl = locate_tile(rm, xi.n, D, qt);
+  if (warp == 1) tmem_alloc(saddr(tmem_slot), 256);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const uint32_t tS = tmem_base, tO = tmem_base + XK;  // P is written over S
+  const int nkb = d / 64;
+  bool ok = live;
+  if (live && warp == 0 && lane == 0) {
+    // ------------------------------------------------------------ TMA
+    const int grow = xi.grow[tl.item] + h * XK;
+    mbar_expect_tx(v_full, X::V_BYTES);
+    tma_load_3d(saddr(sV), &tmV, v_full, 0, h, xi.vrow[tl.item]);
+    if (C::TAIL) tma_load_3d(saddr(sV + X::V_ATOM), &tmV, v_full, 64, h, xi.vrow[tl.item]);
+    for (int k = 0; k < nkb; ++k) {
+      const int st = k % XF_STAGES;
+      if (!mbar_wait(empty0 + 8 * st, ((k / XF_STAGES) & 1) ^ 1, abort_flag)) {
+        *abort_flag = 1;
+        break;
+      }
+      mbar_expect_tx(full0 + 8 * st, X::STAGE);
+      uint8_t* base = smem + st * X::STAGE;
+      tma_load_3d(saddr(base), &tmA, full0 + 8 * st, 0, k, tl.row0);
+      tma_load_3d(saddr(base + X::STAGE_A), &tmG, full0 + 8 * st, 0, k, grow);
+    }
+  } else if (live && warp == 1 && lane == 0) {
+    // ------------------------------------------------------------ MMA
+    const uint64_t da = sw128_desc(saddr(smem)), dg = sw128_desc(saddr(smem + X::STAGE_A));
+    bool good = true;
+    for (int k = 0; k < nkb && good; ++k) {
+      const int st = k % XF_STAGES;
+      if (!mbar_wait(full0 + 8 * st, (k / XF_STAGES) & 1, abort_flag)) {
+        good = false;
+        break;
+      }
+      tc_fence_after();
+      const uint64_t so = uint64_t((st * X::STAGE) >> 4);
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk)
+        umma_bf16(tS, da + so + 2 * kk, dg + so + 2 * kk, X::IDESC_S,
+                  (k > 0 || kk > 0) ? 1u : 0u);
+      umma_commit(empty0 + 8 * st);
+    }
+    if (good) umma_commit(s_full);
+    // P V once every row's P is in TMEM and V has landed
+    if (good && mbar_wait(p_ready, 0, abort_flag) && mbar_wait(v_full, 0, abort_flag)) {
+      tc_fence_after();
+      const uint64_t dv = C::TAIL ? sw128_mnmajor_desc_lbo(saddr(sV), X::V_ATOM)
+                                  : sw128_mnmajor_desc(saddr(sV));
+#pragma unroll
+      for (int kk = 0; kk < XK / 16; ++kk)
+        umma_bf16_ta(tO, tS + 8 * kk, dv + 128 * kk, C::IDESC_PV, kk > 0 ? 1u : 0u);
+      umma_commit(o_full);
+    } else {
+      *abort_flag = 1;
+    }
+  } else if (live && warp >= 2) {
+    // ------------------------------------------------------------ softmax
+    const int sp = warp & 3;
+    const int row = sp * 32 + lane;
+    const uint32_t lane_off = uint32_t(sp * 32) << 16;
+    const int t128 = threadIdx.x - 64;  // 0 .. 127
+    s_kb[t128] = t128 < Nk ? kb[size_t(xi.grow[tl.item]) + size_t(h) * XK + t128] : 0.f;
+    mbar_arrive(kb_ready);
+    ok = mbar_sleep_warp(kb_ready, 0, abort_flag) && mbar_sleep_warp(s_full, 0, abort_flag);
+    float l = 0.f;
+    if (ok) {
+      tc_fence_after();
+      uint32_t r[XK];
+#pragma unroll
+      for (int i = 0; i < XK / 16; ++i) tmem_ld16_nowait(tS + lane_off + 16u * i, r + 16 * i);
+      tmem_wait_ld();
+#pragma unroll
+      for (int c = 0; c < XK; ++c)
+        r[c] = c < Nk ? __float_as_uint(__uint_as_float(r[c]) + s_kb[c])
+                      : __float_as_uint(-INFINITY);
+      float mx8[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) mx8[q] = __uint_as_float(r[q]);
+#pragma unroll
+      for (int c = 8; c < XK; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(r[c]));
+      const float m = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                            fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]))) * scale_log2;
+      const uint64_t sc2 = f32x2(scale_log2, scale_log2), nm2 = f32x2(-m, -m);
+      uint64_t sum2[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) sum2[q] = f32x2(0.f, 0.f);
+#pragma unroll
+      for (int c = 0; c < XK; c += 2) {
+        float a, b;
+        unpack_f32x2(fma_f32x2(f32x2(__uint_as_float(r[c]), __uint_as_float(r[c + 1])), sc2, nm2),
+                     a, b);
+        a = ex2_ftz(a);
+        b = ex2_ftz(b);
+        r[c] = __float_as_uint(a);
+        r[c + 1] = __float_as_uint(b);
+        sum2[(c >> 1) & 3] = add_f32x2(sum2[(c >> 1) & 3], f32x2(a, b));
+      }
+      float s0, s1, s2, s3, s4, s5, s6, s7;
+      unpack_f32x2(sum2[0], s0, s1);
+      unpack_f32x2(sum2[1], s2, s3);
+      unpack_f32x2(sum2[2], s4, s5);
+      unpack_f32x2(sum2[3], s6, s7);
+      l = ((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7));
+      if (CAP && cap.n && row < tl.rows) {  // the localisation scores of the listed keys
+        const int qrow = tl.row0 + row;
+        const int tok = rm.tok ? __ldg(rm.tok + qrow) : qrow;
+        const float inv_l = l > 0.f ? 1.f / l : 0.f;
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          if (q < cap.n) {
+            float pq = 0.f;
+#pragma unroll
+            for (int c = 0; c < XK; ++c)
+              if (c == cap.id[q]) pq = __uint_as_float(r[c]);
+            atomicAdd(cap.out + size_t(tok) * cap.ldo + cap.id[q], cap.w * pq * inv_l);
+          }
+      }
+#pragma unroll
+      for (int h2 = 0; h2 < XK / 32; ++h2) {
+        uint32_t w[16];
+#pragma unroll
+        for (int c = 0; c < 16; ++c)
+          w[c] = pack_bf16x2(__uint_as_float(r[32 * h2 + 2 * c]),
+                             __uint_as_float(r[32 * h2 + 2 * c + 1]));
+        tmem_st16(tS + lane_off + 16u * h2, w);
+      }
+      tmem_wait_st();
+    }
+    tc_fence_before();
+    mbar_arrive(p_ready);  // arrives even on failure so that no wait is left open
+    if (ok) ok = mbar_sleep_warp(o_full, 0, abort_flag);
+    if (ok) {
+      tc_fence_after();
+      uint32_t o[C::DHP];
+#pragma unroll
+      for (int i = 0; i < C::DHP / 16; ++i) tmem_ld16_nowait(tO + lane_off + 16u * i, o + 16 * i);
+      tmem_wait_ld();
+      if (row < tl.rows) {
+        const float inv = l > 0.f ? 1.f / l : 0.f;
+        uint4* dst = reinterpret_cast<uint4*>(O + size_t(tl.row0 + row) * ldo + h * DH);
+#pragma unroll
+        for (int c8 = 0; c8 < DH / 8; ++c8) {
+          uint4 w;
+          w.x = pack_bf16x2(__uint_as_float(o[8 * c8 + 0]) * inv, __uint_as_float(o[8 * c8 + 1]) * inv);
+          w.y = pack_bf16x2(__uint_as_float(o[8 * c8 + 2]) * inv, __uint_as_float(o[8 * c8 + 3]) * inv);
+          w.z = pack_bf16x2(__uint_as_float(o[8 * c8 + 4]) * inv, __uint_as_float(o[8 * c8 + 5]) * inv);
+          w.w = pack_bf16x2(__uint_as_float(o[8 * c8 + 6]) * inv, __uint_as_float(o[8 * c8 + 7]) * inv);
+          dst[c8] = w;
+        }
+      }
+    }
+  }
+  if (live && (!ok || *abort_flag) && threadIdx.x == 64) atomicOr(err, DEVERR_TIMEOUT);
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, 256);
+  }
+}
+
 // Merge of the pieces of the pairs that stream-K cut: one warp per (pair,
 // query row).  The pieces come from CTAs cta_of(first block) .. cta_of(last
 // block); a CTA's piece is its first (slot 0) when its range starts inside
@@ -931,6 +1209,18 @@ int device_sms_attn() {
             cudaSuccess ||
         cudaFuncSetAttribute(xattn_tc_kernel<64, true>,
                              cudaFuncAttributeMaxDynamicSharedMemorySize, int(XCfg<64>::SMEM)) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(xfused_tc_kernel<72, false>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, int(XFCfg<72>::SMEM)) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(xfused_tc_kernel<72, true>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, int(XFCfg<72>::SMEM)) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(xfused_tc_kernel<64, false>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, int(XFCfg<64>::SMEM)) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(xfused_tc_kernel<64, true>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, int(XFCfg<64>::SMEM)) !=
             cudaSuccess)
       return 0;
     sms[dev] = v;
@@ -1023,6 +1313,54 @@ cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* 
                       ldo, heads, rm, ai.n, Nk, grid, err));
     count_launches(1);
   }
+  return cudaSuccess;
+}
+
+cudaError_t launch_xq_fold(const bf16* Kt, int ldk, const bf16* Wq, const float* bq, int M,
+                           int heads, int dh, int d, bf16* G, float* kb, cudaStream_t st) {
+  if (M < 1 || M > XQ_KEYS || dh > 80 || d % FOLD_THREADS || d > FOLD_THREADS * FOLD_COLS)
+    return cudaErrorInvalidValue;
+  RC_TRY(launch_k(xq_fold_kernel, dim3(heads, (M + FOLD_KEYS - 1) / FOLD_KEYS),
+                  dim3(FOLD_THREADS), 0, st, Kt, ldk, Wq, bq, M, dh, d, G, kb));
+  count_launches(1);
+  return cudaSuccess;
+}
+
+cudaError_t launch_xattn_fused(const bf16* xb, int ldx, const bf16* G, const float* kb, int g_rows,
+                               const bf16* V, int ldv, int v_rows, const XqItems& xi, int Nk,
+                               bf16* O, int ldo, int heads, int dh, const RowMap& rm,
+                               unsigned* err, cudaStream_t st, const AttnCapture* capture) {
+  if (rm.bound <= 0) return cudaSuccess;
+  const int d = heads * dh;
+  if ((dh != 72 && dh != 64) || Nk < 1 || Nk > XK || d % 64 || ldx % 8 || ldv % 8)
+    return cudaErrorInvalidValue;
+  if (xi.n < 1 || xi.n > MAX_ITEMS || (xi.n > 1 && !rm.meta)) return cudaErrorInvalidValue;
+  for (int i = 0; i < xi.n; ++i)
+    if (xi.grow[i] < 0 || xi.grow[i] + heads * XK > g_rows || xi.vrow[i] < 0 ||
+        xi.vrow[i] > v_rows - Nk)
+      return cudaErrorInvalidValue;
+  if (!device_sms_attn()) return cudaErrorInvalidDevice;
+  AttnCapture cap{};
+  if (capture && capture->n > 0) {
+    if (capture->n > 8 || !capture->out) return cudaErrorInvalidValue;
+    for (int q = 0; q < capture->n; ++q)
+      if (capture->id[q] < 0 || capture->id[q] >= Nk || capture->id[q] >= capture->ldo)
+        return cudaErrorInvalidValue;
+    cap = *capture;
+  }
+  // xb and G as (64 columns, column block, row) views, V as the head view
+  CUtensorMap ta, tg, tv;
+  RC_TRY(head_map(xb, rm.bound, ldx, d / 64, 64, 64, BQ, &ta));
+  RC_TRY(head_map(G, g_rows, d, d / 64, 64, 64, XK, &tg));
+  RC_TRY(head_map(V, v_rows, ldv, heads, dh, 64, XK, &tv));
+  const float scale_log2 = float(1.4426950408889634 / sqrt(double(dh)));
+  const long long grid = ((long long)(rm.bound + BQ - 1) / BQ + xi.n - 1) * heads;
+  if (grid >= (1ll << 31)) return cudaErrorInvalidValue;
+  auto fn = dh == 72 ? (cap.n ? xfused_tc_kernel<72, true> : xfused_tc_kernel<72, false>)
+                     : (cap.n ? xfused_tc_kernel<64, true> : xfused_tc_kernel<64, false>);
+  RC_TRY(launch_k(fn, dim3(unsigned(grid)), dim3(192), dh == 72 ? XFCfg<72>::SMEM : XFCfg<64>::SMEM,
+                  st, ta, tg, tv, kb, xi, Nk, d, O, ldo, heads, rm, scale_log2, err, cap));
+  count_launches(1);
   return cudaSuccess;
 }
 

@@ -179,4 +179,26 @@ cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* 
                              int dh, const RowMap& rm, unsigned* err, const AttnScratch& as,
                              cudaStream_t st, const AttnCapture* cap = nullptr);
 
+// Text cross-attention with the query projection folded into the keys:
+// S_h = xb W_xq,h^T K_h^T + b_h K_h^T = xb G_h^T + kb_h with G_h = K_h W_xq,h
+// ([XK][d] per (session, layer, head), rows >= text_len zero) and
+// kb_h = K_h b_xq,h.  launch_xq_fold computes G and kb of one (session,
+// layer) for all heads from the text keys (row stride ldk) and W_xq, b_xq.
+constexpr int XQ_KEYS = 128;
+cudaError_t launch_xq_fold(const bf16* Kt, int ldk, const bf16* Wq, const float* bq, int M,
+                           int heads, int dh, int d, bf16* G, float* kb, cudaStream_t st);
+// O[r][h*dh..] = softmax((xb_r G_h^T + kb_h) / sqrt(dh)) V_h over the Nk <= 128
+// text keys of row r's item.  G / kb rows of item i start at grow[i] (+ h *
+// XQ_KEYS); its values at row vrow[i] of V (row stride ldv).  cap as in
+// launch_attention.
+struct XqItems {
+  int n;
+  int grow[MAX_ITEMS];
+  int vrow[MAX_ITEMS];
+};
+cudaError_t launch_xattn_fused(const bf16* xb, int ldx, const bf16* G, const float* kb, int g_rows,
+                               const bf16* V, int ldv, int v_rows, const XqItems& xi, int Nk,
+                               bf16* O, int ldo, int heads, int dh, const RowMap& rm,
+                               unsigned* err, cudaStream_t st, const AttnCapture* cap);
+
 }  // namespace rc

@@ -91,6 +91,10 @@ struct rc_cache {
   int sessions;
   bf16* base = nullptr;  // [sessions][T][L][3 (H,K,V)][N][d] (device-addressable)
   bf16* text = nullptr;  // [sessions][L][M][2d], always in HBM
+  // the text keys with the cross-query projection folded in (HBM):
+  // xg [sessions][L][heads][XQ_KEYS][d] = K_h W_xq,h, xgb [..][XQ_KEYS] = K_h b_xq,h
+  bf16* xg = nullptr;
+  float* xgb = nullptr;
   std::vector<char> text_set;
   // host tier (Section 3.4, Pipelined Execution): the slots live in pinned,
   // mapped host memory (base is its device address).  A step runs layer l on
@@ -123,6 +127,11 @@ struct rc_cache {
   bf16* text_kv(int s, int l) const {
     return text + (size_t(s) * ctx->L + l) * size_t(ctx->M) * 2 * ctx->d;
   }
+  // first xg / xgb row of (session, layer)
+  size_t xg_row(int s, int l) const {
+    return (size_t(s) * ctx->L + l) * size_t(ctx->dims.heads) * rc::XQ_KEYS;
+  }
+  size_t xg_rows() const { return xg_row(sessions, 0); }
 };
 
 namespace {
@@ -306,20 +315,35 @@ rc_status run_block(rc_ctx* c, rc_cache* k, int l, const rc::RowMap& rm, const S
     RC_CUDA(rc::launch_gemm(c->ob, d, static_cast<const bf16*>(w.W_o), rm.bound, rm.count, d, d,
                             e, st), "gemm(out)");
   }
-  // q' = x W_xq^T + b (on the bf16 copy of x)
-  e = rc::GemmEpi{};
-  e.mode = rc::EPI_BIAS_BF16;
-  e.bias = w.b_xq;
-  e.out_bf = c->q;
-  e.ld_out = d;
-  e.gate_off = -1;
-  e.err = c->err;
-  {
-    Probe pr(c, RC_PROBE_GEMM, st);
-    RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_xq), rm.bound, rm.count, d, d,
-                            e, st), "gemm(xq)");
-  }
-  {
+  if (k->xg) {
+    // softmax((x W_xq^T + b) K^T / sqrt(dh)) V per head, with the query
+    // projection folded into the text keys (x G_h^T + kb_h, G_h = K_h W_xq,h):
+    // one kernel on the bf16 copy of x, no cross-query GEMM
+    rc::XqItems xi{};
+    xi.n = si.its.n;
+    for (int i = 0; i < xi.n; ++i) {
+      xi.grow[i] = int(k->xg_row(si.session[i], l));
+      xi.vrow[i] = (si.session[i] * c->L + l) * c->M;
+    }
+    Probe pr(c, RC_PROBE_ATTENTION, st);
+    RC_CUDA(rc::launch_xattn_fused(c->xb, d, k->xg, k->xgb, int(k->xg_rows()), k->text + d, 2 * d,
+                                   k->sessions * c->L * c->M, xi, c->M, c->ob, d, c->dims.heads,
+                                   c->dh, rm, c->err, st, cap),
+            "attention(cross)");
+  } else {
+    // q' = x W_xq^T + b (on the bf16 copy of x)
+    e = rc::GemmEpi{};
+    e.mode = rc::EPI_BIAS_BF16;
+    e.bias = w.b_xq;
+    e.out_bf = c->q;
+    e.ld_out = d;
+    e.gate_off = -1;
+    e.err = c->err;
+    {
+      Probe pr(c, RC_PROBE_GEMM, st);
+      RC_CUDA(rc::launch_gemm(c->xb, d, static_cast<const bf16*>(w.W_xq), rm.bound, rm.count, d,
+                              d, e, st), "gemm(xq)");
+    }
     Probe pr(c, RC_PROBE_ATTENTION, st);
     RC_CUDA(rc::launch_attention(c->q, d, k->text, k->text + d, 2 * d,
                                  k->sessions * c->L * c->M, text_kv_rows(k, si, l), c->M, c->ob,
@@ -492,6 +516,19 @@ rc_status rc_set_schedule(rc_ctx* c, const float* tv, const float* ab) {
   return RC_OK;
 }
 
+// The folded text keys of every (session, layer), zero-filled (rows past the
+// text length stay zero).  Only when the text fits one cross-attention pass.
+static rc_status alloc_xg(rc_cache* k) {
+  const rc_ctx* c = k->ctx;
+  if (c->M > rc::XQ_KEYS) return RC_OK;
+  rc_status s = dalloc(&k->xg, k->xg_rows() * c->d, "folded text keys");
+  if (s == RC_OK) s = dalloc(&k->xgb, k->xg_rows(), "folded text key biases");
+  if (s == RC_OK && (cudaMemset(k->xg, 0, k->xg_rows() * c->d * sizeof(bf16)) != cudaSuccess ||
+                     cudaMemset(k->xgb, 0, k->xg_rows() * sizeof(float)) != cudaSuccess))
+    s = fail(RC_ERR_CUDA, "folded text keys zero fill failed");
+  return s;
+}
+
 rc_status rc_cache_create(rc_ctx* c, int sessions, rc_cache** out) {
   if (!c || !out) return fail(RC_ERR_INVALID_ARG, "rc_cache_create: null argument");
   *out = nullptr;
@@ -510,6 +547,7 @@ rc_status rc_cache_create(rc_ctx* c, int sessions, rc_cache** out) {
   rc_status s = dalloc(&k->base, n, "cache");
   const size_t n_text = size_t(sessions) * c->L * c->M * 2 * c->d;
   if (s == RC_OK) s = dalloc(&k->text, n_text, "text kv");
+  if (s == RC_OK) s = alloc_xg(k);
   // zero-filled: the attention reads whole 64-key blocks, and keys past a
   // slot's end (weighted by zero) come from the next slot, which must be finite
   if (s == RC_OK && (cudaMemset(k->base, 0, n * sizeof(bf16)) != cudaSuccess ||
@@ -519,6 +557,8 @@ rc_status rc_cache_create(rc_ctx* c, int sessions, rc_cache** out) {
   if (s != RC_OK) {
     if (k->base) cudaFree(k->base);
     if (k->text) cudaFree(k->text);
+    if (k->xg) cudaFree(k->xg);
+    if (k->xgb) cudaFree(k->xgb);
     delete k;
     return s;
   }
@@ -546,6 +586,8 @@ void rc_cache_destroy(rc_cache* k) {
     cudaFree(k->base);
   }
   if (k->text) cudaFree(k->text);
+  if (k->xg) cudaFree(k->xg);
+  if (k->xgb) cudaFree(k->xgb);
   delete k;
 }
 
@@ -593,6 +635,7 @@ rc_status rc_cache_create_host(rc_ctx* c, int sessions, rc_cache** out) {
     s = dalloc(&k->window, rc_cache::WINDOWS * 3 * k->slot_elems(), "cache window");
   }
   if (s == RC_OK) s = dalloc(&k->text, n_text, "text kv");
+  if (s == RC_OK) s = alloc_xg(k);
   if (s == RC_OK &&
       (cudaMemset(k->window, 0, rc_cache::WINDOWS * 3 * k->slot_elems() * sizeof(bf16)) !=
            cudaSuccess ||
@@ -646,6 +689,18 @@ rc_status rc_cache_fill(rc_cache* k, int s, int l, int t, const void* H, const v
 rc_status rc_cache_read(rc_cache* k, int s, int l, int t, void* H, void* K, void* V,
                         rc_stream st) {
   return cache_copy(k, s, l, t, H, K, V, false, static_cast<cudaStream_t>(st));
+}
+
+// The cross-query projection folded into the text keys of one session, all
+// layers (Section 3.3's cross-attention, reassociated: see run_block).
+static rc_status fold_text(rc_ctx* c, rc_cache* k, int s, cudaStream_t st) {
+  if (!k->xg) return RC_OK;
+  for (int l = 0; l < c->L; ++l)
+    RC_CUDA(rc::launch_xq_fold(k->text_kv(s, l), 2 * c->d, static_cast<const bf16*>(c->lw[l].W_xq),
+                               c->lw[l].b_xq, c->M, c->dims.heads, c->dh, c->d,
+                               k->xg + k->xg_row(s, l) * c->d, k->xgb + k->xg_row(s, l), st),
+            "fold text keys");
+  return RC_OK;
 }
 
 // Session file: magic, then int32 version, N, hidden, layers, timesteps,
@@ -712,6 +767,15 @@ static rc_status session_file(rc_cache* k, int s, const char* path, bool write) 
                    stage_bytes);
   if (stage) cudaFreeHost(stage);
   if (fclose(f) != 0 && r == RC_OK) r = fail(RC_ERR_IO, "closing %s", path);
+  if (r == RC_OK && !write && hdr[6] != 0) {
+    // the folded text keys are derived data: recomputed from the imported
+    // keys and the context's cross-query weights
+    for (int l = 0; l < c->L && r == RC_OK; ++l)
+      if (!c->lw_set[l]) r = fail(RC_ERR_STATE, "weights of layer %d not set before import", l);
+    if (r == RC_OK) r = fold_text(k->ctx, k, s, nullptr);
+    if (r == RC_OK && cudaStreamSynchronize(nullptr) != cudaSuccess)
+      r = fail(RC_ERR_CUDA, "folding the imported text keys");
+  }
   if (r == RC_OK && !write) k->text_set[s] = char(hdr[6] != 0);
   return r;
 }
@@ -743,6 +807,7 @@ rc_status rc_set_text(rc_ctx* c, rc_cache* k, int s, const void* ctx_bf16, rc_st
                             static_cast<const bf16*>(c->lw[l].W_xkv), c->M, nullptr, 2 * c->d,
                             c->d, e, st), "gemm(text kv)");
   }
+  if ((r = fold_text(c, k, s, st))) return r;
   k->text_set[s] = 1;
   return RC_OK;
 }
