@@ -48,18 +48,20 @@ L2_NOTE = ("inputs larger than L2: each step streams 1.04 GB of weights and a di
            "28 x 28.3 MB cache slice per timestep")
 
 
-def linear_flops_per_token_block(d: synth.Dims) -> float:
-    """2 x (3h^2 + h^2 + h^2 + hF + Fh) per dirty token and block: the GEMM
-    launches (QKV, out, cross-out, fc1, fc2).  The cross-query projection
-    (2 h^2) runs inside the cross-attention kernel, folded into the text keys."""
+def linear_flops_per_token_block(d: synth.Dims, folded: bool = True) -> float:
+    """2 x (3h^2 + h^2 [+ h^2] + h^2 + hF + Fh) per dirty token and block: the
+    GEMM launches (QKV, out, [cross-q,] cross-out, fc1, fc2).  With the
+    cross-query projection folded into the text keys (sparse steps) its 2 h^2
+    run inside the cross-attention kernel instead."""
     h, F = d.hidden, d.mlp
-    return 2.0 * (5 * h * h + 2 * h * F)
+    return 2.0 * ((5 if folded else 6) * h * h + 2 * h * F)
 
 
-def attn_flops_per_token_block(d: synth.Dims) -> float:
-    """Self-attention (4 N h) plus cross-attention with its query projection
-    (4 M h + 2 h^2) per dirty token and block."""
-    return 4.0 * d.tokens * d.hidden + 4.0 * d.text_len * d.hidden + 2.0 * d.hidden * d.hidden
+def attn_flops_per_token_block(d: synth.Dims, folded: bool = True) -> float:
+    """Self-attention (4 N h) plus cross-attention (4 M h), with its query
+    projection (2 h^2) when folded, per dirty token and block."""
+    return (4.0 * d.tokens * d.hidden + 4.0 * d.text_len * d.hidden +
+            (2.0 * d.hidden * d.hidden if folded else 0.0))
 
 
 KERNEL_SOURCES = {
@@ -414,16 +416,21 @@ def kernel_rooflines(d, D, gemm_each, att_each, peak):
     D dirty rows per launch over the CUDA-event launch durations."""
     gemm_ms, gemm_n = sum(gemm_each), len(gemm_each)
     att_ms, att_n = sum(att_each), len(att_each)
-    steps = gemm_n / (5 * d.layers)
-    lin_flops_launch = linear_flops_per_token_block(d) * D / 5
-    gemm_tflops = linear_flops_per_token_block(d) * D * d.layers * steps / (gemm_ms / 1e3) / 1e12
-    att_tflops = attn_flops_per_token_block(d) * D * d.layers * steps / (att_ms / 1e3) / 1e12
+    steps = att_n / (2 * d.layers)
+    per_block = int(round(gemm_n / (steps * d.layers)))  # 5: cross-query folded, 6: not
+    folded = per_block == 5
+    lin = linear_flops_per_token_block(d, folded)
+    lin_flops_launch = lin * D / per_block
+    gemm_tflops = lin * D * d.layers * steps / (gemm_ms / 1e3) / 1e12
+    att_tflops = (attn_flops_per_token_block(d, folded) * D * d.layers * steps /
+                  (att_ms / 1e3) / 1e12)
     roofline = {"bound": "tensor", "achieved": round(gemm_tflops, 2), "peak": peak,
                 "unit": "TFLOP/s", "frac": round(gemm_tflops / peak, 4),
                 "traffic": profiled_traffic("gemm"),
-                "kernel": "gemm (QKV, out, cross-out, fc1, fc2 of every block)",
+                "kernel": "gemm (QKV, out, [cross-q,] cross-out, fc1, fc2 of every block)",
                 "launches": gemm_n, "avg_launch_ms": round(gemm_ms / max(gemm_n, 1), 5),
-                "flops_per_launch": lin_flops_launch}
+                "flops_per_launch": lin_flops_launch,
+                "cross_query_folded_into_attention": folded}
     roof_att = {"bound": "tensor", "achieved": round(att_tflops, 2), "peak": peak,
                 "traffic": profiled_traffic("attention"),
                 "unit": "TFLOP/s", "frac": round(att_tflops / peak, 4), "launches": att_n,
@@ -431,11 +438,11 @@ def kernel_rooflines(d, D, gemm_each, att_each, peak):
     # per-launch breakdown: launches come in block order (GEMMs: QKV, out,
     # cross-q, cross-out, fc1, fc2; attention: self, cross)
     h, F = d.hidden, d.mlp
-    gemm_shapes = [("qkv", 3 * h, h), ("out", h, h), ("cross_out", h, h), ("fc1", F, h),
-                   ("fc2", h, F)]
+    gemm_shapes = [("qkv", 3 * h, h), ("out", h, h)] + ([] if folded else [("cross_q", h, h)]) + [
+        ("cross_out", h, h), ("fc1", F, h), ("fc2", h, F)]
     per_gemm = {}
     for j, (name, n_, k_) in enumerate(gemm_shapes):
-        ts = gemm_each[j::5]
+        ts = gemm_each[j::per_block]
         us = 1e3 * sum(ts) / max(len(ts), 1)
         per_gemm[name] = {"shape": [D, n_, k_], "avg_us": round(us, 2),
                           "tflops": round(2.0 * D * n_ * k_ / (us * 1e-6) / 1e12, 1)}
@@ -443,7 +450,7 @@ def kernel_rooflines(d, D, gemm_each, att_each, peak):
     for j, (name, nk) in enumerate([("self", d.tokens), ("cross", d.text_len)]):
         ts = att_each[j::2]
         us = 1e3 * sum(ts) / max(len(ts), 1)
-        fl = 4.0 * D * nk * h + (2.0 * D * h * h if name == "cross" else 0.0)
+        fl = 4.0 * D * nk * h + (2.0 * D * h * h if name == "cross" and folded else 0.0)
         per_attn[name] = {"queries": D, "keys": nk, "avg_us": round(us, 2),
                           "tflops": round(fl / (us * 1e-6) / 1e12, 1)}
     roofline["per_gemm"] = per_gemm
@@ -523,7 +530,9 @@ def run_ours(args, world, rank, local):
     ln_each = probe(R.RC_PROBE_LN, 2, lambda i: wl.step(i, HEADLINE), K)
     # the same kernels on all 4096 rows (the dense step)
     Kd = max(2, K // 4)
-    gemm_each_d = probe(R.RC_PROBE_GEMM, 5, wl.step_dense, Kd)
+    # 6 GEMMs per block here: at 4096 host-known rows the cross-query projection
+    # runs as its own paired GEMM instead of inside the cross-attention kernel
+    gemm_each_d = probe(R.RC_PROBE_GEMM, 6, wl.step_dense, Kd)
     att_each_d = probe(R.RC_PROBE_ATTENTION, 2, wl.step_dense, Kd)
 
     # sweep and dense baseline (graphs, like the headline)

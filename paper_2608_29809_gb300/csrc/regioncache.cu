@@ -315,7 +315,11 @@ rc_status run_block(rc_ctx* c, rc_cache* k, int l, const rc::RowMap& rm, const S
     RC_CUDA(rc::launch_gemm(c->ob, d, static_cast<const bf16*>(w.W_o), rm.bound, rm.count, d, d,
                             e, st), "gemm(out)");
   }
-  if (k->xg) {
+  // the folded form costs 16 x the query-projection FLOPs (one pass over x
+  // per head); it wins while the rows are few (it saves a launch), the
+  // separate GEMM (CTA pairs) once they are many and known on the host
+  const bool fold = k->xg && (rm.count || rm.bound < 2048);
+  if (fold) {
     // softmax((x W_xq^T + b) K^T / sqrt(dh)) V per head, with the query
     // projection folded into the text keys (x G_h^T + kb_h, G_h = K_h W_xq,h):
     // one kernel on the bf16 copy of x, no cross-query GEMM
