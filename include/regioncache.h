@@ -163,15 +163,21 @@ rc_status rc_cache_read(rc_cache* cache, int session, int layer, int t,
  * raw little-endian bf16, about timesteps * layers * 3 * N * hidden * 2
  * bytes.  Import requires a header equal to the cache's dimensions
  * (RC_ERR_SHAPE otherwise) and marks the session's text as set when the
- * exported session had it.  Errors: RC_ERR_INVALID_ARG, RC_ERR_IO (open,
- * short read / write, bad magic), RC_ERR_SHAPE, RC_ERR_CUDA. */
+ * exported session had it; the folded text keys (see rc_set_text) are not
+ * in the file but recomputed on import, so a session with text needs every
+ * layer's weights set first (RC_ERR_STATE otherwise).  Errors:
+ * RC_ERR_INVALID_ARG, RC_ERR_IO (open, short read / write, bad magic),
+ * RC_ERR_SHAPE, RC_ERR_STATE, RC_ERR_CUDA. */
 rc_status rc_cache_export(rc_cache* cache, int session, const char* path);
 rc_status rc_cache_import(rc_cache* cache, int session, const char* path);
 
 /* Text conditioning of one session for an editing turn: ctx_bf16 is the
  * text context, bf16 [text_len][hidden].  Computes every layer's
  * cross-attention keys/values (ctx W_xkv^T + b_xkv) into the session's
- * cache.  Must precede rc_step / rc_block_forward_region for the session. */
+ * cache, and from them the keys with the cross-query projection folded in
+ * (G_h = K_h W_xq,h, kb_h = K_h b_xq,h per head, device memory owned by the
+ * cache) that sparse steps use instead of a separate query projection.
+ * Must precede rc_step / rc_block_forward_region for the session. */
 rc_status rc_set_text(rc_ctx* ctx, rc_cache* cache, int session, const void* ctx_bf16,
                       rc_stream stream);
 

@@ -315,8 +315,9 @@ rc_status run_block(rc_ctx* c, rc_cache* k, int l, const rc::RowMap& rm, const S
     RC_CUDA(rc::launch_gemm(c->ob, d, static_cast<const bf16*>(w.W_o), rm.bound, rm.count, d, d,
                             e, st), "gemm(out)");
   }
-  // the folded form costs 16 x the query-projection FLOPs (one pass over x
-  // per head); it wins while the rows are few (it saves a launch), the
+  // the folded form multiplies x by 128 padded key rows per head where the
+  // projection multiplies it by dh = 72 (1.8 x the FLOPs, x read once per
+  // head); it wins while the rows are few (one launch less per block), the
   // separate GEMM (CTA pairs) once they are many and known on the host
   const bool fold = k->xg && (rm.count || rm.bound < 2048);
   if (fold) {
