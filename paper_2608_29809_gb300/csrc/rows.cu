@@ -214,6 +214,18 @@ cudaError_t launch_localize(const float* A, int S, int N, int M, int gh, int gw,
 // One warp per row; the row stays in registers (hidden <= 1536, % 128 == 0).
 constexpr int LN_WARPS = 8;
 constexpr int LN_MAXV = 12;  // float4 per lane
+constexpr int LN_SV = (LN_MAXV * 32 + LN_WARPS * 32 - 1) / (LN_WARPS * 32);  // float4 per thread
+                                                                            // and staged vector
+
+// False (and DEVERR_INDEX) when a row's token or item is out of range.
+__device__ __forceinline__ bool row_valid(const RowMap& rm, int n_items, int tok, int item,
+                                          unsigned* err, int lane) {
+  if (tok < 0 || tok >= rm.n_tokens || item < 0 || item >= n_items) {
+    if (lane == 0) atomicOr(err, DEVERR_INDEX);
+    return false;
+  }
+  return true;
+}
 
 // Token and item of compact row r; false (and DEVERR_INDEX) when either is
 // out of range.
@@ -221,11 +233,7 @@ __device__ __forceinline__ bool row_target(const RowMap& rm, int n_items, int r,
                                            int& item, unsigned* err, int lane) {
   tok = rm.tok ? __ldg(rm.tok + r) : r;
   item = rm.item ? __ldg(rm.item + r) : 0;
-  if (tok < 0 || tok >= rm.n_tokens || item < 0 || item >= n_items) {
-    if (lane == 0) atomicOr(err, DEVERR_INDEX);
-    return false;
-  }
-  return true;
+  return row_valid(rm, n_items, tok, item, err, lane);
 }
 
 __global__ void __launch_bounds__(LN_WARPS * 32)
@@ -235,34 +243,58 @@ ln_mod_kernel(const float* __restrict__ x, const float* __restrict__ tab, int k_
   pdl_wait();
   pdl_trigger();
   // shift and scale staged once per CTA: tab (+ the item's tb when the
-  // launch has one item; otherwise each row adds its item's tb)
+  // launch has one item; otherwise each row adds its item's tb).  Loads that
+  // do not depend on one another are all issued before any is used (the
+  // vectors and the live row count, then the row with its token and item),
+  // so a CTA waits for about two L2 round trips before its arithmetic.
   extern __shared__ __align__(16) float s_mod[];  // [2][d]
-  const int D = live_count(rm.count, rm.bound, err);
   const int lane = threadIdx.x & 31;
-  const int nv = d / 128;
+  const int nv = d / 128, nq = d / 4;
   const float* tb0 = it.n == 1 ? it.tb[0] : nullptr;
+  float4 m[4][LN_SV];  // tab shift, tab scale, tb shift, tb scale
+#pragma unroll
+  for (int j = 0; j < LN_SV; ++j) {
+    const int q = threadIdx.x + j * LN_WARPS * 32;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) m[u][j] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (q < nq && tab) {
+      m[0][j] = __ldg(reinterpret_cast<const float4*>(tab + size_t(k_sh) * d) + q);
+      m[1][j] = __ldg(reinterpret_cast<const float4*>(tab + size_t(k_sc) * d) + q);
+    }
+    if (q < nq && tb0) {
+      m[2][j] = __ldg(reinterpret_cast<const float4*>(tb0 + size_t(k_sh) * d) + q);
+      m[3][j] = __ldg(reinterpret_cast<const float4*>(tb0 + size_t(k_sc) * d) + q);
+    }
+  }
+  const int D = live_count(rm.count, rm.bound, err);
   int r = blockIdx.x * LN_WARPS + (threadIdx.x >> 5);
   float4 v[LN_MAXV];
+  int tok = 0, item = 0;
   auto load_row = [&](int rr) {
+    tok = rm.tok ? __ldg(rm.tok + rr) : rr;
+    item = rm.item ? __ldg(rm.item + rr) : 0;
     const float4* xr = reinterpret_cast<const float4*>(x + size_t(rr) * d);
 #pragma unroll
     for (int k = 0; k < LN_MAXV; ++k)
       if (k < nv) v[k] = xr[lane + 32 * k];
   };
-  if (r < D) load_row(r);  // requested before the staging barrier
-  for (int c = threadIdx.x; c < d; c += blockDim.x) {
-    float a = tab ? tab[size_t(k_sh) * d + c] : 0.f, b = tab ? tab[size_t(k_sc) * d + c] : 0.f;
-    if (tb0) {
-      a += tb0[size_t(k_sh) * d + c];
-      b += tb0[size_t(k_sc) * d + c];
+  if (r < D) load_row(r);
+#pragma unroll
+  for (int j = 0; j < LN_SV; ++j) {
+    const int q = threadIdx.x + j * LN_WARPS * 32;
+    if (q < nq) {
+      float4 a = m[0][j], b = m[1][j];
+      if (tb0) {
+        a.x += m[2][j].x; a.y += m[2][j].y; a.z += m[2][j].z; a.w += m[2][j].w;
+        b.x += m[3][j].x; b.y += m[3][j].y; b.z += m[3][j].z; b.w += m[3][j].w;
+      }
+      reinterpret_cast<float4*>(s_mod)[q] = a;
+      reinterpret_cast<float4*>(s_mod + d)[q] = b;
     }
-    s_mod[c] = a;
-    s_mod[d + c] = b;
   }
   __syncthreads();
   while (r < D) {
-    int tok, item;
-    if (row_target(rm, it.n, r, tok, item, err, lane)) {
+    if (row_valid(rm, it.n, tok, item, err, lane)) {
       float s = 0.f;
 #pragma unroll
       for (int k = 0; k < LN_MAXV; ++k)
