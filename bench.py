@@ -188,6 +188,12 @@ def max_over_ranks(x: float, world: int) -> float:
     return float(t.item())
 
 
+def job_rate(units_per_rank: float, ms: float, world: int) -> float:
+    """Whole-job rate of independent replicas (weak scaling): the units all
+    ranks processed over the slowest rank's time (ms)."""
+    return units_per_rank * world / (max_over_ranks(ms, world) / 1e3)
+
+
 # ------------------------------------------------------------------ our arm
 class Workload:
     def __init__(self, R, d: synth.Dims, seed: int, dev: str, fracs=FRACS):
@@ -306,7 +312,7 @@ class Workload:
             R.rc_cache_destroy(hc)
         slot = d.tokens * d.hidden * 2
         h2d = (2 * (d.layers - 1) + 3) * slot
-        return {"steps_per_s": round(K * world / (max_over_ranks(m, world) / 1e3), 3),
+        return {"steps_per_s": round(job_rate(K, m, world), 3),
                 "pool_bytes": d.timesteps * d.layers * 3 * slot,
                 "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": 3 * int(self.cnt.item()) * d.hidden * 2 * d.layers,
@@ -372,9 +378,9 @@ def rate_batched(R, args, world, dev, K, W, n=8):
 
         k = max(2, K // 2)
         m = timed(batched, k, W, world)
-        rate_b = n * k * world / (max_over_ranks(m, world) / 1e3)
+        rate_b = job_rate(n * k, m, world)
         m = timed(one_by_one, k, W, world)
-        rate_1 = n * k * world / (max_over_ranks(m, world) / 1e3)
+        rate_1 = job_rate(n * k, m, world)
         R.rc_sync(model.ctx)
     finally:
         model.close()
@@ -396,10 +402,10 @@ def rate_2048(R, args, world, dev, K, W):
         wl.make_graphs()
         k = max(2, K // 4)
         m = timed(lambda i: wl.gstep(i, HEADLINE), k, W, world)
-        sparse = k * world / (max_over_ranks(m, world) / 1e3)
+        sparse = job_rate(k, m, world)
         D = int(wl.cnt.item())
         m = timed(wl.gstep_dense, k, min(W, 3), world)
-        dense = k * world / (max_over_ranks(m, world) / 1e3)
+        dense = job_rate(k, m, world)
         R.rc_sync(wl.model.ctx)
         wl.free_graphs()
     finally:
@@ -502,7 +508,7 @@ def run_ours(args, world, rank, local):
     value = K * world / (ms_max / 1e3)
     # the same steps issued launch by launch (rc_step)
     m = timed(lambda i: wl.step(i, HEADLINE), K, W, world)
-    direct = K * world / (max_over_ranks(m, world) / 1e3)
+    direct = job_rate(K, m, world)
     if args.quick:
         if rank == 0:
             print(json.dumps({"metric": METRIC, "value": round(value, 3), "unit": UNIT,
@@ -539,12 +545,12 @@ def run_ours(args, world, rank, local):
     sweep, dirty = {}, {}
     for f in FRACS:
         m = timed(lambda i, f=f: wl.gstep(i, f), K, W, world)
-        sweep[f"{f:.2f}"] = round(K * world / (max_over_ranks(m, world) / 1e3), 3)
+        sweep[f"{f:.2f}"] = round(job_rate(K, m, world), 3)
         dirty[f"{f:.2f}"] = int(wl.cnt.item())
     m = timed(wl.gstep_dense, max(2, K // 2), min(W, 3), world)
-    dense = max(2, K // 2) * world / (max_over_ranks(m, world) / 1e3)
+    dense = job_rate(max(2, K // 2), m, world)
     m = timed(wl.step_capture, max(2, K // 2), min(W, 3), world)
-    capture = max(2, K // 2) * world / (max_over_ranks(m, world) / 1e3)
+    capture = job_rate(max(2, K // 2), m, world)
     R.rc_sync(wl.model.ctx)
 
     # batched serving of 8 concurrent 512 px sessions
