@@ -346,7 +346,7 @@ rc_status rc_prompt_similarity(const float* e_minus, const float* e_plus, int di
 rc_status rc_reuse_schedule(float s, float tau_s, float rho, int T, uint8_t* modes_out);
 
 /* CUDA Graph of one rc_step (no counterpart in the paper; serving
- * plumbing): the step's ~320 kernel launches for fixed arguments are
+ * plumbing): the step's ~290 kernel launches for fixed arguments are
  * recorded once and replayed with one launch call.  The arguments are those
  * of rc_step; the graph keeps the device pointers (latent, dirty_idx,
  * dirty_count, the cache slots of (session, t)) and reads and writes their
@@ -396,7 +396,9 @@ rc_status rc_sync(rc_ctx* ctx, rc_stream stream);
 /* Timing probe.  rc_probe_enable(ctx, which, capacity) makes the context
  * record a pair of CUDA events on the launching stream around each of the
  * next `capacity` launches of kernel class `which` (RC_PROBE_GEMM: every
- * tensor-core GEMM of a block; RC_PROBE_ATTENTION: every attention launch;
+ * tensor-core GEMM of a block, five, or six when the cross-query projection
+ * runs as its own GEMM; RC_PROBE_ATTENTION: the self- and the
+ * cross-attention launch of a block;
  * RC_PROBE_LN: both LayerNorm-modulation launches of a block);
  * which = RC_PROBE_OFF disables it.  rc_probe_read waits for the recorded
  * events and returns the summed device time (ms) and the number of launches
