@@ -1,6 +1,7 @@
-"""The binding's ctypes structures have the C header's layout: every field's
-name, order, offset and the structure's size, as a C compiler lays them out
-from include/regioncache.h (gcc, no GPU)."""
+"""The binding matches the C header in include/regioncache.h: its ctypes
+structures have every field's name, order and offset and the structure's
+size as a C compiler (gcc, no GPU) lays them out, and every function's
+argument and return types are those of its prototype."""
 import ctypes
 import os
 import re
@@ -74,3 +75,48 @@ def test_ctypes_structures_match_the_header(R, c_layout):
         for n in names:
             assert getattr(py, n).offset == c_layout[s][n], f"{s}.{n}"
         assert ctypes.sizeof(py) == c_layout[s]["size"], s
+
+
+def header_prototypes():
+    """{name: (return kind, [parameter kinds])} of every function the header
+    declares, kinds being ptr / int / float / double / u64 / none."""
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    src = re.sub(r"#.*", "", src)
+
+    def kind(decl):
+        decl = decl.strip()
+        if "*" in decl or decl.split()[0] == "rc_stream" or " rc_stream " in f" {decl} ":
+            return "ptr"
+        words = [w for w in re.split(r"\s+", decl) if w != "const"]
+        t = words[0]
+        return {"int": "int", "rc_status": "int", "int32_t": "int", "float": "float",
+                "double": "double", "size_t": "u64", "uint64_t": "u64", "void": "none"}[t]
+
+    out = {}
+    for m in re.finditer(r"([A-Za-z_][\w\s\*]*?)\b(rc_\w+)\s*\(([^)]*)\)\s*;", src):
+        ret, name, params = m.group(1), m.group(2), m.group(3).strip()
+        ps = [] if params in ("", "void") else [kind(p) for p in params.split(",")]
+        out[name] = (kind(ret + " x"), ps)
+    return out
+
+
+def ctypes_kind(t):
+    if t is None:
+        return "none"
+    if t in (ctypes.c_void_p, ctypes.c_char_p) or hasattr(t, "_type_") and isinstance(
+            t._type_, type):
+        return "ptr"
+    return {ctypes.c_int: "int", ctypes.c_float: "float", ctypes.c_double: "double",
+            ctypes.c_size_t: "u64", ctypes.c_uint64: "u64"}[t]
+
+
+def test_binding_signatures_match_the_header(R):
+    protos = header_prototypes()
+    assert set(protos) == set(R.header_symbols())
+    for name, (ret, params) in protos.items():
+        f = getattr(R._lib, name)
+        assert f.argtypes is not None, f"{name}: no argtypes in the binding"
+        got = [ctypes_kind(a) for a in f.argtypes]
+        assert got == params, f"{name}: binding {got} vs header {params}"
+        assert ctypes_kind(f.restype) == ret, f"{name}: return {f.restype} vs {ret}"
