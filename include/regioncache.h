@@ -114,7 +114,12 @@ typedef struct rc_cache rc_cache; /* library-owned per-(session, t, layer) cache
 rc_status rc_create(const rc_dims* dims, rc_ctx** out);
 void rc_destroy(rc_ctx* ctx);
 
-/* Registers (borrows) the weights of block `layer` / of the model. */
+/* Registers (borrows) the weights of block `layer` / of the model.  The text
+ * keys / values of every session (and the cross-query keys folded from them,
+ * see rc_set_text) depend on a layer's W_xkv, b_xkv, W_xq and b_xq:
+ * rc_set_layer_weights therefore marks the text of every session of every
+ * cache of this context stale, and steps of a session return RC_ERR_STATE
+ * until rc_set_text (or rc_cache_import) runs for it again. */
 rc_status rc_set_layer_weights(rc_ctx* ctx, int layer, const rc_layer_weights* w);
 rc_status rc_set_global_weights(rc_ctx* ctx, const rc_global_weights* w);
 
@@ -167,7 +172,9 @@ rc_status rc_cache_read(rc_cache* cache, int session, int layer, int t,
  * in the file but recomputed on import, so a session with text needs every
  * layer's weights set first (RC_ERR_STATE otherwise).  Errors:
  * RC_ERR_INVALID_ARG, RC_ERR_IO (open, short read / write, bad magic),
- * RC_ERR_SHAPE, RC_ERR_STATE, RC_ERR_CUDA. */
+ * RC_ERR_SHAPE, RC_ERR_STATE, RC_ERR_CUDA.  An import that fails after the
+ * header check has overwritten part of the session: its text is then marked
+ * unset (steps return RC_ERR_STATE) until rc_set_text or a successful import. */
 rc_status rc_cache_export(rc_cache* cache, int session, const char* path);
 rc_status rc_cache_import(rc_cache* cache, int session, const char* path);
 
@@ -194,7 +201,10 @@ size_t rc_localize_workspace_size(int N, int n_delta);
  *                [0, M); 1 <= n_delta <= 64.
  *   threshold    per delta token j the scores are min-max normalised over the
  *                N tokens and token i is in j's region iff the normalised
- *                value is >= threshold; a constant column gives no token.
+ *                value is >= threshold; a constant column gives no token,
+ *                and so does a column whose averaged scores hold a
+ *                non-finite value (NaN, +-Inf), where the normalisation is
+ *                undefined.
  *   dilation     the union over j is dilated by a (2r+1)^2 square on the
  *                grid_h x grid_w token grid (r = dilation, 0..8), neighbours
  *                outside the grid ignored.
@@ -229,8 +239,10 @@ rc_status rc_localize_mask(const float* xattn, int S, int N, int M, int grid_h, 
  *   Limits: N <= RC_NOALLOC_MAX_TOKENS and n_delta <= RC_NOALLOC_MAX_DELTA;
  *   larger sizes return RC_ERR_SHAPE with a message naming the limit.
  *   Set-up: the first call on each device (with that device current) looks
- *   up the array's device address once; make that first call before any
- *   stream capture.
+ *   up the array's device address once and keeps it for the rest of the
+ *   process; make that first call before any stream capture.  The kept
+ *   address does not survive cudaDeviceReset (or any destruction of the
+ *   device's primary context): do not call this entry point after one.
  *   Sharing: every call on a device uses the same scratch, which keeps the
  *   previous call's contents; no part of it needs to start at zero (each
  *   pass overwrites what the next pass reads).  Calls whose work overlaps on

@@ -191,7 +191,9 @@ def localize_mask(A, delta_ids, grid_h, grid_w, threshold=0.5, dilation=1):
     A: cross-attention scores [S][N][M] (float32); delta_ids: the new/modified
     text tokens j.  a_j = mean over the S slices (summed in ascending s, then
     divided by S); theta_j: a_j is min-max normalised and compared (>=) with
-    `threshold`; a constant column contributes no token; the regions of all
+    `threshold`; a constant column, or one whose averaged scores hold a
+    non-finite value (NaN, +-Inf: the normalisation is undefined there),
+    contributes no token; the regions of all
     delta tokens are united and dilated by a (2r+1)x(2r+1) square on the
     grid, ignoring neighbours outside it.  All arithmetic is float32.
     Returns (mask u8 [N], idx int32 ascending).
@@ -208,6 +210,8 @@ def localize_mask(A, delta_ids, grid_h, grid_w, threshold=0.5, dilation=1):
     union = np.zeros(N, dtype=bool)
     for j in delta_ids:
         a = abar[:, int(j)]
+        if not np.all(np.isfinite(a)):
+            continue
         mn = np.float32(a.min())
         mx = np.float32(a.max())
         rng = np.float32(mx - mn)

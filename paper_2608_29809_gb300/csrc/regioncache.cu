@@ -60,6 +60,10 @@ struct rc_ctx {
   int device;
   std::vector<rc_layer_weights> lw;
   std::vector<char> lw_set;
+  // bumped by every rc_set_layer_weights: a session's text keys (and the
+  // folded cross-query keys derived from them) are valid only for the
+  // generation they were computed with
+  uint64_t wgen = 0;
   rc_global_weights gw;
   bool gw_set = false;
   std::vector<float> t_values, alpha_bar;
@@ -96,6 +100,7 @@ struct rc_cache {
   bf16* xg = nullptr;
   float* xgb = nullptr;
   std::vector<char> text_set;
+  std::vector<uint64_t> text_gen;  // the context's weight generation at rc_set_text / import
   // host tier (Section 3.4, Pipelined Execution): the slots live in pinned,
   // mapped host memory (base is its device address).  A step runs layer l on
   // HBM window l % 3: the copy stream loads layer l + 2's cached K, V into
@@ -203,6 +208,10 @@ rc_status check_ready(const rc_ctx* c, const rc_cache* cache, int session, bool 
   if (need_sched && !c->sched_set) return fail(RC_ERR_STATE, "schedule not set");
   if (!cache->text_set[session])
     return fail(RC_ERR_STATE, "text of session %d not set (rc_set_text)", session);
+  if (cache->text_gen[session] != c->wgen)
+    return fail(RC_ERR_STATE,
+                "layer weights changed after the text of session %d was set: its text keys "
+                "and folded cross-query keys are stale; call rc_set_text again", session);
   return RC_OK;
 }
 
@@ -495,6 +504,7 @@ rc_status rc_set_layer_weights(rc_ctx* c, int layer, const rc_layer_weights* w) 
       return fail(RC_ERR_INVALID_ARG, "layer %d: null or unaligned (16 B) weight", layer);
   c->lw[layer] = *w;
   c->lw_set[layer] = 1;
+  ++c->wgen;
   return RC_OK;
 }
 
@@ -543,6 +553,7 @@ rc_status rc_cache_create(rc_ctx* c, int sessions, rc_cache** out) {
   k->ctx = c;
   k->sessions = sessions;
   k->text_set.assign(sessions, 0);
+  k->text_gen.assign(sessions, 0);
   // attention addresses every cache row with a 32-bit tensor coordinate
   if (k->total_rows() >= (size_t(1) << 31) || size_t(sessions) * c->L * c->M >= (size_t(1) << 31)) {
     delete k;
@@ -605,6 +616,7 @@ rc_status rc_cache_create_host(rc_ctx* c, int sessions, rc_cache** out) {
   k->ctx = c;
   k->sessions = sessions;
   k->text_set.assign(sessions, 0);
+  k->text_gen.assign(sessions, 0);
   k->host_tier = true;
   const size_t n = size_t(sessions) * c->T * c->L * 3 * k->slot_elems();
   const size_t n_text = size_t(sessions) * c->L * c->M * 2 * c->d;
@@ -740,6 +752,7 @@ static rc_status session_file(rc_cache* k, int s, const char* path, bool write) 
   RC_CUDA(cudaDeviceSynchronize(), "synchronise");
   FILE* f = fopen(path, write ? "wb" : "rb");
   if (!f) return fail(RC_ERR_IO, "cannot open %s", path);
+  bool header_ok = write;  // an import overwrites the session only past a good header
   int32_t hdr[7] = {1, c->N, c->d, c->L, c->T, c->M, write ? int32_t(k->text_set[s]) : 0};
   if (write) {
     if (fwrite(kCacheMagic, 1, 8, f) != 8 || fwrite(hdr, sizeof(int32_t), 7, f) != 7)
@@ -754,8 +767,10 @@ static rc_status session_file(rc_cache* k, int s, const char* path, bool write) 
     else if (got[0] != 1 || memcmp(got + 1, hdr + 1, 5 * sizeof(int32_t)) != 0)
       r = fail(RC_ERR_SHAPE, "file dims N %d hidden %d layers %d T %d text %d differ", got[1],
                got[2], got[3], got[4], got[5]);
-    else
+    else {
       hdr[6] = got[6];
+      header_ok = true;
+    }
   }
   void* stage = nullptr;
   const size_t stage_bytes = size_t(64) << 20;
@@ -781,7 +796,13 @@ static rc_status session_file(rc_cache* k, int s, const char* path, bool write) 
     if (r == RC_OK && cudaStreamSynchronize(nullptr) != cudaSuccess)
       r = fail(RC_ERR_CUDA, "folding the imported text keys");
   }
-  if (r == RC_OK && !write) k->text_set[s] = char(hdr[6] != 0);
+  if (!write && header_ok) {
+    // after a good header the session's slots and text are being replaced:
+    // a failure part-way leaves a mix of old and new data, so the session
+    // needs rc_set_text (or another import) before its next step
+    k->text_set[s] = char(r == RC_OK && hdr[6] != 0);
+    k->text_gen[s] = k->ctx->wgen;
+  }
   return r;
 }
 
@@ -814,6 +835,7 @@ rc_status rc_set_text(rc_ctx* c, rc_cache* k, int s, const void* ctx_bf16, rc_st
   }
   if ((r = fold_text(c, k, s, st))) return r;
   k->text_set[s] = 1;
+  k->text_gen[s] = c->wgen;
   return RC_OK;
 }
 

@@ -71,6 +71,9 @@ static MaskWs carve(void* ws, int N, int n_delta) {
 
 // Pass 1: a_j(i) = (sum_s A[s][i][j]) / S for each delta token j (summed in
 // ascending s, f32 round-to-nearest), and per-CTA min / max of each column.
+// A non-finite a_j(i) (NaN, +-Inf) enters the min / max as the pair
+// (-Inf, +Inf): finite values never reach those bounds, so pass 2 reads them
+// as "this column holds a non-finite value" and drops the column.
 __global__ void __launch_bounds__(MASK_ROWS)
 mask_colstats_kernel(const float* __restrict__ A, int S, int N, int M, DeltaIds ids,
                      float* __restrict__ abar, float2* __restrict__ part) {
@@ -88,7 +91,12 @@ mask_colstats_kernel(const float* __restrict__ A, int S, int N, int M, DeltaIds 
       for (int s = 1; s < S; ++s) a = __fadd_rn(a, __ldg(A + s * plane + size_t(i) * M + col));
       a = __fdiv_rn(a, float(S));
       abar[size_t(j) * N + i] = a;
-      lo = hi = a;
+      if (isfinite(a)) {
+        lo = hi = a;
+      } else {
+        lo = -INFINITY;
+        hi = INFINITY;
+      }
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -107,6 +115,7 @@ mask_colstats_kernel(const float* __restrict__ A, int S, int N, int M, DeltaIds 
 
 // Pass 2: column min / max over all CTAs (exact, order-free), then the
 // thresholded union over the delta tokens: ((a - mn) / (mx - mn)) >= tau.
+// A constant column, or one holding a non-finite value, gives no token.
 __global__ void __launch_bounds__(MASK_ROWS)
 mask_threshold_kernel(const float* __restrict__ abar, const float2* __restrict__ part, int nblk,
                       int N, DeltaIds ids, float tau, uint8_t* __restrict__ uni) {
@@ -125,7 +134,7 @@ mask_threshold_kernel(const float* __restrict__ abar, const float2* __restrict__
     float rng = __fsub_rn(hi, lo);
     s_mn[j] = lo;
     s_rng[j] = rng;
-    s_ok[j] = rng > 0.0f;
+    s_ok[j] = rng > 0.0f && lo != -INFINITY && hi != INFINITY;
   }
   __syncthreads();
   const int i = blockIdx.x * MASK_ROWS + threadIdx.x;

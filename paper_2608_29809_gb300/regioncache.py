@@ -41,6 +41,19 @@ class rc_dims(C.Structure):
 RC_MAX_BATCH = 16
 
 
+def header_define(name: str) -> int:
+    """Integer value of a ``#define`` of the header (read from the file)."""
+    m = re.search(r"^#define\s+" + re.escape(name) + r"\s+(\d+)\b", open(HEADER).read(), re.M)
+    if not m:
+        raise KeyError(name)
+    return int(m.group(1))
+
+
+RC_NOALLOC_MAX_TOKENS = header_define("RC_NOALLOC_MAX_TOKENS")
+RC_NOALLOC_MAX_DELTA = header_define("RC_NOALLOC_MAX_DELTA")
+RC_NOALLOC_SCRATCH_BYTES = header_define("RC_NOALLOC_SCRATCH_BYTES")
+
+
 class rc_batch_item(C.Structure):
     _fields_ = [("session", C.c_int), ("latent", C.c_void_p), ("t", C.c_int), ("mode", C.c_int),
                 ("dirty_idx", C.c_void_p), ("D", C.c_int), ("dirty_count", C.c_void_p)]

@@ -69,6 +69,25 @@ def test_workspace_size_grows_with_n(R):
     assert R.rc_localize_workspace_size(0, 4) == 0
 
 
+def test_no_alloc_scratch_equals_the_workspace_at_its_limits(R):
+    # the fixed scratch of rc_localize_mask_noalloc is exactly the workspace
+    # of its largest allowed problem, and anything larger is refused before
+    # the device is touched
+    assert R.RC_NOALLOC_SCRATCH_BYTES == R.rc_localize_workspace_size(
+        R.RC_NOALLOC_MAX_TOKENS, R.RC_NOALLOC_MAX_DELTA)
+    assert R.rc_localize_workspace_size(R.RC_NOALLOC_MAX_TOKENS + 1, R.RC_NOALLOC_MAX_DELTA) > \
+        R.RC_NOALLOC_SCRATCH_BYTES
+    ids = np.arange(2, dtype=np.int32)
+    lib = R._lib
+    st = lib.rc_localize_mask_noalloc(256, 1, 113 * 145, 8, 113, 145, ids.ctypes.data, 2, 0.5, 1,
+                                      256, 256, 256, None)
+    assert st == 2 and "16384" in R.rc_last_error()
+    ids17 = np.arange(17, dtype=np.int32)
+    st = lib.rc_localize_mask_noalloc(256, 1, 64, 32, 8, 8, ids17.ctypes.data, 17, 0.5, 1, 256,
+                                      256, 256, None)
+    assert st == 2 and "n_delta <= 16" in R.rc_last_error()
+
+
 def test_null_handles_are_rejected(R):
     lib = R._lib
     assert lib.rc_step(None, None, 0, None, 0, None, None, 0, None, None) == 1

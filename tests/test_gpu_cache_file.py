@@ -1,6 +1,8 @@
 """Cache export / import: a session written to a file and read into another
 cache (device or host tier) gives back every slot and the text keys/values
-bit for bit, and a step from the imported cache matches the oracle."""
+bit for bit, and a step from the imported cache matches the oracle.  A
+session whose text keys may be stale (an import that failed part-way, layer
+weights set again after rc_set_text) is refused until its text is set."""
 import numpy as np
 import pytest
 import torch
@@ -108,3 +110,45 @@ def test_import_refuses_other_dims_and_bad_files(R, tmp_path):
     finally:
         m.close()
         m2.close()
+
+
+def _reuse_step(R, m, d, x):
+    sched = np.full(d.timesteps, O.MODE_REUSE, np.uint8)
+    R.rc_step(m.ctx, m.cache, 0, x, 0, sched, None, 0, None)
+    R.rc_sync(m.ctx)
+
+
+def test_failed_import_and_new_weights_leave_the_text_unset(R, tmp_path):
+    d = synth.Dims(grid_h=16, grid_w=16, layers=2, timesteps=2)
+    w = synth.make_weights(d, 5)
+    m = R.Model(d, w)
+    try:
+        tv, ab = synth.ddim_tables(d.timesteps)
+        R.rc_set_schedule(m.ctx, tv, ab)
+        text = synth.make_text(d, 5).cuda()
+        R.rc_set_text(m.ctx, m.cache, 0, text)
+        x = synth.make_latent(d, 5).cuda()
+        _reuse_step(R, m, d, x)
+        path = str(tmp_path / "s.rccache")
+        R.rc_cache_export(m.cache, 0, path)
+        # a short file past a good header: the slots were partly overwritten
+        short = tmp_path / "short.rccache"
+        short.write_bytes(open(path, "rb").read()[:100000])
+        with pytest.raises(R.RCError) as ei:
+            R.rc_cache_import(m.cache, 0, str(short))
+        assert ei.value.status == 8
+        with pytest.raises(R.RCError) as ei:
+            _reuse_step(R, m, d, x)
+        assert ei.value.status == 7 and "text" in str(ei.value)
+        R.rc_cache_import(m.cache, 0, path)  # a whole file restores the session
+        _reuse_step(R, m, d, x)
+        # new weights for a layer: the text keys and folded keys are stale
+        w2 = synth.make_weights(d, 6).to("cuda")
+        R.rc_set_layer_weights(m.ctx, 1, w2.layers[1])
+        with pytest.raises(R.RCError) as ei:
+            _reuse_step(R, m, d, x)
+        assert ei.value.status == 7 and "rc_set_text" in str(ei.value)
+        R.rc_set_text(m.ctx, m.cache, 0, text)
+        _reuse_step(R, m, d, x)
+    finally:
+        m.close()

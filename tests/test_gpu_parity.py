@@ -78,6 +78,29 @@ def test_localize_edge_cases(R):
     assert D == 300 and np.array_equal(idx, np.arange(300))
 
 
+def test_localize_non_finite_columns_give_no_token(R):
+    # a delta column whose scores hold NaN or +-Inf contributes nothing; the
+    # finite columns beside it still do (bit-exact with the oracle)
+    d = synth.Dims(grid_h=32, grid_w=32)
+    A, ids = synth.blob_scores(d, 11, n_delta=(4, 4))
+    A = A.copy()
+    A[0, 5, ids[0]] = np.nan
+    A[0, 700, ids[1]] = np.inf
+    A[0, 3, ids[2]] = -np.inf
+    m, idx, D = _gpu_mask(R, A, ids, d.grid_h, d.grid_w, 0.5, 1)
+    m_ref, idx_ref = O.localize_mask(A, ids, d.grid_h, d.grid_w, 0.5, 1)
+    m_last, _ = O.localize_mask(A, ids[3:], d.grid_h, d.grid_w, 0.5, 1)
+    assert np.array_equal(m_ref, m_last) and D > 0
+    assert np.array_equal(m, m_ref) and np.array_equal(idx, idx_ref)
+    # two slices whose finite sum overflows to +Inf in f32: the mean is
+    # non-finite and the column drops out on both sides
+    A2 = np.stack([A[0], A[0]])
+    A2[:, :, ids[3]] = np.nan_to_num(A2[:, :, ids[3]])
+    A2[:, 9, ids[3]] = 3.0e38
+    m2, idx2, D2 = _gpu_mask(R, A2, ids[3:], d.grid_h, d.grid_w, 0.5, 1)
+    assert D2 == 0 and m2.sum() == 0
+
+
 def test_localize_indicator_ellipses_4096(R):
     d = synth.PIXART_1024
     for f in (0.05, 0.1, 0.2, 0.4):

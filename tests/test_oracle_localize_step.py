@@ -64,6 +64,27 @@ def test_localize_constant_column_is_empty():
     assert m.sum() == 0 and idx.size == 0
 
 
+def test_localize_non_finite_column_is_dropped():
+    # NaN or +-Inf anywhere in a delta column: the min-max normalisation is
+    # undefined, the column gives no token, the other columns are unaffected
+    gh, gw = 6, 6
+    A = np.zeros((1, gh * gw, 4), np.float32)
+    A[0, 7, 1] = 1.0
+    A[0, 20, 2] = 1.0
+    for bad in (np.nan, np.inf, -np.inf):
+        B = A.copy()
+        B[0, 30, 2] = bad
+        m, idx = O.localize_mask(B, [1, 2], gh, gw, 0.5, 0)
+        assert idx.tolist() == [7]
+        m, idx = O.localize_mask(B, [2], gh, gw, 0.0, 0)
+        assert idx.size == 0
+    # finite slices whose f32 sum overflows: the mean is +Inf, dropped too
+    C = np.stack([A[0], A[0]])
+    C[:, 20, 2] = 3.0e38
+    m, idx = O.localize_mask(C, [1, 2], gh, gw, 0.5, 0)
+    assert idx.tolist() == [7]
+
+
 def test_localize_plateau_rectangle_grows_by_one():
     gh, gw = 10, 12
     A = rng(3).uniform(0, 0.3, (1, gh * gw, 4)).astype(np.float32)
