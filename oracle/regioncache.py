@@ -345,6 +345,38 @@ def step_capture(G, layers, pos, latent, t, cache_t, tkv_layers, t_values, alpha
     return x_next, eps, new_cache, scores
 
 
+def cached_localization_scores(G, layers, pos, latent, cache_t, tkv_layers, heads, grid_h,
+                               grid_w, patch, delta_ids, M):
+    """Localisation scores of Section 3.2 for a new editing turn, taken from
+    the cached diffusion states instead of a dense step (so that a turn
+    scheduled by Eq. 2 -- REUSE, then SPARSE -- can localise its edit before
+    anything is recomputed).
+
+    For each delta (new or modified) text token j and image token i,
+    a_j(i) = mean over blocks l and heads h of the cross-attention
+    probability of j, softmax over all M text tokens of
+    q'_{l,h}(i) . k_{l,h,j'} / sqrt(dh), where the text keys k are the new
+    turn's (ctx W_xkv^T + b) and the image queries q' = H^l W_xq^T + b_xq are
+    computed from the hidden state entering block l as the cache holds it at
+    this step: H^0 is the patch embedding of `latent` (the state entering the
+    first block; the cache starts at block outputs), H^l for l >= 1 is the
+    cached output of block l - 1.  (Reading: the paper aggregates A_t over
+    heads and layers without naming the operator, taken as the mean; the
+    cached block input stands in for the cross-attention input, which the
+    cache does not hold.)
+    Returns scores [N][M] with the delta columns filled and every other
+    column zero (the [S = 1][N][M] layout the localisation takes)."""
+    N = grid_h * grid_w
+    ids = np.asarray(delta_ids, dtype=np.int64)
+    scores = np.zeros((N, M))
+    for l, Lw in enumerate(layers):
+        h_in = patch_embed(latent, np.arange(N), G, pos, patch) if l == 0 else cache_t[l - 1]["H"]
+        maps = cross_attention_maps(h_in, tkv_layers[l][0], Lw, heads)
+        scores[:, ids] += maps[:, :, ids].sum(axis=0)
+    scores[:, ids] /= len(layers) * heads
+    return scores
+
+
 # ------------------------------------------------------------------ schedules
 def cosine_similarity(e_minus, e_plus):
     """Eq. 1: s = cos(e(tau-), e(tau+))."""
