@@ -345,6 +345,30 @@ rc_status rc_step_capture(rc_ctx* ctx, rc_cache* cache, int session, float* late
                           const int32_t* delta_ids_host, int n_delta, float* scores,
                           rc_stream stream);
 
+/* The localisation scores of Section 3.2 for a new editing turn, computed
+ * from the cached states of the previous turn instead of a dense step, so
+ * that a turn scheduled by Eq. 2 (REUSE steps, then SPARSE steps, no dense
+ * step at all) can localise its edit before anything is recomputed.  Call
+ * it after rc_set_text with the new prompt.  For each of the n_delta (1..8)
+ * new or modified text tokens j in delta_ids_host (host array, values in
+ * [0, text_len)):
+ *   scores[i][j] = mean over blocks l and heads h of
+ *                  softmax_j'(q'_{l,h,i} k_{l,h,j'} / sqrt(head_dim))[j],
+ * where the text keys k are the session's current ones and the image
+ * queries q' = H^l W_xq^T + b_xq use the hidden state entering block l as
+ * the cache holds it at timestep slot t: for l >= 1 the cached output of
+ * block l - 1 (bf16), for l = 0 the patch embedding of `latent` (f32
+ * [in_ch][grid_h*patch][grid_w*patch], the latent of step t).  The cache is
+ * only read.
+ *   scores  device f32 [N][text_len] (caller-owned, 16-B aligned): zeroed,
+ *           then the delta columns written; it is the [S = 1][N][M] score
+ *           map rc_localize_mask takes.
+ * Errors: RC_ERR_INVALID_ARG (bad session, t, ids or n_delta, a host-tier
+ * cache), RC_ERR_STATE (weights or the session's text not set). */
+rc_status rc_localize_scores(rc_ctx* ctx, rc_cache* cache, int session, int t,
+                             const float* latent, const int32_t* delta_ids_host, int n_delta,
+                             float* scores, rc_stream stream);
+
 /* Semantic-aware adaptive reuse scheduling (Section 3.3), host-only.
  * rc_prompt_similarity: Eq. 1, s = cos(e(tau-), e(tau+)) of two token
  *   embeddings (host arrays of dim floats), accumulated in double.

@@ -1221,6 +1221,88 @@ rc_status rc_step_capture(rc_ctx* c, rc_cache* k, int s, float* latent, int t,
   return step_items(c, k, &it, 1, st, &cap);
 }
 
+rc_status rc_localize_scores(rc_ctx* c, rc_cache* k, int s, int t, const float* latent,
+                             const int32_t* delta_ids_host, int n_delta, float* scores,
+                             rc_stream stream) {
+  if (!c || !k || !latent || !delta_ids_host || !scores)
+    return fail(RC_ERR_INVALID_ARG, "rc_localize_scores: null argument");
+  if (k->ctx != c) return fail(RC_ERR_INVALID_ARG, "cache belongs to another context");
+  if (k->host_tier)
+    return fail(RC_ERR_INVALID_ARG, "rc_localize_scores needs a device-tier cache");
+  rc_status r = check_session(k, s);
+  if (r) return r;
+  if (t < 0 || t >= c->T) return fail(RC_ERR_INVALID_ARG, "t %d outside [0, %d)", t, c->T);
+  if (n_delta < 1 || n_delta > 8)
+    return fail(RC_ERR_INVALID_ARG, "n_delta %d not in 1..8", n_delta);
+  if (!aligned16(scores) || !aligned16(latent))
+    return fail(RC_ERR_INVALID_ARG, "scores / latent not 16-B aligned");
+  rc::AttnCapture cap{};
+  cap.n = n_delta;
+  for (int q = 0; q < n_delta; ++q) {
+    if (delta_ids_host[q] < 0 || delta_ids_host[q] >= c->M)
+      return fail(RC_ERR_INVALID_ARG, "delta id %d outside [0, %d)", delta_ids_host[q], c->M);
+    cap.id[q] = delta_ids_host[q];
+  }
+  if ((r = check_ready(c, k, s, false))) return r;
+  cap.out = scores;
+  cap.ldo = c->M;
+  cap.w = 1.f / float(c->L * c->dims.heads);
+  const int N = c->N, d = c->d;
+  const rc_global_weights& g = c->gw;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  RC_CUDA(cudaMemsetAsync(scores, 0, sizeof(float) * size_t(N) * c->M, st), "scores reset");
+  // every token is a query row, in token order
+  const rc::RowMap rm{nullptr, nullptr, nullptr, N, nullptr, N};
+  // the state entering block 0: the patch embedding of the latent (f32),
+  // then its bf16 copy for the query side of the cross-attention
+  rc::Items its{};
+  its.n = 1;
+  its.latent[0] = const_cast<float*>(latent);
+  RC_CUDA(rc::launch_patch_embed(c->dims.grid_h, c->dims.grid_w, c->dims.patch, c->dims.in_ch,
+                                 static_cast<const bf16*>(g.W_e), g.b_e, g.pos, its, rm, c->xf, d,
+                                 c->err, st),
+          "patch_embed");
+  rc::Items cast{};
+  cast.n = 1;
+  cast.slice[0] = c->xb;
+  RC_CUDA(rc::launch_scatter_bf16(c->xf, cast, 0, rm, d, c->err, st), "embedding cast");
+  for (int l = 0; l < c->L; ++l) {
+    // the input of block l as cached at step t: block l - 1's output slot
+    const bf16* h_in = l == 0 ? c->xb : k->slot(s, l - 1, t, 0);
+    if (k->xg) {
+      // (x W_xq^T + b) K^T = x G_h^T + kb_h with the folded text keys; the
+      // kernel's P V output goes to scratch, only the captured columns matter
+      rc::XqItems xi{};
+      xi.n = 1;
+      xi.grow[0] = int(k->xg_row(s, l));
+      xi.vrow[0] = (s * c->L + l) * c->M;
+      RC_CUDA(rc::launch_xattn_fused(h_in, d, k->xg, k->xgb, int(k->xg_rows()), k->text + d,
+                                     2 * d, k->sessions * c->L * c->M, xi, c->M, c->ob, d,
+                                     c->dims.heads, c->dh, rm, c->err, st, &cap),
+              "scores(cross)");
+    } else {
+      rc::GemmEpi e{};
+      e.mode = rc::EPI_BIAS_BF16;
+      e.bias = c->lw[l].b_xq;
+      e.out_bf = c->q;
+      e.ld_out = d;
+      e.gate_off = -1;
+      e.err = c->err;
+      RC_CUDA(rc::launch_gemm(h_in, d, static_cast<const bf16*>(c->lw[l].W_xq), N, nullptr, d,
+                              d, e, st), "gemm(xq)");
+      StepItems si;
+      si.its.n = 1;
+      si.session[0] = s;
+      si.t[0] = t;
+      RC_CUDA(rc::launch_attention(c->q, d, k->text, k->text + d, 2 * d,
+                                   k->sessions * c->L * c->M, text_kv_rows(k, si, l), c->M,
+                                   c->ob, d, c->dims.heads, c->dh, rm, c->err, c->as, st, &cap),
+              "scores(cross)");
+    }
+  }
+  return RC_OK;
+}
+
 rc_status rc_prompt_similarity(const float* e_minus, const float* e_plus, int dim, float* s_out) {
   if (!e_minus || !e_plus || !s_out || dim <= 0)
     return fail(RC_ERR_INVALID_ARG, "rc_prompt_similarity: null argument or dim <= 0");

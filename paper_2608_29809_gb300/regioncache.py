@@ -99,6 +99,7 @@ def load_library(path: str = LIB_PATH) -> C.CDLL:
         "rc_localize_workspace_size": (S, [I, I]),
         "rc_localize_mask": (I, [P, I, I, I, I, I, P, I, F, I, P, P, P, P, S, P]),
         "rc_localize_mask_noalloc": (I, [P, I, I, I, I, I, P, I, F, I, P, P, P, P]),
+        "rc_localize_scores": (I, [P, P, I, I, P, P, I, P, P]),
         "rc_block_forward_region": (I, [P, P, I, I, I, P, P, I, P, P, P]),
         "rc_step": (I, [P, P, I, P, I, P, P, I, P, P]),
         "rc_step_batched": (I, [P, P, C.POINTER(rc_batch_item), I, P]),
@@ -236,6 +237,12 @@ def rc_localize_mask_noalloc(xattn, S, N, M, grid_h, grid_w, delta_ids, threshol
     _check(_lib.rc_localize_mask_noalloc(_ptr(xattn), S, N, M, grid_h, grid_w, ids.ctypes.data,
                                          len(ids), float(threshold), dilation, _ptr(mask),
                                          _ptr(dirty_idx), _ptr(dirty_count), _stream(stream)))
+
+
+def rc_localize_scores(ctx, cache, session, t, latent, delta_ids, scores, stream=None):
+    ids = np.ascontiguousarray(delta_ids, np.int32)
+    _check(_lib.rc_localize_scores(ctx, cache, session, t, _ptr(latent), ids.ctypes.data,
+                                   len(ids), _ptr(scores), _stream(stream)))
 
 
 def rc_block_forward_region(ctx, cache, session, layer, t, hidden, dirty_idx, D, dirty_count,
