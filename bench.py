@@ -224,11 +224,13 @@ class Workload:
             A, ids = synth.indicator_scores(d, blobs, seed)
             self.scores[f] = (torch.from_numpy(A).to(dev), ids, A)
 
-    def localize(self, f, A=None):
+    def localize(self, f, A=None, ids=None):
         d = self.d
-        A_dev, ids, _ = self.scores[f]
-        self.R.rc_localize_mask(A_dev if A is None else A, 1, d.tokens, d.text_len, d.grid_h,
-                                d.grid_w, ids, 0.5, 0, self.mask, self.idx, self.cnt, self.ws)
+        if ids is None:
+            A_dev, ids, _ = self.scores[f]
+            A = A_dev if A is None else A
+        self.R.rc_localize_mask(A, 1, d.tokens, d.text_len, d.grid_h, d.grid_w, ids, 0.5, 0,
+                                self.mask, self.idx, self.cnt, self.ws)
 
     def step(self, i, f):
         t = i % self.d.timesteps
@@ -308,6 +310,7 @@ class Workload:
 
             m = timed(step, K, W, world)
             R.rc_sync(self.model.ctx)
+            thp = thp_state()  # while the pool is still mapped
         finally:
             R.rc_cache_destroy(hc)
         slot = d.tokens * d.hidden * 2
@@ -317,7 +320,30 @@ class Workload:
                 "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": 3 * int(self.cnt.item()) * d.hidden * 2 * d.layers,
                 "h2d_gbs_over_step": round(h2d / (m / K / 1e3) / 1e9, 1),
-                "step": "rc_localize_mask + rc_step(SPARSE) on rc_cache_create_host"}
+                "step": "rc_localize_mask + rc_step(SPARSE) on rc_cache_create_host",
+                "thp": thp}
+
+
+def thp_state():
+    """Transparent-huge-page mode of the host and the anonymous huge pages in
+    use (read while the host-tier pool is mapped): the host tier's rate
+    depends on whether its pool got huge pages."""
+    out = {}
+    for k in ("enabled", "defrag"):
+        try:
+            with open(f"/sys/kernel/mm/transparent_hugepage/{k}") as f:
+                out[k] = f.read().strip()
+        except OSError:
+            out[k] = None
+    try:
+        with open("/proc/meminfo") as f:
+            for ln in f:
+                if ln.startswith(("AnonHugePages:", "Hugepagesize:")):
+                    k, v = ln.split(":", 1)
+                    out[k] = v.strip()
+    except OSError:
+        pass
+    return out
 
 
 def rate_batched(R, args, world, dev, K, W, n=8):
@@ -390,6 +416,205 @@ def rate_batched(R, args, world, dev, K, W, n=8):
             "session_steps_per_s_one_by_one": round(rate_1, 3),
             "speedup_of_batching": round(rate_b / rate_1, 3),
             "step": "rc_step_batched over all sessions (vs one rc_step per session)"}
+
+
+def pct(xs, q):
+    """q-th percentile (nearest rank) of a list."""
+    xs = sorted(xs)
+    return xs[min(len(xs) - 1, max(0, int(np.ceil(q / 100.0 * len(xs))) - 1))]
+
+
+def rate_server(R, args, world, dev, n=8, turns_per_session=2):
+    """Persistent serving through the cross-session scheduler (rc_server_*):
+    n 512 px sessions (1024 tokens, 28 blocks), turns arriving on a seeded
+    schedule (exponential gaps, mean 2.5 ticks; a session's next turn queues
+    until its previous one ends), each turn = T SPARSE steps over the
+    session's own ragged region (dirty fraction from U(2 %, 35 %)).  Every
+    tick is one rc_server_tick (one batched step over up to n running turns);
+    CUDA events around each tick give the per-tick latency, and a turn's
+    latency runs from the start of the tick at which it arrived to the end of
+    its last tick."""
+    from dataclasses import replace
+    d = replace(synth.PIXART_512, timesteps=args.resident_steps)
+    T = d.timesteps
+    seed = SEED + 13
+    w = synth.make_weights(d, seed, device=dev)
+    model = R.Model(d, w, sessions=n, device=dev, max_batch=n)
+    srv = None
+    try:
+        for s in range(n):
+            R.rc_set_text(model.ctx, model.cache, s, synth.make_text(d, seed + s, dev))
+            for t in range(T):
+                for l in range(d.layers):
+                    H, K_, V = synth.make_cache_slice(d, seed, s, l, t, device=dev)
+                    R.rc_cache_fill(model.cache, s, l, t, H, K_, V)
+        tv, ab = synth.ddim_tables(T)
+        R.rc_set_schedule(model.ctx, tv, ab)
+        rng = np.random.default_rng(seed)
+        fracs = rng.uniform(0.02, 0.35, size=n)
+        N = d.tokens
+        idx, cnt, lat0, lat = [], [], [], []
+        for s in range(n):
+            blobs = synth.ellipse_blobs(d, seed + s, float(fracs[s]))
+            A, ids = synth.indicator_scores(d, blobs, seed + s)
+            ws = torch.empty(R.rc_localize_workspace_size(N, len(ids)), dtype=torch.uint8,
+                             device=dev)
+            mask = torch.zeros(N, dtype=torch.uint8, device=dev)
+            idx.append(torch.zeros(N, dtype=torch.int32, device=dev))
+            cnt.append(torch.zeros(1, dtype=torch.int32, device=dev))
+            R.rc_localize_mask(torch.from_numpy(A).to(dev), A.shape[0], N, A.shape[2], d.grid_h,
+                               d.grid_w, ids, 0.5, 0, mask, idx[s], cnt[s], ws)
+            lat0.append(synth.make_latent(d, seed + s, dev))
+            lat.append(lat0[s].clone())
+        torch.cuda.synchronize()
+        dirty = [int(c.item()) for c in cnt]
+        sparse = np.full(T, R.RC_MODE_SPARSE, np.uint8)
+        # seeded arrivals: (tick, session), sessions in turn order
+        gaps = rng.exponential(2.5, size=n * turns_per_session)
+        arrivals = [(int(np.floor(g)), k % n) for k, g in enumerate(np.cumsum(gaps) - gaps[0])]
+        srv = R.rc_server_create(model.ctx, model.cache, n)
+
+        def run(record):
+            pending = list(arrivals)
+            waiting, started, done = [], {}, []
+            ev = []
+            tick = 0
+            while pending or waiting or R.rc_server_running(srv):
+                while pending and pending[0][0] <= tick:
+                    waiting.append(pending.pop(0))
+                for a in list(waiting):
+                    s = a[1]
+                    if R.rc_server_state(srv, s) < 0:
+                        lat[s].copy_(lat0[s])
+                        R.rc_server_admit(srv, s, lat[s], sparse, idx[s], -1, cnt[s])
+                        started[s] = (a[0], tick)
+                        waiting.remove(a)
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record()
+                stepped = R.rc_server_tick(srv, n)
+                e1.record()
+                ev.append((e0, e1, stepped))
+                for s in list(started):
+                    if R.rc_server_state(srv, s) < 0 and s in stepped:
+                        done.append((started.pop(s), tick))
+                tick += 1
+            torch.cuda.synchronize()
+            if not record:
+                return None
+            tick_ms = [a.elapsed_time(b) for a, b, st in ev if st]
+            t0 = ev[0][0]
+            start_of = [t0.elapsed_time(a) for a, _, _ in ev]
+            end_of = [t0.elapsed_time(b) for _, b, _ in ev]
+            turn_ms = [end_of[e] - start_of[a_tick] for (a_tick, _), e in done]
+            total_ms = end_of[-1]
+            steps = sum(len(st) for _, _, st in ev)
+            return tick_ms, turn_ms, total_ms, steps, len(ev)
+
+        run(False)  # warm-up pass (tensor maps, tables)
+        tick_ms, turn_ms, total_ms, steps, ticks = run(True)
+        R.rc_sync(model.ctx)
+    finally:
+        if srv:
+            R.rc_server_destroy(srv)
+        model.close()
+    return {"workload": f"persistent serving: {n} sessions x pixart-alpha-512px ({d.tokens} "
+                        f"tokens, {d.layers} blocks, {T} timesteps), "
+                        f"{n * turns_per_session} turns on a seeded arrival schedule",
+            "dirty_tokens": dirty, "turns": len(turn_ms), "ticks": ticks,
+            "session_steps": steps,
+            "session_steps_per_s": round(steps / (total_ms / 1e3) * world, 3),
+            "tick_ms_p50": round(pct(tick_ms, 50), 3), "tick_ms_p99": round(pct(tick_ms, 99), 3),
+            "turn_ms_p50": round(pct(turn_ms, 50), 2), "turn_ms_p99": round(pct(turn_ms, 99), 2),
+            "step": "rc_server_tick: one rc_step_batched over up to 8 running turns, "
+                    "least recently stepped first"}
+
+
+def rate_session(wl, R, d, seed, turns=5):
+    """Multi-turn editing session at 1024 px (4096 tokens, 28 blocks, T = 20),
+    the cache updated in place from turn to turn.  Per turn: a new prompt
+    (rc_set_text), a seeded similarity s ~ U(0, 1) giving k = 2 (1 + min(3,
+    floor(4 (1 - s)))) fully recomputed leading steps -- the first one
+    rc_step_capture (DENSE + the delta tokens' scores), the rest DENSE graphs
+    -- then the turn's region (an ellipse map of f ~ U(5 %, 20 %): the
+    random-init model's own attention is not localised) through
+    rc_localize_mask, and SPARSE graphs for steps k .. T-1.  A second
+    session runs the paper's Eq. 2 schedule instead: T_reuse = floor(0.2 T)
+    REUSE steps, then the region localised from the cached states
+    (rc_localize_scores + rc_localize_mask) and SPARSE steps."""
+    T = d.timesteps
+    rng = np.random.default_rng(seed)
+    sims = rng.uniform(0.0, 1.0, size=turns)
+    fr = rng.uniform(0.05, 0.20, size=turns)
+    plans = []
+    for j in range(turns):
+        blobs = synth.ellipse_blobs(d, seed + 10 * j, float(fr[j]))
+        A, ids = synth.indicator_scores(d, blobs, seed + 10 * j)
+        # the workload's leading dense steps: k = 2 (1 + min(3, floor(4 (1 - s))))
+        k = 2 * (1 + min(3, int(np.floor(4.0 * (1.0 - float(sims[j]))))))
+        plans.append((k, torch.from_numpy(A).to(wl.dev), ids,
+                      synth.make_text(d, seed + 10 * j, wl.dev)))
+    cap = torch.empty(d.tokens, d.text_len, device=wl.dev)
+    ctx, cache = wl.model.ctx, wl.model.cache
+
+    def first_k():
+        ks = []
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for k, A, ids, text in plans:
+            R.rc_set_text(ctx, cache, 0, text)
+            wl.latent.copy_(wl.latent0)
+            R.rc_step_capture(ctx, cache, 0, wl.latent, 0, ids[:8], cap)
+            for t in range(1, k):
+                R.rc_graph_launch(wl.dense_graphs[t])
+            wl.localize(None, A=A, ids=ids)
+            for t in range(k, T):
+                R.rc_graph_launch(wl.graphs[t])
+            ks.append(k)
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1), ks
+
+    lat_scores = torch.empty(d.tokens, d.text_len, device=wl.dev)
+    t_reuse = int(np.floor(0.2 * T))
+    reuse = R.rc_reuse_schedule(0.0, 1.0, T, 0.2)
+
+    def eq2():
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for k, A, ids, text in plans:
+            R.rc_set_text(ctx, cache, 0, text)
+            wl.latent.copy_(wl.latent0)
+            for t in range(t_reuse):
+                R.rc_step(ctx, cache, 0, wl.latent, t, reuse, None, 0, None)
+            R.rc_localize_scores(ctx, cache, 0, t_reuse, wl.latent, ids[:8], lat_scores)
+            # the region of the random-init model's scores is not compact: the
+            # turn's ellipse map stands in for the mask (the score pass is timed)
+            wl.localize(None, A=A, ids=ids)
+            for t in range(t_reuse, T):
+                R.rc_graph_launch(wl.graphs[t])
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1)
+
+    first_k()
+    ms, ks = first_k()
+    eq2()
+    ms_eq2 = eq2()
+    steps = turns * T
+    return {"workload": f"{turns}-turn editing session, pixart-alpha-1024px ({d.tokens} tokens, "
+                        f"{d.layers} blocks, {T} timesteps), cache updated in place",
+            "first_k_dense": {"k_per_turn": ks, "session_ms": round(ms, 2),
+                              "steps_per_s": round(steps / (ms / 1e3), 3),
+                              "step": "rc_set_text, rc_step_capture, k-1 DENSE graphs, "
+                                      "rc_localize_mask, T-k SPARSE graphs per turn"},
+            "eq2_reuse_then_sparse": {"t_reuse": t_reuse, "session_ms": round(ms_eq2, 2),
+                                      "steps_per_s": round(steps / (ms_eq2 / 1e3), 3),
+                                      "step": "rc_set_text, T_reuse REUSE steps, "
+                                              "rc_localize_scores, rc_localize_mask, "
+                                              "T-T_reuse SPARSE graphs per turn"}}
 
 
 def rate_2048(R, args, world, dev, K, W):
@@ -489,6 +714,15 @@ def run_ours(args, world, rank, local):
     K, W = args.steps, args.warmup
     wl = Workload(R, d, SEED + rank, dev)
     peaks = load_peaks()
+    if args.dense_only:
+        m = timed(wl.step_dense, K, W, world)
+        R.rc_sync(wl.model.ctx)
+        if rank == 0:
+            print(json.dumps({"metric": METRIC, "dense_only": True, "unit": UNIT,
+                              "dense_steps_per_s": round(job_rate(K, m, world), 3),
+                              "steps": K, "warmup": W}), flush=True)
+        wl.model.close()
+        return
 
     # headline: 20 % dirty, each step = localisation + the CUDA graph of
     # rc_step for the timestep; clock sampler running, no probe events
@@ -558,6 +792,12 @@ def run_ours(args, world, rank, local):
     if not args.no_batched:
         batch = rate_batched(R, args, world, dev, K, W)
 
+    # persistent serving: turns arriving on a seeded schedule, through the
+    # cross-session scheduler
+    server = None
+    if not args.no_server:
+        server = rate_server(R, args, world, dev)
+
     # the same step at 2048 px (16 384 tokens, 63.4 GB cache resident)
     big = None
     if not args.no_2048:
@@ -598,11 +838,19 @@ def run_ours(args, world, rank, local):
            "h2d_bytes_per_step": int(A_host.numel() * 4 + lat_host.numel() * 4),
            "d2h_bytes_per_step": int(lat_host.numel() * 4)}
 
-    peak = peaks["bf16_tflops_sustained"]
+    # the 5-turn editing session at size (first k dense, then sparse), and
+    # the same turns under Eq. 2 with the region localised from the cache
+    session = None
+    if not args.no_session:
+        session = rate_session(wl, R, d, SEED + 17)
+
+    # burst peak: each launch is timed on its own (tens of microseconds), far
+    # shorter than the seconds-long loop the sustained figure needs
+    peak = peaks["bf16_tflops"]
     roofline, roof_att = kernel_rooflines(d, D, gemm_each, att_each, peak)
     roofline.update({"timing": "CUDA events around each launch, separate pass of the same "
                                "K steps",
-                     "peak_source": f"{peaks['source']} bf16_tflops_sustained"})
+                     "peak_source": f"{peaks['source']} bf16_tflops (burst)"})
     roof_dense, roof_att_dense = kernel_rooflines(d, d.tokens, gemm_each_d, att_each_d, peak)
     # LayerNorm-modulation launches (HBM-bound class): bytes per launch are
     # the D rows read as f32 and written as bf16, plus the bf16 H rows the
@@ -635,12 +883,15 @@ def run_ours(args, world, rank, local):
         "host_tier": host_tier,
         "pixart2048": big,
         "batched_serving": batch,
+        "persistent_serving": server,
+        "editing_session": session,
         "direct_steps_per_s": round(direct, 3),
         "speedup_vs_dense": {k: round(v / dense, 3) for k, v in sweep.items()},
         "roofline": roofline, "roofline_attention": roof_att,
         "roofline_dense": {"rows": d.tokens, "gemm": roof_dense, "attention": roof_att_dense},
         "roofline_ln": roof_ln,
-        "e2e": e2e, "gpu_launches": int(launches), "clocks": clk,
+        "e2e": e2e, "gpu_launches": int(launches),
+        "launches_per_step": round(launches / K, 2), "clocks": clk,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(d, SEED, HEADLINE, layers_sample=args.cpu_layers)
@@ -692,7 +943,7 @@ def cpu_baseline(d, seed, f, layers_sample=2):
     t_fin = time.perf_counter() - t0
     step_s = t_loc + d.layers * t_blk + t_fin
     return {"value": round(1.0 / step_s, 6), "unit": UNIT, "cores": os.cpu_count(),
-            "kind": "oracle",
+            "kind": "oracle", "extrapolated": True,
             "sample": f"one step of the headline workload ({int(f * 100)} % dirty, D={len(idx)}) "
                       f"timed as localisation + {layers_sample} of {d.layers} region blocks "
                       f"(scaled x{d.layers}/{layers_sample}) + final layer; float64 numpy",
@@ -724,20 +975,26 @@ def run_reference(args, world, rank):
     for i in range(args.warmup):
         one(i)
     ts = [one(i) for i in range(args.steps)]
-    step_s = t_fixed + d.layers * (sum(ts) / len(ts))
+    block_s = sum(ts) / len(ts)
+    step_s = t_fixed + d.layers * block_s
     v = 1.0 / step_s
-    sample = (f"each timed step is one of {layers_sample} oracle region blocks of the headline "
-              f"workload ({int(HEADLINE * 100)} % dirty, D={len(idx)}); steps/s = 1 / "
-              f"({d.layers} x mean block time + localisation + final layer)")
+    sample = (f"each timed step is ONE of the {d.layers} oracle region blocks of a headline step "
+              f"({int(HEADLINE * 100)} % dirty, D={len(idx)}; blocks {layers_sample} apart in "
+              f"weights and cache); value = 1 / ({d.layers} x mean block time + localisation + "
+              f"final layer), extrapolated to whole steps")
+    # "steps" / "ms_per_step" describe what was timed (blocks); the value is
+    # the extrapolated whole-step rate
     out = {"metric": METRIC, "value": round(v, 6), "unit": UNIT, "n_gpus": world,
-           "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_s * 1e3, 3),
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(block_s * 1e3, 3),
+           "timed_unit": f"one region block (1/{d.layers} of a step)", "extrapolated": True,
+           "ms_per_whole_step": round(step_s * 1e3, 3),
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
            "data": "synthetic", "impl": "reference",
            "config": {"workload": WORKLOAD, "tokens": d.tokens, "dirty_frac": HEADLINE,
                       "dirty_tokens": int(len(idx)), "layers": d.layers,
                       "timesteps": d.timesteps},
            "cpu_baseline": {"value": round(v, 6), "unit": UNIT, "cores": os.cpu_count(),
-                            "kind": "oracle", "sample": sample},
+                            "kind": "oracle", "sample": sample, "extrapolated": True},
            "e2e": {"value": round(v, 6), "unit": UNIT, "h2d_bytes_per_step": 0,
                    "d2h_bytes_per_step": 0}}
     print(json.dumps(out), flush=True)
@@ -759,6 +1016,13 @@ def main():
                     help="skip the 2048 px (16 384-token, 63 GB cache) measurement")
     ap.add_argument("--no-host-tier", action="store_true",
                     help="skip the host-tier cache measurement (a pinned host pool)")
+    ap.add_argument("--no-server", action="store_true",
+                    help="skip the persistent-serving measurement (rc_server, 8 x 512 px)")
+    ap.add_argument("--no-session", action="store_true",
+                    help="skip the 5-turn editing-session measurement")
+    ap.add_argument("--dense-only", action="store_true",
+                    help="profiling mode: K launch-by-launch DENSE steps of the headline model "
+                         "and nothing else (prints one line)")
     ap.add_argument("--resident-steps", type=int, default=20,
                     help="timesteps held in the cache (1 keeps a profiling run to ~2 GB)")
     args = ap.parse_args()

@@ -401,6 +401,43 @@ rc_status rc_step_graph_create(rc_ctx* ctx, rc_cache* cache, int session, float*
 rc_status rc_graph_launch(rc_graph* graph, rc_stream stream);
 void rc_graph_destroy(rc_graph* graph);
 
+/* Cross-session serving scheduler (no counterpart in the paper, which serves
+ * one request at a time): editing sessions join and leave between steps,
+ * and every tick runs ONE rc_step_batched over up to max_items of the turns
+ * in progress, each at its own timestep, so that one pass over the weights
+ * serves them all.  A turn = the steps t = 0 .. timesteps-1 of one session,
+ * in order, each computed exactly as rc_step would compute it.  When more
+ * turns are running than a tick takes, the least recently stepped go first
+ * (ties: admission order), so every turn advances in round robin.  Host
+ * state only; drive a server from one host thread, and let no other call
+ * step the sessions it is running.
+ *   rc_server_create   max_items in [1, the context's max_batch] (1 for a
+ *                      host-tier cache).
+ *   rc_server_admit    starts a turn of `session` (not already running):
+ *                      latent f32 [in_ch][grid_h*patch][grid_w*patch]
+ *                      device, in/out; schedule_host[timesteps] modes
+ *                      (copied); dirty_idx / D / dirty_count as in rc_step,
+ *                      read at each SPARSE step (borrowed until the turn
+ *                      ends).
+ *   rc_server_tick     one batched step on `stream`; sessions_out (host,
+ *                      max_items entries, may be null) receives the sessions
+ *                      stepped, *n_out their number (0 when no turn is
+ *                      running).  A turn whose last step ran leaves the
+ *                      server.  On an error nothing advances.
+ *   rc_server_state    *next_t = the next step of the session's running
+ *                      turn, or -1 when it has none.
+ *   rc_server_running  number of turns in progress.
+ * Errors: RC_ERR_INVALID_ARG, and those of rc_step_batched. */
+typedef struct rc_server rc_server;
+rc_status rc_server_create(rc_ctx* ctx, rc_cache* cache, int max_items, rc_server** out);
+void rc_server_destroy(rc_server* server);
+rc_status rc_server_admit(rc_server* server, int session, float* latent,
+                          const uint8_t* schedule_host, const int32_t* dirty_idx, int D,
+                          const int32_t* dirty_count);
+rc_status rc_server_tick(rc_server* server, rc_stream stream, int* sessions_out, int* n_out);
+rc_status rc_server_state(const rc_server* server, int session, int* next_t);
+int rc_server_running(const rc_server* server);
+
 /* Full-recompute baseline: rc_step with mode DENSE. */
 rc_status rc_step_dense(rc_ctx* ctx, rc_cache* cache, int session, float* latent, int t,
                         rc_stream stream);

@@ -6,14 +6,25 @@
 #include <stddef.h>
 #include <stdint.h>
 
+struct rc_ctx;
+struct rc_cache;
+
 namespace rc {
 
 typedef __nv_bfloat16 bf16;
 
 // Kernels launched by this library in this process (reported by rc_launch_count).
 void count_launches(int n);
+
 // Sets the calling thread's rc_last_error() text.
 void set_last_error(const char* msg);
+
+// Facts about a context / cache for host code outside regioncache.cu.
+int ctx_max_batch(const ::rc_ctx* c);
+int ctx_timesteps(const ::rc_ctx* c);
+const ::rc_ctx* cache_context(const ::rc_cache* k);
+int cache_sessions(const ::rc_cache* k);
+bool cache_host_tier(const ::rc_cache* k);
 
 // ------------------------------------------------------------- localisation
 struct DeltaIds {

@@ -139,6 +139,14 @@ struct rc_cache {
   size_t xg_rows() const { return xg_row(sessions, 0); }
 };
 
+namespace rc {
+int ctx_max_batch(const ::rc_ctx* c) { return c->max_batch; }
+int ctx_timesteps(const ::rc_ctx* c) { return c->T; }
+const ::rc_ctx* cache_context(const ::rc_cache* k) { return k->ctx; }
+int cache_sessions(const ::rc_cache* k) { return k->sessions; }
+bool cache_host_tier(const ::rc_cache* k) { return k->host_tier; }
+}  // namespace rc
+
 namespace {
 
 __global__ void iota_kernel(int* p, int n) {

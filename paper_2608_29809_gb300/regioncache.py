@@ -100,6 +100,12 @@ def load_library(path: str = LIB_PATH) -> C.CDLL:
         "rc_localize_mask": (I, [P, I, I, I, I, I, P, I, F, I, P, P, P, P, S, P]),
         "rc_localize_mask_noalloc": (I, [P, I, I, I, I, I, P, I, F, I, P, P, P, P]),
         "rc_localize_scores": (I, [P, P, I, I, P, P, I, P, P]),
+        "rc_server_create": (I, [P, P, I, C.POINTER(P)]),
+        "rc_server_destroy": (None, [P]),
+        "rc_server_admit": (I, [P, I, P, P, P, I, P]),
+        "rc_server_tick": (I, [P, P, P, C.POINTER(I)]),
+        "rc_server_state": (I, [P, I, C.POINTER(I)]),
+        "rc_server_running": (I, [P]),
         "rc_block_forward_region": (I, [P, P, I, I, I, P, P, I, P, P, P]),
         "rc_step": (I, [P, P, I, P, I, P, P, I, P, P]),
         "rc_step_batched": (I, [P, P, C.POINTER(rc_batch_item), I, P]),
@@ -243,6 +249,40 @@ def rc_localize_scores(ctx, cache, session, t, latent, delta_ids, scores, stream
     ids = np.ascontiguousarray(delta_ids, np.int32)
     _check(_lib.rc_localize_scores(ctx, cache, session, t, _ptr(latent), ids.ctypes.data,
                                    len(ids), _ptr(scores), _stream(stream)))
+
+
+def rc_server_create(ctx, cache, max_items) -> int:
+    out = C.c_void_p()
+    _check(_lib.rc_server_create(ctx, cache, max_items, C.byref(out)))
+    return out.value
+
+
+def rc_server_destroy(server):
+    _lib.rc_server_destroy(server)
+
+
+def rc_server_admit(server, session, latent, schedule, dirty_idx, D, dirty_count):
+    sch = np.ascontiguousarray(schedule, np.uint8)
+    _check(_lib.rc_server_admit(server, session, _ptr(latent), sch.ctypes.data, _ptr(dirty_idx),
+                                D, _ptr(dirty_count)))
+
+
+def rc_server_tick(server, max_items, stream=None):
+    """One tick; returns the list of sessions it stepped."""
+    buf = (C.c_int * max(1, max_items))()
+    n = C.c_int()
+    _check(_lib.rc_server_tick(server, _stream(stream), buf, C.byref(n)))
+    return [buf[i] for i in range(n.value)]
+
+
+def rc_server_state(server, session) -> int:
+    t = C.c_int()
+    _check(_lib.rc_server_state(server, session, C.byref(t)))
+    return t.value
+
+
+def rc_server_running(server) -> int:
+    return int(_lib.rc_server_running(server))
 
 
 def rc_block_forward_region(ctx, cache, session, layer, t, hidden, dirty_idx, D, dirty_count,

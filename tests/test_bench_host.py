@@ -54,3 +54,11 @@ def test_kernel_rooflines_from_event_times(per_block):
     assert roof_att["achieved"] == pytest.approx(att / (sum(att_each) / 1e3) / 1e12, abs=0.006)
     assert roof_att["per_launch"]["self"]["keys"] == d.tokens
     assert roof_att["per_launch"]["cross"]["keys"] == d.text_len
+
+
+def test_nearest_rank_percentiles():
+    xs = [5.0, 1.0, 4.0, 2.0, 3.0]
+    assert bench.pct(xs, 50) == 3.0
+    assert bench.pct(xs, 99) == 5.0
+    assert bench.pct(xs, 1) == 1.0
+    assert bench.pct(list(range(1, 101)), 99) == 99

@@ -43,30 +43,31 @@ def _normalised(col):
     return (col - lo) / (hi - lo)
 
 
-def _gpu_mask(R, scores, ids, d):
+def _gpu_mask(R, scores, ids, d, dil=1):
     N = d.tokens
     ws = torch.empty(R.rc_localize_workspace_size(N, len(ids)), dtype=torch.uint8, device="cuda")
     mask = torch.zeros(N, dtype=torch.uint8, device="cuda")
     idx = torch.zeros(N, dtype=torch.int32, device="cuda")
     cnt = torch.zeros(1, dtype=torch.int32, device="cuda")
-    R.rc_localize_mask(scores, 1, N, d.text_len, d.grid_h, d.grid_w, ids, 0.5, 1, mask, idx,
+    R.rc_localize_mask(scores, 1, N, d.text_len, d.grid_h, d.grid_w, ids, 0.5, dil, mask, idx,
                        cnt, ws)
     torch.cuda.synchronize()
     return mask, idx, cnt
 
 
-def _check_mask(mask_gpu, ref, ids, d):
+def _check_mask(mask_gpu, ref, ids, d, dil=1):
     """The GPU mask equals the oracle's except on tokens whose normalised
     oracle score lies within 0.02 of the threshold (or next to one, through
     the dilation)."""
-    m_ref, _ = O.localize_mask(ref.astype(np.float32)[None], ids, d.grid_h, d.grid_w, 0.5, 1)
+    m_ref, _ = O.localize_mask(ref.astype(np.float32)[None], ids, d.grid_h, d.grid_w, 0.5, dil)
     diff = np.flatnonzero(mask_gpu != m_ref)
     if len(diff):
         near = np.zeros(d.tokens, bool)
         for j in ids:
             near |= np.abs(_normalised(ref[:, j]) - 0.5) <= 0.02
-        near = binary_dilation(near.reshape(d.grid_h, d.grid_w), np.ones((3, 3), bool))
-        near = near.reshape(-1)
+        if dil:
+            near = binary_dilation(near.reshape(d.grid_h, d.grid_w),
+                                   np.ones((2 * dil + 1, 2 * dil + 1), bool)).reshape(-1)
         assert np.all(near[diff]), diff[~near[diff]]
     return m_ref
 
@@ -93,7 +94,9 @@ def test_cached_scores_small(R, ids):
 
 def test_cached_scores_then_localise_512px(R):
     """28 blocks at 1024 tokens: scores from the cache feed the localisation
-    kernel; the normalised scores agree with the oracle's to 0.02."""
+    kernel; the normalised scores agree with the oracle's to 0.02.  (The
+    synthetic states are unrelated to the text, so the regions are scattered:
+    no dilation, or the union would cover the grid.)"""
     d = synth.PIXART_512
     p = Problem(R, d, 1234 + 521, ts=(3,))
     try:
@@ -105,8 +108,8 @@ def test_cached_scores_then_localise_512px(R):
         for j in ids:
             assert np.max(np.abs(_normalised(got[:, j]) - _normalised(ref[:, j]))) <= 0.02
         mask, idx, cnt = _gpu_mask(R, torch.from_numpy(got.astype(np.float32)[None]).cuda(),
-                                   ids, d)
-        _check_mask(mask.cpu().numpy(), ref, ids, d)
+                                   ids, d, 0)
+        _check_mask(mask.cpu().numpy(), ref, ids, d, 0)
         assert 0 < int(cnt.item()) < d.tokens
     finally:
         p.close()
@@ -138,9 +141,10 @@ def test_eq2_turn_localised_from_the_cache_1024_tokens(R):
                 got = _gpu_scores(R, p, t, x, ids)
                 ref = _ref_scores(p, t, x64, ids)
                 block_close(got[:, ids], ref[:, ids], f"cached scores at t = {t}")
+                # (scattered regions on synthetic states: no dilation)
                 mask, idx_dev, cnt = _gpu_mask(
-                    R, torch.from_numpy(got.astype(np.float32)[None]).cuda(), ids, d)
-                _check_mask(mask.cpu().numpy(), ref, ids, d)
+                    R, torch.from_numpy(got.astype(np.float32)[None]).cuda(), ids, d, 0)
+                _check_mask(mask.cpu().numpy(), ref, ids, d, 0)
                 D = int(cnt.item())
                 assert 0 < D < d.tokens
                 idx_host = idx_dev[:D].cpu().numpy()
