@@ -49,9 +49,11 @@ constexpr int STAGING_BYTES = 12 * STAGING_WARP;
 
 // Operand ring: stages of A (16 KB) + B (BN x 128 B), as many as fit.
 constexpr int RING_BYTES = 168 * 1024;
-constexpr int MAX_STAGES = 8;
+constexpr int MAX_STAGES = 9;
 constexpr int TMEM_COLS = 512;  // two accumulators of up to 256 columns
-constexpr size_t SMEM_BYTES = size_t(RING_BYTES) + STAGING_BYTES + 1024 + 256;
+// per-tile column vectors of the epilogue: bias and gate of up to 256 columns
+constexpr int VEC_BYTES = 2 * 256 * 4;
+constexpr size_t SMEM_BYTES = size_t(RING_BYTES) + STAGING_BYTES + VEC_BYTES + 1024 + 256;
 // Instruction descriptor, kind::f16: D f32, A and B bf16, both K-major,
 // M >> 4 at bit 24; N >> 3 goes to bit 17 at run time.
 constexpr uint32_t IDESC_BASE = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(BM >> 4) << 24);
@@ -87,34 +89,70 @@ __device__ __forceinline__ void red_add_v4(float* p, float a, float b, float c, 
                : "memory");
 }
 
-// Epilogue values of columns c0 .. c0+31 of one output row: bias (when
-// with_bias: a split gated residual adds it with its first piece only, its
-// update being a sum over pieces), tanh-GELU, gate.
-__device__ __forceinline__ void epilogue_values(const GemmEpi& ep, int c0, int item, float* v,
-                                                bool with_bias) {
-  if (ep.bias && with_bias) {
-    float b[32];
-    load32(ep.bias + c0, b);
+__device__ __forceinline__ bool gated(const GemmEpi& ep) {
+  return (ep.mode == EPI_GATE_RES || ep.mode == EPI_GATE_RES_CAST) && ep.gate_tab;
+}
+// The gate's per-item part comes with each row (from its item's timestep
+// vector) only when the launch has several items; with one item it is
+// folded into the staged gate vector.
+__device__ __forceinline__ bool row_gate(const GemmEpi& ep) {
+  return gated(ep) && ep.gate_off >= 0 && ep.its.n > 1;
+}
+
+// The column vectors of one tile (columns col0 .. col0 + BN - 1) in shared
+// memory, written by the 384 epilogue threads before the accumulator is
+// ready: sv[c] = bias (0 when absent, or when this piece of a split gated
+// residual does not start at k = 0: the update is a sum over pieces, so the
+// bias goes with one of them), sv[256 + c] = gate (table part, plus the
+// item's timestep part when the launch has one item).
+__device__ __forceinline__ void stage_vectors(const GemmEpi& ep, int col0, int BN, bool with_bias,
+                                              float* sv, int etid) {
+  const float* tb0 = (ep.its.n == 1 && ep.gate_off >= 0) ? ep.its.tb[0] : nullptr;
+  for (int c = etid; c < BN; c += 384) {
+    const int col = col0 + c;
+    sv[c] = (ep.bias && with_bias) ? __ldg(ep.bias + col) : 0.f;
+    if (gated(ep)) sv[256 + c] = __ldg(ep.gate_tab + col) + (tb0 ? __ldg(tb0 + ep.gate_off + col) : 0.f);
+  }
+}
+
+// Epilogue values of columns c0 .. c0+31 of one output row (cl = c0 within
+// the tile): bias, tanh-GELU, gate, from the staged vectors (plus the row's
+// item gate when the launch has several items).
+__device__ __forceinline__ void epilogue_values(const GemmEpi& ep, int c0, int cl, int item,
+                                                float* v, const float* sv) {
+  const float4* b4 = reinterpret_cast<const float4*>(sv + cl);
 #pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] += b[i];
+  for (int i = 0; i < 8; ++i) {
+    const float4 b = b4[i];
+    v[4 * i] += b.x; v[4 * i + 1] += b.y; v[4 * i + 2] += b.z; v[4 * i + 3] += b.w;
   }
   if (ep.mode == EPI_GELU_BF16) {
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] = gelu_tanh(v[i]);
-  } else if ((ep.mode == EPI_GATE_RES || ep.mode == EPI_GATE_RES_CAST) && ep.gate_tab) {
+  } else if (gated(ep)) {
     float g[32];
-    load32(ep.gate_tab + c0, g);
-    const float* tb = ep.gate_off >= 0 ? ep.its.tb[item] : nullptr;
-    if (tb) {
-      float g2[32];
-      load32(tb + ep.gate_off + c0, g2);
+    const float4* g4 = reinterpret_cast<const float4*>(sv + 256 + cl);
 #pragma unroll
-      for (int i = 0; i < 32; ++i) g[i] += g2[i];
+    for (int i = 0; i < 8; ++i) {
+      const float4 a = g4[i];
+      g[4 * i] = a.x; g[4 * i + 1] = a.y; g[4 * i + 2] = a.z; g[4 * i + 3] = a.w;
+    }
+    if (row_gate(ep)) {
+      const float* tb = ep.its.tb[item];
+      if (tb) {
+        float g2[32];
+        load32(tb + ep.gate_off + c0, g2);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) g[i] += g2[i];
+      }
     }
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] *= g[i];
   }
 }
+
+// Named barrier of the 12 epilogue warps.
+__device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, 384;" ::: "memory"); }
 
 // Destination of columns c0 .. c0+31 of output row r, or null when the row is
 // beyond the live count (or its token / item index is bad: QKV raises
@@ -250,6 +288,10 @@ __device__ __forceinline__ void store_chunk(int mode, uint8_t* stg, int lane, co
 struct Sched {
   int BN, stages, mt, nt, tiles, kbt, G, whole, Gr, S;
   bool pair;
+  // every CTA holds at most one work item: its epilogue starts only once
+  // all of its MMAs have read the ring, so the ring may run on over the
+  // epilogue staging buffers that follow it
+  bool alias;
   long long Wr;
   // S > 0: split-S (requires tiles * S <= grid); S == 0: waves (+ stream-K)
   __host__ __device__ void plan(int M, int bn, int n, int k, int grid, bool additive, int s,
@@ -264,10 +306,13 @@ struct Sched {
     kbt = k / BK;
     G = pair ? grid / 2 : grid;
     S = s;
+    alias = false;
     if (S > 0) {
       whole = 0;
       Wr = 0;
       Gr = 0;
+      alias = true;  // one piece per CTA
+      stages = stages_for(bn, pr, true);
       return;
     }
     const int R = tiles % G;
@@ -277,14 +322,16 @@ struct Sched {
     long long g = Wr / MIN_KB_PER_CTA;
     if (g < 1) g = 1;
     Gr = split ? int(g < G ? g : G) : 0;
+    alias = whole <= G && Gr == 0;
+    stages = stages_for(bn, pr, alias);
   }
   // bytes of one stage in one CTA: A (128 x 64) and B (BN x 64, half of it
   // in each CTA of a pair)
   __host__ __device__ static int stage_bytes(int bn, bool pr) {
     return STAGE_A + (pr ? bn * BK : bn * BK * 2);
   }
-  __host__ __device__ static int stages_for(int bn, bool pr) {
-    const int s = RING_BYTES / stage_bytes(bn, pr);
+  __host__ __device__ static int stages_for(int bn, bool pr, bool alias = false) {
+    const int s = (RING_BYTES + (alias ? STAGING_BYTES : 0)) / stage_bytes(bn, pr);
     return s < MAX_STAGES ? s : MAX_STAGES;
   }
   // Estimated duration (SM cycles): k-blocks on the busiest CTA x per-k-block
@@ -394,8 +441,11 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   // 1024-aligned operand ring, epilogue staging, then barriers
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
+  // the staging buffers follow the ring; a CTA with one work item lets its
+  // ring run on over them (see Sched::alias)
   uint8_t* sStg = smem + RING_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sStg + STAGING_BYTES);
+  float* sVec = reinterpret_cast<float*>(sStg + STAGING_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sStg + STAGING_BYTES + VEC_BYTES);
   // bars: full[MAX_STAGES], empty[MAX_STAGES], tfull[2], tempty[2]
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * MAX_STAGES + 4);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -536,42 +586,52 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     // the accumulator is drained once every epilogue warp of the pair (or
     // CTA) has arrived on rank 0's barrier
     const uint32_t tempty_r0 = PAIR ? mapa_shared(tempty0, 0) : tempty0;
+    // every epilogue warp passes the same number of epi_sync barriers, also
+    // after a failed wait (it then skips the rest of the work), so that no
+    // warp is ever left waiting at one
+    bool ok = true;
     while (sg.next(t, kb0, kb1)) {
       const int mq = t % sc.mt, nn = t / sc.mt;
       const int m = PAIR ? 2 * mq + int(rank) : mq;
-      if (!mbar_wait_warp(tfull0 + 8 * acc, acc_phase, abort_flag)) goto timeout;
-      tc_fence_after();
+      // everything that does not depend on the accumulator first, while the
+      // main loop runs: the row's token / item, the tile's column vectors
       const int row = sp * 32 + lane;
       const int r = m * BM + row;
-      const uint32_t tbase = tmem_base + uint32_t(acc * 256) + (uint32_t(sp * 32) << 16);
       int tok = 0, item = 0;
       if (r < M) {
         if (ep.mode == EPI_QKV) tok = ep.tok ? __ldg(ep.tok + r) : r;
         if (ep.item) item = __ldg(ep.item + r);
       }
-      // a piece of a split tile only occurs for the gated residual, whose
-      // update is a sum: the bias goes with the piece that starts at k = 0
+      epi_sync();  // the previous tile's readers of sVec are done
+      stage_vectors(ep, nn * BN, BN, kb0 == 0, sVec, int(threadIdx.x) - 64);
+      epi_sync();
+      if (ok && !mbar_wait_warp(tfull0 + 8 * acc, acc_phase, abort_flag)) ok = false;
+      if (ok) {
+        tc_fence_after();
+        const uint32_t tbase = tmem_base + uint32_t(acc * 256) + (uint32_t(sp * 32) << 16);
 #pragma unroll 1
-      for (int ch = (warp - 2) >> 2; ch < BN / 32; ch += 3) {
-        float v[32];
-        tmem_ld32(tbase + uint32_t(ch * 32), v);
-        const int c0 = nn * BN + ch * 32;
-        epilogue_values(ep, c0, item, v, kb0 == 0);
-        bf16* xb_row = (ep.mode == EPI_GATE_RES_CAST && r < M)
-                           ? ep.out_bf + size_t(r) * ep.ld_out + c0 : nullptr;
-        store_chunk(ep.mode, sStg + (warp - 2) * STAGING_WARP, lane, v, chunk_dst(ep, r, M, tok, item, c0),
-                    xb_row);
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) {
-        if (PAIR)
-          mbar_arrive_cluster(tempty_r0 + 8 * acc);
-        else
-          mbar_arrive(tempty0 + 8 * acc);
+        for (int ch = (warp - 2) >> 2; ch < BN / 32; ch += 3) {
+          float v[32];
+          tmem_ld32(tbase + uint32_t(ch * 32), v);
+          const int c0 = nn * BN + ch * 32;
+          epilogue_values(ep, c0, ch * 32, item, v, sVec);
+          bf16* xb_row = (ep.mode == EPI_GATE_RES_CAST && r < M)
+                             ? ep.out_bf + size_t(r) * ep.ld_out + c0 : nullptr;
+          store_chunk(ep.mode, sStg + (warp - 2) * STAGING_WARP, lane, v,
+                      chunk_dst(ep, r, M, tok, item, c0), xb_row);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          if (PAIR)
+            mbar_arrive_cluster(tempty_r0 + 8 * acc);
+          else
+            mbar_arrive(tempty0 + 8 * acc);
+        }
       }
       if (++acc == 2) { acc = 0; acc_phase ^= 1; }
     }
+    if (!ok) goto timeout;
   }
   goto done;
 timeout:
