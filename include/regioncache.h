@@ -487,6 +487,18 @@ rc_status rc_probe_enable(rc_ctx* ctx, int which, int capacity);
 rc_status rc_probe_read(rc_ctx* ctx, double* total_ms, int* launches);
 rc_status rc_probe_read_each(rc_ctx* ctx, float* ms_out, int capacity, int* launches);
 
+/* Self-test of the device-side failure path (no counterpart in the paper):
+ * every kernel of this library that waits on another agent (an mbarrier, a
+ * flag) gives up after a bounded time, records RC_ERR_TIMEOUT in the
+ * context's error word and returns, so the context stays usable.  This
+ * entry point runs that bounded wait on its own: one thread polls a
+ * context-owned device flag for at most timeout_us (1 .. 10^6)
+ * microseconds; with set_flag = 0 nothing raises the flag, the wait gives
+ * up and the next rc_sync returns RC_ERR_TIMEOUT; with set_flag = 1 the
+ * flag is raised first and the wait ends at once.  Nothing faults or traps.
+ * Errors: RC_ERR_INVALID_ARG. */
+rc_status rc_selftest_wait(rc_ctx* ctx, int timeout_us, int set_flag, rc_stream stream);
+
 /* Number of kernels this library has launched in the calling process. */
 uint64_t rc_launch_count(void);
 

@@ -83,6 +83,7 @@ struct rc_ctx {
   int* b_item = nullptr; // [R] item of each compact row (batched steps)
   int* b_meta = nullptr; // [META_INTS] row offsets / counts / query tiles per item
   unsigned* err = nullptr;
+  unsigned* wait_flag = nullptr;  // the self-test's flag (rc_selftest_wait)
   rc::AttnScratch as{};  // key-split partial outputs
   // timing probe
   int probe_which = RC_PROBE_OFF;
@@ -149,6 +150,30 @@ bool cache_host_tier(const ::rc_cache* k) { return k->host_tier; }
 
 namespace {
 
+// The bounded device wait every waiting kernel of this library uses, on its
+// own: one thread polls `flag` until it is non-zero or `ns` nanoseconds of
+// the global timer have passed; then it records DEVERR_TIMEOUT in the error
+// word and returns.  With set_first the flag is raised first (the wait ends
+// at once).
+__global__ void selftest_wait_kernel(unsigned* flag, unsigned long long ns, int set_first,
+                                     unsigned* err) {
+  if (threadIdx.x != 0) return;
+  volatile unsigned* f = flag;
+  if (set_first) *f = 1u;
+  unsigned long long t0;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
+  while (*f == 0u) {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    if (t - t0 > ns) {
+      atomicOr(err, rc::DEVERR_TIMEOUT);
+      return;
+    }
+    __nanosleep(1000);
+  }
+  *f = 0u;  // lowered again for the next call
+}
+
 __global__ void iota_kernel(int* p, int n) {
   int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n) p[i] = i;
@@ -197,7 +222,7 @@ void free_ctx(rc_ctx* c) {
   probe_free(c);
   void* ps[] = {c->xf,   c->xb,   c->ob,   c->q,    c->u,      c->fbuf,
                 c->h1,   c->temb, c->tb,   c->iota, c->b_tok,  c->b_item,
-                c->b_meta, c->err, c->as.part};
+                c->b_meta, c->err, c->wait_flag, c->as.part};
   for (void* p : ps)
     if (p) cudaFree(p);
   delete c;
@@ -478,7 +503,7 @@ rc_status rc_create(const rc_dims* dims, rc_ctx** out) {
       (s = dalloc(&c->iota, N, "iota")) || (s = dalloc(&c->b_tok, R, "batch tok")) ||
       (s = dalloc(&c->b_item, R, "batch item")) ||
       (s = dalloc(&c->b_meta, size_t(rc::META_INTS), "batch meta")) ||
-      (s = dalloc(&c->err, 1, "err"))) {
+      (s = dalloc(&c->err, 1, "err")) || (s = dalloc(&c->wait_flag, 1, "wait flag"))) {
     free_ctx(c);
     return s;
   }
@@ -490,6 +515,7 @@ rc_status rc_create(const rc_dims* dims, rc_ctx** out) {
   iota_kernel<<<int((N + 255) / 256), 256>>>(c->iota, int(N));
   rc::count_launches(1);
   cudaError_t e = cudaMemset(c->err, 0, sizeof(unsigned));
+  if (e == cudaSuccess) e = cudaMemset(c->wait_flag, 0, sizeof(unsigned));
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
   if (e != cudaSuccess) {
     free_ctx(c);
@@ -1419,6 +1445,17 @@ rc_status rc_probe_read(rc_ctx* c, double* total_ms, int* launches) {
   double tot = 0.0;
   for (float v : ms) tot += v;
   *total_ms = tot;
+  return RC_OK;
+}
+
+rc_status rc_selftest_wait(rc_ctx* c, int timeout_us, int set_flag, rc_stream stream) {
+  if (!c) return fail(RC_ERR_INVALID_ARG, "rc_selftest_wait: null context");
+  if (timeout_us < 1 || timeout_us > 1000000)
+    return fail(RC_ERR_INVALID_ARG, "rc_selftest_wait: timeout %d us not in 1 .. 10^6", timeout_us);
+  selftest_wait_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(
+      c->wait_flag, 1000ull * unsigned(timeout_us), set_flag ? 1 : 0, c->err);
+  RC_CUDA(cudaGetLastError(), "selftest wait");
+  rc::count_launches(1);
   return RC_OK;
 }
 

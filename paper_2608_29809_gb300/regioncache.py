@@ -106,6 +106,7 @@ def load_library(path: str = LIB_PATH) -> C.CDLL:
         "rc_server_tick": (I, [P, P, P, C.POINTER(I)]),
         "rc_server_state": (I, [P, I, C.POINTER(I)]),
         "rc_server_running": (I, [P]),
+        "rc_selftest_wait": (I, [P, I, I, P]),
         "rc_block_forward_region": (I, [P, P, I, I, I, P, P, I, P, P, P]),
         "rc_step": (I, [P, P, I, P, I, P, P, I, P, P]),
         "rc_step_batched": (I, [P, P, C.POINTER(rc_batch_item), I, P]),
@@ -359,6 +360,10 @@ def rc_linear(ctx, x, W, b, y, rows, n, k, stream=None):
 def rc_attention(ctx, Q, ldq, K, V, ldkv, Nq, Nk, O, ldo, stream=None):
     _check(_lib.rc_attention(ctx, _ptr(Q), ldq, _ptr(K), _ptr(V), ldkv, Nq, Nk, _ptr(O), ldo,
                              _stream(stream)))
+
+
+def rc_selftest_wait(ctx, timeout_us, set_flag, stream=None):
+    _check(_lib.rc_selftest_wait(ctx, timeout_us, 1 if set_flag else 0, _stream(stream)))
 
 
 def rc_sync(ctx, stream=None):
