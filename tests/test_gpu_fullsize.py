@@ -184,3 +184,87 @@ def test_c4_multi_turn_session(R):
                                     f"turn {turn} t {t} layer {l} {key}")
     finally:
         p.close()
+
+
+def test_c4_session_at_full_size_sampled(R):
+    """The 5-turn session at its stated size: 4096 tokens, 28 blocks, T = 20
+    (15.85 GB cache), the cache updated in place across turns.  Every turn
+    sets a new prompt (rc_set_text), runs its first step as rc_step_capture
+    (DENSE + the delta tokens' scores) and k - 1 more DENSE steps, then its
+    region (an ellipse map, localised on the device) in SPARSE steps.  The
+    oracle cannot run 100 whole steps at this size, so it checks what it can
+    compute from the device's state: the dirty count of every turn; at the
+    first SPARSE step of the last turn, block 0 over all dirty rows (from the
+    step's input latent and the cache rows read back before the step)
+    against the H / K / V rows the device wrote; and at two SPARSE steps of
+    the last turn the clean rows of every layer, bitwise unchanged."""
+    d = synth.PIXART_1024
+    seed = 1234 + 330
+    T = d.timesteps
+    w = synth.make_weights(d, seed)
+    m = R.Model(d, w)
+    try:
+        L0 = {k: O.to64(v) for k, v in w.layers[0].items()}
+        G64 = {k: O.to64(v) for k, v in w.glob.items()}
+        pos64 = O.to64(w.pos)
+        for t in range(T):
+            for l in range(d.layers):
+                H, K, V = synth.make_cache_slice(d, seed, 0, l, t, device="cuda")
+                R.rc_cache_fill(m.cache, 0, l, t, H, K, V)
+        tv, ab = synth.ddim_tables(T)
+        R.rc_set_schedule(m.ctx, tv, ab)
+        scores = torch.empty(d.tokens, d.text_len, device="cuda")
+        n_turns = 5
+        for turn in range(n_turns):
+            last = turn == n_turns - 1
+            text = synth.make_text(d, seed + 10 * turn)
+            R.rc_set_text(m.ctx, m.cache, 0, text.cuda())
+            k = O.k_from_similarity(synth.similarity(seed, turn))
+            sched = O.schedule_first_k_dense(k, T)
+            f = synth.turn_dirty_fraction(seed, turn)
+            blobs = synth.ellipse_blobs(d, seed + turn, f)
+            A, ids = synth.indicator_scores(d, blobs, seed + turn)
+            x = synth.make_latent(d, seed + 17 * turn).cuda()
+            R.rc_step_capture(m.ctx, m.cache, 0, x, 0, ids[:8], scores)
+            for t in range(1, k):
+                R.rc_step(m.ctx, m.cache, 0, x, t, sched, None, 0, None)
+            _, idx_d, cnt = _localize(R, A, ids, d, 0)
+            _, idx = O.localize_mask(A, ids, d.grid_h, d.grid_w, 0.5, 0)
+            torch.cuda.synchronize()
+            assert int(cnt.item()) == len(idx) > 0
+            clean = torch.from_numpy(np.setdiff1d(np.arange(d.tokens), idx)).cuda()
+            for t in range(k, T):
+                check = last and t in (k, T - 1)
+                if check:
+                    x_before = x.cpu()
+                    before = []
+                    for l in range(d.layers):
+                        bufs = [torch.empty(d.tokens, d.hidden, dtype=torch.bfloat16,
+                                            device="cuda") for _ in range(3)]
+                        R.rc_cache_read(m.cache, 0, l, t, *bufs)
+                        before.append(bufs)
+                R.rc_step(m.ctx, m.cache, 0, x, t, sched, idx_d, -1, cnt)
+                if not check:
+                    continue
+                R.rc_sync(m.ctx)
+                for l in range(d.layers):
+                    after = [torch.empty(d.tokens, d.hidden, dtype=torch.bfloat16,
+                                         device="cuda") for _ in range(3)]
+                    R.rc_cache_read(m.cache, 0, l, t, *after)
+                    for b, a in zip(before[l], after):
+                        assert torch.equal(b[clean], a[clean]), (t, l)
+                    if l == 0 and t == k:
+                        got = {key: O.to64(v.cpu()) for key, v in zip("HKV", after)}
+                cache0 = {key: O.to64(v.cpu()) for key, v in zip("HKV", before[0])}
+                if t == k:
+                    temb = O.t_embed(float(tv[t]), G64)
+                    m6 = L0["table"] + O.t_block(temb, G64)
+                    xd = O.patch_embed(O.to64(x_before), idx, G64, pos64, d.patch)
+                    tkv = O.text_kv(O.to64(text), L0)
+                    new, _ = O.region_block(xd, idx, cache0, L0, m6, tkv, d.heads)
+                    for key in "HKV":
+                        block_close(got[key][idx], new[key][idx], f"block 0 {key}, t {t}")
+            R.rc_sync(m.ctx)
+            assert torch.isfinite(x).all()
+    finally:
+        m.close()
