@@ -790,7 +790,7 @@ xq_fold_kernel(const bf16* __restrict__ Kt, int ldk, const bf16* __restrict__ Wq
 // One (query tile, head) per CTA: S = xb_tile G_h^T accumulated over d in
 // 64-column k-blocks (TMA ring, M = 128, N = 128), then the softmax of
 // (S + kb) / sqrt(dh) per row, P over S in TMEM, O = P V, O / l stored.
-constexpr int XF_STAGES = 4;
+constexpr int XF_STAGES = 6;
 template <int DH>
 struct XFCfg {
   using C = ACfg<DH>;

@@ -249,13 +249,17 @@ __global__ void __launch_bounds__(LN_WARPS * 32)
 ln_mod_kernel(const float* __restrict__ x, const float* __restrict__ tab, int k_sh, int k_sc,
               const __grid_constant__ Items it, bf16* __restrict__ out, RowMap rm,
               long long hprev_off, int d, unsigned* err) {
-  pdl_wait();
-  pdl_trigger();
   // shift and scale staged once per CTA: tab (+ the item's tb when the
   // launch has one item; otherwise each row adds its item's tb).  Loads that
   // do not depend on one another are all issued before any is used (the
   // vectors and the live row count, then the row with its token and item),
   // so a CTA waits for about two L2 round trips before its arithmetic.
+  // The vectors and the row count are requested before the programmatic-
+  // dependency wait: this kernel is never the first of a step or a block
+  // call, and every kernel here waits for its predecessor before letting its
+  // successor start, so whatever was written two or more launches earlier
+  // (the modulation table and timestep vector, the dirty count) is complete
+  // when this kernel starts; only the rows x come from the predecessor.
   extern __shared__ __align__(16) float s_mod[];  // [2][d]
   const int lane = threadIdx.x & 31;
   const int nv = d / 128, nq = d / 4;
@@ -276,6 +280,8 @@ ln_mod_kernel(const float* __restrict__ x, const float* __restrict__ tab, int k_
     }
   }
   const int D = live_count(rm.count, rm.bound, err);
+  pdl_wait();
+  pdl_trigger();
   int r = blockIdx.x * LN_WARPS + (threadIdx.x >> 5);
   float4 v[LN_MAXV];
   int tok = 0, item = 0;
