@@ -255,11 +255,16 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
   const uint32_t tmem_base = *tmem_slot;
   const uint32_t tS0 = tmem_base, tO = tmem_base + 2 * BKV, tP = tO + 80;
 
-  pdl_wait();
-  pdl_trigger();
+  // the live row count (and, for several items, the row table) was written
+  // two or more launches earlier: read before the programmatic-dependency
+  // wait (every kernel of the library waits for its predecessor before
+  // letting its successor start); Q and the fresh K / V rows come from the
+  // predecessor
   const int D = live_count(rm.count, rm.bound, err);
   AttnSched sc;
   sc.init(query_tiles(rm, ai.n, D), heads, Nk, gridDim.x);
+  pdl_wait();
+  pdl_trigger();
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA
@@ -838,13 +843,16 @@ xfused_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  pdl_wait();
-  pdl_trigger();
+  // Before the programmatic-dependency wait this kernel reads only what was
+  // written two or more launches earlier (every kernel of the library waits
+  // for its predecessor before letting its successor start): the live row
+  // count and the turn's folded keys, key biases and text values.  Only the
+  // bf16 rows of x come from the predecessor.
   const int D = live_count(rm.count, rm.bound, err);
   const int qtiles = query_tiles(rm, xi.n, D);
   const int qt = int(blockIdx.x) / heads, h = int(blockIdx.x) - (int(blockIdx.x) / heads) * heads;
   // the grid covers the bound of the query tiles: CTAs past the live ones
-  // leave before taking tensor memory
+  // leave at once, before taking tensor memory
   if (qt >= qtiles) return;
   const bool live = true;
   const TileLoc tl = locate_tile(rm, xi.n, D, qt);
@@ -858,23 +866,35 @@ xfused_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
   bool ok = live;
   if (live && warp == 0 && lane == 0) {
     // ------------------------------------------------------------ TMA
+    // V and the folded keys of the first stages before the wait (each stage
+    // barrier expects both halves of its bytes), the x rows after it
     const int grow = xi.grow[tl.item] + h * XK;
     mbar_expect_tx(v_full, X::V_BYTES);
     tma_load_3d(saddr(sV), &tmV, v_full, 0, h, xi.vrow[tl.item]);
     if (C::TAIL) tma_load_3d(saddr(sV + X::V_ATOM), &tmV, v_full, 64, h, xi.vrow[tl.item]);
+    const int pre = nkb < XF_STAGES ? nkb : XF_STAGES;
+    for (int k = 0; k < pre; ++k) {
+      mbar_expect_tx(full0 + 8 * k, X::STAGE);
+      tma_load_3d(saddr(smem + k * X::STAGE + X::STAGE_A), &tmG, full0 + 8 * k, 0, k, grow);
+    }
+    pdl_wait();
+    pdl_trigger();
     for (int k = 0; k < nkb; ++k) {
       const int st = k % XF_STAGES;
-      if (!mbar_wait(empty0 + 8 * st, ((k / XF_STAGES) & 1) ^ 1, abort_flag)) {
-        *abort_flag = 1;
-        break;
-      }
-      mbar_expect_tx(full0 + 8 * st, X::STAGE);
       uint8_t* base = smem + st * X::STAGE;
+      if (k >= pre) {
+        if (!mbar_wait(empty0 + 8 * st, ((k / XF_STAGES) & 1) ^ 1, abort_flag)) {
+          *abort_flag = 1;
+          break;
+        }
+        mbar_expect_tx(full0 + 8 * st, X::STAGE);
+        tma_load_3d(saddr(base + X::STAGE_A), &tmG, full0 + 8 * st, 0, k, grow);
+      }
       tma_load_3d(saddr(base), &tmA, full0 + 8 * st, 0, k, tl.row0);
-      tma_load_3d(saddr(base + X::STAGE_A), &tmG, full0 + 8 * st, 0, k, grow);
     }
   } else if (live && warp == 1 && lane == 0) {
     // ------------------------------------------------------------ MMA
+    pdl_wait();
     const uint64_t da = sw128_desc(saddr(smem)), dg = sw128_desc(saddr(smem + X::STAGE_A));
     bool good = true;
     for (int k = 0; k < nkb && good; ++k) {
@@ -911,6 +931,7 @@ xfused_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
     const uint32_t lane_off = uint32_t(sp * 32) << 16;
     const int t128 = threadIdx.x - 64;  // 0 .. 127
     s_kb[t128] = t128 < Nk ? kb[size_t(xi.grow[tl.item]) + size_t(h) * XK + t128] : 0.f;
+    pdl_wait();  // (before any global write: the predecessor reads O's buffer)
     mbar_arrive(kb_ready);
     ok = mbar_sleep_warp(kb_ready, 0, abort_flag) && mbar_sleep_warp(s_full, 0, abort_flag);
     float l = 0.f;
@@ -1021,11 +1042,13 @@ template <int DH>
 __global__ void __launch_bounds__(256)
 attn_combine_kernel(const float* __restrict__ part, bf16* __restrict__ O, int ldo, int heads,
                     RowMap rm, int n_items, int Nk, int attn_grid, unsigned* err) {
-  pdl_wait();
-  pdl_trigger();
+  // the row count predates the attention launch (see attn_tc_kernel): read
+  // before the wait; the pieces come from the predecessor
   const int D = live_count(rm.count, rm.bound, err);
   AttnSched sc;
   sc.init(query_tiles(rm, n_items, D), heads, Nk, attn_grid);
+  pdl_wait();
+  pdl_trigger();
   if (!sc.streamk) return;
   const int lane = threadIdx.x & 31;
   for (int gw = blockIdx.x * 8 + (threadIdx.x >> 5); gw < sc.pairs * BQ; gw += gridDim.x * 8) {

@@ -485,13 +485,16 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   // arrivals can reach them
   if (PAIR) cluster_sync();
 
-  // everything above is private set-up; inputs written by earlier kernels
-  // are read only after the predecessor has completed
-  pdl_wait();
-  pdl_trigger();
+  // everything above is private set-up.  The live row count was written two
+  // or more launches earlier (a step's dirty count before its first block;
+  // every kernel of the library waits for its predecessor before letting its
+  // successor start), so it and the schedule come before the programmatic-
+  // dependency wait; the operands and the residual are read after it
   const int M = live_count(dcount, Mbound, ep.err);
   Sched sc;
   sc.init(M, n, k, int(gridDim.x), ep.mode, bt.w64, PAIR);
+  pdl_wait();
+  pdl_trigger();
   const int BN = sc.BN, STAGES = sc.stages;
   const int STAGE = Sched::stage_bytes(BN, PAIR);
   // schedule position: the pair (its row tiles 2p + rank) or the CTA
