@@ -1032,12 +1032,25 @@ xfused_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
   }
 }
 
-// Merge of the pieces of the pairs that stream-K cut: one warp per (pair,
-// query row).  The pieces come from CTAs cta_of(first block) .. cta_of(last
-// block); a CTA's piece is its first (slot 0) when its range starts inside
-// the pair, else its last (slot 1).  Lanes take the pieces' row max / sum in
-// turn, the warp reduces them, then lanes < DH / 4 accumulate 4 head-dim
-// columns each over the pieces.
+// Merge of the pieces of the pairs that stream-K cut.  The (pair, query row)
+// sequence is cut into equal contiguous runs, one per warp, so a warp's rows
+// mostly share one pair and its bookkeeping (which CTAs hold its pieces,
+// which workspace slot) is worked out once per pair.  The pieces of a pair
+// come from CTAs cta_of(first block) .. cta_of(last block); a CTA's piece is
+// its first (slot 0) when its range starts inside the pair, else its last
+// (slot 1).  Per row, lanes take the pieces' row max / sum in turn, the warp
+// reduces them, and lanes < DH / 4 accumulate 4 head-dim columns each over
+// the pieces.  With at most four pieces (the usual case) a row's loads go
+// out in one round, and the next row's before the current one is reduced.
+template <int DH>
+struct CombineRow {
+  float2 ml;     // lane q < np: piece q's row max / sum
+  float4 v[4];   // lanes < DH / 4: pieces 0..3, head-dim columns 4 lane ..
+  int qrow;      // output row; -1: nothing to do
+  int h;         // head
+  bool many;     // more than four pieces: the general path
+};
+
 template <int DH>
 __global__ void __launch_bounds__(256)
 attn_combine_kernel(const float* __restrict__ part, bf16* __restrict__ O, int ldo, int heads,
@@ -1051,86 +1064,78 @@ attn_combine_kernel(const float* __restrict__ part, bf16* __restrict__ O, int ld
   pdl_trigger();
   if (!sc.streamk) return;
   const int lane = threadIdx.x & 31;
-  for (int gw = blockIdx.x * 8 + (threadIdx.x >> 5); gw < sc.pairs * BQ; gw += gridDim.x * 8) {
+  const int total = sc.pairs * BQ;
+  const int nwarps = int(gridDim.x) * 8;
+  const int per = (total + nwarps - 1) / nwarps;
+  const int w = int(blockIdx.x) * 8 + (int(threadIdx.x) >> 5);
+  const int r0 = w * per, r1 = min(total, r0 + per);
+  // bookkeeping of the current pair
+  int cpair = -1, c_lo = 0, np = 0, slot_lo = 0, h = 0;
+  TileLoc tl{0, 0, 0};
+  auto piece = [&](int q, int row) {
+    const int c = c_lo + q;
+    return part + (size_t(c) * 2 + (q == 0 ? slot_lo : 0)) * (BQ * PART_STRIDE) +
+           size_t(row) * PART_STRIDE;
+  };
+  auto prep = [&](int gw, CombineRow<DH>& cr) {
+    cr.qrow = -1;
+    cr.many = false;
+    if (gw >= r1) return;
     const int pair = gw / BQ, row = gw - pair * BQ;
-    const int lo = pair * sc.nkb;
-    const int c_lo = sc.cta_of(lo), c_hi = sc.cta_of(lo + sc.nkb - 1);
-    if (c_lo == c_hi) continue;  // one CTA held the whole pair
-    const int qt = pair % sc.qtiles, h = pair / sc.qtiles;
-    const TileLoc tl = locate_tile(rm, n_items, D, qt);
-    if (row >= tl.rows) continue;
-    const int np = c_hi - c_lo + 1;
-    // CTAs after c_lo start inside the pair (their first piece); c_lo's
-    // piece is its first only when its range starts exactly at the pair
-    const int slot_lo = sc.bound(c_lo) == lo ? 0 : 1;
-    const float* base = part + size_t(row) * PART_STRIDE;
-    auto piece = [&](int q) {
-      const int c = c_lo + q;
-      return base + (size_t(c) * 2 + (q == 0 ? slot_lo : 0)) * (BQ * PART_STRIDE);
-    };
-    if (np <= 32) {
-      // lane q holds piece q's row max / sum; the first four pieces' columns
-      // are requested in the same round
-      float2 ml = make_float2(-INFINITY, 0.f);
-      if (lane < np) ml = __ldcg(reinterpret_cast<const float2*>(piece(lane) + DH));
-      float4 v0[4];
+    if (pair != cpair) {
+      cpair = pair;
+      const int lo = pair * sc.nkb;
+      c_lo = sc.cta_of(lo);
+      np = sc.cta_of(lo + sc.nkb - 1) - c_lo + 1;
+      slot_lo = sc.bound(c_lo) == lo ? 0 : 1;
+      const int qt = pair % sc.qtiles;
+      h = pair / sc.qtiles;
+      tl = locate_tile(rm, n_items, D, qt);
+    }
+    if (np == 1 || row >= tl.rows) return;  // one CTA held the whole pair
+    cr.qrow = tl.row0 + row;
+    cr.h = h;
+    if (np > 4) {
+      cr.many = true;
+      return;
+    }
+    cr.ml = lane < np ? __ldcg(reinterpret_cast<const float2*>(piece(lane, row) + DH))
+                      : make_float2(-INFINITY, 0.f);
 #pragma unroll
-      for (int e = 0; e < 4; ++e)
-        v0[e] = (e < np && lane < DH / 4)
-                    ? __ldcg(reinterpret_cast<const float4*>(piece(e)) + lane)
+    for (int e = 0; e < 4; ++e)
+      cr.v[e] = (e < np && lane < DH / 4)
+                    ? __ldcg(reinterpret_cast<const float4*>(piece(e, row)) + lane)
                     : make_float4(0.f, 0.f, 0.f, 0.f);
-      float M = ml.x;
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-      const float w = lane < np ? ex2_ftz(ml.x - M) : 0.f;
-      float L = w * ml.y;
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-      // lanes < DH / 4 accumulate 4 columns each, four pieces' loads in flight
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int q0 = 0; q0 < np; q0 += 4) {
-        float4 v[4];
-        float wq[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          wq[e] = __shfl_sync(0xffffffffu, w, (q0 + e) & 31);
-          v[e] = q0 == 0 ? v0[e]
-                 : (q0 + e < np && lane < DH / 4)
-                     ? __ldcg(reinterpret_cast<const float4*>(piece(q0 + e)) + lane)
-                     : make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float ww = q0 + e < np ? wq[e] : 0.f;
-          acc.x += ww * v[e].x;
-          acc.y += ww * v[e].y;
-          acc.z += ww * v[e].z;
-          acc.w += ww * v[e].w;
-        }
-      }
-      if (lane < DH / 4) {
-        const float inv = L > 0.f ? 1.f / L : 0.f;
-        const int qrow = tl.row0 + row;
-        *reinterpret_cast<uint2*>(O + size_t(qrow) * ldo + h * DH + 4 * lane) = make_uint2(
-            pack_bf16x2(acc.x * inv, acc.y * inv), pack_bf16x2(acc.z * inv, acc.w * inv));
-      }
-    } else {
-      // many pieces (very long key ranges): plain loops
+  };
+  auto store = [&](int qrow, int hh, float4 acc, float L) {
+    if (lane < DH / 4) {
+      const float inv = L > 0.f ? 1.f / L : 0.f;
+      *reinterpret_cast<uint2*>(O + size_t(qrow) * ldo + hh * DH + 4 * lane) = make_uint2(
+          pack_bf16x2(acc.x * inv, acc.y * inv), pack_bf16x2(acc.z * inv, acc.w * inv));
+    }
+  };
+  CombineRow<DH> cur, nxt;
+  prep(r0, cur);
+  for (int gw = r0; gw < r1; ++gw) {
+    const int np_cur = np;  // (prep of the next row may move to the next pair)
+    const int row_cur = gw - (gw / BQ) * BQ;
+    if (cur.many) {
+      // many pieces (very long key ranges): plain loops, no prefetch
       float M = -INFINITY;
-      for (int q = lane; q < np; q += 32) M = fmaxf(M, __ldcg(piece(q) + DH));
+      for (int q = lane; q < np_cur; q += 32) M = fmaxf(M, __ldcg(piece(q, row_cur) + DH));
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
       float L = 0.f;
-      for (int q = lane; q < np; q += 32) {
-        const float2 ml = __ldcg(reinterpret_cast<const float2*>(piece(q) + DH));
+      for (int q = lane; q < np_cur; q += 32) {
+        const float2 ml = __ldcg(reinterpret_cast<const float2*>(piece(q, row_cur) + DH));
         L += ex2_ftz(ml.x - M) * ml.y;
       }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
       if (lane < DH / 4) {
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int q = 0; q < np; ++q) {
-          const float* b = piece(q);
+        for (int q = 0; q < np_cur; ++q) {
+          const float* b = piece(q, row_cur);
           const float wq = ex2_ftz(__ldcg(b + DH) - M);
           const float4 v = __ldcg(reinterpret_cast<const float4*>(b) + lane);
           acc.x += wq * v.x;
@@ -1138,12 +1143,32 @@ attn_combine_kernel(const float* __restrict__ part, bf16* __restrict__ O, int ld
           acc.z += wq * v.z;
           acc.w += wq * v.w;
         }
-        const float inv = L > 0.f ? 1.f / L : 0.f;
-        const int qrow = tl.row0 + row;
-        *reinterpret_cast<uint2*>(O + size_t(qrow) * ldo + h * DH + 4 * lane) = make_uint2(
-            pack_bf16x2(acc.x * inv, acc.y * inv), pack_bf16x2(acc.z * inv, acc.w * inv));
+      }
+      store(cur.qrow, cur.h, acc, L);
+      prep(gw + 1, nxt);
+    } else {
+      prep(gw + 1, nxt);  // the next row's loads go out before this row's reduction
+      if (cur.qrow >= 0) {
+        float M = cur.ml.x;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+        const float wl = lane < np_cur ? ex2_ftz(cur.ml.x - M) : 0.f;
+        float L = wl * cur.ml.y;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float ww = e < np_cur ? __shfl_sync(0xffffffffu, wl, e) : 0.f;
+          acc.x += ww * cur.v[e].x;
+          acc.y += ww * cur.v[e].y;
+          acc.z += ww * cur.v[e].z;
+          acc.w += ww * cur.v[e].w;
+        }
+        store(cur.qrow, cur.h, acc, L);
       }
     }
+    cur = nxt;
   }
 }
 
