@@ -382,8 +382,8 @@ patch_embed_kernel(int gh, int gw, int p, int C, const bf16* __restrict__ We,
                    const float* __restrict__ be, const float* __restrict__ pos,
                    const __grid_constant__ Items it, RowMap rm, float* __restrict__ xf, int d,
                    unsigned* err) {
-  pdl_wait();
-  pdl_trigger();
+  // W_e is staged before the programmatic-dependency wait (weights never
+  // change during a step); the latent, the row map and xf after it
   extern __shared__ __align__(16) uint8_t pe_smem[];
   bf16* s_w = reinterpret_cast<bf16*>(pe_smem);  // [d][16], zero beyond P
   const int P = C * p * p;                         // <= 16
@@ -397,6 +397,8 @@ patch_embed_kernel(int gh, int gw, int p, int C, const bf16* __restrict__ We,
       s_w[e] = k < P ? We[size_t(o) * P + k] : f2bf(0.f);
     }
   }
+  pdl_wait();
+  pdl_trigger();
   __syncthreads();
   const int D = live_count(rm.count, rm.bound, err);
   const int lane = threadIdx.x & 31;
@@ -528,8 +530,11 @@ final_ddim_kernel(const bf16* __restrict__ H, const float* __restrict__ temb,
                   const float* __restrict__ table_f, const bf16* __restrict__ Wf,
                   const float* __restrict__ bfin, float* __restrict__ latent, int gh, int gw,
                   int p, int c_in, int c_out, int d, float ab_t, float ab_next) {
-  pdl_wait();
-  pdl_trigger();
+  // the modulation vectors and the eps rows of W_f are staged before the
+  // programmatic-dependency wait: the weights never change during a step and
+  // temb was written at its start, two or more launches earlier (every
+  // kernel of the library waits for its predecessor before letting its
+  // successor start); H and the latent are read after the wait
   extern __shared__ uint8_t smem_raw[];
   float* s_shift = reinterpret_cast<float*>(smem_raw);
   float* s_scale = s_shift + d;
@@ -547,6 +552,8 @@ final_ddim_kernel(const bf16* __restrict__ H, const float* __restrict__ temb,
     reinterpret_cast<uint4*>(s_w + size_t(e) * d)[c8] =
         __ldg(reinterpret_cast<const uint4*>(Wf + size_t(sub * c_out + ch) * d) + c8);
   }
+  pdl_wait();
+  pdl_trigger();
   __syncthreads();
   const int N = gh * gw;
   const int lane = threadIdx.x & 31;
