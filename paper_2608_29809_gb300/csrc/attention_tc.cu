@@ -95,10 +95,13 @@ struct ACfg {
   // is a single MMA of N = DHP per 16 keys (MN-major B spanning the atoms)
   static constexpr int K_BYTES = K128 + K32;
   static constexpr int V_BYTES = TAIL ? 2 * K128 : K128;
-  static constexpr int STAGES = TAIL ? 3 : 4;
+  // separate rings: K (read by the S MMAs, refilled by the thread that
+  // issues them) and V (read by the P V MMAs, refilled by their issuer)
+  static constexpr int K_STAGES = TAIL ? 4 : 5;
+  static constexpr int V_STAGES = TAIL ? 3 : 4;
   static constexpr int Q_BYTES = Q128 + Q32;
-  static constexpr int KV_BYTES = K_BYTES + V_BYTES;  // K then V
-  static constexpr size_t SMEM = size_t(Q_BYTES) + STAGES * KV_BYTES + 1024 + 256;
+  static constexpr size_t SMEM =
+      size_t(Q_BYTES) + K_STAGES * K_BYTES + V_STAGES * V_BYTES + 1024 + 256;
   // kind::f16, D f32, A/B bf16; S: both K-major; PV: B (V) MN-major (bit 16)
   static constexpr uint32_t IDESC_S = (1u << 4) | (1u << 7) | (1u << 10) |
                                       (uint32_t(BKV >> 3) << 17) | (uint32_t(BQ >> 4) << 24);
@@ -204,17 +207,19 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
+  constexpr int KS = C::K_STAGES, VS = C::V_STAGES;
   uint8_t* sQ = smem;
-  uint8_t* sKV = sQ + C::Q_BYTES;
-  constexpr int KV_STAGES = C::STAGES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sKV + KV_STAGES * C::KV_BYTES);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 24);
+  uint8_t* sK = sQ + C::Q_BYTES;
+  uint8_t* sV = sK + KS * C::K_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sV + VS * C::V_BYTES);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 30);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   // barrier addresses
   const uint32_t b0 = saddr(bars);
   const uint32_t q_full = b0, q_empty = b0 + 8;
-  const uint32_t kv_full = b0 + 16, kv_empty = kv_full + 8 * KV_STAGES;
-  const uint32_t s_full = kv_empty + 8 * KV_STAGES;  // [2]: S of a block is in TMEM
+  const uint32_t k_full = b0 + 16, k_empty = k_full + 8 * KS;
+  const uint32_t v_full = k_empty + 8 * KS, v_empty = v_full + 8 * VS;
+  const uint32_t s_full = v_empty + 8 * VS;          // [2]: S of a block is in TMEM
   const uint32_t s_free = s_full + 16;               // [2]: the softmax has read it
   const uint32_t p_ready = s_free + 16;              // P of the next block is in TMEM
   const uint32_t pv_done = p_ready + 8;              // one phase per completed P V
@@ -224,9 +229,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
     mbar_init(q_empty, 1);
-    for (int s = 0; s < KV_STAGES; ++s) {
-      mbar_init(kv_full + 8 * s, 1);
-      mbar_init(kv_empty + 8 * s, 1);
+    for (int s = 0; s < KS; ++s) {
+      mbar_init(k_full + 8 * s, 1);
+      mbar_init(k_empty + 8 * s, 1);
+    }
+    for (int s = 0; s < VS; ++s) {
+      mbar_init(v_full + 8 * s, 1);
+      mbar_init(v_empty + 8 * s, 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(s_full + 8 * b, 1);
@@ -266,94 +275,147 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
   pdl_wait();
   pdl_trigger();
 
+  // Two issuing threads, so that neither MMA stream waits behind the other's
+  // instruction issue: warp 0 loads Q and K and issues the S MMAs, warp 1
+  // loads V and issues the P V MMAs.  Each refills its own ring.
   if (warp == 0) {
-    // ------------------------------------------------------------ TMA
+    // ------------------------------------------------- Q, K loads and S = Q K^T
+    // K runs KS - 1 key blocks ahead of the S MMAs: the K stage of block
+    // g + KS - 1 is the one block g - 1 used, whose S has completed by the
+    // time S(g) is issued.  S(g) goes into the S buffer the softmax of block
+    // g - 2 has read.
     if (lane == 0) {
-      int g = 0, uc = 0;
+      const uint32_t qb = saddr(sQ), kb_0 = saddr(sK);
+      const uint64_t dq = sw128_desc(qb), dqt = sw32_kmajor_desc(qb + C::Q128);
+      // stage descriptors differ only in the start address field (address >>
+      // 4, which never carries out of its 14 bits here)
+      const uint64_t dk = sw128_desc(kb_0), dkt = sw32_kmajor_desc(kb_0 + C::K128);
+      int gl = 0, gs = 0, uc = 0;
+      AttnSeg itl;
+      itl.init(sc, blockIdx.x);
+      int l_kb = 0, l_kb1 = 0, l_h = 0, l_row = 0;
+      bool l_more = true;
+      // requests K of the next key block to load (false: a wait gave up)
+      auto load_k = [&]() -> bool {
+        while (l_kb >= l_kb1) {
+          int pair, kb0, kb1, slot;
+          if (!itl.next(pair, kb0, kb1, slot)) {
+            l_more = false;
+            return true;
+          }
+          const TileLoc tl = locate_tile(rm, ai.n, D, pair % sc.qtiles);
+          l_h = pair / sc.qtiles;
+          l_row = ai.krow[tl.item];
+          l_kb = kb0;
+          l_kb1 = kb1;
+        }
+        const int st = gl % KS;
+        if (!mbar_sleep(k_empty + 8 * st, ((gl / KS) & 1) ^ 1, abort_flag)) return false;
+        mbar_expect_tx(k_full + 8 * st, C::K_BYTES);
+        uint8_t* base = sK + st * C::K_BYTES;
+        tma_load_3d(saddr(base), &tmK, k_full + 8 * st, 0, l_h, l_row + l_kb * BKV);
+        if (C::TAIL)
+          tma_load_3d(saddr(base + C::K128), &tmKt, k_full + 8 * st, 64, l_h, l_row + l_kb * BKV);
+        ++l_kb;
+        ++gl;
+        return true;
+      };
       AttnSeg it;
       it.init(sc, blockIdx.x);
       int pair, kb0, kb1, slot;
       for (; it.next(pair, kb0, kb1, slot); ++uc) {
         const int qt = pair % sc.qtiles, h = pair / sc.qtiles;
         const TileLoc tl = locate_tile(rm, ai.n, D, qt);
-        const int krow = ai.krow[tl.item], vrow = ai.vrow[tl.item];
+        const int n = kb1 - kb0;
+        // Q of the unit, once the previous unit's S MMAs have read the buffer
         if (!mbar_sleep(q_empty, (uc + 1) & 1, abort_flag)) goto timeout;
         mbar_expect_tx(q_full, C::Q_BYTES);
         tma_load_3d(saddr(sQ), &tmQ, q_full, 0, h, tl.row0);
         if (C::TAIL) tma_load_3d(saddr(sQ + C::Q128), &tmQt, q_full, 64, h, tl.row0);
-        for (int kb = kb0; kb < kb1; ++kb, ++g) {
-          const int st = g % KV_STAGES;
-          if (!mbar_sleep(kv_empty + 8 * st, ((g / KV_STAGES) & 1) ^ 1, abort_flag)) goto timeout;
-          mbar_expect_tx(kv_full + 8 * st, C::KV_BYTES);
-          uint8_t* base = sKV + st * C::KV_BYTES;
-          const uint32_t fb = kv_full + 8 * st;
-          tma_load_3d(saddr(base), &tmK, fb, 0, h, krow + kb * BKV);
-          if (C::TAIL) tma_load_3d(saddr(base + C::K128), &tmKt, fb, 64, h, krow + kb * BKV);
-          tma_load_3d(saddr(base + C::K_BYTES), &tmV, fb, 0, h, vrow + kb * BKV);
-          if (C::TAIL)
-            tma_load_3d(saddr(base + C::K_BYTES + C::K128), &tmV, fb, 64, h, vrow + kb * BKV);
-        }
-      }
-    }
-  } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA
-    // In a fixed order, sleeping on each input: S of the unit's first two
-    // blocks, then per block j: P V of block j (once its P is in TMEM), then
-    // S of block j + 2 into the S buffer the softmax of block j has read.
-    // S(j + 2) is first needed after the softmax of block j + 1, so issuing it
-    // after P V(j) costs nothing, and no warp spins.
-    if (lane == 0) {
-      int g = 0, uc = 0;
-      // descriptors of stage 0; a stage's differ only in the start address
-      // field (address >> 4, which never carries out of its 14 bits here)
-      const uint32_t qb = saddr(sQ), kb_0 = saddr(sKV);
-      const uint64_t dq = sw128_desc(qb), dqt = sw32_kmajor_desc(qb + C::Q128);
-      const uint64_t dk = sw128_desc(kb_0), dkt = sw32_kmajor_desc(kb_0 + C::K128);
-      const uint64_t dv = sw128_mnmajor_desc_lbo(kb_0 + C::K_BYTES, C::K128);
-      AttnSeg it;
-      it.init(sc, blockIdx.x);
-      int pair, kb0, kb1, slot;
-      for (; it.next(pair, kb0, kb1, slot); ++uc) {
-        const int n = kb1 - kb0;
-        if (!mbar_sleep(q_full, uc & 1, abort_flag)) goto timeout;
-        tc_fence_after();
-        // S of block ns of the unit
-        auto issue_s = [&](int ns) -> bool {
-          const int gs = g + ns;
-          const int st = gs % KV_STAGES;
-          if (!mbar_sleep(kv_full + 8 * st, (gs / KV_STAGES) & 1, abort_flag) ||
+        for (int ns = 0; ns < n; ++ns, ++gs) {
+          while (l_more && gl < gs + KS) {
+            if (!load_k()) goto timeout;
+          }
+          if (ns == 0 && !mbar_sleep(q_full, uc & 1, abort_flag)) goto timeout;
+          const int st = gs % KS;
+          if (!mbar_sleep(k_full + 8 * st, (gs / KS) & 1, abort_flag) ||
               !mbar_sleep(s_free + 8 * (gs & 1), ((gs >> 1) + 1) & 1, abort_flag))
-            return false;
+            goto timeout;
           tc_fence_after();
-          const uint64_t so = uint64_t(st * (C::KV_BYTES >> 4));
+          const uint64_t so = uint64_t(st * (C::K_BYTES >> 4));
           const uint32_t sd = tS0 + uint32_t(BKV) * uint32_t(gs & 1);
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)
             umma_bf16(sd, dq + 2 * kk, dk + so + 2 * kk, C::IDESC_S, kk > 0 ? 1u : 0u);
           if (C::TAIL) umma_bf16(sd, dqt, dkt + so, C::IDESC_S, 1u);
+          umma_commit(k_empty + 8 * st);
           umma_commit(s_full + 8 * (gs & 1));
           if (ns == n - 1) umma_commit(q_empty);  // last S of the unit issued
-          return true;
-        };
-        if (!issue_s(0) || (n > 1 && !issue_s(1))) goto timeout;
-        for (int np = 0; np < n; ++np) {
-          const int gp = g + np;
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------ V loads and O += P V
+    // V runs VS key blocks ahead: after P V(g) the thread waits for it to
+    // complete (it has time: P(g + 1) takes a whole softmax) and refills the
+    // stage with V(g + VS).
+    if (lane == 0) {
+      const uint64_t dv = sw128_mnmajor_desc_lbo(saddr(sV), C::K128);
+      int gv = 0, g = 0, uc = 0;
+      AttnSeg itl;
+      itl.init(sc, blockIdx.x);
+      int l_kb = 0, l_kb1 = 0, l_h = 0, l_row = 0;
+      bool l_more = true;
+      auto load_v = [&]() -> bool {
+        while (l_kb >= l_kb1) {
+          int pair, kb0, kb1, slot;
+          if (!itl.next(pair, kb0, kb1, slot)) {
+            l_more = false;
+            return true;
+          }
+          const TileLoc tl = locate_tile(rm, ai.n, D, pair % sc.qtiles);
+          l_h = pair / sc.qtiles;
+          l_row = ai.vrow[tl.item];
+          l_kb = kb0;
+          l_kb1 = kb1;
+        }
+        const int st = gv % VS;
+        if (!mbar_sleep(v_empty + 8 * st, ((gv / VS) & 1) ^ 1, abort_flag)) return false;
+        mbar_expect_tx(v_full + 8 * st, C::V_BYTES);
+        uint8_t* base = sV + st * C::V_BYTES;
+        tma_load_3d(saddr(base), &tmV, v_full + 8 * st, 0, l_h, l_row + l_kb * BKV);
+        if (C::TAIL)
+          tma_load_3d(saddr(base + C::K128), &tmV, v_full + 8 * st, 64, l_h, l_row + l_kb * BKV);
+        ++l_kb;
+        ++gv;
+        return true;
+      };
+      while (l_more && gv < VS) {
+        if (!load_v()) goto timeout;
+      }
+      AttnSeg it;
+      it.init(sc, blockIdx.x);
+      int pair, kb0, kb1, slot;
+      for (; it.next(pair, kb0, kb1, slot); ++uc) {
+        const int n = kb1 - kb0;
+        for (int np = 0; np < n; ++np, ++g) {
           if (np == 0 && !mbar_sleep(o_free, (uc + 1) & 1, abort_flag)) goto timeout;
-          if (!mbar_sleep(p_ready, gp & 1, abort_flag)) goto timeout;
+          const int st = g % VS;
+          if (!mbar_sleep(p_ready, g & 1, abort_flag) ||
+              !mbar_sleep(v_full + 8 * st, (g / VS) & 1, abort_flag))
+            goto timeout;
           tc_fence_after();
-          const int st = gp % KV_STAGES;
-          const uint64_t vd = dv + uint64_t(st * (C::KV_BYTES >> 4));
+          const uint64_t vd = dv + uint64_t(st * (C::V_BYTES >> 4));
           // 16 keys per MMA: P columns 8 kk .., V rows 16 kk .. (2 KB)
 #pragma unroll
           for (int kk = 0; kk < BKV / 16; ++kk)
             umma_bf16_ta(tO, tP + 8 * kk, vd + 128 * kk, C::IDESC_PV,
                          (np > 0 || kk > 0) ? 1u : 0u);
-          umma_commit(kv_empty + 8 * st);
+          umma_commit(v_empty + 8 * st);
           umma_commit(pv_done);
-          if (np + 2 < n && !issue_s(np + 2)) goto timeout;
+          if (np == n - 1) umma_commit(o_full);
+          if (l_more && !load_v()) goto timeout;  // V(g + VS) into this stage
         }
-        g += n;
-        umma_commit(o_full);
       }
     }
   } else {
