@@ -218,8 +218,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
   const uint32_t b0 = saddr(bars);
   const uint32_t q_full = b0, q_empty = b0 + 8;
   const uint32_t k_full = b0 + 16, k_empty = k_full + 8 * KS;
-  const uint32_t v_full = k_empty + 8 * KS, v_empty = v_full + 8 * VS;
-  const uint32_t s_full = v_empty + 8 * VS;          // [2]: S of a block is in TMEM
+  const uint32_t v_full = k_empty + 8 * KS;
+  const uint32_t s_full = v_full + 8 * VS;           // [2]: S of a block is in TMEM
   const uint32_t s_free = s_full + 16;               // [2]: the softmax has read it
   const uint32_t p_ready = s_free + 16;              // P of the next block is in TMEM
   const uint32_t pv_done = p_ready + 8;              // one phase per completed P V
@@ -233,10 +233,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
       mbar_init(k_full + 8 * s, 1);
       mbar_init(k_empty + 8 * s, 1);
     }
-    for (int s = 0; s < VS; ++s) {
-      mbar_init(v_full + 8 * s, 1);
-      mbar_init(v_empty + 8 * s, 1);
-    }
+    for (int s = 0; s < VS; ++s) mbar_init(v_full + 8 * s, 1);
     for (int b = 0; b < 2; ++b) {
       mbar_init(s_full + 8 * b, 1);
       mbar_init(s_free + 8 * b, 128);
@@ -280,10 +277,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
   // loads V and issues the P V MMAs.  Each refills its own ring.
   if (warp == 0) {
     // ------------------------------------------------- Q, K loads and S = Q K^T
-    // K runs KS - 1 key blocks ahead of the S MMAs: the K stage of block
-    // g + KS - 1 is the one block g - 1 used, whose S has completed by the
-    // time S(g) is issued.  S(g) goes into the S buffer the softmax of block
-    // g - 2 has read.
+    // K runs KS - 2 key blocks ahead of the S MMAs: the K stage of block
+    // g + KS - 2 is the one block g - 2 used, whose S has long completed, so
+    // the refill never waits on the MMA just issued.  S(g) goes into the S
+    // buffer the softmax of block g - 2 has read.
     if (lane == 0) {
       const uint32_t qb = saddr(sQ), kb_0 = saddr(sK);
       const uint64_t dq = sw128_desc(qb), dqt = sw32_kmajor_desc(qb + C::Q128);
@@ -333,7 +330,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         tma_load_3d(saddr(sQ), &tmQ, q_full, 0, h, tl.row0);
         if (C::TAIL) tma_load_3d(saddr(sQ + C::Q128), &tmQt, q_full, 64, h, tl.row0);
         for (int ns = 0; ns < n; ++ns, ++gs) {
-          while (l_more && gl < gs + KS) {
+          while (l_more && gl < gs + KS - 1) {
             if (!load_k()) goto timeout;
           }
           if (ns == 0 && !mbar_sleep(q_full, uc & 1, abort_flag)) goto timeout;
@@ -357,8 +354,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
   } else if (warp == 1) {
     // ------------------------------------------------------ V loads and O += P V
     // V runs VS key blocks ahead: after P V(g) the thread waits for it to
-    // complete (it has time: P(g + 1) takes a whole softmax) and refills the
-    // stage with V(g + VS).
+    // complete (pv_done, which the softmax waits for too; the thread has time:
+    // P(g + 1) takes a whole softmax) and refills the stage with V(g + VS).
     if (lane == 0) {
       const uint64_t dv = sw128_mnmajor_desc_lbo(saddr(sV), C::K128);
       int gv = 0, g = 0, uc = 0;
@@ -380,7 +377,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
           l_kb1 = kb1;
         }
         const int st = gv % VS;
-        if (!mbar_sleep(v_empty + 8 * st, ((gv / VS) & 1) ^ 1, abort_flag)) return false;
+        // the stage's previous block, gv - VS, is the P V just issued
+        if (gv >= VS && !mbar_sleep(pv_done, (gv - VS) & 1, abort_flag)) return false;
         mbar_expect_tx(v_full + 8 * st, C::V_BYTES);
         uint8_t* base = sV + st * C::V_BYTES;
         tma_load_3d(saddr(base), &tmV, v_full + 8 * st, 0, l_h, l_row + l_kb * BKV);
@@ -411,7 +409,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
           for (int kk = 0; kk < BKV / 16; ++kk)
             umma_bf16_ta(tO, tP + 8 * kk, vd + 128 * kk, C::IDESC_PV,
                          (np > 0 || kk > 0) ? 1u : 0u);
-          umma_commit(v_empty + 8 * st);
           umma_commit(pv_done);
           if (np == n - 1) umma_commit(o_full);
           if (l_more && !load_v()) goto timeout;  // V(g + VS) into this stage
