@@ -41,7 +41,12 @@ namespace {
 using namespace rc::tc;
 
 constexpr int BM = 128, BK = 64;
-constexpr int THREADS = 448;  // TMA warp, MMA warp, 12 epilogue warps
+// TMA warp (A, or A and W for CTA pairs), MMA warp, 12 epilogue warps, and
+// a second TMA warp that loads W for unpaired CTAs: each TMA request takes
+// long enough to issue that one thread issuing both operands bounds the
+// main loop
+constexpr int THREADS = 480;
+constexpr int W_WARP = 14;
 constexpr int STAGE_A = BM * BK * 2;   // bytes
 constexpr int MIN_KB_PER_CTA = 4;
 constexpr int STAGING_WARP = 32 * 128;  // epilogue staging: 32 rows of 128 B per warp
@@ -526,10 +531,32 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             tma_load_2d_pair(saddr(st), &tmA, fb, kb * BK, m * BM);
             tma_load_2d_pair(saddr(st + STAGE_A), tmW, fb, kb * BK, nn * BN + int(rank) * brows);
           } else {
+            // W comes from the W warp on the same barrier (which may see
+            // its bytes before this expectation: the phase still needs this
+            // arrival)
             mbar_expect_tx(full0 + 8 * stage, STAGE);
             tma_load_2d(saddr(st), &tmA, full0 + 8 * stage, kb * BK, m * BM);
-            tma_load_2d(saddr(st + STAGE_A), tmW, full0 + 8 * stage, kb * BK, nn * BN);
           }
+          if (++stage == STAGES) { stage = 0; phase ^= 1; }
+        }
+      }
+    }
+  } else if (warp == W_WARP) {
+    // ------------------------------------------------------- TMA: W (unpaired)
+    if (!PAIR && lane == 0) {
+      const CUtensorMap* tmW = &tmB.m[bmap_index(BN)];
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tmW)) : "memory");
+      int stage = 0;
+      uint32_t phase = 0;
+      Segs sg;
+      sg.init(sc, pos);
+      int t, kb0, kb1;
+      while (sg.next(t, kb0, kb1)) {
+        const int nn = t / sc.mt;
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(empty0 + 8 * stage, phase ^ 1, abort_flag)) goto timeout;
+          tma_load_2d(saddr(smem + stage * STAGE + STAGE_A), tmW, full0 + 8 * stage, kb * BK,
+                      nn * BN);
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
         }
       }
