@@ -218,6 +218,7 @@ class Workload:
         self.cnt = torch.zeros(1, dtype=torch.int32, device=dev)
         self.ws = torch.empty(R.rc_localize_workspace_size(N, 8), dtype=torch.uint8, device=dev)
         self.sparse = np.full(d.timesteps, R.RC_MODE_SPARSE, np.uint8)
+        self.dilation = 0
         self.scores = {}
         for f in fracs:
             blobs = synth.ellipse_blobs(d, seed, f)
@@ -229,8 +230,8 @@ class Workload:
         if ids is None:
             A_dev, ids, _ = self.scores[f]
             A = A_dev if A is None else A
-        self.R.rc_localize_mask(A, 1, d.tokens, d.text_len, d.grid_h, d.grid_w, ids, 0.5, 0,
-                                self.mask, self.idx, self.cnt, self.ws)
+        self.R.rc_localize_mask(A, 1, d.tokens, d.text_len, d.grid_h, d.grid_w, ids, 0.5,
+                                self.dilation, self.mask, self.idx, self.cnt, self.ws)
 
     def step(self, i, f):
         t = i % self.d.timesteps
@@ -642,6 +643,119 @@ def rate_2048(R, args, world, dev, K, W):
             "cache_bytes": d.timesteps * d.layers * 3 * d.tokens * d.hidden * 2}
 
 
+def rate_c1(R, world, dev, K, W, seed, with_oracle):
+    """One PixArt-alpha block at 256 tokens (16 x 16) on a seeded ~15 % dirty
+    rectangle: rc_block_forward_region with the block input restored before
+    each launch sequence, blocks/s; beside it the oracle's region_block on
+    the same shapes, timed whole on the host cores."""
+    d = synth.ONE_BLOCK_256
+    w = synth.make_weights(d, seed)
+    text = synth.make_text(d, seed)
+    mod6 = synth.make_mod6(d, w.layers[0]["table"], seed)
+    x0 = synth.make_hidden(d, seed)
+    slot = synth.make_cache_slice(d, seed, 0, 0, 0)
+    idx = np.flatnonzero(synth.rectangle_mask(d, seed)).astype(np.int32)
+    m = R.Model(d, w, device=dev)
+    try:
+        R.rc_cache_fill(m.cache, 0, 0, 0, *(a.to(dev) for a in slot))
+        R.rc_set_text(m.ctx, m.cache, 0, text.to(dev))
+        idx_d, mod6_d = torch.from_numpy(idx).to(dev), mod6.to(dev)
+        x0_d = x0.to(dev)
+        x = x0_d.clone()
+
+        def blk(i):
+            x.copy_(x0_d)
+            R.rc_block_forward_region(m.ctx, m.cache, 0, 0, 0, x, idx_d, len(idx), None, mod6_d)
+
+        k = 10 * K
+        ms = timed(blk, k, W, world)
+        R.rc_sync(m.ctx)
+    finally:
+        m.close()
+    out = {"workload": f"one PixArt-alpha block, {d.tokens} tokens ({d.grid_h} x {d.grid_w}), "
+                       "bf16 weights and cache, seeded rectangle",
+           "dirty_tokens": int(len(idx)), "unit": "blocks/s",
+           "blocks_per_s": round(job_rate(k, ms, world), 3),
+           "ms_per_block": round(ms / k, 5),
+           "timed": "copy of the block input + rc_block_forward_region, CUDA events"}
+    if with_oracle:
+        import oracle as O
+        L64 = {kk: O.to64(v) for kk, v in w.layers[0].items()}
+        cache = dict(zip("HKV", (O.to64(a) for a in slot)))
+        tkv = O.text_kv(O.to64(text), L64)
+        x64, m64 = O.to64(x0)[idx], O.to64(mod6)
+        n, t0 = 0, time.perf_counter()
+        while n < 3 or time.perf_counter() - t0 < 2.0:
+            O.region_block(x64, idx.astype(np.int64), cache, L64, m64, tkv, d.heads)
+            n += 1
+        sec = (time.perf_counter() - t0) / n
+        out["oracle"] = {"value": round(1.0 / sec, 3), "unit": "blocks/s",
+                         "cores": os.cpu_count(), "kind": "oracle", "extrapolated": False,
+                         "sample": f"{n} whole region blocks, float64 numpy",
+                         "seconds_per_block": round(sec, 5)}
+    return out
+
+
+def rate_c2(R, args, world, dev, K, W, seed, with_oracle):
+    """Whole steps of the 28-block model at 512 px (32 x 32 = 1024 tokens, all
+    timesteps resident): localisation on a seeded score map with 3-8 delta
+    tokens (threshold 0.5, one token of dilation) + the CUDA graph of rc_step
+    (SPARSE), and the dense path; beside them one whole oracle step
+    (localisation, 28 region blocks, final layer and DDIM update)."""
+    from dataclasses import replace
+    d = replace(synth.PIXART_512, timesteps=args.resident_steps)
+    A, ids = synth.blob_scores(d, seed)
+    wl = Workload(R, d, seed, dev, fracs=())
+    try:
+        wl.scores["c2"] = (torch.from_numpy(A).to(dev), ids, A)
+        wl.dilation = 1
+        wl.make_graphs()
+        ms = timed(lambda i: wl.gstep(i, "c2"), K, W, world)
+        sparse = job_rate(K, ms, world)
+        D = int(wl.cnt.item())
+        m = timed(wl.gstep_dense, K, min(W, 3), world)
+        dense = job_rate(K, m, world)
+        R.rc_sync(wl.model.ctx)
+        wl.free_graphs()
+    finally:
+        wl.model.close()
+    out = {"workload": f"pixart-alpha-512px: {d.tokens} tokens, {d.layers} blocks, "
+                       f"{d.timesteps} timesteps, batch 1; dirty set localised from a seeded "
+                       f"score map ({len(ids)} delta tokens, threshold 0.5, dilation 1)",
+           "dirty_tokens": D, "dirty_frac": round(D / d.tokens, 4),
+           "steps_per_s": round(sparse, 3), "ms_per_step": round(ms / K, 4),
+           "dense_steps_per_s": round(dense, 3), "speedup_vs_dense": round(sparse / dense, 3)}
+    if with_oracle:
+        import oracle as O
+        w = synth.make_weights(d, seed)
+        L64 = [{kk: O.to64(v) for kk, v in L.items()} for L in w.layers]
+        G64 = {kk: O.to64(v) for kk, v in w.glob.items()}
+        pos = O.to64(w.pos)
+        del w
+        ctx = O.to64(synth.make_text(d, seed))
+        tkv = [O.text_kv(ctx, L) for L in L64]
+        t = 5
+        cache = [dict(zip("HKV", (O.to64(a) for a in synth.make_cache_slice(d, seed, 0, l, t))))
+                 for l in range(d.layers)]
+        lat = O.to64(synth.make_latent(d, seed))
+        tv, ab = synth.ddim_tables(d.timesteps)
+        tv, ab = tv.astype(np.float64), ab.astype(np.float64)
+        secs = []
+        for _ in range(2):
+            t0 = time.perf_counter()
+            _, idx = O.localize_mask(A, ids, d.grid_h, d.grid_w, 0.5, 1)
+            O.step(G64, L64, pos, lat, t, O.MODE_SPARSE, idx, cache, tkv, tv, ab, d.heads,
+                   d.grid_h, d.grid_w, d.patch, d.in_ch)
+            secs.append(time.perf_counter() - t0)
+        sec = min(secs)
+        out["oracle"] = {"value": round(1.0 / sec, 5), "unit": UNIT, "cores": os.cpu_count(),
+                         "kind": "oracle", "extrapolated": False, "dirty_tokens": int(len(idx)),
+                         "sample": "2 whole steps (localisation, 28 region blocks, final "
+                                   "layer, DDIM update), float64 numpy; the faster one",
+                         "seconds_per_step": round(sec, 3)}
+    return out
+
+
 def kernel_rooflines(d, D, gemm_each, att_each, peak):
     """GEMM and attention rooflines of one probe pass: algorithmic FLOPs of
     D dirty rows per launch over the CUDA-event launch durations."""
@@ -775,6 +889,13 @@ def run_ours(args, world, rank, local):
     gemm_each_d = probe(R.RC_PROBE_GEMM, 6, wl.step_dense, Kd)
     att_each_d = probe(R.RC_PROBE_ATTENTION, 2, wl.step_dense, Kd)
 
+    # the same launch-by-launch steps with the gated residuals on whole tiles
+    # (rc_set_deterministic: bit-reproducible results)
+    R.rc_set_deterministic(wl.model.ctx, True)
+    m = timed(lambda i: wl.step(i, HEADLINE), K, W, world)
+    R.rc_set_deterministic(wl.model.ctx, False)
+    direct_det = job_rate(K, m, world)
+
     # sweep and dense baseline (graphs, like the headline)
     sweep, dirty = {}, {}
     for f in FRACS:
@@ -802,6 +923,14 @@ def run_ours(args, world, rank, local):
     big = None
     if not args.no_2048:
         big = rate_2048(R, args, world, dev, K, W)
+
+    # the two smaller configurations: one block at 256 tokens, whole steps at
+    # 512 px, each with the oracle timed whole beside it
+    small = None
+    if not args.no_small:
+        with_oracle = rank == 0 and world == 1 and not args.no_cpu_baseline
+        small = {"c1_one_block_256": rate_c1(R, world, dev, K, W, SEED + 11, with_oracle),
+                 "c2_512px": rate_c2(R, args, world, dev, K, W, SEED + 13, with_oracle)}
 
     # the same headline steps on a host-tier cache (pinned host pool, each
     # layer's K, V streamed into HBM windows while the previous layer runs)
@@ -882,10 +1011,12 @@ def run_ours(args, world, rank, local):
         "dense_capture_steps_per_s": round(capture, 3),
         "host_tier": host_tier,
         "pixart2048": big,
+        "small_configs": small,
         "batched_serving": batch,
         "persistent_serving": server,
         "editing_session": session,
         "direct_steps_per_s": round(direct, 3),
+        "deterministic_direct_steps_per_s": round(direct_det, 3),
         "speedup_vs_dense": {k: round(v / dense, 3) for k, v in sweep.items()},
         "roofline": roofline, "roofline_attention": roof_att,
         "roofline_dense": {"rows": d.tokens, "gemm": roof_dense, "attention": roof_att_dense},
@@ -1018,6 +1149,8 @@ def main():
                     help="skip the host-tier cache measurement (a pinned host pool)")
     ap.add_argument("--no-server", action="store_true",
                     help="skip the persistent-serving measurement (rc_server, 8 x 512 px)")
+    ap.add_argument("--no-small", action="store_true",
+                    help="skip the one-block 256-token and 512 px lines")
     ap.add_argument("--no-session", action="store_true",
                     help="skip the 5-turn editing-session measurement")
     ap.add_argument("--dense-only", action="store_true",

@@ -129,6 +129,23 @@ rc_status rc_set_global_weights(rc_ctx* ctx, const rc_global_weights* w);
  * DDIM (eta = 0) update after step t: alpha_bar[t] -> alpha_bar[t+1]. */
 rc_status rc_set_schedule(rc_ctx* ctx, const float* t_values_host, const float* alpha_bar_host);
 
+/* Reproducible sums.  By default the three gated-residual projections of a
+ * block (x += g (y W^T + b) after attention, cross-attention and the MLP,
+ * Section 3.3's region block) may split their reduction over k between
+ * CTAs that add their partial products into x with atomic reductions, so a
+ * step's result can differ in the last bits from run to run (always within
+ * the documented tolerances).  With on != 0 every such GEMM runs on whole
+ * output tiles (one reduction per element, k summed in a fixed order), and
+ * rc_step, rc_step_batched, rc_step_dense, rc_block_forward_region and the
+ * graphs captured from them give bit-identical results for bit-identical
+ * inputs on the same GPU and build.  It costs about a tenth of the step
+ * rate at 831 dirty tokens of 4096 (fewer CTAs share the residual GEMMs).
+ * The score sums of rc_step_capture and rc_localize_scores (over heads, with
+ * atomic adds) stay order-dependent either way.  Takes effect at the next
+ * launch; graphs keep the schedule they were captured with.  Never fails
+ * except on a null context. */
+rc_status rc_set_deterministic(rc_ctx* ctx, int on);
+
 /* ------------------------------------------------------------------ cache */
 
 /* Cache pool of Section 3.2 (Hidden-State-Oriented Caching): for every

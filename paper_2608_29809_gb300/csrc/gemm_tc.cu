@@ -94,6 +94,12 @@ __device__ __forceinline__ void red_add_v4(float* p, float a, float b, float c, 
                : "memory");
 }
 
+// The mode a schedule is planned for: a gated residual held to whole tiles
+// plans like any other 4-byte epilogue whose tiles are not split.
+__host__ __device__ inline int sched_mode(const GemmEpi& ep) {
+  return ep.mode == EPI_GATE_RES && ep.whole_tiles ? int(EPI_F32) : ep.mode;
+}
+
 __device__ __forceinline__ bool gated(const GemmEpi& ep) {
   return (ep.mode == EPI_GATE_RES || ep.mode == EPI_GATE_RES_CAST) && ep.gate_tab;
 }
@@ -497,7 +503,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   // dependency wait; the operands and the residual are read after it
   const int M = live_count(dcount, Mbound, ep.err);
   Sched sc;
-  sc.init(M, n, k, int(gridDim.x), ep.mode, bt.w64, PAIR);
+  sc.init(M, n, k, int(gridDim.x), sched_mode(ep), bt.w64, PAIR);
   pdl_wait();
   pdl_trigger();
   const int BN = sc.BN, STAGES = sc.stages;
@@ -846,7 +852,7 @@ cudaError_t launch_gemm(const bf16* A, int lda, const bf16* W, int Mbound, const
   // count must be known here: a device-side count keeps CTAs unpaired.
   const bool pair = shp.pair && !dcount && Mbound >= PAIR_MIN_ROWS;
   const int grid = pair ? shp.grid : device_sms();
-  const BnTable bt = bn_table(n, k, grid, ep.mode, (Mbound + BM - 1) / BM, pair);
+  const BnTable bt = bn_table(n, k, grid, sched_mode(ep), (Mbound + BM - 1) / BM, pair);
   if (pair)
     RC_TRY(launch_k_cluster(gemm_tc_kernel<true>, dim3(shp.grid), dim3(THREADS), SMEM_BYTES, 2,
                             st, ta, tb, Mbound, dcount, n, k, ep, bt));

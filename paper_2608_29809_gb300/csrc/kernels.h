@@ -144,6 +144,7 @@ struct GemmEpi {
   int n_tokens;            // bound of token indices
   unsigned* err;
   Items its;               // per-item cache slices and modulation vectors
+  int whole_tiles;         // GATE_RES: no k split (one reduction per element, reproducible)
 };
 
 // C[M][n] = A[M][k] W[n][k]^T, epilogue `ep`.  M = *dcount if non-null (bounded

@@ -68,6 +68,8 @@ struct rc_ctx {
   bool gw_set = false;
   std::vector<float> t_values, alpha_bar;
   bool sched_set = false;
+  // gated residual GEMMs on whole tiles only (rc_set_deterministic)
+  bool deterministic = false;
   // device scratch (R = max_batch * N compact rows)
   float* xf = nullptr;   // [R][d] residual rows of the dirty tokens (compact)
   bf16* xb = nullptr;    // [R][d] GEMM input: modulated rows / residual copy
@@ -344,6 +346,7 @@ rc_status run_block(rc_ctx* c, rc_cache* k, int l, const rc::RowMap& rm, const S
     g.n_tokens = N;
     g.err = c->err;
     g.its = si.its;
+    g.whole_tiles = c->deterministic ? 1 : 0;
     return g;
   };
   // (whole tiles, read-modify-write, also leaving xb = bf16(x) for the
@@ -562,6 +565,12 @@ rc_status rc_set_schedule(rc_ctx* c, const float* tv, const float* ab) {
   c->t_values.assign(tv, tv + c->T);
   c->alpha_bar.assign(ab, ab + c->T + 1);
   c->sched_set = true;
+  return RC_OK;
+}
+
+rc_status rc_set_deterministic(rc_ctx* c, int on) {
+  if (!c) return fail(RC_ERR_INVALID_ARG, "rc_set_deterministic: null context");
+  c->deterministic = on != 0;
   return RC_OK;
 }
 

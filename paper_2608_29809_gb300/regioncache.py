@@ -85,6 +85,7 @@ def load_library(path: str = LIB_PATH) -> C.CDLL:
         "rc_set_layer_weights": (I, [P, I, C.POINTER(rc_layer_weights)]),
         "rc_set_global_weights": (I, [P, C.POINTER(rc_global_weights)]),
         "rc_set_schedule": (I, [P, P, P]),
+        "rc_set_deterministic": (I, [P, I]),
         "rc_cache_create": (I, [P, I, C.POINTER(P)]),
         "rc_cache_create_host": (I, [P, I, C.POINTER(P)]),
         "rc_cache_export": (I, [P, I, C.c_char_p]),
@@ -184,6 +185,10 @@ def rc_set_schedule(ctx, t_values, alpha_bar):
     tv = np.ascontiguousarray(t_values, np.float32)
     ab = np.ascontiguousarray(alpha_bar, np.float32)
     _check(_lib.rc_set_schedule(ctx, tv.ctypes.data, ab.ctypes.data))
+
+
+def rc_set_deterministic(ctx, on: bool):
+    _check(_lib.rc_set_deterministic(ctx, 1 if on else 0))
 
 
 def rc_cache_create(ctx, sessions) -> int:
