@@ -17,13 +17,16 @@
 // into equal k-block ranges (stream-K).  Its casting variant (x += ..., then
 // xb = bf16(x), read-modify-write) and the other epilogues see whole tiles.
 //
-// CTA = 14 warps: warp 0 issues TMA loads, warp 1 owns TMEM and issues the
-// MMAs (one thread), warps 2..13 drain the accumulator (one TMEM lane = one
-// output row per thread; three warps per TMEM lane quarter take every third
-// 32-column chunk; re-staged through shared memory so that global writes
-// are whole row pieces).  The epilogue is latency-bound (a CTA holds one
-// tile at small row counts), so its width is worth more than a deeper ring.  Two TMEM accumulators of up to 256 columns
-// let the epilogue of one tile overlap the main loop of the next.
+// CTA = 16 warps: warp 0 issues TMA loads (A), warp 14 those of W, warp 1
+// owns TMEM and issues the MMAs (one thread), warps 2..13 drain the
+// accumulator (one TMEM lane = one output row per thread; three warps per
+// TMEM lane quarter take every third 32-column chunk; re-staged through
+// shared memory so that global writes are whole row pieces), and warp 15
+// is a second MMA issuer when every CTA holds one work item (the item's odd
+// k-blocks into the second accumulator, see split2).  The epilogue is
+// latency-bound (a CTA holds one tile at small row counts), so its width is
+// worth more than a deeper ring.  Otherwise two TMEM accumulators of up to
+// 256 columns let the epilogue of one tile overlap the main loop of the next.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -41,12 +44,13 @@ namespace {
 using namespace rc::tc;
 
 constexpr int BM = 128, BK = 64;
-// TMA warp (A, or A and W for CTA pairs), MMA warp, 12 epilogue warps, and
-// a second TMA warp that loads W for unpaired CTAs: each TMA request takes
-// long enough to issue that one thread issuing both operands bounds the
-// main loop
-constexpr int THREADS = 480;
+// TMA warp (A, or A and W for CTA pairs), MMA warp, 12 epilogue warps, a
+// second TMA warp that loads W for unpaired CTAs (each TMA request takes long
+// enough to issue that one thread issuing both operands bounds the main
+// loop), and a second MMA warp
+constexpr int THREADS = 512;
 constexpr int W_WARP = 14;
+constexpr int MMA2_WARP = 15;
 constexpr int STAGE_A = BM * BK * 2;   // bytes
 constexpr int MIN_KB_PER_CTA = 4;
 constexpr int STAGING_WARP = 32 * 128;  // epilogue staging: 32 rows of 128 B per warp
@@ -160,6 +164,53 @@ __device__ __forceinline__ void epilogue_values(const GemmEpi& ep, int c0, int c
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] *= g[i];
   }
+}
+
+// 32 consecutive f32 columns of this thread's TMEM lane, summed over the two
+// accumulators at taddr and taddr + 256 (a tile whose k-blocks two MMA
+// threads split between them).
+__device__ __forceinline__ void tmem_ld32_sum2(uint32_t taddr, float* v) {
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    uint32_t a[16], b[16];
+    tmem_ld16_nowait(taddr + uint32_t(16 * h), a);
+    tmem_ld16_nowait(taddr + 256u + uint32_t(16 * h), b);
+    tmem_wait_ld();
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[16 * h + i] = __uint_as_float(a[i]) + __uint_as_float(b[i]);
+  }
+}
+// The k-blocks of parity `par` of a CTA's one work item (k-blocks [kb0, kb1),
+// ring stages from 0), issued by one of two MMA threads into accumulator
+// `par` (TMEM columns 256 par ..); its tfull barrier is committed at the end.
+// Returns false when a bounded wait gave up.
+__device__ __forceinline__ bool mma_half(int par, int kb0, int kb1, int STAGES, int STAGE,
+                                         uint32_t ring, uint32_t tmem_base, uint32_t idesc,
+                                         uint32_t full0, uint32_t empty0, uint32_t tfull0,
+                                         uint32_t tempty0, volatile int* abort_flag) {
+  if (!mbar_wait(tempty0 + 8 * par, 1, abort_flag)) return false;
+  tc_fence_after();
+  const uint64_t da = sw128_desc(ring), db = sw128_desc(ring + STAGE_A);
+  const uint32_t dtm = tmem_base + uint32_t(par * 256);
+  int stage = par;
+  uint32_t phase = 0;
+  for (int kb = kb0 + par; kb < kb1; kb += 2) {
+    if (!mbar_wait(full0 + 8 * stage, phase, abort_flag)) return false;
+    tc_fence_after();
+    const uint64_t so = uint64_t((stage * STAGE) >> 4);
+#pragma unroll
+    for (int kk = 0; kk < BK / 16; ++kk)
+      umma_bf16(dtm, da + so + 2 * kk, db + so + 2 * kk, idesc,
+                (kb > kb0 + par || kk > 0) ? 1u : 0u);
+    umma_commit(empty0 + 8 * stage);
+    stage += 2;
+    if (stage >= STAGES) {
+      stage -= STAGES;
+      phase ^= 1;
+    }
+  }
+  umma_commit(tfull0 + 8 * par);
+  return true;
 }
 
 // Named barrier of the 12 epilogue warps.
@@ -508,6 +559,14 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   pdl_trigger();
   const int BN = sc.BN, STAGES = sc.stages;
   const int STAGE = Sched::stage_bytes(BN, PAIR);
+  // split2: when every CTA holds one work item (so the second accumulator is
+  // free), two MMA threads take the item's even and odd k-blocks into the two
+  // accumulators, which the epilogue adds.  One thread issues a tcgen05.mma
+  // only about every 140 cycles when the ring stage is known at run time,
+  // whatever N; two threads together issue about twice as fast (measured).
+  // It shortens the main loop where few rows leave it bound by that issue
+  // rate (a sparse step at 5 % dirty: 397 -> 428 steps/s).
+  const bool split2 = !PAIR && sc.alias && sc.kbt >= 2;
   // schedule position: the pair (its row tiles 2p + rank) or the CTA
   const int pos = PAIR ? int(blockIdx.x) >> 1 : int(blockIdx.x);
 
@@ -569,7 +628,16 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     }
   } else if (warp == 1) {
     // ------------------------------------------------------- MMA issuer
-    if (lane == 0 && rank == 0) {
+    if (lane == 0 && rank == 0 && split2) {
+      Segs sg;
+      sg.init(sc, pos);
+      int t, kb0, kb1;
+      if (sg.next(t, kb0, kb1) &&
+          !mma_half(0, kb0, kb1, STAGES, STAGE, saddr(smem), tmem_base,
+                    IDESC_BASE | (uint32_t(BN >> 3) << 17), full0, empty0, tfull0, tempty0,
+                    abort_flag))
+        goto timeout;
+    } else if (lane == 0 && rank == 0) {
       const uint32_t idesc = (PAIR ? IDESC_PAIR : IDESC_BASE) | (uint32_t(BN >> 3) << 17);
       const uint64_t da = sw128_desc(saddr(smem)), db = sw128_desc(saddr(smem + STAGE_A));
       int stage = 0;
@@ -611,6 +679,18 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         if (++acc == 2) { acc = 0; acc_phase ^= 1; }
       }
     }
+  } else if (warp == MMA2_WARP) {
+    // ------------------------------------------------------- second MMA issuer
+    if (lane == 0 && split2) {
+      Segs sg;
+      sg.init(sc, pos);
+      int t, kb0, kb1;
+      if (sg.next(t, kb0, kb1) &&
+          !mma_half(1, kb0, kb1, STAGES, STAGE, saddr(smem), tmem_base,
+                    IDESC_BASE | (uint32_t(BN >> 3) << 17), full0, empty0, tfull0, tempty0,
+                    abort_flag))
+        goto timeout;
+    }
   } else {
     // ------------------------------------------------------- epilogue (warps 2..13)
     const int sp = warp & 3;  // TMEM lane sub-partition this warp may access
@@ -642,13 +722,17 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       stage_vectors(ep, nn * BN, BN, kb0 == 0, sVec, int(threadIdx.x) - 64);
       epi_sync();
       if (ok && !mbar_wait_warp(tfull0 + 8 * acc, acc_phase, abort_flag)) ok = false;
+      if (ok && split2 && !mbar_wait_warp(tfull0 + 8, 0, abort_flag)) ok = false;
       if (ok) {
         tc_fence_after();
         const uint32_t tbase = tmem_base + uint32_t(acc * 256) + (uint32_t(sp * 32) << 16);
 #pragma unroll 1
         for (int ch = (warp - 2) >> 2; ch < BN / 32; ch += 3) {
           float v[32];
-          tmem_ld32(tbase + uint32_t(ch * 32), v);
+          if (split2)
+            tmem_ld32_sum2(tbase + uint32_t(ch * 32), v);
+          else
+            tmem_ld32(tbase + uint32_t(ch * 32), v);
           const int c0 = nn * BN + ch * 32;
           epilogue_values(ep, c0, ch * 32, item, v, sVec);
           bf16* xb_row = (ep.mode == EPI_GATE_RES_CAST && r < M)
