@@ -854,7 +854,12 @@ xq_fold_kernel(const bf16* __restrict__ Kt, int ldk, const bf16* __restrict__ Wq
 // One (query tile, head) per CTA: S = xb_tile G_h^T accumulated over d in
 // 64-column k-blocks (TMA ring, M = 128, N = 128), then the softmax of
 // (S + kb) / sqrt(dh) per row, P over S in TMEM, O = P V, O / l stored.
+// Two threads issue the S MMAs, the even k-blocks into S0 and the odd ones
+// into S1 (TMEM columns 0 / 128; the softmax adds them): one thread issues
+// a tcgen05.mma only about every 140 cycles from a ring whose stage is known
+// at run time, and the 72 MMAs of the d = 1152 loop were bound by that.
 constexpr int XF_STAGES = 6;
+constexpr int XF_THREADS = 224;  // TMA, MMA, 4 softmax warps, second MMA warp
 template <int DH>
 struct XFCfg {
   using C = ACfg<DH>;
@@ -869,7 +874,7 @@ struct XFCfg {
 };
 
 template <int DH, bool CAP>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(XF_THREADS, 1)
 xfused_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmG,
                  const __grid_constant__ CUtensorMap tmV, const float* __restrict__ kb,
                  const __grid_constant__ XqItems xi, int Nk, int d, bf16* __restrict__ O,
@@ -895,7 +900,7 @@ xfused_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
       mbar_init(empty0 + 8 * i, 1);
     }
     mbar_init(v_full, 1);
-    mbar_init(s_full, 1);
+    mbar_init(s_full, 2);  // both MMA threads commit their half of S
     mbar_init(p_ready, 128);
     mbar_init(o_full, 1);
     mbar_init(kb_ready, 128);
@@ -915,12 +920,14 @@ xfused_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
   if (qt >= qtiles) return;
   const bool live = true;
   const TileLoc tl = locate_tile(rm, xi.n, D, qt);
-  if (warp == 1) tmem_alloc(saddr(tmem_slot), 256);
+  // one CTA per SM (its shared memory), so all 512 columns are there
+  if (warp == 1) tmem_alloc(saddr(tmem_slot), 512);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const uint32_t tS = tmem_base, tO = tmem_base + XK;  // P is written over S
+  // S0 | S1 | O; P is written over S0
+  const uint32_t tS = tmem_base, tS1 = tmem_base + XK, tO = tmem_base + 2 * XK;
   const int nkb = d / 64;
   bool ok = live;
   if (live && warp == 0 && lane == 0) {
@@ -951,12 +958,15 @@ xfused_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
       }
       tma_load_3d(saddr(base), &tmA, full0 + 8 * st, 0, k, tl.row0);
     }
-  } else if (live && warp == 1 && lane == 0) {
+  } else if (live && (warp == 1 || warp == 6) && lane == 0) {
     // ------------------------------------------------------------ MMA
+    // warp 1: the even k-blocks into S0, then P V; warp 6: the odd ones into S1
     pdl_wait();
+    const int par = warp == 1 ? 0 : 1;
+    const uint32_t dS = par ? tS1 : tS;
     const uint64_t da = sw128_desc(saddr(smem)), dg = sw128_desc(saddr(smem + X::STAGE_A));
     bool good = true;
-    for (int k = 0; k < nkb && good; ++k) {
+    for (int k = par; k < nkb && good; k += 2) {
       const int st = k % XF_STAGES;
       if (!mbar_wait(full0 + 8 * st, (k / XF_STAGES) & 1, abort_flag)) {
         good = false;
@@ -966,11 +976,15 @@ xfused_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
       const uint64_t so = uint64_t((st * X::STAGE) >> 4);
 #pragma unroll
       for (int kk = 0; kk < 4; ++kk)
-        umma_bf16(tS, da + so + 2 * kk, dg + so + 2 * kk, X::IDESC_S,
-                  (k > 0 || kk > 0) ? 1u : 0u);
+        umma_bf16(dS, da + so + 2 * kk, dg + so + 2 * kk, X::IDESC_S,
+                  (k > par || kk > 0) ? 1u : 0u);
       umma_commit(empty0 + 8 * st);
     }
-    if (good) umma_commit(s_full);
+    if (good) umma_commit(s_full);  // (arrives at once when this half has no k-block)
+    if (par) {
+      if (!good) *abort_flag = 1;
+      goto xf_done;
+    }
     // P V once every row's P is in TMEM and V has landed
     if (good && mbar_wait(p_ready, 0, abort_flag) && mbar_wait(v_full, 0, abort_flag)) {
       tc_fence_after();
@@ -983,7 +997,7 @@ xfused_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
     } else {
       *abort_flag = 1;
     }
-  } else if (live && warp >= 2) {
+  } else if (live && warp >= 2 && warp < 6) {
     // ------------------------------------------------------------ softmax
     const int sp = warp & 3;
     const int row = sp * 32 + lane;
@@ -1000,6 +1014,18 @@ xfused_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
 #pragma unroll
       for (int i = 0; i < XK / 16; ++i) tmem_ld16_nowait(tS + lane_off + 16u * i, r + 16 * i);
       tmem_wait_ld();
+      if (nkb > 1) {  // S = S0 + S1 (the odd k-blocks)
+#pragma unroll
+        for (int j = 0; j < XK / 32; ++j) {
+          uint32_t q[32];
+          tmem_ld16_nowait(tS1 + lane_off + 32u * j, q);
+          tmem_ld16_nowait(tS1 + lane_off + 32u * j + 16u, q + 16);
+          tmem_wait_ld();
+#pragma unroll
+          for (int c = 0; c < 32; ++c)
+            r[32 * j + c] = __float_as_uint(__uint_as_float(r[32 * j + c]) + __uint_as_float(q[c]));
+        }
+      }
 #pragma unroll
       for (int c = 0; c < XK; ++c)
         r[c] = c < Nk ? __float_as_uint(__uint_as_float(r[c]) + s_kb[c])
@@ -1081,13 +1107,14 @@ xfused_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
       }
     }
   }
+xf_done:
   if (live && (!ok || *abort_flag) && threadIdx.x == 64) atomicOr(err, DEVERR_TIMEOUT);
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tmem_base, 256);
+    tmem_dealloc(tmem_base, 512);
   }
 }
 
@@ -1465,7 +1492,7 @@ cudaError_t launch_xattn_fused(const bf16* xb, int ldx, const bf16* G, const flo
   if (grid >= (1ll << 31)) return cudaErrorInvalidValue;
   auto fn = dh == 72 ? (cap.n ? xfused_tc_kernel<72, true> : xfused_tc_kernel<72, false>)
                      : (cap.n ? xfused_tc_kernel<64, true> : xfused_tc_kernel<64, false>);
-  RC_TRY(launch_k(fn, dim3(unsigned(grid)), dim3(192), dh == 72 ? XFCfg<72>::SMEM : XFCfg<64>::SMEM,
+  RC_TRY(launch_k(fn, dim3(unsigned(grid)), dim3(XF_THREADS), dh == 72 ? XFCfg<72>::SMEM : XFCfg<64>::SMEM,
                   st, ta, tg, tv, kb, xi, Nk, d, O, ldo, heads, rm, scale_log2, err, cap));
   count_launches(1);
   return cudaSuccess;
