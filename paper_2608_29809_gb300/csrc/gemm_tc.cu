@@ -565,8 +565,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   // only about every 140 cycles when the ring stage is known at run time,
   // whatever N; two threads together issue about twice as fast (measured).
   // It shortens the main loop where few rows leave it bound by that issue
-  // rate (a sparse step at 5 % dirty: 397 -> 428 steps/s).
-  const bool split2 = !PAIR && sc.alias && sc.kbt >= 2;
+  // rate (a sparse step at 5 % dirty: 397 -> 428 steps/s).  A 256-wide MMA
+  // keeps the tensor pipe busy about as long as one thread takes to issue
+  // it, so 256-wide tiles keep one issuer (the second accumulator's read in
+  // the epilogue would cost more than it saves: 298.7 -> 301.8 steps/s at
+  // 20 % dirty without it there).
+  const bool split2 = !PAIR && sc.alias && sc.kbt >= 2 && BN <= 192;
   // schedule position: the pair (its row tiles 2p + rank) or the CTA
   const int pos = PAIR ? int(blockIdx.x) >> 1 : int(blockIdx.x);
 
