@@ -116,11 +116,15 @@ def test_localize_indicator_ellipses_4096(R):
 # the tile width is chosen on the device from the row count: these shapes
 # take 64 (1, 37, 128, 1000 rows), 128 (300 x 3456), 192 (831 x 3456) and 256
 # (831 x 4608); from 2048 rows (known on the host) CTA pairs share M = 256
-# MMAs, including a ragged last pair (2900 rows: 23 row tiles) and split k
+# MMAs, including a ragged last pair (2900 rows: 23 row tiles) and split k.
+# When every CTA holds one tile, tiles up to 192 wide are issued by two MMA
+# threads (even / odd k-blocks into two accumulators): 2, 3 and 19 k-blocks
+# give them equal and unequal shares, 1 k-block leaves the second idle.
 @pytest.mark.parametrize("rows,n,k", [(1, 128, 64), (37, 1152, 1152), (128, 256, 4608),
                                       (300, 3456, 1152), (1000, 1152, 4608), (831, 3456, 1152),
                                       (831, 4608, 1152), (2048, 1152, 1152), (2900, 1152, 4608),
-                                      (3001, 3456, 1152), (4096, 4608, 1152)])
+                                      (3001, 3456, 1152), (4096, 4608, 1152), (96, 384, 128),
+                                      (200, 256, 192), (831, 1152, 1216), (500, 640, 64)])
 def test_linear_matches_fp64(R, rows, n, k):
     g = torch.Generator().manual_seed(rows * 7 + n)
     x = torch.randn(rows, k, generator=g).to(torch.bfloat16)
