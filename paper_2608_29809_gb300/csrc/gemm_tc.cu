@@ -397,11 +397,14 @@ struct Sched {
     return s < MAX_STAGES ? s : MAX_STAGES;
   }
   // Estimated duration (SM cycles): k-blocks on the busiest CTA x per-k-block
-  // time (operands at ~60 B/clk per SM) plus its exposed epilogues (~20 B/clk
-  // per SM with twelve epilogue warps; both rates measured); a stream-K CTA
-  // holds two pieces.
+  // time (operands at ~60 B/clk per SM, but no less than the MMA issue time)
+  // plus its exposed epilogues (~20 B/clk per SM with twelve epilogue warps;
+  // all rates measured); a stream-K CTA holds two pieces.
   __host__ __device__ float cost(int out_bytes) const {
-    const float ckb = float(stage_bytes(BN, pair)) * (1.f / 60.f);
+    // one thread issues a tcgen05.mma about every 140 cycles (4 per k-block),
+    // two together twice as fast (one work item per CTA, tiles up to 192)
+    const float cmma = (alias && !pair && BN <= 192) ? 280.f : 560.f;
+    const float ckb = fmaxf(float(stage_bytes(BN, pair)) * (1.f / 60.f), cmma);
     const float cep = float(BM * BN * out_bytes) * (1.f / 20.f);
     if (S > 0) return float((kbt + S - 1) / S) * ckb + cep;
     const int waves = (whole + G - 1) / G;
