@@ -372,29 +372,59 @@ cudaError_t launch_ln_mod(const float* x, const float* tab, int k_sh, int k_sc, 
 
 // ============================================================ patch embed
 // x_r = W_e patch(idx[r]) + b_e + pos[idx[r]], the patch vector ordered
-// (channel, py, px).  W_e (<= 16 inputs per output) sits in shared memory;
-// one warp per dirty token, grid-stride over the tokens.
+// (channel, py, px).  W_e (<= 16 inputs per output) and b_e sit in shared
+// memory; one warp per dirty token, grid-stride over the tokens.  A lane
+// owns outputs lane + 32 m; a token's pos row (read from DRAM once per step)
+// and its latent pixels are requested together before any is used, so a
+// token costs one memory round trip instead of one per output group.
 constexpr int PE_WARPS = 8;
 constexpr int PE_MAXD = 1536;
+constexpr int PE_MAXM = PE_MAXD / 32;  // outputs per lane
 
 __global__ void __launch_bounds__(PE_WARPS * 32)
 patch_embed_kernel(int gh, int gw, int p, int C, const bf16* __restrict__ We,
                    const float* __restrict__ be, const float* __restrict__ pos,
                    const __grid_constant__ Items it, RowMap rm, float* __restrict__ xf, int d,
                    unsigned* err) {
-  // W_e is staged before the programmatic-dependency wait (weights never
-  // change during a step); the latent, the row map and xf after it
+  // W_e and b_e are staged before the programmatic-dependency wait (weights
+  // never change during a step); the latent, the row map and xf after it
   extern __shared__ __align__(16) uint8_t pe_smem[];
-  bf16* s_w = reinterpret_cast<bf16*>(pe_smem);  // [d][16], zero beyond P
-  const int P = C * p * p;                         // <= 16
+  bf16* s_w = reinterpret_cast<bf16*>(pe_smem);                    // [d][16], zero beyond P
+  float* s_b = reinterpret_cast<float*>(pe_smem + size_t(d) * 32);  // [d]
+  const int P = C * p * p;                                          // <= 16
   if (P == 16 && (reinterpret_cast<uintptr_t>(We) & 15u) == 0) {
-    // rows of 16 weights are 32 bytes: a straight 16-byte copy
-    for (int v = threadIdx.x; v < d * 2; v += blockDim.x)
-      reinterpret_cast<uint4*>(s_w)[v] = __ldg(reinterpret_cast<const uint4*>(We) + v);
+    // rows of 16 weights are 32 bytes: a straight 16-byte copy, every load of
+    // a thread in flight before its first store
+    constexpr int NV = (PE_MAXD * 2 + PE_WARPS * 32 - 1) / (PE_WARPS * 32);
+    uint4 t[NV];
+#pragma unroll
+    for (int j = 0; j < NV; ++j) {
+      const int v = threadIdx.x + j * PE_WARPS * 32;
+      if (v < d * 2) t[j] = __ldg(reinterpret_cast<const uint4*>(We) + v);
+    }
+#pragma unroll
+    for (int j = 0; j < NV; ++j) {
+      const int v = threadIdx.x + j * PE_WARPS * 32;
+      if (v < d * 2) reinterpret_cast<uint4*>(s_w)[v] = t[j];
+    }
   } else {
     for (int e = threadIdx.x; e < d * 16; e += blockDim.x) {
       const int o = e >> 4, k = e & 15;
       s_w[e] = k < P ? We[size_t(o) * P + k] : f2bf(0.f);
+    }
+  }
+  {
+    constexpr int NB = (PE_MAXD + PE_WARPS * 32 - 1) / (PE_WARPS * 32);
+    float t[NB];
+#pragma unroll
+    for (int j = 0; j < NB; ++j) {
+      const int o = threadIdx.x + j * PE_WARPS * 32;
+      if (o < d) t[j] = __ldg(be + o);
+    }
+#pragma unroll
+    for (int j = 0; j < NB; ++j) {
+      const int o = threadIdx.x + j * PE_WARPS * 32;
+      if (o < d) s_b[o] = t[j];
     }
   }
   pdl_wait();
@@ -403,6 +433,7 @@ patch_embed_kernel(int gh, int gw, int p, int C, const bf16* __restrict__ We,
   const int D = live_count(rm.count, rm.bound, err);
   const int lane = threadIdx.x & 31;
   const int W = gw * p, H = gh * p;
+  const int nm = d / 32;
   for (int r = blockIdx.x * PE_WARPS + (threadIdx.x >> 5); r < D; r += gridDim.x * PE_WARPS) {
     int i, item;
     if (!row_target(rm, it.n, r, i, item, err, lane)) continue;
@@ -414,10 +445,19 @@ patch_embed_kernel(int gh, int gw, int p, int C, const bf16* __restrict__ We,
       const int py = rem / p, px = rem - py * p;
       pv = latent[(size_t(c) * H + gy * p + py) * W + gx * p + px];
     }
+    const float* prow = pos + size_t(i) * d;
+    float pp[PE_MAXM];
+#pragma unroll
+    for (int m = 0; m < PE_MAXM; ++m)
+      if (m < nm) pp[m] = __ldg(prow + lane + 32 * m);
     float patch[16];
 #pragma unroll
     for (int k = 0; k < 16; ++k) patch[k] = __shfl_sync(0xffffffffu, pv, k);
-    for (int o = lane; o < d; o += 32) {
+    float* xrow = xf + size_t(r) * d;
+#pragma unroll
+    for (int m = 0; m < PE_MAXM; ++m) {
+      if (m >= nm) break;
+      const int o = lane + 32 * m;
       const uint4* w4 = reinterpret_cast<const uint4*>(s_w + o * 16);
       float acc = 0.f;
 #pragma unroll
@@ -434,7 +474,7 @@ patch_embed_kernel(int gh, int gw, int p, int C, const bf16* __restrict__ We,
         acc = fmaf(e2.x, patch[8 * q + 6], acc);
         acc = fmaf(e2.y, patch[8 * q + 7], acc);
       }
-      xf[size_t(r) * d + o] = acc + be[o] + pos[size_t(i) * d + o];
+      xrow[o] = acc + s_b[o] + pp[m];
     }
   }
 }
@@ -443,10 +483,16 @@ cudaError_t launch_patch_embed(int gh, int gw, int p, int C, const bf16* We, con
                                const float* pos, const Items& it, const RowMap& rm, float* xf,
                                int d, unsigned* err, cudaStream_t st) {
   if (rm.bound <= 0) return cudaSuccess;
-  if (d > PE_MAXD || C * p * p > 16) return cudaErrorInvalidValue;
+  if (d > PE_MAXD || d % 32 || C * p * p > 16) return cudaErrorInvalidValue;
+  static bool attr_set = false;  // (55 KB at the largest hidden size)
+  if (!attr_set) {
+    RC_TRY(cudaFuncSetAttribute(patch_embed_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                int(size_t(PE_MAXD) * (16 * sizeof(bf16) + sizeof(float)))));
+    attr_set = true;
+  }
   RC_TRY(launch_k(patch_embed_kernel, dim3(row_grid(rm.bound, PE_WARPS, 1)), dim3(PE_WARPS * 32),
-                  size_t(d) * 16 * sizeof(bf16), st, gh, gw, p, C, We, be, pos, it, rm, xf, d,
-                  err));
+                  size_t(d) * (16 * sizeof(bf16) + sizeof(float)), st, gh, gw, p, C, We, be, pos,
+                  it, rm, xf, d, err));
   count_launches(1);
   return cudaSuccess;
 }
@@ -540,17 +586,51 @@ final_ddim_kernel(const bf16* __restrict__ H, const float* __restrict__ temb,
   float* s_scale = s_shift + d;
   bf16* s_w = reinterpret_cast<bf16*>(s_scale + d);  // [n_eps][d]
   const int n_eps = p * p * c_in;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) {
-    s_shift[c] = table_f[c] + temb[c];
-    s_scale[c] = table_f[d + c] + temb[c];
+  // every load of a thread is issued before its first store (a loop of
+  // dependent load / store pairs would wait one memory round trip each)
+  {
+    constexpr int NC = (FIN_MAXV * 128 + FIN_WARPS * 32 - 1) / (FIN_WARPS * 32);
+    float a[NC], b[NC], e[NC];
+#pragma unroll
+    for (int j = 0; j < NC; ++j) {
+      const int c = threadIdx.x + j * FIN_WARPS * 32;
+      if (c < d) {
+        a[j] = table_f[c];
+        b[j] = table_f[d + c];
+        e[j] = temb[c];
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < NC; ++j) {
+      const int c = threadIdx.x + j * FIN_WARPS * 32;
+      if (c < d) {
+        s_shift[c] = a[j] + e[j];
+        s_scale[c] = b[j] + e[j];
+      }
+    }
   }
   // the eps rows of W_f, 16 bytes per thread and step (d % 8 == 0)
   const int d8 = d / 8;
-  for (int v = threadIdx.x; v < n_eps * d8; v += blockDim.x) {
-    const int e = v / d8, c8 = v - e * d8;
-    const int sub = e / c_in, ch = e - sub * c_in;
-    reinterpret_cast<uint4*>(s_w + size_t(e) * d)[c8] =
-        __ldg(reinterpret_cast<const uint4*>(Wf + size_t(sub * c_out + ch) * d) + c8);
+  {
+    constexpr int NW = (FIN_MAXO * FIN_MAXV * 16 + FIN_WARPS * 32 - 1) / (FIN_WARPS * 32);
+    uint4 t[NW];
+#pragma unroll
+    for (int j = 0; j < NW; ++j) {
+      const int v = threadIdx.x + j * FIN_WARPS * 32;
+      if (v < n_eps * d8) {
+        const int e = v / d8, c8 = v - e * d8;
+        const int sub = e / c_in, ch = e - sub * c_in;
+        t[j] = __ldg(reinterpret_cast<const uint4*>(Wf + size_t(sub * c_out + ch) * d) + c8);
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < NW; ++j) {
+      const int v = threadIdx.x + j * FIN_WARPS * 32;
+      if (v < n_eps * d8) {
+        const int e = v / d8, c8 = v - e * d8;
+        reinterpret_cast<uint4*>(s_w + size_t(e) * d)[c8] = t[j];
+      }
+    }
   }
   pdl_wait();
   pdl_trigger();
@@ -643,9 +723,12 @@ cudaError_t launch_final_ddim(const bf16* H, const float* temb, const float* tab
     attr_set = true;
   }
   const int N = gh * gw;
-  // a warp per token: the per-token reductions are latency-bound chains
+  // a warp per token (grid-stride): the per-token reductions are
+  // latency-bound chains.  One wave of CTAs (two fit an SM by their
+  // registers), so that each SM stages W_f and the modulation once per CTA
+  // it holds rather than once per token group
   int grid = cdiv(N, FIN_WARPS);
-  const int cap = 8 * device_sm_count();
+  const int cap = 2 * device_sm_count();
   if (grid > cap) grid = cap;
   RC_TRY(launch_k(final_ddim_kernel, dim3(grid), dim3(FIN_WARPS * 32), smem, st, H, temb, table_f,
                   Wf, bf, latent, gh, gw, p, c_in, c_out, d, ab_t, ab_next));
