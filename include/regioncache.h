@@ -121,6 +121,12 @@ void rc_destroy(rc_ctx* ctx);
  * cache of this context stale, and steps of a session return RC_ERR_STATE
  * until rc_set_text (or rc_cache_import) runs for it again. */
 rc_status rc_set_layer_weights(rc_ctx* ctx, int layer, const rc_layer_weights* w);
+/* The timestep embedding and t_block modulation of every scheduled timestep
+ * depend only on W_t1 .. b_tb and the schedule: they are computed once, at
+ * the first step or graph capture after rc_set_global_weights or
+ * rc_set_schedule, and reused by every later step.  Weights changed in place
+ * therefore need rc_set_global_weights again.  (A step captured by the
+ * caller into a graph before they exist computes its own.) */
 rc_status rc_set_global_weights(rc_ctx* ctx, const rc_global_weights* w);
 
 /* Sampling schedule, copied: timestep values t_values_host[timesteps] fed to

@@ -80,6 +80,12 @@ struct rc_ctx {
   float* h1 = nullptr;   // [d]
   float* temb = nullptr; // [RC_MAX_BATCH][d] timestep embedding per item
   float* tb = nullptr;   // [RC_MAX_BATCH][6d] t_block modulation per item
+  // the same for every scheduled timestep, [T][d] and [T][6d]: they depend
+  // only on the global weights and the schedule, so they are computed once
+  // (t_ready) and reused by every step
+  float* temb_tab = nullptr;
+  float* tb_tab = nullptr;
+  bool t_ready = false;
   int* iota = nullptr;   // [N] identity row map (dense path)
   int* b_tok = nullptr;  // [R] token of each compact row (batched steps)
   int* b_item = nullptr; // [R] item of each compact row (batched steps)
@@ -224,7 +230,7 @@ void free_ctx(rc_ctx* c) {
   probe_free(c);
   void* ps[] = {c->xf,   c->xb,   c->ob,   c->q,    c->u,      c->fbuf,
                 c->h1,   c->temb, c->tb,   c->iota, c->b_tok,  c->b_item,
-                c->b_meta, c->err, c->wait_flag, c->as.part};
+                c->b_meta, c->err, c->wait_flag, c->as.part, c->temb_tab, c->tb_tab};
   for (void* p : ps)
     if (p) cudaFree(p);
   delete c;
@@ -503,6 +509,8 @@ rc_status rc_create(const rc_dims* dims, rc_ctx** out) {
       (s = dalloc(&c->h1, D.hidden, "h1")) ||
       (s = dalloc(&c->temb, size_t(RC_MAX_BATCH) * D.hidden, "temb")) ||
       (s = dalloc(&c->tb, size_t(RC_MAX_BATCH) * 6 * D.hidden, "tb")) ||
+      (s = dalloc(&c->temb_tab, size_t(D.timesteps) * D.hidden, "temb table")) ||
+      (s = dalloc(&c->tb_tab, size_t(D.timesteps) * 6 * D.hidden, "tb table")) ||
       (s = dalloc(&c->iota, N, "iota")) || (s = dalloc(&c->b_tok, R, "batch tok")) ||
       (s = dalloc(&c->b_item, R, "batch item")) ||
       (s = dalloc(&c->b_meta, size_t(rc::META_INTS), "batch meta")) ||
@@ -554,6 +562,7 @@ rc_status rc_set_global_weights(rc_ctx* c, const rc_global_weights* w) {
       return fail(RC_ERR_INVALID_ARG, "global weights: null or unaligned (16 B) pointer");
   c->gw = *w;
   c->gw_set = true;
+  c->t_ready = false;
   return RC_OK;
 }
 
@@ -565,6 +574,7 @@ rc_status rc_set_schedule(rc_ctx* c, const float* tv, const float* ab) {
   c->t_values.assign(tv, tv + c->T);
   c->alpha_bar.assign(ab, ab + c->T + 1);
   c->sched_set = true;
+  c->t_ready = false;
   return RC_OK;
 }
 
@@ -1003,6 +1013,24 @@ static rc_status host_writeback(rc_ctx* c, rc_cache* k, int s, int t, int l,
   return RC_OK;
 }
 
+// The timestep embedding and t_block modulation of every scheduled timestep
+// into temb_tab / tb_tab, queued on st, when the global weights or the
+// schedule changed since they were last computed.
+static rc_status fill_t_tables(rc_ctx* c, cudaStream_t st) {
+  if (c->t_ready) return RC_OK;
+  const rc_global_weights& g = c->gw;
+  const int d = c->d;
+  for (int t = 0; t < c->T; ++t)
+    RC_CUDA(rc::launch_t_embed(c->t_values[t], c->dims.freq_dim, d,
+                               static_cast<const bf16*>(g.W_t1), g.b_t1,
+                               static_cast<const bf16*>(g.W_t2), g.b_t2,
+                               static_cast<const bf16*>(g.W_tb), g.b_tb, c->fbuf, c->h1,
+                               c->temb_tab + size_t(t) * d, c->tb_tab + size_t(t) * 6 * d, st),
+            "t_embed");
+  c->t_ready = true;
+  return RC_OK;
+}
+
 // Denoising steps of n items (validated by the callers); cap (DENSE single
 // item only) captures cross-attention probabilities of listed text tokens.
 // On a host-tier cache (one item) the layers run on HBM windows while the
@@ -1017,12 +1045,27 @@ static rc_status step_items(rc_ctx* c, rc_cache* k, const rc_batch_item* items, 
   rc::BatchIn bin{};
   bin.n = n;
   long long rows = 0;
+  // the per-timestep tables, unless this stream is being captured before
+  // they exist (a capture by the caller: the step then computes its items'
+  // embeddings itself, as part of the captured work)
+  bool tables = c->t_ready;
+  if (!tables) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    RC_CUDA(cudaStreamIsCapturing(st, &cs), "capture status");
+    if (cs == cudaStreamCaptureStatusNone) {
+      rc_status r = fill_t_tables(c, st);
+      if (r) return r;
+      tables = true;
+    }
+  }
+  const float* temb_of[rc::MAX_ITEMS] = {};
   for (int i = 0; i < n; ++i) {
     const rc_batch_item& it = items[i];
     si.session[i] = it.session;
     si.t[i] = it.t;
     si.its.slice[i] = k->slot(it.session, 0, it.t, 0);
-    si.its.tb[i] = c->tb + size_t(i) * 6 * d;
+    si.its.tb[i] = tables ? c->tb_tab + size_t(it.t) * 6 * d : c->tb + size_t(i) * 6 * d;
+    temb_of[i] = tables ? c->temb_tab + size_t(it.t) * d : c->temb + size_t(i) * d;
     si.its.latent[i] = it.latent;
     if (it.mode == RC_MODE_DENSE) {
       bin.idx[i] = c->iota;
@@ -1033,12 +1076,13 @@ static rc_status step_items(rc_ctx* c, rc_cache* k, const rc_batch_item* items, 
       bin.bound[i] = it.D < 0 ? N : it.D;
     }
     rows += bin.bound[i];
-    RC_CUDA(rc::launch_t_embed(c->t_values[it.t], c->dims.freq_dim, d,
-                               static_cast<const bf16*>(g.W_t1), g.b_t1,
-                               static_cast<const bf16*>(g.W_t2), g.b_t2,
-                               static_cast<const bf16*>(g.W_tb), g.b_tb, c->fbuf, c->h1,
-                               c->temb + size_t(i) * d, c->tb + size_t(i) * 6 * d, st),
-            "t_embed");
+    if (!tables)
+      RC_CUDA(rc::launch_t_embed(c->t_values[it.t], c->dims.freq_dim, d,
+                                 static_cast<const bf16*>(g.W_t1), g.b_t1,
+                                 static_cast<const bf16*>(g.W_t2), g.b_t2,
+                                 static_cast<const bf16*>(g.W_tb), g.b_tb, c->fbuf, c->h1,
+                                 c->temb + size_t(i) * d, c->tb + size_t(i) * 6 * d, st),
+              "t_embed");
   }
   const bool host = k->host_tier;
   const int s0 = items[0].session, t0 = items[0].t, L = c->L;
@@ -1107,7 +1151,7 @@ static rc_status step_items(rc_ctx* c, rc_cache* k, const rc_batch_item* items, 
   for (int i = 0; i < n; ++i) {
     const rc_batch_item& it = items[i];
     RC_CUDA(rc::launch_final_ddim(host ? win_last : k->slot(it.session, L - 1, it.t, 0),
-                                  c->temb + size_t(i) * d,
+                                  temb_of[i],
                                   g.table_f, static_cast<const bf16*>(g.W_f), g.b_f, it.latent,
                                   c->dims.grid_h, c->dims.grid_w, c->dims.patch, c->dims.in_ch,
                                   c->dims.out_ch, d, c->alpha_bar[it.t], c->alpha_bar[it.t + 1],
@@ -1187,6 +1231,15 @@ rc_status rc_step_graph_create(rc_ctx* c, rc_cache* k, int s, float* latent, int
   if (e != cudaSuccess) {
     delete gr;
     return cuda_fail(e, "capture stream");
+  }
+  // the per-timestep embedding tables first, outside the capture, so that
+  // replays read them instead of recomputing them
+  r = fill_t_tables(c, cs);
+  if (r == RC_OK && (e = cudaStreamSynchronize(cs)) != cudaSuccess) r = cuda_fail(e, "t tables");
+  if (r != RC_OK) {
+    cudaStreamDestroy(cs);
+    delete gr;
+    return r;
   }
   const uint64_t n0 = rc_launch_count();
   e = cudaStreamBeginCapture(cs, cudaStreamCaptureModeRelaxed);
