@@ -314,6 +314,33 @@ def test_step_parity_small(R, step_problem, mode):
     _reset(R, p, t)
 
 
+def test_step_after_schedule_change(R, step_problem):
+    """The per-timestep embeddings are computed once per schedule: after
+    rc_set_schedule with other timestep values, a step uses the new ones."""
+    p = step_problem
+    t = 3
+    lat = synth.make_latent(p.d, p.seed)
+    idx = np.flatnonzero(synth.rectangle_mask(p.d, p.seed))
+    _reset(R, p, t)
+    _gpu_step(R, p, lat, t, O.MODE_SPARSE, idx)  # embeddings of the first schedule
+    tv0 = p.tv
+    tv1 = (np.float32(999.0) - tv0).astype(np.float32)  # the schedule reversed
+    ref0, _, _ = p.oracle_step(O.to64(lat), t, O.MODE_SPARSE, idx)
+    try:
+        R.rc_set_schedule(p.model.ctx, tv1, p.ab)
+        p.tv = tv1
+        _reset(R, p, t)
+        got = _gpu_step(R, p, lat, t, O.MODE_SPARSE, idx)
+        ref, _, _ = p.oracle_step(O.to64(lat), t, O.MODE_SPARSE, idx)
+        # the two schedules give results far apart, so stale embeddings fail
+        assert rel_l2(ref0, ref) > 2 * LATENT_REL_L2
+        assert rel_l2(got, ref) <= LATENT_REL_L2
+    finally:
+        R.rc_set_schedule(p.model.ctx, tv0, p.ab)
+        p.tv = tv0
+        _reset(R, p, t)
+
+
 @pytest.fixture(scope="module")
 def c2_problem(R):
     p = Problem(R, synth.PIXART_512, 1234 + 200, ts=(5,))
