@@ -413,7 +413,12 @@ rc_status rc_reuse_schedule(float s, float tau_s, float rho, int T, uint8_t* mod
  * dirty_count contents (use D = -1 with a device count whose bound is N).
  * Mode schedule_host[t] and the host bound D are fixed at creation.  The
  * graph reuses the context's scratch: replays of graphs of one context are
- * serialised on one stream, like its steps.  Creation enqueues nothing.
+ * serialised on one stream, like its steps.  Creation enqueues nothing on
+ * the caller's streams; when the per-timestep embedding tables are stale
+ * (see rc_set_global_weights) it computes them first, on a private stream
+ * that it waits for.  A replay reads those tables but keeps the DDIM
+ * coefficients of the schedule at creation: create graphs again after
+ * rc_set_schedule or rc_set_global_weights.
  * Errors: as rc_step; RC_ERR_INVALID_ARG for a host-tier cache or while a
  * timing probe is enabled; RC_ERR_CUDA when capture or instantiation fails. */
 typedef struct rc_graph rc_graph;
