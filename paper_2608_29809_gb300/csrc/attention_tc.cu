@@ -135,9 +135,20 @@ __device__ __forceinline__ int query_tiles(const RowMap& rm, int n_items, int D)
 // results (unnormalised O, row max and sum) that the combine kernel merges.
 // With fewer key blocks (the text cross-attention) every pair is one unit,
 // handed out round-robin.
+//
+// G: as many CTAs as the grid holds (at least MIN_KB_PER_SPLIT key blocks
+// each), unless ranges of r key blocks, r a power of two dividing the pair's
+// count, cost less: then every CTA holds exactly one piece of one pair.  The
+// estimate is the busiest CTA's key blocks plus PIECE_COST per piece it
+// holds (a piece costs a Q load, a drained O and a stored partial; the equal
+// cut leaves most CTAs two).  Measured on the 4096-token step: at 205 dirty
+// queries (2048 key blocks) 304 ranges of 6-7 blocks gave 441 steps/s, 256
+// of 8 blocks 460; at 410 (4096 key blocks) 304 of 13-14 gave 363, 256 of 16
+// gave 389; from 831 queries on, the equal cut stays.
 struct AttnSched {
   int qtiles, pairs, nkb, G, total;
   bool streamk;
+  static constexpr int PIECE_COST = 4;  // key blocks
   __device__ void init(int tiles, int heads, int Nk, int grid) {
     qtiles = tiles;
     pairs = qtiles * heads;
@@ -145,7 +156,23 @@ struct AttnSched {
     total = pairs * nkb;
     streamk = nkb >= 2 * MIN_KB_PER_SPLIT;
     G = grid;
-    if (streamk) G = max(1, min(grid, total / MIN_KB_PER_SPLIT));
+    if (!streamk) return;
+    G = pick_ctas(total, nkb, grid);
+  }
+  // (powers of two only, found with shifts: every thread of the attention
+  // and combine kernels runs this before its first load, and a search with
+  // run-time divisors cost more than the better ranges saved; not inlined,
+  // so that its temporaries do not raise the kernels' register counts)
+  static __device__ __noinline__ int pick_ctas(int total, int nkb, int grid) {
+    const int G = max(1, min(grid, total / MIN_KB_PER_SPLIT));
+    if (nkb & (nkb - 1)) return G;
+    int lg = 0;
+    while ((1 << lg) < MIN_KB_PER_SPLIT) ++lg;
+    while ((1 << lg) < nkb && (total >> lg) > grid) ++lg;
+    if ((1 << lg) > nkb || (total >> lg) > grid) return G;
+    const int r0 = (total + G - 1) / G;
+    const bool one_piece = total % G == 0 && nkb % r0 == 0;
+    return (1 << lg) + PIECE_COST < r0 + PIECE_COST * (one_piece ? 1 : 2) ? total >> lg : G;
   }
   // unsigned 32-bit arithmetic: the launcher checks total * G < 2^32
   __device__ int bound(int c) const { return int(unsigned(total) * unsigned(c) / unsigned(G)); }
