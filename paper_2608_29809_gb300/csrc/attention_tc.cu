@@ -49,7 +49,10 @@ using namespace rc::tc;
 constexpr int BQ = 128, BKV = 64, THREADS = 192;
 constexpr int TMEM_COLS = 256;     // S0 | S1 (64 columns each) | O (80) | P (32)
 constexpr int CTAS_PER_SM = 2;
-constexpr int PART_STRIDE = 76;    // floats per row of a split's partial result
+// floats per row of a workspace slot: a piece's DH columns, its row max and
+// sum (stored as column planes, see attn_combine_kernel)
+constexpr int PART_STRIDE = 76;
+static_assert(72 + 2 <= PART_STRIDE, "a slot holds DH + 2 floats per row");
 constexpr float LAZY_RESCALE = 8.f;
 constexpr int MIN_KB_PER_SPLIT = 4;  // key blocks per CTA range, at least
 
@@ -596,14 +599,15 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
       } else {
         // a piece of the pair's keys: unnormalised O with its row max and
         // sum; the combine kernel merges the pieces
-        float* mine = part + (size_t(blockIdx.x) * 2 + slot) * (BQ * PART_STRIDE) +
-                      size_t(row) * PART_STRIDE;
+        // (the workspace slot's planes: column group c4 of every row, then
+        // the rows' (max, sum); a warp's stores are whole 512-byte runs)
+        float* mine = part + (size_t(blockIdx.x) * 2 + slot) * (BQ * PART_STRIDE);
 #pragma unroll
         for (int c4 = 0; c4 < DH / 4; ++c4)
-          __stcg(reinterpret_cast<float4*>(mine) + c4,
+          __stcg(reinterpret_cast<float4*>(mine) + c4 * BQ + row,
                  make_float4(__uint_as_float(o[4 * c4]), __uint_as_float(o[4 * c4 + 1]),
                              __uint_as_float(o[4 * c4 + 2]), __uint_as_float(o[4 * c4 + 3])));
-        __stcg(reinterpret_cast<float2*>(mine + DH), make_float2(m, l));
+        __stcg(reinterpret_cast<float2*>(mine + DH * BQ) + row, make_float2(m, l));
       }
     }
   }
@@ -1145,27 +1149,21 @@ xf_done:
   }
 }
 
-// Merge of the pieces of the pairs that stream-K cut.  The (pair, query row)
-// sequence is cut into equal contiguous runs, one per warp, so a warp's rows
-// mostly share one pair and its bookkeeping (which CTAs hold its pieces,
-// which workspace slot) is worked out once per pair.  The pieces of a pair
+// Merge of the pieces of the pairs that stream-K cut.  The pieces of a pair
 // come from CTAs cta_of(first block) .. cta_of(last block); a CTA's piece is
 // its first (slot 0) when its range starts inside the pair, else its last
-// (slot 1).  Per row, lanes take the pieces' row max / sum in turn, the warp
-// reduces them, and lanes < DH / 4 accumulate 4 head-dim columns each over
-// the pieces.  With at most four pieces (the usual case) a row's loads go
-// out in one round, and the next row's before the current one is reduced.
+// (slot 1).  A workspace slot holds its piece as DH / 4 planes of 128 float4
+// (head-dim columns 4 c .. 4 c + 3 of the tile's rows), then the rows' (max,
+// sum) pairs, so that the attention kernel's softmax threads (one row each)
+// and this kernel's lanes (one row each) access whole 512-byte runs.  A work
+// unit is 32 consecutive rows of one cut pair and COMBINE_CH of the column
+// planes; units go to warps in turn.  Per row: the largest of the pieces'
+// maxima M, then the pieces' columns weighted by 2^(m_q - M), over the
+// weighted sums, stored as bf16.  Each of the two passes keeps several
+// pieces' loads in flight.
+constexpr int COMBINE_THREADS = 256, COMBINE_CH = 3;
 template <int DH>
-struct CombineRow {
-  float2 ml;     // lane q < np: piece q's row max / sum
-  float4 v[4];   // lanes < DH / 4: pieces 0..3, head-dim columns 4 lane ..
-  int qrow;      // output row; -1: nothing to do
-  int h;         // head
-  bool many;     // more than four pieces: the general path
-};
-
-template <int DH>
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(COMBINE_THREADS, 2)
 attn_combine_kernel(const float* __restrict__ part, bf16* __restrict__ O, int ldo, int heads,
                     RowMap rm, int n_items, int Nk, int attn_grid, unsigned* err) {
   // the row count predates the attention launch (see attn_tc_kernel): read
@@ -1176,112 +1174,61 @@ attn_combine_kernel(const float* __restrict__ part, bf16* __restrict__ O, int ld
   pdl_wait();
   pdl_trigger();
   if (!sc.streamk) return;
+  constexpr int C4 = DH / 4, NCH = (C4 + COMBINE_CH - 1) / COMBINE_CH;
+  constexpr int PER_PAIR = (BQ / 32) * NCH;  // units of one pair
   const int lane = threadIdx.x & 31;
-  const int total = sc.pairs * BQ;
-  const int nwarps = int(gridDim.x) * 8;
-  const int per = (total + nwarps - 1) / nwarps;
-  const int w = int(blockIdx.x) * 8 + (int(threadIdx.x) >> 5);
-  const int r0 = w * per, r1 = min(total, r0 + per);
-  // bookkeeping of the current pair
-  int cpair = -1, c_lo = 0, np = 0, slot_lo = 0, h = 0;
-  TileLoc tl{0, 0, 0};
-  auto piece = [&](int q, int row) {
-    const int c = c_lo + q;
-    return part + (size_t(c) * 2 + (q == 0 ? slot_lo : 0)) * (BQ * PART_STRIDE) +
-           size_t(row) * PART_STRIDE;
-  };
-  auto prep = [&](int gw, CombineRow<DH>& cr) {
-    cr.qrow = -1;
-    cr.many = false;
-    if (gw >= r1) return;
-    const int pair = gw / BQ, row = gw - pair * BQ;
-    if (pair != cpair) {
-      cpair = pair;
-      const int lo = pair * sc.nkb;
-      c_lo = sc.cta_of(lo);
-      np = sc.cta_of(lo + sc.nkb - 1) - c_lo + 1;
-      slot_lo = sc.bound(c_lo) == lo ? 0 : 1;
-      const int qt = pair % sc.qtiles;
-      h = pair / sc.qtiles;
-      tl = locate_tile(rm, n_items, D, qt);
-    }
-    if (np == 1 || row >= tl.rows) return;  // one CTA held the whole pair
-    cr.qrow = tl.row0 + row;
-    cr.h = h;
-    if (np > 4) {
-      cr.many = true;
-      return;
-    }
-    cr.ml = lane < np ? __ldcg(reinterpret_cast<const float2*>(piece(lane, row) + DH))
-                      : make_float2(-INFINITY, 0.f);
+  const int units = sc.pairs * PER_PAIR;
+  const int nwarps = int(gridDim.x) * (COMBINE_THREADS / 32);
+  for (int u = int(blockIdx.x) * (COMBINE_THREADS / 32) + (int(threadIdx.x) >> 5); u < units;
+       u += nwarps) {
+    const int pair = u / PER_PAIR, rest = u - pair * PER_PAIR;
+    const int row = (rest / NCH) * 32 + lane, c0 = (rest - (rest / NCH) * NCH) * COMBINE_CH;
+    const int lo = pair * sc.nkb;
+    const int c_lo = sc.cta_of(lo);
+    const int np = sc.cta_of(lo + sc.nkb - 1) - c_lo + 1;
+    if (np == 1) continue;  // one CTA held the whole pair (warp-uniform)
+    const int slot_lo = sc.bound(c_lo) == lo ? 0 : 1;
+    const TileLoc tl = locate_tile(rm, n_items, D, pair % sc.qtiles);
+    const int h = pair / sc.qtiles;
+    auto slot = [&](int q) {
+      return part + (size_t(c_lo + q) * 2 + (q == 0 ? slot_lo : 0)) * (BQ * PART_STRIDE);
+    };
+    float M = -INFINITY;
+#pragma unroll 8
+    for (int q = 0; q < np; ++q)
+      M = fmaxf(M, __ldcg(reinterpret_cast<const float2*>(slot(q) + DH * BQ) + row).x);
+    float L = 0.f;
+    float4 acc[COMBINE_CH];
 #pragma unroll
-    for (int e = 0; e < 4; ++e)
-      cr.v[e] = (e < np && lane < DH / 4)
-                    ? __ldcg(reinterpret_cast<const float4*>(piece(e, row)) + lane)
-                    : make_float4(0.f, 0.f, 0.f, 0.f);
-  };
-  auto store = [&](int qrow, int hh, float4 acc, float L) {
-    if (lane < DH / 4) {
+    for (int c = 0; c < COMBINE_CH; ++c) acc[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+    for (int q = 0; q < np; ++q) {
+      const float* b = slot(q);
+      const float2 ml = __ldcg(reinterpret_cast<const float2*>(b + DH * BQ) + row);
+      float4 v[COMBINE_CH];
+#pragma unroll
+      for (int c = 0; c < COMBINE_CH; ++c)
+        if (c0 + c < C4) v[c] = __ldcg(reinterpret_cast<const float4*>(b) + (c0 + c) * BQ + row);
+      const float wq = ex2_ftz(ml.x - M);
+      L += wq * ml.y;
+#pragma unroll
+      for (int c = 0; c < COMBINE_CH; ++c)
+        if (c0 + c < C4) {
+          acc[c].x += wq * v[c].x;
+          acc[c].y += wq * v[c].y;
+          acc[c].z += wq * v[c].z;
+          acc[c].w += wq * v[c].w;
+        }
+    }
+    if (row < tl.rows) {
       const float inv = L > 0.f ? 1.f / L : 0.f;
-      *reinterpret_cast<uint2*>(O + size_t(qrow) * ldo + hh * DH + 4 * lane) = make_uint2(
-          pack_bf16x2(acc.x * inv, acc.y * inv), pack_bf16x2(acc.z * inv, acc.w * inv));
+      uint2* dst = reinterpret_cast<uint2*>(O + size_t(tl.row0 + row) * ldo + h * DH) + c0;
+#pragma unroll
+      for (int c = 0; c < COMBINE_CH; ++c)
+        if (c0 + c < C4)
+          dst[c] = make_uint2(pack_bf16x2(acc[c].x * inv, acc[c].y * inv),
+                              pack_bf16x2(acc[c].z * inv, acc[c].w * inv));
     }
-  };
-  CombineRow<DH> cur, nxt;
-  prep(r0, cur);
-  for (int gw = r0; gw < r1; ++gw) {
-    const int np_cur = np;  // (prep of the next row may move to the next pair)
-    const int row_cur = gw - (gw / BQ) * BQ;
-    if (cur.many) {
-      // many pieces (very long key ranges): plain loops, no prefetch
-      float M = -INFINITY;
-      for (int q = lane; q < np_cur; q += 32) M = fmaxf(M, __ldcg(piece(q, row_cur) + DH));
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-      float L = 0.f;
-      for (int q = lane; q < np_cur; q += 32) {
-        const float2 ml = __ldcg(reinterpret_cast<const float2*>(piece(q, row_cur) + DH));
-        L += ex2_ftz(ml.x - M) * ml.y;
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (lane < DH / 4) {
-        for (int q = 0; q < np_cur; ++q) {
-          const float* b = piece(q, row_cur);
-          const float wq = ex2_ftz(__ldcg(b + DH) - M);
-          const float4 v = __ldcg(reinterpret_cast<const float4*>(b) + lane);
-          acc.x += wq * v.x;
-          acc.y += wq * v.y;
-          acc.z += wq * v.z;
-          acc.w += wq * v.w;
-        }
-      }
-      store(cur.qrow, cur.h, acc, L);
-      prep(gw + 1, nxt);
-    } else {
-      prep(gw + 1, nxt);  // the next row's loads go out before this row's reduction
-      if (cur.qrow >= 0) {
-        float M = cur.ml.x;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-        const float wl = lane < np_cur ? ex2_ftz(cur.ml.x - M) : 0.f;
-        float L = wl * cur.ml.y;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float ww = e < np_cur ? __shfl_sync(0xffffffffu, wl, e) : 0.f;
-          acc.x += ww * cur.v[e].x;
-          acc.y += ww * cur.v[e].y;
-          acc.z += ww * cur.v[e].z;
-          acc.w += ww * cur.v[e].w;
-        }
-        store(cur.qrow, cur.h, acc, L);
-      }
-    }
-    cur = nxt;
   }
 }
 
@@ -1464,14 +1411,15 @@ cudaError_t launch_attention(const bf16* Q, int ldq, const bf16* K, const bf16* 
   // stream-K (and so partial pieces) only with at least 2 MIN_KB_PER_SPLIT key blocks
   if ((Nk + BKV - 1) / BKV >= 2 * MIN_KB_PER_SPLIT) {
     const int tiles = (rm.bound + BQ - 1) / BQ + ai.n - 1;  // bound of the query tiles
-    const int warps = tiles * heads * BQ;
-    const int cgrid = min((warps + 7) / 8, 4 * sms);
+    // units of 32 rows and COMBINE_CH column planes of a pair
+    const int units = tiles * heads * (BQ / 32) * ((dh / 4 + COMBINE_CH - 1) / COMBINE_CH);
+    const int cgrid = min((units + COMBINE_THREADS / 32 - 1) / (COMBINE_THREADS / 32), 2 * sms);
     if (dh == 72)
-      RC_TRY(launch_k(attn_combine_kernel<72>, dim3(cgrid), dim3(256), 0, st, as.part, O,
-                      ldo, heads, rm, ai.n, Nk, grid, err));
+      RC_TRY(launch_k(attn_combine_kernel<72>, dim3(cgrid), dim3(COMBINE_THREADS), 0, st,
+                      as.part, O, ldo, heads, rm, ai.n, Nk, grid, err));
     else
-      RC_TRY(launch_k(attn_combine_kernel<64>, dim3(cgrid), dim3(256), 0, st, as.part, O,
-                      ldo, heads, rm, ai.n, Nk, grid, err));
+      RC_TRY(launch_k(attn_combine_kernel<64>, dim3(cgrid), dim3(COMBINE_THREADS), 0, st,
+                      as.part, O, ldo, heads, rm, ai.n, Nk, grid, err));
     count_launches(1);
   }
   return cudaSuccess;
