@@ -27,8 +27,9 @@
 // Two CTAs share an SM (256 TMEM columns and ~100 KB of shared memory each),
 // so the softmax of one overlaps the MMAs and exponentials of the other.
 // Key splits of the same (query tile, head) leave their unnormalised O and
-// row max / sum in a workspace; a small combine kernel, launched right after,
-// merges them (one warp per row, coalesced).
+// row max / sum in a workspace (as column planes, so that the softmax
+// threads' stores are whole 512-byte runs); a small combine kernel, launched
+// right after, merges them (one lane per row).
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <math.h>
